@@ -1,0 +1,150 @@
+/*
+ * grkv.h — C ABI of the GRKV prefill-time KV-cache compression path.
+ *
+ * GRKV (arXiv 2605.31105) compresses each layer's KV cache right after its
+ * prefill.  For every *unit* (one layer x KV head of one sequence) the path:
+ *   1. scores every cached key with the window queries (the last w prompt
+ *      queries, Sec. 3.2, Eq. 4): softmax(Q_win K^T / sqrt(d));
+ *   2. keeps the B - w keys with the best span-pooled score plus the window
+ *      (SnapKV-style span retention, Sec. 1-2);
+ *   3. forms the full-cache target Y = A_win^full V_full (Algorithm 1);
+ *   4. runs GRKV's value step: the ridge regression of Eq. 6 solved in dual
+ *      (Woodbury) form, Sec. 3.4 and App. D.1, over the free retained tokens
+ *      (fixed tokens, Sec. 3.4 and App. D.3, stay as they are).
+ *
+ * Units are independent.  Query heads are grouped onto their KV head (GQA):
+ * the g query heads that read one KV head stack their w window rows into
+ * m = g*w rows r = h*w + a; window slot a sits at position n - w + a.
+ *
+ * Layouts (row-major, contiguous, `dtype` elements unless stated):
+ *   q        [U][g][w][d]      window queries
+ *   k, v     [U][n][d]         full key / value caches
+ *   scores   [U][n-w]  fp32    per-key prefix score c_j = sum_r A_rj
+ *   y        [U][m][d] fp32    target Y
+ *   row_stats[U][m][2] fp32    (M_r, L_r): row max of the logits and
+ *                              sum_j exp(l_rj - M_r)
+ *   idx      [U][B]    int32   retained positions, ascending; the last w are
+ *                              the window n-w..n-1
+ *   k_out, v_out [U][B][d]     compressed cache
+ *
+ * Ownership and ordering: every pointer except `params` and the output
+ * `bytes` / `device_status` is DEVICE memory owned by the caller.  The
+ * library allocates nothing, keeps no pointer after a call returns, and
+ * enqueues all work asynchronously on `stream` (a cudaStream_t passed as
+ * void*, NULL = legacy default stream).  Device pointers must be 16-byte
+ * aligned.  Nothing is written if host-side validation fails.
+ *
+ * Errors: calls return GRKV_OK (0) or a negative code.  Host-detected errors
+ * are returned directly.  Errors found on the device (a non-positive Cholesky
+ * pivot, an expired bounded wait) are written to a status word at the start
+ * of the workspace; every call clears that word first, so it reports the
+ * most recent call; read it with grkv_status().
+ */
+#ifndef GRKV_H
+#define GRKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define GRKV_OK                       0
+#define GRKV_ERR_INVALID_ARG         -1  /* a parameter is out of range         */
+#define GRKV_ERR_UNSUPPORTED         -2  /* valid but not implemented (d != 128) */
+#define GRKV_ERR_WORKSPACE_TOO_SMALL -3
+#define GRKV_ERR_MISALIGNED          -4  /* a device pointer is not 16-B aligned */
+#define GRKV_ERR_CUDA                -5  /* a CUDA call or launch failed          */
+#define GRKV_ERR_NUMERIC             -6  /* device: Cholesky pivot <= 0 (lambda ~ 0) */
+#define GRKV_ERR_TIMEOUT             -7  /* device: a bounded wait expired        */
+
+#define GRKV_F32  0
+#define GRKV_BF16 1
+
+#define GRKV_POOL_MAX 0
+#define GRKV_POOL_AVG 1
+
+#define GRKV_UPDATE_K      0x1u  /* key step (Sec. 3.4, Eq. key_dual_update): not implemented */
+#define GRKV_FORCE_SIMT    0x2u  /* use the portable CUDA-core kernels even for bf16 */
+
+typedef struct {
+  int32_t units;        /* U >= 0: independent (batch x layer x KV head) problems   */
+  int32_t group;        /* g >= 1: query heads per KV head                          */
+  int32_t n;            /* context length, window included, n >= window             */
+  int32_t d;            /* head dimension; 128 only                                 */
+  int32_t window;       /* w >= 1: positions n-w..n-1, always retained              */
+  int32_t budget;       /* B: window <= B <= n, window included                     */
+  int32_t pool_kernel;  /* odd >= 1 (7)                                             */
+  int32_t pool_type;    /* GRKV_POOL_MAX (default) or GRKV_POOL_AVG                 */
+  int32_t n_sink;       /* >= 0: retained tokens j < n_sink stay fixed (4)          */
+  float   beta;         /* [0, 1): floor(beta*B) best-scored retained prefix
+                           tokens stay fixed (0.10)                                 */
+  float   lambda_v;     /* >= 0 (may be +inf: values unchanged): ridge weight of
+                           the value step, Eq. 6                                    */
+  float   lambda_k;     /* reserved for the key step                               */
+  float   scale;        /* logit scale; 0 -> fp32(1/sqrt(d))                        */
+  int32_t causal;       /* 1: window slot a sees keys j <= n-w+a; 0: all n keys      */
+  int32_t dtype;        /* GRKV_BF16 or GRKV_F32 for q, k, v, k_out, v_out          */
+  uint32_t flags;       /* GRKV_FORCE_SIMT; GRKV_UPDATE_K -> GRKV_ERR_UNSUPPORTED    */
+} grkv_params;
+
+/* Fills `p` with the defaults above for the given sizes (bf16, lambda 1e-2,
+ * max pool 7, 4 sinks, beta 0.10, causal). */
+void grkv_params_init(grkv_params* p, int32_t units, int32_t group, int32_t n,
+                      int32_t window, int32_t budget);
+
+/* Workspace bytes that every call below needs for `p` (the largest of them).
+ * Returns GRKV_ERR_INVALID_ARG / UNSUPPORTED like the calls would. */
+int grkv_workspace_size(const grkv_params* p, size_t* bytes);
+
+/* Steps 1 and 3: window attention statistics, prefix scores and target.
+ *   row_stats = (max_j l_rj, sum_j exp(l_rj - M_r)),  l_rj = scale * q_r.k_j
+ *   scores[j] = sum_r exp(l_rj - M_r) / L_r  for j < n - w  (Eq. 4, summed
+ *               over the window rows: SnapKV's aggregated window attention)
+ *   y         = A_win^full V_full                     (Algorithm 1, target Y) */
+int grkv_score(const grkv_params* p, const void* q, const void* k, const void* v,
+               float* scores, float* y, float* row_stats,
+               void* ws, size_t ws_bytes, void* stream);
+
+/* Step 2: pool the prefix scores with kernel `pool_kernel` (max over the
+ * in-range neighbours, or the zero-padded mean), keep the B - w largest
+ * (ties to the smaller position), sort them ascending and append the window. */
+int grkv_select(const grkv_params* p, const float* scores, int32_t* idx,
+                void* ws, size_t ws_bytes, void* stream);
+
+/* Step 4 given the retained set: gather K0 = K[idx], V0 = V[idx]; fixed set F
+ * = retained sinks + window + the floor(beta*B) retained prefix non-sink
+ * tokens with the largest scores[j] (ties to the smaller position); retained
+ * attention X = softmax(Q_win K0^T * scale) over the B retained keys;
+ *   R = Y - X V0,  Z = (X_G X_G^T + lambda_v I_m)^-1 R,
+ *   V_out[G] = V0[G] + X_G^T Z,  V_out[F] = V0[F],  K_out = K0
+ * (Algorithm 1 value step; App. D.1 dual form; App. D.3 fixed tokens).
+ * Outputs are rounded to `dtype` (round to nearest even). */
+int grkv_merge(const grkv_params* p, const void* q, const void* k, const void* v,
+               const float* scores, const float* y, const int32_t* idx,
+               void* k_out, void* v_out, void* ws, size_t ws_bytes, void* stream);
+
+/* The whole path: grkv_score, grkv_select and grkv_merge with every
+ * intermediate in the workspace.  Writes idx, k_out and v_out. */
+int grkv_compress(const grkv_params* p, const void* q, const void* k, const void* v,
+                  void* k_out, void* v_out, int32_t* idx,
+                  void* ws, size_t ws_bytes, void* stream);
+
+/* Synchronises `stream`, then stores in *device_status the device-side
+ * status of the most recent call that used `ws` (GRKV_OK, GRKV_ERR_NUMERIC or
+ * GRKV_ERR_TIMEOUT).  Returns GRKV_ERR_CUDA if the stream reports an error. */
+int grkv_status(const void* ws, int* device_status, void* stream);
+
+/* Static description of an error code. */
+const char* grkv_strerror(int code);
+
+/* Diagnostic with no counterpart in the paper: the number of CUDA kernels
+ * this library has enqueued in the calling process so far (all calls, all
+ * streams).  Lets a caller count the library's launches in a timed region. */
+uint64_t grkv_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* GRKV_H */

@@ -1,0 +1,251 @@
+// C ABI of the GRKV compression path: host-side validation, workspace plan
+// and the launch sequence of each entry point declared in grkv.h.
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+
+#include "grkv_internal.cuh"
+
+using namespace grkv;
+
+namespace {
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+int make_shape(const grkv_params* p, Shape* s) {
+  if (!p) return GRKV_ERR_INVALID_ARG;
+  if (p->units < 0 || p->group < 1 || p->window < 1 || p->n < p->window) return GRKV_ERR_INVALID_ARG;
+  if (p->budget < p->window || p->budget > p->n) return GRKV_ERR_INVALID_ARG;
+  if (p->pool_kernel < 1 || (p->pool_kernel & 1) == 0) return GRKV_ERR_INVALID_ARG;
+  if (p->pool_type != GRKV_POOL_MAX && p->pool_type != GRKV_POOL_AVG) return GRKV_ERR_INVALID_ARG;
+  if (p->n_sink < 0) return GRKV_ERR_INVALID_ARG;
+  if (!(p->beta >= 0.f && p->beta < 1.f)) return GRKV_ERR_INVALID_ARG;
+  if (!(p->lambda_v >= 0.f)) return GRKV_ERR_INVALID_ARG;          // rejects NaN
+  if (!(p->scale >= 0.f) || std::isinf(p->scale)) return GRKV_ERR_INVALID_ARG;
+  if (p->causal != 0 && p->causal != 1) return GRKV_ERR_INVALID_ARG;
+  if (p->dtype != GRKV_F32 && p->dtype != GRKV_BF16) return GRKV_ERR_INVALID_ARG;
+  if (p->flags & ~(GRKV_UPDATE_K | GRKV_FORCE_SIMT)) return GRKV_ERR_INVALID_ARG;
+  if (p->d < 1) return GRKV_ERR_INVALID_ARG;
+  if (p->flags & GRKV_UPDATE_K) return GRKV_ERR_UNSUPPORTED;
+  if (p->d != kD) return GRKV_ERR_UNSUPPORTED;
+  if ((int64_t)p->group * p->window > kMaxM) return GRKV_ERR_UNSUPPORTED;
+  if ((int64_t)p->n * kD > (int64_t)1 << 31) return GRKV_ERR_UNSUPPORTED;
+  s->U = p->units;
+  s->g = p->group;
+  s->n = p->n;
+  s->d = p->d;
+  s->w = p->window;
+  s->B = p->budget;
+  s->m = p->group * p->window;
+  s->P = p->n - p->window;
+  s->kk = p->budget - p->window;
+  s->pool_k = p->pool_kernel;
+  s->pool_type = p->pool_type;
+  s->n_sink = p->n_sink;
+  s->n_fix = (int)std::floor((double)p->beta * (double)p->budget);
+  s->causal = p->causal;
+  s->dtype = p->dtype;
+  s->lambda = p->lambda_v;
+  s->lambda_inf = std::isinf(p->lambda_v) ? 1 : 0;
+  s->scale = p->scale != 0.f ? p->scale : (float)(1.0 / std::sqrt((double)p->d));
+  return GRKV_OK;
+}
+
+int check_ws(const WsLayout& L, const void* ws, size_t ws_bytes) {
+  if (!ws) return GRKV_ERR_INVALID_ARG;
+  if (!aligned16(ws)) return GRKV_ERR_MISALIGNED;
+  if (ws_bytes < L.total) return GRKV_ERR_WORKSPACE_TOO_SMALL;
+  return GRKV_OK;
+}
+
+// Non-null (unless the array is empty) and 16-byte aligned.
+int check_ptr(const void* p, size_t elems) {
+  if (elems == 0) return GRKV_OK;
+  if (!p) return GRKV_ERR_INVALID_ARG;
+  return aligned16(p) ? GRKV_OK : GRKV_ERR_MISALIGNED;
+}
+
+int cuda_rc(cudaError_t e) { return e == cudaSuccess ? GRKV_OK : GRKV_ERR_CUDA; }
+
+#define GRKV_TRY(expr)            \
+  do {                            \
+    const int rc_ = (expr);       \
+    if (rc_ != GRKV_OK) return rc_; \
+  } while (0)
+
+int check_inputs(const Shape& s, const void* q, const void* k, const void* v) {
+  GRKV_TRY(check_ptr(q, (size_t)s.U * s.m));
+  GRKV_TRY(check_ptr(k, (size_t)s.U * s.n));
+  GRKV_TRY(check_ptr(v, (size_t)s.U * s.n));
+  return GRKV_OK;
+}
+
+}  // namespace
+
+namespace grkv {
+
+static std::atomic<uint64_t> g_launches{0};
+
+void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+
+WsLayout plan_workspace(const Shape& s) {
+  WsLayout L{};
+  const size_t U = (size_t)s.U, m = (size_t)s.m, d = (size_t)kD;
+  L.chunk = std::max(1024, ((s.n + 15) / 16 + 63) / 64 * 64);
+  L.nchunk = (s.n + L.chunk - 1) / L.chunk;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align256(off + bytes);
+    return at;
+  };
+  L.status = take(256);
+  L.pstats = take(U * L.nchunk * m * 8);
+  L.ypart = take(U * L.nchunk * m * d * 4);
+  L.pooled = take(U * (size_t)s.P * 4);
+  L.xbuf = take(U * m * (size_t)s.B * 4);
+  L.flags = take(U * (size_t)s.B);
+  L.gram = take(U * m * m * 8);
+  L.rz = take(U * m * d * 8);
+  L.scores = take(U * (size_t)s.P * 4);
+  L.y = take(U * m * d * 4);
+  L.rstats = take(U * m * 8);
+  L.total = off;
+  return L;
+}
+
+}  // namespace grkv
+
+extern "C" {
+
+void grkv_params_init(grkv_params* p, int32_t units, int32_t group, int32_t n, int32_t window,
+                      int32_t budget) {
+  if (!p) return;
+  p->units = units;
+  p->group = group;
+  p->n = n;
+  p->d = kD;
+  p->window = window;
+  p->budget = budget;
+  p->pool_kernel = 7;
+  p->pool_type = GRKV_POOL_MAX;
+  p->n_sink = 4;
+  p->beta = 0.10f;
+  p->lambda_v = 1e-2f;
+  p->lambda_k = 1e-2f;
+  p->scale = 0.f;
+  p->causal = 1;
+  p->dtype = GRKV_BF16;
+  p->flags = 0;
+}
+
+int grkv_workspace_size(const grkv_params* p, size_t* bytes) {
+  Shape s;
+  GRKV_TRY(make_shape(p, &s));
+  if (!bytes) return GRKV_ERR_INVALID_ARG;
+  *bytes = plan_workspace(s).total;
+  return GRKV_OK;
+}
+
+int grkv_score(const grkv_params* p, const void* q, const void* k, const void* v, float* scores,
+               float* y, float* row_stats, void* ws, size_t ws_bytes, void* stream) {
+  Shape s;
+  GRKV_TRY(make_shape(p, &s));
+  const WsLayout L = plan_workspace(s);
+  GRKV_TRY(check_ws(L, ws, ws_bytes));
+  GRKV_TRY(check_inputs(s, q, k, v));
+  GRKV_TRY(check_ptr(scores, (size_t)s.U * s.P));
+  GRKV_TRY(check_ptr(y, (size_t)s.U * s.m));
+  GRKV_TRY(check_ptr(row_stats, (size_t)s.U * s.m));
+  cudaStream_t st = (cudaStream_t)stream;
+  char* w = (char*)ws;
+  GRKV_TRY(cuda_rc(cudaMemsetAsync(w + L.status, 0, 4, st)));
+  if (s.U == 0) return GRKV_OK;
+  return cuda_rc(launch_score_simt(s, q, k, v, scores, y, row_stats, w, L, st));
+}
+
+int grkv_select(const grkv_params* p, const float* scores, int32_t* idx, void* ws,
+                size_t ws_bytes, void* stream) {
+  Shape s;
+  GRKV_TRY(make_shape(p, &s));
+  const WsLayout L = plan_workspace(s);
+  GRKV_TRY(check_ws(L, ws, ws_bytes));
+  GRKV_TRY(check_ptr(scores, (size_t)s.U * s.P));
+  GRKV_TRY(check_ptr(idx, (size_t)s.U * s.B));
+  cudaStream_t st = (cudaStream_t)stream;
+  char* w = (char*)ws;
+  GRKV_TRY(cuda_rc(cudaMemsetAsync(w + L.status, 0, 4, st)));
+  if (s.U == 0) return GRKV_OK;
+  return cuda_rc(launch_select(s, scores, idx, w, L, st));
+}
+
+int grkv_merge(const grkv_params* p, const void* q, const void* k, const void* v,
+               const float* scores, const float* y, const int32_t* idx, void* k_out, void* v_out,
+               void* ws, size_t ws_bytes, void* stream) {
+  Shape s;
+  GRKV_TRY(make_shape(p, &s));
+  const WsLayout L = plan_workspace(s);
+  GRKV_TRY(check_ws(L, ws, ws_bytes));
+  GRKV_TRY(check_inputs(s, q, k, v));
+  GRKV_TRY(check_ptr(scores, (size_t)s.U * s.P));
+  GRKV_TRY(check_ptr(y, (size_t)s.U * s.m));
+  GRKV_TRY(check_ptr(idx, (size_t)s.U * s.B));
+  GRKV_TRY(check_ptr(k_out, (size_t)s.U * s.B));
+  GRKV_TRY(check_ptr(v_out, (size_t)s.U * s.B));
+  cudaStream_t st = (cudaStream_t)stream;
+  char* w = (char*)ws;
+  GRKV_TRY(cuda_rc(cudaMemsetAsync(w + L.status, 0, 4, st)));
+  if (s.U == 0) return GRKV_OK;
+  return cuda_rc(launch_merge_simt(s, q, k, v, scores, y, idx, k_out, v_out, w, L, st));
+}
+
+int grkv_compress(const grkv_params* p, const void* q, const void* k, const void* v, void* k_out,
+                  void* v_out, int32_t* idx, void* ws, size_t ws_bytes, void* stream) {
+  Shape s;
+  GRKV_TRY(make_shape(p, &s));
+  const WsLayout L = plan_workspace(s);
+  GRKV_TRY(check_ws(L, ws, ws_bytes));
+  GRKV_TRY(check_inputs(s, q, k, v));
+  GRKV_TRY(check_ptr(idx, (size_t)s.U * s.B));
+  GRKV_TRY(check_ptr(k_out, (size_t)s.U * s.B));
+  GRKV_TRY(check_ptr(v_out, (size_t)s.U * s.B));
+  cudaStream_t st = (cudaStream_t)stream;
+  char* w = (char*)ws;
+  GRKV_TRY(cuda_rc(cudaMemsetAsync(w + L.status, 0, 4, st)));
+  if (s.U == 0) return GRKV_OK;
+  float* scores = (float*)(w + L.scores);
+  float* y = (float*)(w + L.y);
+  float* rstats = (float*)(w + L.rstats);
+  GRKV_TRY(cuda_rc(launch_score_simt(s, q, k, v, scores, y, rstats, w, L, st)));
+  GRKV_TRY(cuda_rc(launch_select(s, scores, idx, w, L, st)));
+  return cuda_rc(launch_merge_simt(s, q, k, v, scores, y, idx, k_out, v_out, w, L, st));
+}
+
+int grkv_status(const void* ws, int* device_status, void* stream) {
+  if (!ws || !device_status) return GRKV_ERR_INVALID_ARG;
+  if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return GRKV_ERR_CUDA;
+  int h = 0;
+  if (cudaMemcpy(&h, ws, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess) return GRKV_ERR_CUDA;
+  *device_status = h;
+  return GRKV_OK;
+}
+
+uint64_t grkv_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+const char* grkv_strerror(int code) {
+  switch (code) {
+    case GRKV_OK: return "ok";
+    case GRKV_ERR_INVALID_ARG: return "invalid argument";
+    case GRKV_ERR_UNSUPPORTED: return "unsupported configuration";
+    case GRKV_ERR_WORKSPACE_TOO_SMALL: return "workspace too small";
+    case GRKV_ERR_MISALIGNED: return "device pointer not 16-byte aligned";
+    case GRKV_ERR_CUDA: return "CUDA error";
+    case GRKV_ERR_NUMERIC: return "non-positive Cholesky pivot";
+    case GRKV_ERR_TIMEOUT: return "bounded device wait expired";
+    default: return "unknown error";
+  }
+}
+
+}  // extern "C"

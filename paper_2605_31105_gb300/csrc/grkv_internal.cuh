@@ -1,0 +1,77 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stddef.h>
+#include <stdint.h>
+#include <string.h>
+
+#include "grkv.h"
+
+namespace grkv {
+
+constexpr int kD = 128;          // supported head dimension
+constexpr int kMaxM = 256;       // stacked window rows g*w supported
+
+// Validated problem sizes, derived once on the host.
+struct Shape {
+  int U, g, n, d, w, B, m;
+  int P;          // prefix length n - w (scored, pooled, selectable)
+  int kk;         // prefix tokens kept: B - w
+  int pool_k, pool_type, n_sink, n_fix, causal, dtype;
+  float lambda, scale;
+  int lambda_inf; // lambda_v == +inf: values stay V0
+};
+
+// Byte offsets of the workspace regions (each 256-B aligned).
+struct WsLayout {
+  size_t status;  // int32 device status word
+  // score path (portable kernels)
+  size_t pstats;  // float2 [U][nchunk][m]      per-chunk (max, sum)
+  size_t ypart;   // float  [U][nchunk][m][d]   per-chunk target partials
+  int chunk, nchunk;
+  // select
+  size_t pooled;  // float [U][P]
+  // merge
+  size_t xbuf;    // float [U][m][B]   retained logits, then X
+  size_t flags;   // uint8 [U][B]      fixed-token flags
+  size_t gram;    // acc   [U][m][m]   X_G X_G^T + lambda I, then its Cholesky factor
+  size_t rz;      // acc   [U][m][d]   residual R, then Z
+  // compress intermediates
+  size_t scores;  // float [U][P]
+  size_t y;       // float [U][m][d]
+  size_t rstats;  // float2 [U][m]
+  size_t total;
+};
+
+WsLayout plan_workspace(const Shape& s);
+
+// Order-preserving map of an fp32 value to an unsigned key.
+__host__ __device__ inline uint32_t order_key(float f) {
+#ifdef __CUDA_ARCH__
+  uint32_t b = __float_as_uint(f);
+#else
+  uint32_t b;
+  memcpy(&b, &f, 4);
+#endif
+  return b ^ ((b >> 31) ? 0xFFFFFFFFu : 0x80000000u);
+}
+
+__device__ inline void set_status(int* status, int code) { atomicCAS(status, 0, code); }
+
+// Adds n to the process-wide count of kernels this library enqueued.
+void count_launches(int n);
+
+// Launchers (all asynchronous on `st`).
+cudaError_t launch_score_simt(const Shape& s, const void* q, const void* k, const void* v,
+                              float* scores, float* y, float* row_stats, char* ws,
+                              const WsLayout& L, cudaStream_t st);
+cudaError_t launch_select(const Shape& s, const float* scores, int32_t* idx, char* ws,
+                          const WsLayout& L, cudaStream_t st);
+cudaError_t launch_merge_simt(const Shape& s, const void* q, const void* k, const void* v,
+                              const float* scores, const float* y, const int32_t* idx,
+                              void* k_out, void* v_out, char* ws, const WsLayout& L,
+                              cudaStream_t st);
+
+}  // namespace grkv

@@ -1,0 +1,170 @@
+"""Helpers of the GPU parity tests: seeded cases, C-ABI calls, tolerances.
+
+Tolerances follow from the arithmetic of the CUDA path (fp32 accumulation of
+exact bf16 or fp32 products, fp32 exponentials):
+  * a logit l = s * sum_t q_t k_t accumulated in fp32 over d terms is off by
+    at most s * gamma_d * sum_t |q_t k_t|, gamma_d = d u / (1 - d u), u = 2^-24;
+  * a probability exp(l - M) / L then has relative error <= 2 * that bound
+    (its own logit and the row log-normaliser) plus a few ulps of exp/divide;
+  * a prefix score is a sum of m such probabilities: add m u.
+The merged values are held to the bar of the method's statement: for every
+retained row, max |gpu - oracle| / ||oracle row||_2 <= 1e-4 (fp32 inputs) or
+2e-2 (bf16 inputs).
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import torch
+
+import grkv_inputs as gi
+import oracle as O
+from paper_2605_31105_gb300 import binding as b
+
+U = 2.0 ** -24
+V_TOL = {"f32": 1e-4, "bf16": 2e-2}
+
+
+def oracle_params(wl: gi.Workload, **over) -> O.Params:
+    kw = dict(group=wl.group, n=wl.n, d=wl.d, window=wl.window, budget=wl.budget,
+              pool_kernel=wl.pool_kernel, lambda_v=wl.lambda_v)
+    kw.update(over)
+    return O.Params(**kw)
+
+
+def lib_params(wl: gi.Workload, units: int, **over) -> b.grkv_params:
+    p = b.params(units, wl.group, wl.n, wl.window, wl.budget, pool_kernel=wl.pool_kernel,
+                 lambda_v=wl.lambda_v, dtype=wl.dtype)
+    for key, val in over.items():
+        if key == "pool_type":
+            val = {"max": b.GRKV_POOL_MAX, "avg": b.GRKV_POOL_AVG}[val]
+        if key == "causal":
+            val = int(val)
+        setattr(p, key, val)
+    return p
+
+
+def to_device(x: np.ndarray, dtype: str) -> torch.Tensor:
+    if dtype == "bf16":
+        return torch.from_numpy(gi.bf16_bits(x).view(np.int16)).view(torch.bfloat16).cuda()
+    return torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32)).cuda()
+
+
+def to_host(t: torch.Tensor) -> np.ndarray:
+    return t.float().cpu().numpy()
+
+
+class Case:
+    """Seeded inputs of some units of a workload, on the host and the device."""
+
+    def __init__(self, wl: gi.Workload, units=None):
+        self.wl = wl
+        self.units = list(range(wl.units)) if units is None else list(units)
+        arrs = [gi.unit_arrays(wl, u) for u in self.units]
+        self.q = np.stack([a[0] for a in arrs])
+        self.k = np.stack([a[1] for a in arrs])
+        self.v = np.stack([a[2] for a in arrs])
+        self.dq = to_device(self.q, wl.dtype)
+        self.dk = to_device(self.k, wl.dtype)
+        self.dv = to_device(self.v, wl.dtype)
+
+    @property
+    def U(self):
+        return len(self.units)
+
+
+def workspace(p) -> torch.Tensor:
+    return torch.empty(max(256, b.grkv_workspace_size(p)), dtype=torch.uint8, device="cuda")
+
+
+def run_score(c: Case, p):
+    m, P = p.group * p.window, p.n - p.window
+    scores = torch.empty((c.U, P), dtype=torch.float32, device="cuda")
+    y = torch.empty((c.U, m, 128), dtype=torch.float32, device="cuda")
+    rs = torch.empty((c.U, m, 2), dtype=torch.float32, device="cuda")
+    ws = workspace(p)
+    b.grkv_score(p, c.dq, c.dk, c.dv, scores, y, rs, ws)
+    assert b.grkv_status(ws) == b.GRKV_OK
+    return to_host(scores), to_host(y), to_host(rs)
+
+
+def run_select(p, scores: np.ndarray):
+    d_scores = torch.from_numpy(np.ascontiguousarray(scores, dtype=np.float32)).cuda()
+    idx = torch.empty((scores.shape[0], p.budget), dtype=torch.int32, device="cuda")
+    ws = workspace(p)
+    b.grkv_select(p, d_scores, idx, ws)
+    assert b.grkv_status(ws) == b.GRKV_OK
+    return idx.cpu().numpy()
+
+
+def _out_dtype(c: Case):
+    return torch.bfloat16 if c.wl.dtype == "bf16" else torch.float32
+
+
+def run_merge(c: Case, p, scores, y, idx, expect_status=b.GRKV_OK):
+    ko = torch.empty((c.U, p.budget, 128), dtype=_out_dtype(c), device="cuda")
+    vo = torch.empty_like(ko)
+    ws = workspace(p)
+    b.grkv_merge(p, c.dq, c.dk, c.dv,
+                 torch.from_numpy(np.ascontiguousarray(scores, np.float32)).cuda(),
+                 torch.from_numpy(np.ascontiguousarray(y, np.float32)).cuda(),
+                 torch.from_numpy(np.ascontiguousarray(idx, np.int32)).cuda(), ko, vo, ws)
+    assert b.grkv_status(ws) == expect_status
+    return to_host(ko), to_host(vo)
+
+
+def run_compress(c: Case, p):
+    ko = torch.empty((c.U, p.budget, 128), dtype=_out_dtype(c), device="cuda")
+    vo = torch.empty_like(ko)
+    idx = torch.empty((c.U, p.budget), dtype=torch.int32, device="cuda")
+    ws = workspace(p)
+    b.grkv_compress(p, c.dq, c.dk, c.dv, ko, vo, idx, ws)
+    assert b.grkv_status(ws) == b.GRKV_OK
+    return idx.cpu().numpy(), to_host(ko), to_host(vo)
+
+
+# ----------------------------------------------------------------- bounds --
+def logit_bound(q, k, op: O.Params) -> float:
+    """s * gamma_d * max_{r,j} sum_t |q_rt k_jt|: worst fp32 error of a logit."""
+    Q = np.abs(q.reshape(op.m, op.d)).astype(np.float64)
+    K = np.abs(k).astype(np.float64)
+    gam = op.d * U / (1 - op.d * U)
+    return O.effective_scale(op) * gam * float((Q @ K.T).max())
+
+
+def score_rel_tol(q, k, op: O.Params) -> float:
+    return 2.0 * logit_bound(q, k, op) + (op.m + 8) * U + 1e-6
+
+
+def assert_scores(gpu, ora, tol_rel, what="scores"):
+    err = np.abs(gpu.astype(np.float64) - ora)
+    lim = tol_rel * np.abs(ora) + 1e-30
+    bad = err > lim
+    assert not bad.any(), (f"{what}: {bad.sum()} of {bad.size} beyond tolerance; worst rel "
+                           f"{(err / np.maximum(np.abs(ora), 1e-30)).max():.3e} vs {tol_rel:.3e}")
+
+
+def assert_values(gpu, ora, dtype: str, what="v_out"):
+    """max_j ||gpu_j - ora_j||_inf / ||ora_j||_2 within the method's bar."""
+    den = np.maximum(np.linalg.norm(ora, axis=-1), 1e-30)
+    rel = np.abs(gpu.astype(np.float64) - ora).max(axis=-1) / den
+    assert rel.max() <= V_TOL[dtype], f"{what}: max row-relative error {rel.max():.3e}"
+    return float(rel.max())
+
+
+def idx_tie_check(gpu_idx, ora, op: O.Params, tol_rel: float):
+    """Retained sets must agree except where the oracle's pooled scores sit
+    within the score tolerance of the cut: returns the number of such swaps."""
+    g, o = set(gpu_idx.tolist()), set(ora["idx"].tolist())
+    diff = g ^ o
+    if not diff:
+        return 0
+    pooled = ora["pooled"].astype(np.float64)
+    kk = op.budget - op.window
+    cut = np.sort(pooled)[::-1][kk - 1]
+    for j in diff:
+        assert j < op.n - op.window, f"window position {j} differs"
+        assert abs(pooled[j] - cut) <= 2 * tol_rel * cut, \
+            f"idx differs at {j}: pooled {pooled[j]:.9e} vs cut {cut:.9e}"
+    return len(diff) // 2

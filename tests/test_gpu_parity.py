@@ -1,0 +1,203 @@
+"""GPU parity: every stage of the CUDA path against the fp64 oracle, through
+the C ABI, element by element on the same seeded inputs.
+
+Stage tests feed both sides identical inputs (the oracle's fp32 scores, its
+fp32 target and its retained set), so integer results must match bit for bit
+and merged values within the method's bar; the end-to-end test checks the
+retained set up to score ties within the derived score tolerance.
+"""
+import math
+
+import numpy as np
+import pytest
+
+import grkv_inputs as gi
+import oracle as O
+from paper_2605_31105_gb300 import binding as b
+from tests import gpu_cases as G
+
+pytestmark = pytest.mark.gpu
+
+RAGGED = gi.Workload("ragged_g3_w5_n1000", 3, 3, 1000, 128, 5, 77, 5, 1e-2, "bf16", "lowrank", 777)
+M256 = gi.Workload("m256_spans_n8192", 2, 4, 8192, 128, 64, 512, 7, 1e-1, "bf16", "spans", 888)
+
+CASES = {
+    "c0_full": (gi.workload(0), {}),
+    "c1_full": (gi.workload(1), {}),
+    "ragged_causal": (RAGGED, {}),
+    "ragged_noncausal_avgpool": (RAGGED, dict(causal=False, pool_type="avg")),
+    "ragged_f32": (RAGGED.replace(dtype="f32"), {}),
+    "m256_spans": (M256, {}),
+    "c2_recipe_n8192": (gi.workload(2).replace(units=3, n=8192, budget=1024), {}),
+    "g1_w1": (RAGGED.replace(group=1, window=1, budget=40, seed=5), dict(n_sink=0, beta=0.0)),
+}
+
+
+class Prepared:
+    def __init__(self, wl, over):
+        self.wl = wl
+        self.over = over
+        self.case = G.Case(wl)
+        self.op = G.oracle_params(wl, **over)
+        self.p = G.lib_params(wl, self.case.U, **over)
+        self.ora = [O.compress_unit(self.case.q[i], self.case.k[i], self.case.v[i], self.op)
+                    for i in range(self.case.U)]
+        self.tol = [G.score_rel_tol(self.case.q[i], self.case.k[i], self.op)
+                    for i in range(self.case.U)]
+
+
+@pytest.fixture(scope="module", params=list(CASES))
+def prep(request, grkv_lib):
+    wl, over = CASES[request.param]
+    return Prepared(wl, over)
+
+
+def test_score_stage(prep):
+    c, op = prep.case, prep.op
+    scores, y, rs = G.run_score(c, prep.p)
+    for i, ora in enumerate(prep.ora):
+        lb = G.logit_bound(c.q[i], c.k[i], op)
+        np.testing.assert_allclose(rs[i, :, 0], ora["row_max"], rtol=0, atol=lb + 1e-6)
+        G.assert_scores(rs[i, :, 1], ora["row_sum"], prep.tol[i] + op.n * G.U, "row_sum")
+        G.assert_scores(scores[i], ora["scores"], prep.tol[i])
+        s_abs = ora["attn"] @ np.abs(c.v[i].astype(np.float64))
+        lim = (prep.tol[i] + op.n * G.U) * s_abs + 1e-7
+        err = np.abs(y[i] - ora["y"])
+        assert (err <= lim).all(), f"y: worst excess {(err - lim).max():.3e}"
+
+
+def test_select_stage_bit_exact(prep):
+    scores32 = np.stack([o["scores32"] for o in prep.ora])
+    idx = G.run_select(prep.p, scores32)
+    for i, ora in enumerate(prep.ora):
+        np.testing.assert_array_equal(idx[i], ora["idx"])
+
+
+def test_merge_stage(prep):
+    c, op = prep.case, prep.op
+    scores32 = np.stack([o["scores32"] for o in prep.ora])
+    y32 = np.stack([o["y"].astype(np.float32) for o in prep.ora])
+    idx = np.stack([o["idx"] for o in prep.ora])
+    ko, vo = G.run_merge(c, prep.p, scores32, y32, idx)
+    for i in range(c.U):
+        ref = O.merge_unit(c.q[i], c.k[i], c.v[i], scores32[i], y32[i], idx[i], op)
+        np.testing.assert_array_equal(ko[i], c.k[i][idx[i]])            # K_out = K0
+        fixed = ref["fixed"]
+        np.testing.assert_array_equal(vo[i][fixed], c.v[i][idx[i]][fixed])  # F rows as V0
+        G.assert_values(vo[i], ref["v_out"], c.wl.dtype)
+
+
+def test_compress_end_to_end(prep):
+    c, op = prep.case, prep.op
+    idx, ko, vo = G.run_compress(c, prep.p)
+    compared = 0
+    for i, ora in enumerate(prep.ora):
+        swaps = G.idx_tie_check(idx[i], ora, op, prep.tol[i])
+        np.testing.assert_array_equal(ko[i], c.k[i][idx[i]])
+        if swaps == 0:
+            G.assert_values(vo[i], ora["v_out"], c.wl.dtype)
+            compared += 1
+    assert compared >= max(1, c.U // 2)
+
+
+# ------------------------------------------------------------- edge cases --
+EDGE = gi.Workload("edge_n600", 2, 2, 600, 128, 8, 64, 7, 1e-2, "bf16", "lowrank", 4242)
+
+
+@pytest.mark.parametrize("over", [
+    dict(budget=8),                       # B = w: only the window is kept
+    dict(budget=600),                     # B = n: nothing evicted, zero update
+    dict(pool_kernel=1),
+    dict(lambda_v=math.inf),              # values unchanged
+    dict(lambda_v=1e6),
+    dict(lambda_v=1e-5),
+    dict(n_sink=0, beta=0.0),
+    dict(beta=0.5, n_sink=64),
+], ids=lambda d: ",".join(f"{k}={v}" for k, v in d.items()))
+def test_edge_cases(grkv_lib, over):
+    wl = EDGE.replace(budget=over.get("budget", EDGE.budget))
+    over = {k: v for k, v in over.items() if k != "budget"}
+    c = G.Case(wl)
+    op = G.oracle_params(wl, **over)
+    p = G.lib_params(wl, c.U, **over)
+    idx, ko, vo = G.run_compress(c, p)
+    for i in range(c.U):
+        ora = O.compress_unit(c.q[i], c.k[i], c.v[i], op)
+        assert G.idx_tie_check(idx[i], ora, op, G.score_rel_tol(c.q[i], c.k[i], op)) == 0
+        G.assert_values(vo[i], ora["v_out"], wl.dtype)
+        if wl.budget == wl.n:
+            G.assert_values(vo[i], c.v[i].astype(np.float64), wl.dtype, "B = n leaves V")
+        if math.isinf(op.lambda_v):
+            np.testing.assert_array_equal(vo[i], c.v[i][idx[i]])
+
+
+def test_select_ties_take_smaller_positions(grkv_lib):
+    wl = EDGE
+    p = G.lib_params(wl, 2)
+    op = G.oracle_params(wl)
+    P = wl.n - wl.window
+    flat = np.full((2, P), 0.25, np.float32)             # every score tied
+    steps = np.repeat(np.arange(P // 8, dtype=np.float32), 8)[:P][None].repeat(2, 0)
+    steps = np.concatenate([steps, np.zeros((2, P - steps.shape[1]), np.float32)], 1)
+    for s in (flat, steps):
+        idx = G.run_select(p, s)
+        for i in range(2):
+            np.testing.assert_array_equal(idx[i], O.select(O.pool(s[i], op), op))
+
+
+def test_zero_units_is_a_no_op(grkv_lib):
+    import torch
+    p = b.params(0, 4, 1024, 32, 128)
+    ws = torch.empty(1024, dtype=torch.uint8, device="cuda")
+    z = torch.empty(16, dtype=torch.bfloat16, device="cuda")
+    zi = torch.empty(16, dtype=torch.int32, device="cuda")
+    assert b.grkv_compress(p, z, z, z, z, z, zi, ws) == b.GRKV_OK
+    assert b.grkv_status(ws) == b.GRKV_OK
+
+
+def test_singular_dual_system_reports_numeric_status(grkv_lib):
+    """lambda = 0 with every retained token fixed: X_G = 0, the dual matrix is
+    0 and its first Cholesky pivot is exactly 0; the device reports
+    GRKV_ERR_NUMERIC through the status word and the context stays usable."""
+    wl = EDGE.replace(budget=EDGE.window)
+    c = G.Case(wl)
+    p = G.lib_params(wl, c.U, lambda_v=0.0)
+    op = G.oracle_params(wl, lambda_v=0.0)
+    ora = [O.compress_unit(c.q[i], c.k[i], c.v[i], G.oracle_params(wl)) for i in range(c.U)]
+    scores32 = np.stack([o["scores32"] for o in ora])
+    y32 = np.stack([o["y"].astype(np.float32) for o in ora])
+    idx = np.stack([o["idx"] for o in ora])
+    G.run_merge(c, p, scores32, y32, idx, expect_status=b.GRKV_ERR_NUMERIC)
+    # the next call on the same context is unaffected
+    p2 = G.lib_params(wl, c.U)
+    _, vo = G.run_merge(c, p2, scores32, y32, idx)
+    assert op.lambda_v == 0.0 and np.isfinite(vo).all()
+
+
+def test_full_size_c2_sampled_units(grkv_lib):
+    """The 32-layer, 32K-token workload at full size, in the launch
+    configuration the bench times; sampled units against the oracle."""
+    import torch
+    wl = gi.workload(2)
+    q = np.empty((wl.units, wl.group, wl.window, wl.d), np.uint16)
+    k = np.empty((wl.units, wl.n, wl.d), np.uint16)
+    v = np.empty_like(k)
+    gi.fill_units(wl, q, k, v)
+    as_dev = lambda x: torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).cuda()
+    dq, dk, dv = as_dev(q), as_dev(k), as_dev(v)
+    p = G.lib_params(wl, wl.units)
+    ko = torch.empty((wl.units, wl.budget, wl.d), dtype=torch.bfloat16, device="cuda")
+    vo = torch.empty_like(ko)
+    idx = torch.empty((wl.units, wl.budget), dtype=torch.int32, device="cuda")
+    ws = G.workspace(p)
+    b.grkv_compress(p, dq, dk, dv, ko, vo, idx, ws)
+    assert b.grkv_status(ws) == b.GRKV_OK
+    idx, ko, vo = idx.cpu().numpy(), G.to_host(ko), G.to_host(vo)
+    op = G.oracle_params(wl)
+    for u in (0, 131, 255):
+        qu, ku, vu = gi.unit_arrays(wl, u)
+        ora = O.compress_unit(qu, ku, vu, op)
+        swaps = G.idx_tie_check(idx[u], ora, op, G.score_rel_tol(qu, ku, op))
+        np.testing.assert_array_equal(ko[u], ku[idx[u]])
+        if swaps == 0:
+            G.assert_values(vo[u], ora["v_out"], wl.dtype)
