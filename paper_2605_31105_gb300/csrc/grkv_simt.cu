@@ -15,6 +15,10 @@ namespace {
 
 constexpr int QP = kD + 1;  // padded row stride (floats) of q / key tiles in shared memory
 
+// Float count rounded up to a multiple of 4, so the next shared-memory region
+// starts on a 16-byte boundary.
+__host__ __device__ constexpr int pad4(int n) { return (n + 3) & ~3; }
+
 __device__ __forceinline__ float ldv(const float* p, size_t i) { return p[i]; }
 __device__ __forceinline__ float ldv(const __nv_bfloat16* p, size_t i) {
   return __bfloat162float(p[i]);
@@ -127,10 +131,10 @@ template <typename T>
 __global__ void __launch_bounds__(256) k_stats_chunk(const T* __restrict__ q,
                                                      const T* __restrict__ k, Shape s, int chunk,
                                                      int nchunk, float2* __restrict__ pstats) {
-  extern __shared__ float sm[];
-  float* qs = sm;                          // [m][QP]
-  float* ks = qs + s.m * QP;               // [64][kD]
-  float2* red = (float2*)(ks + 64 * kD);   // [256]
+  extern __shared__ __align__(16) float sm[];
+  float* qs = sm;                          // [m][QP], padded to 16 bytes
+  float* ks = qs + pad4(s.m * QP);         // [64][kD]
+  float2* red = (float2*)(ks + 64 * kD);   // [256], 8-byte aligned
   const int u = blockIdx.y, c = blockIdx.x, tid = threadIdx.x;
   const int j0 = c * chunk, j1 = min(s.n, j0 + chunk);
   const T* qu = q + (size_t)u * s.m * kD;
@@ -209,7 +213,7 @@ __global__ void __launch_bounds__(512) k_prob_chunk(const T* __restrict__ q,
                                                     int nchunk, const float* __restrict__ row_stats,
                                                     float* __restrict__ scores,
                                                     float* __restrict__ ypart) {
-  extern __shared__ float sm[];
+  extern __shared__ __align__(16) float sm[];
   float* qs = sm;                 // [m][QP]
   float* ks = qs + s.m * QP;      // [32][QP]
   float* vs = ks + 32 * QP;       // [32][kD]
@@ -359,7 +363,7 @@ __global__ void __launch_bounds__(512) k_merge(
     const float* __restrict__ scores, const float* __restrict__ y, const int32_t* __restrict__ idx,
     T* __restrict__ k_out, T* __restrict__ v_out, Shape s, float* __restrict__ xbuf,
     uint8_t* __restrict__ flags, A* __restrict__ gram, A* __restrict__ rz, int* status) {
-  extern __shared__ float sm[];
+  extern __shared__ __align__(16) float sm[];
   __shared__ int hist[256];
   __shared__ int sh[48];
   const int u = blockIdx.x, tid = threadIdx.x, m = s.m, B = s.B;
@@ -587,7 +591,7 @@ cudaError_t score_impl(const Shape& s, const T* q, const T* k, const T* v, float
                        cudaStream_t st) {
   float2* pstats = (float2*)(ws + L.pstats);
   float* ypart = (float*)(ws + L.ypart);
-  const size_t smA = ((size_t)s.m * QP + 64 * kD) * 4 + 256 * sizeof(float2);
+  const size_t smA = ((size_t)pad4(s.m * QP) + 64 * kD) * 4 + 256 * sizeof(float2);
   cudaError_t e = cudaFuncSetAttribute(k_stats_chunk<T>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smA);
   if (e != cudaSuccess) return e;
