@@ -131,6 +131,24 @@ int grkv_compress(const grkv_params* p, const void* q, const void* k, const void
                   void* k_out, void* v_out, int32_t* idx,
                   void* ws, size_t ws_bytes, void* stream);
 
+/* grkv_select without a workspace.  The paper has no counterpart: this entry
+ * point exists for callers that cannot give the library scratch device
+ * memory, such as a plugin inside an inference engine that owns all device
+ * memory through its own pool and passes plugins no workspace, or a serving
+ * loop that must not call cudaMalloc on the request path (it synchronises the
+ * device and fails once a pool has taken the free memory).  It allocates
+ * nothing: the pooled scores go to a 16 MiB array in the library's device
+ * image, which every GPU that loads the library holds until the process exits.
+ * Limit: units * (n - window) <= 4,194,304 floats; larger sizes return
+ * GRKV_ERR_WORKSPACE_TOO_SMALL.  The first call on a device looks up the
+ * array's device address (cudaGetSymbolAddress) with that device current;
+ * make that first call before any stream capture.  All calls share the array
+ * and it keeps the last call's contents; every element a call reads is first
+ * written by the same call, so nothing needs clearing.  Calls that overlap on
+ * the GPU (two streams, or two host threads) race on the array: serialise
+ * them.  scores and idx are device pointers laid out as for grkv_select. */
+int grkv_select_noalloc(const grkv_params* p, const float* scores, int32_t* idx, void* stream);
+
 /* Synchronises `stream`, then stores in *device_status the device-side
  * status of the most recent call that used `ws` (GRKV_OK, GRKV_ERR_NUMERIC or
  * GRKV_ERR_TIMEOUT).  Returns GRKV_ERR_CUDA if the stream reports an error. */

@@ -30,7 +30,8 @@ GRKV_UPDATE_K = 0x1
 GRKV_FORCE_SIMT = 0x2
 
 EXPORTS = ("grkv_params_init", "grkv_workspace_size", "grkv_score", "grkv_select", "grkv_merge",
-           "grkv_compress", "grkv_status", "grkv_strerror", "grkv_launch_count")
+           "grkv_compress", "grkv_status", "grkv_strerror", "grkv_launch_count",
+           "grkv_select_noalloc")
 
 
 class grkv_params(ctypes.Structure):
@@ -75,6 +76,8 @@ def load():
     lib.grkv_status.argtypes = [_vp, ctypes.POINTER(ctypes.c_int), _vp]
     lib.grkv_strerror.argtypes = [ctypes.c_int]
     lib.grkv_strerror.restype = ctypes.c_char_p
+    lib.grkv_select_noalloc.argtypes = [_P, _vp, _vp, _vp]
+    lib.grkv_select_noalloc.restype = ctypes.c_int
     lib.grkv_launch_count.argtypes = []
     lib.grkv_launch_count.restype = ctypes.c_uint64
     for name in ("grkv_workspace_size", "grkv_score", "grkv_select", "grkv_merge",
@@ -162,6 +165,12 @@ def grkv_compress(p, q, k, v, k_out, v_out, idx, ws, ws_bytes=None, stream=None,
     rc = load().grkv_compress(ctypes.byref(p), _ptr(q), _ptr(k), _ptr(v), _ptr(k_out),
                               _ptr(v_out), _ptr(idx), _ptr(ws), ws_bytes, _stream(stream))
     return _check(rc, "grkv_compress", check)
+
+
+def grkv_select_noalloc(p, scores, idx, stream=None, check=True):
+    """grkv_select with the library's built-in scratch array (no workspace)."""
+    rc = load().grkv_select_noalloc(ctypes.byref(p), _ptr(scores), _ptr(idx), _stream(stream))
+    return _check(rc, "grkv_select_noalloc", check)
 
 
 def grkv_launch_count() -> int:

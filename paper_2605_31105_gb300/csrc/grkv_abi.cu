@@ -14,6 +14,39 @@ size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
+int check_ws(const WsLayout& L, const void* ws, size_t ws_bytes) {
+  if (!ws) return GRKV_ERR_INVALID_ARG;
+  if (!aligned16(ws)) return GRKV_ERR_MISALIGNED;
+  if (ws_bytes < L.total) return GRKV_ERR_WORKSPACE_TOO_SMALL;
+  return GRKV_OK;
+}
+
+// Non-null (unless the array is empty) and 16-byte aligned.
+int check_ptr(const void* p, size_t elems) {
+  if (elems == 0) return GRKV_OK;
+  if (!p) return GRKV_ERR_INVALID_ARG;
+  return aligned16(p) ? GRKV_OK : GRKV_ERR_MISALIGNED;
+}
+
+int cuda_rc(cudaError_t e) { return e == cudaSuccess ? GRKV_OK : GRKV_ERR_CUDA; }
+
+#define GRKV_TRY(expr)            \
+  do {                            \
+    const int rc_ = (expr);       \
+    if (rc_ != GRKV_OK) return rc_; \
+  } while (0)
+
+int check_inputs(const Shape& s, const void* q, const void* k, const void* v) {
+  GRKV_TRY(check_ptr(q, (size_t)s.U * s.m));
+  GRKV_TRY(check_ptr(k, (size_t)s.U * s.n));
+  GRKV_TRY(check_ptr(v, (size_t)s.U * s.n));
+  return GRKV_OK;
+}
+
+}  // namespace
+
+namespace grkv {
+
 int make_shape(const grkv_params* p, Shape* s) {
   if (!p) return GRKV_ERR_INVALID_ARG;
   if (p->units < 0 || p->group < 1 || p->window < 1 || p->n < p->window) return GRKV_ERR_INVALID_ARG;
@@ -52,39 +85,6 @@ int make_shape(const grkv_params* p, Shape* s) {
   s->scale = p->scale != 0.f ? p->scale : (float)(1.0 / std::sqrt((double)p->d));
   return GRKV_OK;
 }
-
-int check_ws(const WsLayout& L, const void* ws, size_t ws_bytes) {
-  if (!ws) return GRKV_ERR_INVALID_ARG;
-  if (!aligned16(ws)) return GRKV_ERR_MISALIGNED;
-  if (ws_bytes < L.total) return GRKV_ERR_WORKSPACE_TOO_SMALL;
-  return GRKV_OK;
-}
-
-// Non-null (unless the array is empty) and 16-byte aligned.
-int check_ptr(const void* p, size_t elems) {
-  if (elems == 0) return GRKV_OK;
-  if (!p) return GRKV_ERR_INVALID_ARG;
-  return aligned16(p) ? GRKV_OK : GRKV_ERR_MISALIGNED;
-}
-
-int cuda_rc(cudaError_t e) { return e == cudaSuccess ? GRKV_OK : GRKV_ERR_CUDA; }
-
-#define GRKV_TRY(expr)            \
-  do {                            \
-    const int rc_ = (expr);       \
-    if (rc_ != GRKV_OK) return rc_; \
-  } while (0)
-
-int check_inputs(const Shape& s, const void* q, const void* k, const void* v) {
-  GRKV_TRY(check_ptr(q, (size_t)s.U * s.m));
-  GRKV_TRY(check_ptr(k, (size_t)s.U * s.n));
-  GRKV_TRY(check_ptr(v, (size_t)s.U * s.n));
-  return GRKV_OK;
-}
-
-}  // namespace
-
-namespace grkv {
 
 static std::atomic<uint64_t> g_launches{0};
 

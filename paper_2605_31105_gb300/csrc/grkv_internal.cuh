@@ -69,6 +69,11 @@ cudaError_t launch_score_simt(const Shape& s, const void* q, const void* k, cons
                               const WsLayout& L, cudaStream_t st);
 cudaError_t launch_select(const Shape& s, const float* scores, int32_t* idx, char* ws,
                           const WsLayout& L, cudaStream_t st);
+// Selection with the pooled-score scratch [U][n-w] given directly.
+cudaError_t launch_select_pooled(const Shape& s, const float* scores, int32_t* idx,
+                                 float* pooled, cudaStream_t st);
+// Host-side parameter validation shared by the entry points.
+int make_shape(const grkv_params* p, Shape* s);
 cudaError_t launch_merge_simt(const Shape& s, const void* q, const void* k, const void* v,
                               const float* scores, const float* y, const int32_t* idx,
                               void* k_out, void* v_out, char* ws, const WsLayout& L,

@@ -651,6 +651,13 @@ cudaError_t launch_select(const Shape& s, const float* scores, int32_t* idx, cha
   return cudaGetLastError();
 }
 
+cudaError_t launch_select_pooled(const Shape& s, const float* scores, int32_t* idx,
+                                 float* pooled, cudaStream_t st) {
+  k_select<<<s.U, 1024, 0, st>>>(scores, s, pooled, idx);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_merge_simt(const Shape& s, const void* q, const void* k, const void* v,
                               const float* scores, const float* y, const int32_t* idx,
                               void* k_out, void* v_out, char* ws, const WsLayout& L,
