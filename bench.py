@@ -43,6 +43,8 @@ def args_():
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--path", choices=("default", "two_pass", "portable"), default="default",
+                    help="scoring kernels to use (default: fused tensor-core rounds)")
     return ap.parse_args()
 
 
@@ -271,7 +273,9 @@ def run_ours(a):
     gi.fill_units(wl, view(hq), view(hk), view(hv))
     dq, dk, dv = hq.cuda(), hk.cuda(), hv.cuda()
     p = b.params(U, wl.group, n, wl.window, B, pool_kernel=wl.pool_kernel,
-                 lambda_v=wl.lambda_v, dtype=wl.dtype)
+                 lambda_v=wl.lambda_v, dtype=wl.dtype,
+                 flags={"default": 0, "two_pass": b.GRKV_TWO_PASS,
+                        "portable": b.GRKV_FORCE_SIMT}[a.path])
     ws = torch.empty(b.grkv_workspace_size(p), dtype=torch.uint8, device="cuda")
     ko = torch.empty((U, B, d), dtype=tdt, device="cuda")
     vo = torch.empty_like(ko)
@@ -389,6 +393,7 @@ def run_ours(a):
                    "group": wl.group, "d": d, "lambda_v": wl.lambda_v,
                    "pool_kernel": wl.pool_kernel, "l2": "inputs (K+V %.1f GB) exceed L2" %
                    (read / 1e9), "parallelism": f"units sharded, {world} rank(s)"},
+        "path": a.path,
         "roofline": {"bound": "hbm", "kernel": "grkv_score stage (window scoring + target)",
                      "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind, "traffic": None,

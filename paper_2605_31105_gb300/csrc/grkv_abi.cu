@@ -30,6 +30,14 @@ int check_ptr(const void* p, size_t elems) {
 
 int cuda_rc(cudaError_t e) { return e == cudaSuccess ? GRKV_OK : GRKV_ERR_CUDA; }
 
+cudaError_t launch_score(const Shape& s, const void* q, const void* k, const void* v,
+                         float* scores, float* y, float* row_stats, char* ws, const WsLayout& L,
+                         cudaStream_t st) {
+  if (s.tc)
+    return launch_score_tc(s, q, k, v, scores, y, row_stats, ws, L, s.two_pass ? 0 : 2, st);
+  return launch_score_simt(s, q, k, v, scores, y, row_stats, ws, L, st);
+}
+
 #define GRKV_TRY(expr)            \
   do {                            \
     const int rc_ = (expr);       \
@@ -59,7 +67,7 @@ int make_shape(const grkv_params* p, Shape* s) {
   if (!(p->scale >= 0.f) || std::isinf(p->scale)) return GRKV_ERR_INVALID_ARG;
   if (p->causal != 0 && p->causal != 1) return GRKV_ERR_INVALID_ARG;
   if (p->dtype != GRKV_F32 && p->dtype != GRKV_BF16) return GRKV_ERR_INVALID_ARG;
-  if (p->flags & ~(GRKV_UPDATE_K | GRKV_FORCE_SIMT)) return GRKV_ERR_INVALID_ARG;
+  if (p->flags & ~(GRKV_UPDATE_K | GRKV_FORCE_SIMT | GRKV_TWO_PASS)) return GRKV_ERR_INVALID_ARG;
   if (p->d < 1) return GRKV_ERR_INVALID_ARG;
   if (p->flags & GRKV_UPDATE_K) return GRKV_ERR_UNSUPPORTED;
   if (p->d != kD) return GRKV_ERR_UNSUPPORTED;
@@ -83,6 +91,8 @@ int make_shape(const grkv_params* p, Shape* s) {
   s->lambda = p->lambda_v;
   s->lambda_inf = std::isinf(p->lambda_v) ? 1 : 0;
   s->scale = p->scale != 0.f ? p->scale : (float)(1.0 / std::sqrt((double)p->d));
+  s->tc = (p->flags & GRKV_FORCE_SIMT) ? 0 : (score_tc_supported(*s) ? 1 : 0);
+  s->two_pass = (p->flags & GRKV_TWO_PASS) ? 1 : 0;
   return GRKV_OK;
 }
 
@@ -102,8 +112,14 @@ WsLayout plan_workspace(const Shape& s) {
     return at;
   };
   L.status = take(256);
-  L.pstats = take(U * L.nchunk * m * 8);
-  L.ypart = take(U * L.nchunk * m * d * 4);
+  if (s.tc) {
+    int maxc, gu, rounds;
+    L.pstats_tc = take(score_tc_pstats_bytes(s, &maxc, &gu, &rounds, kMaxScoreCtas));
+    L.rounds_tc = take((size_t)rounds * sizeof(int));
+  } else {
+    L.pstats = take(U * L.nchunk * m * 8);
+    L.ypart = take(U * L.nchunk * m * d * 4);
+  }
   L.pooled = take(U * (size_t)s.P * 4);
   L.xbuf = take(U * m * (size_t)s.B * 4);
   L.flags = take(U * (size_t)s.B);
@@ -163,7 +179,7 @@ int grkv_score(const grkv_params* p, const void* q, const void* k, const void* v
   char* w = (char*)ws;
   GRKV_TRY(cuda_rc(cudaMemsetAsync(w + L.status, 0, 4, st)));
   if (s.U == 0) return GRKV_OK;
-  return cuda_rc(launch_score_simt(s, q, k, v, scores, y, row_stats, w, L, st));
+  return cuda_rc(launch_score(s, q, k, v, scores, y, row_stats, w, L, st));
 }
 
 int grkv_select(const grkv_params* p, const float* scores, int32_t* idx, void* ws,
@@ -218,7 +234,7 @@ int grkv_compress(const grkv_params* p, const void* q, const void* k, const void
   float* scores = (float*)(w + L.scores);
   float* y = (float*)(w + L.y);
   float* rstats = (float*)(w + L.rstats);
-  GRKV_TRY(cuda_rc(launch_score_simt(s, q, k, v, scores, y, rstats, w, L, st)));
+  GRKV_TRY(cuda_rc(launch_score(s, q, k, v, scores, y, rstats, w, L, st)));
   GRKV_TRY(cuda_rc(launch_select(s, scores, idx, w, L, st)));
   return cuda_rc(launch_merge_simt(s, q, k, v, scores, y, idx, k_out, v_out, w, L, st));
 }

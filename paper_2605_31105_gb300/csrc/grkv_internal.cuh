@@ -13,6 +13,7 @@ namespace grkv {
 
 constexpr int kD = 128;          // supported head dimension
 constexpr int kMaxM = 256;       // stacked window rows g*w supported
+constexpr int kMaxScoreCtas = 256;  // persistent score grid bound used to size slots
 
 // Validated problem sizes, derived once on the host.
 struct Shape {
@@ -22,6 +23,8 @@ struct Shape {
   int pool_k, pool_type, n_sink, n_fix, causal, dtype;
   float lambda, scale;
   int lambda_inf; // lambda_v == +inf: values stay V0
+  int tc;         // bf16, m <= 128, not forced portable: tensor-core scoring
+  int two_pass;   // tensor-core scoring as two launches
 };
 
 // Byte offsets of the workspace regions (each 256-B aligned).
@@ -31,6 +34,9 @@ struct WsLayout {
   size_t pstats;  // float2 [U][nchunk][m]      per-chunk (max, sum)
   size_t ypart;   // float  [U][nchunk][m][d]   per-chunk target partials
   int chunk, nchunk;
+  // score path (tensor cores)
+  size_t pstats_tc;  // float2 [U][maxc][2][128] pass-A statistics slots
+  size_t rounds_tc;  // int [rounds] finished pass-A blocks per round
   // select
   size_t pooled;  // float [U][P]
   // merge
@@ -69,6 +75,15 @@ cudaError_t launch_score_simt(const Shape& s, const void* q, const void* k, cons
                               const WsLayout& L, cudaStream_t st);
 cudaError_t launch_select(const Shape& s, const float* scores, int32_t* idx, char* ws,
                           const WsLayout& L, cudaStream_t st);
+// Tensor-core window scoring (bf16, m <= 128); mode 2 = fused rounds,
+// otherwise two launches.
+bool score_tc_supported(const Shape& s);
+size_t score_tc_pstats_bytes(const Shape& s, int* maxc, int* gu, int* rounds, int sms);
+int sm_count();
+cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const void* v,
+                            float* scores, float* y, float* row_stats, char* ws,
+                            const WsLayout& L, int mode, cudaStream_t st);
+
 // Selection with the pooled-score scratch [U][n-w] given directly.
 cudaError_t launch_select_pooled(const Shape& s, const float* scores, int32_t* idx,
                                  float* pooled, cudaStream_t st);

@@ -1,0 +1,672 @@
+// Window scoring on the 5th-generation tensor cores (bf16, d = 128, m <= 128).
+//
+// For every unit the path needs, over all n keys, the row statistics of the
+// window logits (pass A: M_r, L_r) and then, with those, the probabilities,
+// the per-key prefix scores c_j = sum_r P_rj and the target Y = P V (pass B);
+// Eq. 4 and Algorithm 1 of the paper.  The row normaliser depends on every
+// key, so the keys are read twice.  This kernel is persistent (one CTA per
+// SM) and processes the units in rounds small enough that a round's keys stay
+// in L2: each CTA runs pass A of round r+1 and then pass B of round r, so the
+// second read of K is served from L2 and only K and V cross HBM once.
+//
+// Roles (384 threads): warp 0 issues TMA loads (Q per segment, K and V
+// tiles of 128 tokens through a 4-slot ring), warp 1 issues tcgen05 MMAs
+// (S = Q K^T into TMEM; Y += P V with P read from TMEM), warps 4-7 and 8-11
+// are two compute groups that take alternate tiles.  A compute thread owns
+// one window row (one TMEM lane): pass A keeps its running max / sum in
+// registers, pass B writes exp2(l - Lambda_r) back into TMEM as bf16 (the A
+// operand of the Y MMA) and sums probabilities over rows with a warp
+// transpose-reduction plus a 4-way shared-memory sum.  Per-unit statistics of
+// the CTAs that share a unit meet in a global slot array; pass B of round r
+// waits (bounded) on a per-round counter of finished pass-A blocks.  Y
+// partials of the CTAs sharing a unit are added with float4 atomics.
+#include <algorithm>
+#include <cmath>
+
+#include "grkv_internal.cuh"
+#include "sm100.cuh"
+#include "tmap.cuh"
+
+namespace grkv {
+namespace {
+
+using namespace sm100;
+
+constexpr int kTile = 128;            // tokens per tile
+constexpr int kRows = 128;            // window rows (m padded to 128)
+constexpr int kRing = 4;              // K / V ring slots
+constexpr int kThreads = 384;
+constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KB
+constexpr long long kWaitBudget = 1ll << 32;      // cycles (~2 s) before a wait gives up
+
+// Shared-memory layout (offsets from a 1024-byte aligned base).
+constexpr uint32_t kOffQ = 0;                                   // 2 x 32 KB
+constexpr uint32_t kOffRing = kOffQ + 2 * kTileBytes;           // 4 x 32 KB
+constexpr uint32_t kOffRed = kOffRing + kRing * kTileBytes;     // [2 wg][2 buf][4][128] fp32
+constexpr uint32_t kOffBar = kOffRed + 2 * 2 * 4 * kTile * 4;
+constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;           // + alignment slack
+
+// TMEM columns: two S buffers, two Y accumulators.
+constexpr uint32_t kColS = 0, kColY = 256;
+
+struct Args {
+  int U, n, w, m, P, causal;
+  int tpu;        // tiles per unit
+  int mode;       // 0: pass A only, 1: pass B only, 2: both, in rounds
+  int gu;         // units per round
+  int rounds;
+  int maxc;       // stats slots per unit
+  float sl2;      // scale * log2(e)
+  float* scores;  // [U][P]
+  float* y;       // [U][m][128], zeroed by the host
+  float* row_stats;  // [U][m][2]
+  float2* pstats;    // [U][maxc][2][128]  (max in log2 units, sum)
+  int* round_done;   // [rounds], zeroed by the host
+  int* status;
+};
+
+// ------------------------------------------------------------ job schedule
+struct Job {
+  int kind;       // 0 = pass A, 1 = pass B
+  int u, r;       // unit, round
+  int j0, len;    // first token, tokens in the tile
+  int seg_first, seg_last;
+};
+
+// The CTA's sequence of blocks is A(0), then A(r+1), B(r) for each round r,
+// ending with B(R-1) (mode 2), or a single A or B block over all units.
+struct Sched {
+  int U, tpu, G, cta, mode, gu, rounds;
+  __device__ int nblocks() const { return mode == 2 ? 2 * rounds : 1; }
+  __device__ void block(int p, int* kind, int* r) const {
+    if (mode != 2) {
+      *kind = mode;
+      *r = 0;
+      return;
+    }
+    if (p == 0) { *kind = 0; *r = 0; }
+    else if (p == 2 * rounds - 1) { *kind = 1; *r = rounds - 1; }
+    else if (p & 1) { *kind = 0; *r = (p + 1) / 2; }
+    else { *kind = 1; *r = p / 2 - 1; }
+  }
+  __device__ int round_units(int r) const { return min(gu, U - r * gu); }
+  __device__ long long tiles(int r) const { return (long long)round_units(r) * tpu; }
+  __device__ long long start(int r, int c) const { return tiles(r) * c / G; }
+  // CTA whose range holds round-local tile t.
+  __device__ int owner(int r, long long t) const {
+    const long long T = tiles(r);
+    return (int)(((t + 1) * G + T - 1) / T) - 1;
+  }
+  __device__ int first_cta(int u) const {
+    const int r = u / gu;
+    return owner(r, (long long)(u - r * gu) * tpu);
+  }
+  __device__ int nslots(int u) const {
+    const int r = u / gu;
+    const long long t0 = (long long)(u - r * gu) * tpu;
+    return owner(r, t0 + tpu - 1) - owner(r, t0) + 1;
+  }
+};
+
+struct JobIter {
+  const Sched* sc;
+  int n;
+  int p, kind, r;
+  long long t, t_end, t_begin;
+  __device__ void init(const Sched* s, int n_) {
+    sc = s;
+    n = n_;
+    p = -1;
+    t = t_end = 0;
+  }
+  // Advances to the next block; returns false when none are left.
+  __device__ bool next_block() {
+    if (++p >= sc->nblocks()) return false;
+    sc->block(p, &kind, &r);
+    t_begin = t = sc->start(r, sc->cta);
+    t_end = sc->start(r, sc->cta + 1);
+    return true;
+  }
+  __device__ bool has_job() const { return t < t_end; }
+  __device__ Job job() const {
+    Job j;
+    j.kind = kind;
+    j.r = r;
+    const int lu = (int)(t / sc->tpu), ti = (int)(t % sc->tpu);
+    j.u = r * sc->gu + lu;
+    j.j0 = ti * kTile;
+    j.len = min(kTile, n - j.j0);
+    j.seg_first = (t == t_begin) || ti == 0;
+    j.seg_last = (t + 1 == t_end) || ti == sc->tpu - 1;
+    return j;
+  }
+  __device__ void advance() { ++t; }
+};
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);   // .x (low half) = lo
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st_wait() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+// D[tmem] (+)= A[tmem] * B[smem]^T, kind::f16.
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
+                                            uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ int ld_acquire(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+struct Bars {
+  uint64_t ring_full[kRing], ring_empty[kRing];
+  uint64_t q_full[2], q_empty[2];
+  uint64_t s_full[2], s_done[2];
+  uint64_t y_full[2], y_empty[2];
+  uint64_t drain;
+  uint32_t tmem;
+  int abort;
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_score_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+               const __grid_constant__ CUtensorMap tmV, Args a) {
+  extern __shared__ __align__(1024) uint8_t smraw[];
+  uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
+  Bars* bars = (Bars*)(sm + kOffBar);
+  float* red = (float*)(sm + kOffRed);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+  Sched sc{a.U, a.tpu, (int)gridDim.x, (int)blockIdx.x, a.mode, a.gu, a.rounds};
+
+  if (tid == 0) {
+    for (int i = 0; i < kRing; ++i) {
+      mbar_init(&bars->ring_full[i], 1);
+      mbar_init(&bars->ring_empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bars->q_full[i], 1);
+      mbar_init(&bars->q_empty[i], 1);
+      mbar_init(&bars->s_full[i], 1);
+      mbar_init(&bars->s_done[i], 128);
+      mbar_init(&bars->y_full[i], 1);
+      mbar_init(&bars->y_empty[i], 128);
+    }
+    mbar_init(&bars->drain, 1);
+    bars->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&bars->tmem, 512);
+    tmem_relinquish();
+  }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem;
+  volatile int* abort_flag = &bars->abort;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      prefetch_tensormap(&tmQ);
+      prefetch_tensormap(&tmK);
+      prefetch_tensormap(&tmV);
+      const uint64_t keep = l2_evict_last(), stream = l2_evict_first();
+      JobIter it;
+      it.init(&sc, a.n);
+      uint32_t slot = 0, ring_use = 0;   // ring_use counts loads
+      int seg = 0, qissued = 0;
+      bool ok = true;
+      while (ok && it.next_block()) {
+        for (; ok && it.has_job(); it.advance()) {
+          const Job j = it.job();
+          if (j.seg_first) {
+            const int qs = seg & 1;
+            if (seg >= 2) ok = mbar_wait(&bars->q_empty[qs], ((seg >> 1) - 1) & 1, abort_flag,
+                                         kWaitBudget);
+            if (!ok) break;
+            ++qissued;
+            mbar_expect_tx(&bars->q_full[qs], kTileBytes);
+            uint8_t* dq = sm + kOffQ + qs * kTileBytes;
+            tma_load_3d(dq, &tmQ, &bars->q_full[qs], 0, 0, j.u, keep);
+            tma_load_3d(dq + kTileBytes / 2, &tmQ, &bars->q_full[qs], 64, 0, j.u, keep);
+          }
+          const int loads = j.kind == 1 ? 2 : 1;
+          for (int l = 0; l < loads && ok; ++l) {
+            if (ring_use >= kRing)
+              ok = mbar_wait(&bars->ring_empty[slot], ((ring_use / kRing) - 1) & 1, abort_flag,
+                             kWaitBudget);
+            if (!ok) break;
+            const CUtensorMap* map = l == 0 ? &tmK : &tmV;
+            const uint64_t pol = (l == 0 && j.kind == 0 && a.mode == 2) ? keep : stream;
+            uint8_t* dst = sm + kOffRing + slot * kTileBytes;
+            mbar_expect_tx(&bars->ring_full[slot], kTileBytes);
+            tma_load_3d(dst, map, &bars->ring_full[slot], 0, j.j0, j.u, pol);
+            tma_load_3d(dst + kTileBytes / 2, map, &bars->ring_full[slot], 64, j.j0, j.u, pol);
+            ++ring_use;
+            slot = (slot + 1) % kRing;
+          }
+          if (j.seg_last) ++seg;
+        }
+      }
+      // let every issued load land before the CTA can exit
+      for (uint32_t i = ring_use > kRing ? ring_use - kRing : 0; i < ring_use; ++i)
+        mbar_wait(&bars->ring_full[i % kRing], (i / kRing) & 1, abort_flag, kWaitBudget);
+      const int qloads = qissued;
+      for (int i = qloads > 2 ? qloads - 2 : 0; i < qloads; ++i)
+        mbar_wait(&bars->q_full[i & 1], (i >> 1) & 1, abort_flag, kWaitBudget);
+    }
+  } else if (warp == 1) {
+    // ----------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      const uint32_t id_s = idesc_bf16(kRows, kTile, 0, 0);   // S = Q K^T, both K-major
+      const uint32_t id_y = idesc_bf16(kRows, kD, 0, 1);      // Y += P V, V MN-major
+      JobIter it;
+      it.init(&sc, a.n);
+      uint32_t slot = 0, ring_use = 0;
+      int seg = 0, bseg = 0, i = 0;
+      bool ok = true;
+      // the pending pass-B job whose Y MMA is issued after the next S MMA
+      bool pend = false;
+      Job pj{};
+      int p_i = 0, p_yb = 0;
+      uint32_t p_vslot = 0, p_vuse = 0;
+      int ybuf_uses[2] = {0, 0};
+      while (ok && it.next_block()) {
+        for (; ok && it.has_job(); it.advance()) {
+          const Job j = it.job();
+          const int b = i & 1, use = i >> 1;
+          if (j.seg_first) {
+            ok = mbar_wait(&bars->q_full[seg & 1], (seg >> 1) & 1, abort_flag, kWaitBudget);
+            if (!ok) break;
+          }
+          const uint32_t kslot = slot, kuse = ring_use;
+          ok = mbar_wait(&bars->ring_full[kslot], (kuse / kRing) & 1, abort_flag, kWaitBudget);
+          if (ok && use >= 1)
+            ok = mbar_wait(&bars->s_done[b], (use - 1) & 1, abort_flag, kWaitBudget);
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t qa = smem_u32(sm + kOffQ + (seg & 1) * kTileBytes);
+          const uint32_t ka = smem_u32(sm + kOffRing + kslot * kTileBytes);
+#pragma unroll
+          for (int kk = 0; kk < kD / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
+            mma_bf16(tmem + kColS + b * kTile, sw128_desc(qa + off, 16, 1024),
+                     sw128_desc(ka + off, 16, 1024), id_s, kk > 0);
+          }
+          mma_commit(&bars->ring_empty[kslot]);
+          mma_commit(&bars->s_full[b]);
+          ++ring_use;
+          slot = (slot + 1) % kRing;
+          if (j.seg_last) {
+            mma_commit(&bars->q_empty[seg & 1]);
+            ++seg;
+          }
+          uint32_t vslot = 0, vuse = 0;
+          if (j.kind == 1) {
+            vslot = slot;
+            vuse = ring_use;
+            ++ring_use;
+            slot = (slot + 1) % kRing;
+          }
+          // Y MMA of the previous pass-B job (its P is ready once s_done fires)
+          if (pend) {
+            const int pb = p_i & 1, puse = p_i >> 1;
+            const int yb = p_yb;
+            if (pj.seg_first && ybuf_uses[yb] >= 1)
+              ok = mbar_wait(&bars->y_empty[yb], (ybuf_uses[yb] - 1) & 1, abort_flag,
+                             kWaitBudget);
+            if (ok) ok = mbar_wait(&bars->s_done[pb], puse & 1, abort_flag, kWaitBudget);
+            if (ok)
+              ok = mbar_wait(&bars->ring_full[p_vslot], (p_vuse / kRing) & 1, abort_flag,
+                             kWaitBudget);
+            if (!ok) break;
+            tc_fence_after();
+            const uint32_t va = smem_u32(sm + kOffRing + p_vslot * kTileBytes);
+#pragma unroll
+            for (int kk = 0; kk < kTile / 16; ++kk)
+              mma_bf16_ts(tmem + kColY + yb * kD, tmem + kColS + pb * kTile + kk * 8,
+                          sw128_desc(va + kk * 2048, kTileBytes / 2, 1024), id_y,
+                          (pj.seg_first && kk == 0) ? 0u : 1u);
+            mma_commit(&bars->ring_empty[p_vslot]);
+            if (pj.seg_last) {
+              mma_commit(&bars->y_full[yb]);
+              ++ybuf_uses[yb];
+            }
+            pend = false;
+          }
+          if (j.kind == 1) {
+            pend = true;
+            pj = j;
+            p_i = i;
+            p_vslot = vslot;
+            p_vuse = vuse;
+            if (j.seg_first) p_yb = bseg & 1;
+            if (j.seg_last) ++bseg;
+          }
+          ++i;
+        }
+      }
+      if (ok && pend) {
+        const int pb = p_i & 1, puse = p_i >> 1;
+        const int yb = p_yb;
+        if (pj.seg_first && ybuf_uses[yb] >= 1)
+          ok = mbar_wait(&bars->y_empty[yb], (ybuf_uses[yb] - 1) & 1, abort_flag, kWaitBudget);
+        if (ok) ok = mbar_wait(&bars->s_done[pb], puse & 1, abort_flag, kWaitBudget);
+        if (ok)
+          ok = mbar_wait(&bars->ring_full[p_vslot], (p_vuse / kRing) & 1, abort_flag,
+                         kWaitBudget);
+        if (ok) {
+          tc_fence_after();
+          const uint32_t va = smem_u32(sm + kOffRing + p_vslot * kTileBytes);
+#pragma unroll
+          for (int kk = 0; kk < kTile / 16; ++kk)
+            mma_bf16_ts(tmem + kColY + yb * kD, tmem + kColS + pb * kTile + kk * 8,
+                        sw128_desc(va + kk * 2048, kTileBytes / 2, 1024), id_y,
+                        (pj.seg_first && kk == 0) ? 0u : 1u);
+          mma_commit(&bars->ring_empty[p_vslot]);
+          if (pj.seg_last) mma_commit(&bars->y_full[yb]);
+        }
+      }
+      // every MMA issued so far completes before TMEM can be released
+      mma_commit(&bars->drain);
+      mbar_wait(&bars->drain, 0, abort_flag, kWaitBudget);
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------------- compute groups
+    const int wg = (warp - 4) >> 2, q = warp & 3;
+    const int row = q * 32 + lane;
+    const bool row_ok = row < a.m;
+    const int lim = a.causal ? a.n - a.w + (row_ok ? row % a.w : 0) : a.n - 1;
+    const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
+    const uint32_t bar_id = 1 + wg;
+    JobIter it;
+    it.init(&sc, a.n);
+    int i = 0, bseg = 0, mine = 0;
+    bool ok = true;
+    float M = -INFINITY, L = 0.f;     // pass-A running stats (log2 units)
+    float lam = INFINITY;             // pass-B log2 normaliser of this row
+    int yuse[2] = {0, 0};
+    while (ok && it.next_block()) {
+      if (it.kind == 1 && a.mode == 2 && it.has_job()) {
+        // every CTA must have finished pass A of this round
+        const long long t0 = clock64();
+        const int target = 2 * (int)gridDim.x;
+        while (ld_acquire(&a.round_done[it.r]) < target) {
+          if (*abort_flag || clock64() - t0 > kWaitBudget) {
+            *abort_flag = 1;
+            ok = false;
+            break;
+          }
+        }
+      }
+      for (; ok && it.has_job(); it.advance(), ++i) {
+        const Job j = it.job();
+        const int b = i & 1;
+        if (j.seg_first) {
+          if (j.kind == 0) {
+            M = -INFINITY;
+            L = 0.f;
+          } else {
+            // combine the pass-A slots of this unit
+            const int ns = sc.nslots(j.u);
+            float Mr = -INFINITY, Lr = 0.f;
+            for (int k = 0; k < ns; ++k)
+              for (int g = 0; g < 2; ++g) {
+                const float2 pr = a.pstats[(((size_t)j.u * a.maxc + k) * 2 + g) * kRows + row];
+                if (pr.x == -INFINITY) continue;
+                if (pr.x > Mr) {
+                  Lr = Lr * fast_exp2(Mr - pr.x) + pr.y;
+                  Mr = pr.x;
+                } else {
+                  Lr += pr.y * fast_exp2(pr.x - Mr);
+                }
+              }
+            lam = (row_ok && Lr > 0.f) ? Mr + __log2f(Lr) : INFINITY;
+            if (wg == 0 && row_ok && sc.first_cta(j.u) == (int)blockIdx.x) {
+              a.row_stats[((size_t)j.u * a.m + row) * 2 + 0] = Mr * 0.69314718055994531f;
+              a.row_stats[((size_t)j.u * a.m + row) * 2 + 1] = Lr;
+            }
+          }
+        }
+        if (b == wg) {
+          ok = mbar_wait(&bars->s_full[b], (i >> 1) & 1, abort_flag, kWaitBudget);
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t sbase = lane_addr + kColS + b * kTile;
+          if (j.kind == 0) {
+#pragma unroll 1
+            for (int c = 0; c < 4; ++c) {
+              float v[32];
+              tmem_ld32(sbase + c * 32, v);
+              tmem_ld_wait();
+              float vmax = -INFINITY;
+#pragma unroll
+              for (int e = 0; e < 32; ++e) {
+                const int jj = j.j0 + c * 32 + e;
+                if (jj > lim || jj >= a.n || !row_ok) v[e] = -INFINITY;
+                vmax = fmaxf(vmax, v[e]);
+              }
+              if (vmax == -INFINITY) continue;
+              const float cm = vmax * a.sl2;
+              if (cm > M) {
+                L *= fast_exp2(M - cm);
+                M = cm;
+              }
+              float s = 0.f;
+#pragma unroll
+              for (int e = 0; e < 32; ++e) s += fast_exp2(fmaf(v[e], a.sl2, -M));
+              L += s;
+            }
+            tc_fence_before();
+            mbar_arrive(&bars->s_done[b]);
+          } else {
+            float* rb = red + ((wg * 2 + (mine & 1)) * 4) * kTile;
+#pragma unroll 1
+            for (int c = 0; c < 4; ++c) {
+              float v[32];
+              tmem_ld32(sbase + c * 32, v);
+              tmem_ld_wait();
+#pragma unroll
+              for (int e = 0; e < 32; ++e) {
+                const int jj = j.j0 + c * 32 + e;
+                v[e] = (jj > lim || jj >= a.n || !row_ok) ? 0.f
+                                                          : fast_exp2(fmaf(v[e], a.sl2, -lam));
+              }
+              uint32_t pk[16];
+#pragma unroll
+              for (int e = 0; e < 16; ++e) pk[e] = pack_bf16(v[2 * e], v[2 * e + 1]);
+              tmem_st16(sbase + c * 16, pk);
+              // transpose-reduce: lane t ends with the warp's sum for token 32c + t
+#pragma unroll
+              for (int h = 16; h >= 1; h >>= 1) {
+                const bool up = (lane & h) != 0;
+#pragma unroll
+                for (int e = 0; e < h; ++e) {
+                  const float send = up ? v[e] : v[e + h];
+                  const float keep = up ? v[e + h] : v[e];
+                  v[e] = keep + __shfl_xor_sync(0xffffffffu, send, h);
+                }
+              }
+              rb[q * kTile + c * 32 + lane] = v[0];
+            }
+            tmem_st_wait();
+            tc_fence_before();
+            mbar_arrive(&bars->s_done[b]);
+            named_bar(bar_id, 128);
+            const int jj = q * 32 + lane;
+            const float cs = ((rb[jj] + rb[kTile + jj]) + rb[2 * kTile + jj]) + rb[3 * kTile + jj];
+            if (j.j0 + jj < a.P && jj < j.len) a.scores[(size_t)j.u * a.P + j.j0 + jj] = cs;
+            ++mine;
+          }
+        }
+        if (j.seg_last) {
+          if (j.kind == 0) {
+            const int k = (int)blockIdx.x - sc.first_cta(j.u);
+            // k < maxc always holds (the host sizes maxc from the same
+            // partition); the check only keeps a broken launch in bounds.
+            if (k >= 0 && k < a.maxc)
+              a.pstats[(((size_t)j.u * a.maxc + k) * 2 + wg) * kRows + row] = make_float2(M, L);
+          } else {
+            const int yb = bseg & 1;
+            if (b == wg) {   // this group ran the segment's last tile: it flushes Y
+              ok = mbar_wait(&bars->y_full[yb], yuse[yb] & 1, abort_flag, kWaitBudget);
+              if (!ok) break;
+              tc_fence_after();
+              const uint32_t ybase = lane_addr + kColY + yb * kD;
+#pragma unroll 1
+              for (int c = 0; c < 4; ++c) {
+                float v[32];
+                tmem_ld32(ybase + c * 32, v);
+                tmem_ld_wait();
+                if (row_ok) {
+                  float4* dst = (float4*)(a.y + ((size_t)j.u * a.m + row) * kD + c * 32);
+#pragma unroll
+                  for (int e = 0; e < 8; ++e)
+                    atomicAdd(dst + e, make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2],
+                                                   v[4 * e + 3]));
+                }
+              }
+              tc_fence_before();
+              mbar_arrive(&bars->y_empty[yb]);
+            }
+            ++yuse[yb];
+            ++bseg;
+          }
+        }
+      }
+      if (ok && it.kind == 0 && a.mode == 2) {
+        // this group's pass-A statistics of the round are in place
+        __threadfence();
+        named_bar(bar_id, 128);
+        if (q == 0 && lane == 0) atomicAdd(&a.round_done[it.r], 1);
+      }
+    }
+    if (!ok && row == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
+int g_num_sms[64] = {};
+
+}  // namespace
+
+bool score_tc_supported(const Shape& s) { return s.dtype == GRKV_BF16 && s.m <= kRows; }
+
+size_t score_tc_pstats_bytes(const Shape& s, int* maxc, int* gu, int* rounds, int sms) {
+  const int tpu = (s.n + kTile - 1) / kTile;
+  const size_t unit_k = (size_t)s.n * kD * 2;
+  const size_t budget = (size_t)64 << 20;   // K of two rounds resident in L2
+  int g = (int)std::max<size_t>(1, budget / (2 * unit_k));
+  g = std::min(g, s.U);
+  const int R = (s.U + g - 1) / g;
+  const int last = s.U - (R - 1) * g;
+  const long long tmin = (long long)std::min(g, last) * tpu;
+  const int mc = (int)std::min<long long>(sms, ((long long)tpu * sms + tmin - 1) / tmin + 2);
+  *maxc = mc;
+  *gu = g;
+  *rounds = R;
+  return (size_t)s.U * mc * 2 * kRows * sizeof(float2);
+}
+
+int sm_count() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (!g_num_sms[dev] &&
+      cudaDeviceGetAttribute(&g_num_sms[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    g_num_sms[dev] = 0;
+  return g_num_sms[dev];
+}
+
+cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const void* v,
+                            float* scores, float* y, float* row_stats, char* ws,
+                            const WsLayout& L, int mode, cudaStream_t st) {
+  CUtensorMap mq, mk, mv;
+  if (!encode_bf16_3d(&mq, q, kD, s.m, s.U, 64, kRows) ||
+      !encode_bf16_3d(&mk, k, kD, s.n, s.U, 64, kTile) ||
+      !encode_bf16_3d(&mv, v, kD, s.n, s.U, 64, kTile))
+    return cudaErrorInvalidValue;
+  const int G = sm_count();
+  if (G <= 0 || G > kMaxScoreCtas) return cudaErrorInvalidDevice;
+  Args a{};
+  a.U = s.U;
+  a.n = s.n;
+  a.w = s.w;
+  a.m = s.m;
+  a.P = s.P;
+  a.causal = s.causal;
+  a.tpu = (s.n + kTile - 1) / kTile;
+  int maxc, gu, rounds;
+  score_tc_pstats_bytes(s, &maxc, &gu, &rounds, G);
+  a.maxc = maxc;
+  a.gu = gu;
+  a.rounds = rounds;
+  a.sl2 = (float)((double)s.scale * 1.4426950408889634);
+  a.scores = scores;
+  a.y = y;
+  a.row_stats = row_stats;
+  a.pstats = (float2*)(ws + L.pstats_tc);
+  a.round_done = (int*)(ws + L.rounds_tc);
+  a.status = (int*)(ws + L.status);
+  cudaError_t e = cudaMemsetAsync(y, 0, (size_t)s.U * s.m * kD * sizeof(float), st);
+  if (e != cudaSuccess) return e;
+  e = cudaMemsetAsync(a.round_done, 0, (size_t)rounds * sizeof(int), st);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(k_score_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+  if (e != cudaSuccess) return e;
+  auto launch = [&](int md) {
+    a.mode = md;
+    if (md != 2) {
+      a.gu = s.U;
+      a.rounds = 1;
+    } else {
+      a.gu = gu;
+      a.rounds = rounds;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(G);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = md == 2 ? 1 : 0;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    count_launches(1);
+    return cudaLaunchKernelEx(&cfg, k_score_tc, mq, mk, mv, a);
+  };
+  if (mode == 2) return launch(2);
+  e = launch(0);
+  if (e != cudaSuccess) return e;
+  return launch(1);
+}
+
+}  // namespace grkv

@@ -33,6 +33,18 @@ def oracle_params(wl: gi.Workload, **over) -> O.Params:
     return O.Params(**kw)
 
 
+def uses_tensor_cores(p) -> bool:
+    """The library scores on the tensor cores for bf16 with m <= 128."""
+    return (p.dtype == b.GRKV_BF16 and p.group * p.window <= 128
+            and not (p.flags & b.GRKV_FORCE_SIMT))
+
+
+def y_tol_extra(p) -> float:
+    """The tensor-core path rounds P to bf16 before Y = P V: relative 2^-9
+    per term, counted as 2^-8."""
+    return 2.0 ** -8 if uses_tensor_cores(p) else 0.0
+
+
 def lib_params(wl: gi.Workload, units: int, **over) -> b.grkv_params:
     p = b.params(units, wl.group, wl.n, wl.window, wl.budget, pool_kernel=wl.pool_kernel,
                  lambda_v=wl.lambda_v, dtype=wl.dtype)
