@@ -30,6 +30,14 @@ int check_ptr(const void* p, size_t elems) {
 
 int cuda_rc(cudaError_t e) { return e == cudaSuccess ? GRKV_OK : GRKV_ERR_CUDA; }
 
+cudaError_t launch_merge(const Shape& s, const void* q, const void* k, const void* v,
+                         const float* scores, const float* y, const int32_t* idx, void* k_out,
+                         void* v_out, char* ws, const WsLayout& L, cudaStream_t st) {
+  if (s.tc_merge)
+    return launch_merge_tc(s, q, k, v, scores, y, idx, k_out, v_out, ws, L, st);
+  return launch_merge_simt(s, q, k, v, scores, y, idx, k_out, v_out, ws, L, st);
+}
+
 cudaError_t launch_score(const Shape& s, const void* q, const void* k, const void* v,
                          float* scores, float* y, float* row_stats, char* ws, const WsLayout& L,
                          cudaStream_t st) {
@@ -92,6 +100,7 @@ int make_shape(const grkv_params* p, Shape* s) {
   s->lambda_inf = std::isinf(p->lambda_v) ? 1 : 0;
   s->scale = p->scale != 0.f ? p->scale : (float)(1.0 / std::sqrt((double)p->d));
   s->tc = (p->flags & GRKV_FORCE_SIMT) ? 0 : (score_tc_supported(*s) ? 1 : 0);
+  s->tc_merge = (s->tc && merge_tc_supported(*s)) ? 1 : 0;
   s->two_pass = (p->flags & GRKV_TWO_PASS) ? 1 : 0;
   return GRKV_OK;
 }
@@ -121,10 +130,12 @@ WsLayout plan_workspace(const Shape& s) {
     L.ypart = take(U * L.nchunk * m * d * 4);
   }
   L.pooled = take(U * (size_t)s.P * 4);
-  L.xbuf = take(U * m * (size_t)s.B * 4);
-  L.flags = take(U * (size_t)s.B);
-  L.gram = take(U * m * m * 8);
-  L.rz = take(U * m * d * 8);
+  if (!s.tc_merge) {
+    L.xbuf = take(U * m * (size_t)s.B * 4);
+    L.flags = take(U * (size_t)s.B);
+    L.gram = take(U * m * m * 8);
+    L.rz = take(U * m * d * 8);
+  }
   L.scores = take(U * (size_t)s.P * 4);
   L.y = take(U * m * d * 4);
   L.rstats = take(U * m * 8);
@@ -214,7 +225,7 @@ int grkv_merge(const grkv_params* p, const void* q, const void* k, const void* v
   char* w = (char*)ws;
   GRKV_TRY(cuda_rc(cudaMemsetAsync(w + L.status, 0, 4, st)));
   if (s.U == 0) return GRKV_OK;
-  return cuda_rc(launch_merge_simt(s, q, k, v, scores, y, idx, k_out, v_out, w, L, st));
+  return cuda_rc(launch_merge(s, q, k, v, scores, y, idx, k_out, v_out, w, L, st));
 }
 
 int grkv_compress(const grkv_params* p, const void* q, const void* k, const void* v, void* k_out,
@@ -236,7 +247,7 @@ int grkv_compress(const grkv_params* p, const void* q, const void* k, const void
   float* rstats = (float*)(w + L.rstats);
   GRKV_TRY(cuda_rc(launch_score(s, q, k, v, scores, y, rstats, w, L, st)));
   GRKV_TRY(cuda_rc(launch_select(s, scores, idx, w, L, st)));
-  return cuda_rc(launch_merge_simt(s, q, k, v, scores, y, idx, k_out, v_out, w, L, st));
+  return cuda_rc(launch_merge(s, q, k, v, scores, y, idx, k_out, v_out, w, L, st));
 }
 
 int grkv_status(const void* ws, int* device_status, void* stream) {

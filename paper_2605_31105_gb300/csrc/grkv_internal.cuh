@@ -24,6 +24,7 @@ struct Shape {
   float lambda, scale;
   int lambda_inf; // lambda_v == +inf: values stay V0
   int tc;         // bf16, m <= 128, not forced portable: tensor-core scoring
+  int tc_merge;   // ... and B <= 32768: tensor-core value merge
   int two_pass;   // tensor-core scoring as two launches
 };
 
@@ -83,6 +84,12 @@ int sm_count();
 cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const void* v,
                             float* scores, float* y, float* row_stats, char* ws,
                             const WsLayout& L, int mode, cudaStream_t st);
+
+// Tensor-core value merge (bf16, m <= 128, B <= 32768).
+bool merge_tc_supported(const Shape& s);
+cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const void* v,
+                            const float* scores, const float* y, const int32_t* idx, void* k_out,
+                            void* v_out, char* ws, const WsLayout& L, cudaStream_t st);
 
 // Selection with the pooled-score scratch [U][n-w] given directly.
 cudaError_t launch_select_pooled(const Shape& s, const float* scores, int32_t* idx,

@@ -101,6 +101,8 @@ struct Sched {
     const int r = u / gu;
     return owner(r, (long long)(u - r * gu) * tpu);
   }
+  // True if CTA c holds no tile of round r (more CTAs than tiles).
+  __device__ bool empty(int r, int c) const { return start(r, c) == start(r, c + 1); }
   __device__ int nslots(int u) const {
     const int r = u / gu;
     const long long t0 = (long long)(u - r * gu) * tpu;
@@ -433,9 +435,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             L = 0.f;
           } else {
             // combine the pass-A slots of this unit
-            const int ns = sc.nslots(j.u);
+            const int ns = sc.nslots(j.u), c0 = sc.first_cta(j.u);
             float Mr = -INFINITY, Lr = 0.f;
-            for (int k = 0; k < ns; ++k)
+            for (int k = 0; k < ns; ++k) {
+              if (sc.empty(j.r, c0 + k)) continue;   // that CTA wrote no slot
               for (int g = 0; g < 2; ++g) {
                 const float2 pr = a.pstats[(((size_t)j.u * a.maxc + k) * 2 + g) * kRows + row];
                 if (pr.x == -INFINITY) continue;
@@ -446,6 +449,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                   Lr += pr.y * fast_exp2(pr.x - Mr);
                 }
               }
+            }
             lam = (row_ok && Lr > 0.f) ? Mr + __log2f(Lr) : INFINITY;
             if (wg == 0 && row_ok && sc.first_cta(j.u) == (int)blockIdx.x) {
               a.row_stats[((size_t)j.u * a.m + row) * 2 + 0] = Mr * 0.69314718055994531f;

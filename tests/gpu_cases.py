@@ -87,7 +87,10 @@ class Case:
 
 
 def workspace(p) -> torch.Tensor:
-    return torch.empty(max(256, b.grkv_workspace_size(p)), dtype=torch.uint8, device="cuda")
+    """A workspace filled with a NaN byte pattern, so a kernel that reads a
+    workspace byte it did not write first cannot pass by luck."""
+    return torch.full((max(256, b.grkv_workspace_size(p)),), 0xFF, dtype=torch.uint8,
+                      device="cuda")
 
 
 def run_score(c: Case, p):

@@ -79,12 +79,15 @@ def test_select_stage_bit_exact(prep):
         np.testing.assert_array_equal(idx[i], ora["idx"])
 
 
-def test_merge_stage(prep):
+@pytest.mark.parametrize("path", ["default", "portable"])
+def test_merge_stage(prep, path):
     c, op = prep.case, prep.op
     scores32 = np.stack([o["scores32"] for o in prep.ora])
     y32 = np.stack([o["y"].astype(np.float32) for o in prep.ora])
     idx = np.stack([o["idx"] for o in prep.ora])
-    ko, vo = G.run_merge(c, prep.p, scores32, y32, idx)
+    p = G.lib_params(prep.wl, c.U, **prep.over)
+    p.flags = PATHS[path]
+    ko, vo = G.run_merge(c, p, scores32, y32, idx)
     for i in range(c.U):
         ref = O.merge_unit(c.q[i], c.k[i], c.v[i], scores32[i], y32[i], idx[i], op)
         np.testing.assert_array_equal(ko[i], c.k[i][idx[i]])            # K_out = K0
