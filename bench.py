@@ -40,11 +40,14 @@ def args_():
     ap.add_argument("--workload", default="c2_llama_32k_bf16")
     ap.add_argument("--n", type=int, default=0, help="override N (sweep points)")
     ap.add_argument("--budget", type=int, default=0, help="override B (sweep points)")
+    ap.add_argument("--units", type=int, default=0,
+                    help="take only the first U units of the workload (profiling slices)")
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
-    ap.add_argument("--path", choices=("default", "two_pass", "portable"), default="default",
-                    help="scoring kernels to use (default: fused tensor-core rounds)")
+    ap.add_argument("--path", choices=("default", "fused", "portable"), default="default",
+                    help="scoring kernels: default (two tensor-core launches), fused (one launch "
+                         "in L2-sized rounds) or portable (CUDA cores)")
     return ap.parse_args()
 
 
@@ -55,6 +58,8 @@ def workload(a):
         n, bud = a.n or wl.n, a.budget or wl.budget
         wl = wl.replace(name=f"{wl.name}_n{n}_b{bud}", n=n, budget=bud,
                         seed=gi.seed_for(wl.seed, n, bud))
+    if a.units:
+        wl = wl.replace(name=f"{wl.name}_first{a.units}", units=min(a.units, wl.units))
     return wl
 
 
@@ -274,7 +279,7 @@ def run_ours(a):
     dq, dk, dv = hq.cuda(), hk.cuda(), hv.cuda()
     p = b.params(U, wl.group, n, wl.window, B, pool_kernel=wl.pool_kernel,
                  lambda_v=wl.lambda_v, dtype=wl.dtype,
-                 flags={"default": 0, "two_pass": b.GRKV_TWO_PASS,
+                 flags={"default": 0, "fused": b.GRKV_FUSED_SCORE,
                         "portable": b.GRKV_FORCE_SIMT}[a.path])
     ws = torch.empty(b.grkv_workspace_size(p), dtype=torch.uint8, device="cuda")
     ko = torch.empty((U, B, d), dtype=tdt, device="cuda")

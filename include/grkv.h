@@ -67,9 +67,9 @@ extern "C" {
 
 #define GRKV_UPDATE_K      0x1u  /* key step (Sec. 3.4, Eq. key_dual_update): not implemented */
 #define GRKV_FORCE_SIMT    0x2u  /* use the portable CUDA-core kernels even for bf16 */
-#define GRKV_TWO_PASS      0x4u  /* tensor-core scoring: run the statistics and the
-                                    probability pass as two launches (no L2 reuse of K
-                                    between them); for measurement */
+#define GRKV_FUSED_SCORE   0x4u  /* tensor-core scoring in one persistent launch whose
+                                    L2-sized rounds let the probability pass re-read K
+                                    from L2 (default: two launches, K read twice) */
 
 typedef struct {
   int32_t units;        /* U >= 0: independent (batch x layer x KV head) problems   */

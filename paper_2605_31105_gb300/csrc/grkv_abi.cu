@@ -42,7 +42,7 @@ cudaError_t launch_score(const Shape& s, const void* q, const void* k, const voi
                          float* scores, float* y, float* row_stats, char* ws, const WsLayout& L,
                          cudaStream_t st) {
   if (s.tc)
-    return launch_score_tc(s, q, k, v, scores, y, row_stats, ws, L, s.two_pass ? 0 : 2, st);
+    return launch_score_tc(s, q, k, v, scores, y, row_stats, ws, L, s.fused ? 2 : 0, st);
   return launch_score_simt(s, q, k, v, scores, y, row_stats, ws, L, st);
 }
 
@@ -75,7 +75,7 @@ int make_shape(const grkv_params* p, Shape* s) {
   if (!(p->scale >= 0.f) || std::isinf(p->scale)) return GRKV_ERR_INVALID_ARG;
   if (p->causal != 0 && p->causal != 1) return GRKV_ERR_INVALID_ARG;
   if (p->dtype != GRKV_F32 && p->dtype != GRKV_BF16) return GRKV_ERR_INVALID_ARG;
-  if (p->flags & ~(GRKV_UPDATE_K | GRKV_FORCE_SIMT | GRKV_TWO_PASS)) return GRKV_ERR_INVALID_ARG;
+  if (p->flags & ~(GRKV_UPDATE_K | GRKV_FORCE_SIMT | GRKV_FUSED_SCORE)) return GRKV_ERR_INVALID_ARG;
   if (p->d < 1) return GRKV_ERR_INVALID_ARG;
   if (p->flags & GRKV_UPDATE_K) return GRKV_ERR_UNSUPPORTED;
   if (p->d != kD) return GRKV_ERR_UNSUPPORTED;
@@ -101,7 +101,7 @@ int make_shape(const grkv_params* p, Shape* s) {
   s->scale = p->scale != 0.f ? p->scale : (float)(1.0 / std::sqrt((double)p->d));
   s->tc = (p->flags & GRKV_FORCE_SIMT) ? 0 : (score_tc_supported(*s) ? 1 : 0);
   s->tc_merge = (s->tc && merge_tc_supported(*s)) ? 1 : 0;
-  s->two_pass = (p->flags & GRKV_TWO_PASS) ? 1 : 0;
+  s->fused = (p->flags & GRKV_FUSED_SCORE) ? 1 : 0;
   return GRKV_OK;
 }
 
@@ -124,7 +124,8 @@ WsLayout plan_workspace(const Shape& s) {
   if (s.tc) {
     int maxc, gu, rounds;
     L.pstats_tc = take(score_tc_pstats_bytes(s, &maxc, &gu, &rounds, kMaxScoreCtas));
-    L.rounds_tc = take((size_t)rounds * sizeof(int));
+    L.ustats_tc = take(U * 128 * sizeof(float2));
+    L.flags_tc = take(2 * U * sizeof(int));
   } else {
     L.pstats = take(U * L.nchunk * m * 8);
     L.ypart = take(U * L.nchunk * m * d * 4);

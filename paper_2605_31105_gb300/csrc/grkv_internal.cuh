@@ -25,7 +25,7 @@ struct Shape {
   int lambda_inf; // lambda_v == +inf: values stay V0
   int tc;         // bf16, m <= 128, not forced portable: tensor-core scoring
   int tc_merge;   // ... and B <= 32768: tensor-core value merge
-  int two_pass;   // tensor-core scoring as two launches
+  int fused;      // tensor-core scoring as one launch in L2-sized rounds
 };
 
 // Byte offsets of the workspace regions (each 256-B aligned).
@@ -37,7 +37,8 @@ struct WsLayout {
   int chunk, nchunk;
   // score path (tensor cores)
   size_t pstats_tc;  // float2 [U][maxc][2][128] pass-A statistics slots
-  size_t rounds_tc;  // int [rounds] finished pass-A blocks per round
+  size_t ustats_tc;  // float2 [U][128] combined pass-A statistics per unit
+  size_t flags_tc;   // int [2][U] slots written / statistics ready per unit
   // select
   size_t pooled;  // float [U][P]
   // merge

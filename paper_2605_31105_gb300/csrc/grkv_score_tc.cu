@@ -7,7 +7,9 @@
 // key, so the keys are read twice.  This kernel is persistent (one CTA per
 // SM) and processes the units in rounds small enough that a round's keys stay
 // in L2: each CTA runs pass A of round r+1 and then pass B of round r, so the
-// second read of K is served from L2 and only K and V cross HBM once.
+// second read of K is served from L2 and only K and V cross HBM once (mode 2,
+// GRKV_FUSED_SCORE).  By default the two passes run as two launches over all
+// units (modes 0 and 1), which reads K twice but needs no cross-CTA waits.
 //
 // Roles (384 threads): warp 0 issues TMA loads (Q per segment, K and V
 // tiles of 128 tokens through a 4-slot ring), warp 1 issues tcgen05 MMAs
@@ -35,7 +37,7 @@ using namespace sm100;
 constexpr int kTile = 128;            // tokens per tile
 constexpr int kRows = 128;            // window rows (m padded to 128)
 constexpr int kRing = 4;              // K / V ring slots
-constexpr int kThreads = 384;
+constexpr int kThreads = 512;
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KB
 constexpr long long kWaitBudget = 1ll << 32;      // cycles (~2 s) before a wait gives up
 
@@ -43,7 +45,9 @@ constexpr long long kWaitBudget = 1ll << 32;      // cycles (~2 s) before a wait
 constexpr uint32_t kOffQ = 0;                                   // 2 x 32 KB
 constexpr uint32_t kOffRing = kOffQ + 2 * kTileBytes;           // 4 x 32 KB
 constexpr uint32_t kOffRed = kOffRing + kRing * kTileBytes;     // [2 wg][2 buf][4][128] fp32
-constexpr uint32_t kOffBar = kOffRed + 2 * 2 * 4 * kTile * 4;
+constexpr uint32_t kOffAstat = kOffRed + 2 * 2 * 4 * kTile * 4;   // [2 buf][2 wg][128] float2
+constexpr uint32_t kOffLam = kOffAstat + 2 * 2 * kRows * 8;       // [2 buf][128] float
+constexpr uint32_t kOffBar = kOffLam + 2 * kRows * 4;
 constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;           // + alignment slack
 
 // TMEM columns: two S buffers, two Y accumulators.
@@ -61,7 +65,9 @@ struct Args {
   float* y;       // [U][m][128], zeroed by the host
   float* row_stats;  // [U][m][2]
   float2* pstats;    // [U][maxc][2][128]  (max in log2 units, sum)
-  int* round_done;   // [rounds], zeroed by the host
+  float2* ustats;    // [U][128] combined statistics of each unit (log2 units)
+  int* unit_cnt;     // [U] pass-A slots written, zeroed by the host
+  int* unit_ready;   // [U] 1 once ustats of the unit is in place, zeroed by the host
   int* status;
 };
 
@@ -103,6 +109,13 @@ struct Sched {
   }
   // True if CTA c holds no tile of round r (more CTAs than tiles).
   __device__ bool empty(int r, int c) const { return start(r, c) == start(r, c + 1); }
+  // Pass-A statistics slots written for unit u (one per CTA that holds its tiles).
+  __device__ int writers(int u) const {
+    const int r = u / gu, c0 = first_cta(u), ns = nslots(u);
+    int w = 0;
+    for (int k = 0; k < ns; ++k) w += empty(r, c0 + k) ? 0 : 1;
+    return w;
+  }
   __device__ int nslots(int u) const {
     const int r = u / gu;
     const long long t0 = (long long)(u - r * gu) * tpu;
@@ -178,6 +191,66 @@ __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, ui
       : "memory");
 }
 
+// 32 fp32 TMEM columns of this thread's lane; the values are valid only after
+// tmem_wait32 on the same array, which ties the registers to the wait.
+__device__ __forceinline__ void tmem_ld32f(uint32_t taddr, float* v) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, "
+      "%28, %29, %30, %31}, [%32];"
+      : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]), "=f"(v[4]), "=f"(v[5]), "=f"(v[6]),
+        "=f"(v[7]), "=f"(v[8]), "=f"(v[9]), "=f"(v[10]), "=f"(v[11]), "=f"(v[12]),
+        "=f"(v[13]), "=f"(v[14]), "=f"(v[15]), "=f"(v[16]), "=f"(v[17]), "=f"(v[18]),
+        "=f"(v[19]), "=f"(v[20]), "=f"(v[21]), "=f"(v[22]), "=f"(v[23]), "=f"(v[24]),
+        "=f"(v[25]), "=f"(v[26]), "=f"(v[27]), "=f"(v[28]), "=f"(v[29]), "=f"(v[30]),
+        "=f"(v[31])
+      : "r"(taddr)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_wait32(float* v) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+f"(v[0]), "+f"(v[1]), "+f"(v[2]), "+f"(v[3]), "+f"(v[4]), "+f"(v[5]),
+                 "+f"(v[6]), "+f"(v[7]), "+f"(v[8]), "+f"(v[9]), "+f"(v[10]), "+f"(v[11]),
+                 "+f"(v[12]), "+f"(v[13]), "+f"(v[14]), "+f"(v[15]), "+f"(v[16]), "+f"(v[17]),
+                 "+f"(v[18]), "+f"(v[19]), "+f"(v[20]), "+f"(v[21]), "+f"(v[22]), "+f"(v[23]),
+                 "+f"(v[24]), "+f"(v[25]), "+f"(v[26]), "+f"(v[27]), "+f"(v[28]), "+f"(v[29]),
+                 "+f"(v[30]), "+f"(v[31])
+               :
+               : "memory");
+}
+
+__device__ __forceinline__ float max32(const float* v) {
+  float m[16];
+#pragma unroll
+  for (int e = 0; e < 16; ++e) m[e] = fmaxf(v[e], v[e + 16]);
+#pragma unroll
+  for (int h = 8; h >= 1; h >>= 1)
+#pragma unroll
+    for (int e = 0; e < h; ++e) m[e] = fmaxf(m[e], m[e + h]);
+  return m[0];
+}
+
+// Pass A on 32 logits: online row max / sum of exp2 in log2 units.
+__device__ __forceinline__ void stats_chunk(float* v, bool full, int j0, int lim, int n,
+                                            bool row_ok, float sl2, float& M, float& L) {
+  if (!full) {
+#pragma unroll
+    for (int e = 0; e < 32; ++e)
+      if (j0 + e > lim || j0 + e >= n || !row_ok) v[e] = -INFINITY;
+  }
+  const float vmax = max32(v);
+  if (vmax == -INFINITY) return;
+  const float cm = vmax * sl2;
+  if (cm > M) {
+    L *= fast_exp2(M - cm);
+    M = cm;
+  }
+  float s[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int e = 0; e < 32; ++e) s[e & 3] += fast_exp2(fmaf(v[e], sl2, -M));
+  L += (s[0] + s[1]) + (s[2] + s[3]);
+}
+
 __device__ __forceinline__ int ld_acquire(const int* p) {
   int v;
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -189,6 +262,8 @@ struct Bars {
   uint64_t q_full[2], q_empty[2];
   uint64_t s_full[2], s_done[2];
   uint64_t y_full[2], y_empty[2];
+  uint64_t astat_full[2], astat_empty[2];   // compute groups -> statistics publisher
+  uint64_t lam_full[2], lam_empty[2];       // statistics fetcher -> compute groups
   uint64_t drain;
   uint32_t tmem;
   int abort;
@@ -217,6 +292,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars->s_done[i], 128);
       mbar_init(&bars->y_full[i], 1);
       mbar_init(&bars->y_empty[i], 128);
+      mbar_init(&bars->astat_full[i], 256);
+      mbar_init(&bars->astat_empty[i], 1);
+      mbar_init(&bars->lam_full[i], 1);
+      mbar_init(&bars->lam_empty[i], 256);
     }
     mbar_init(&bars->drain, 1);
     bars->abort = 0;
@@ -398,6 +477,162 @@ __global__ void __launch_bounds__(kThreads, 1)
       mma_commit(&bars->drain);
       mbar_wait(&bars->drain, 0, abort_flag, kWaitBudget);
     }
+  } else if (warp == 2) {
+    // ----------------------------------------------- statistics publisher
+    // Copies each pass-A segment's row statistics to its global slot; the
+    // unit's last writer combines all slots once and raises its ready flag.
+    float2* astat = (float2*)(sm + kOffAstat);
+    JobIter it;
+    it.init(&sc, a.n);
+    int aseg = 0;
+    bool ok = true;
+    while (ok && it.next_block()) {
+      for (; ok && it.has_job(); it.advance()) {
+        const Job j = it.job();
+        if (!(j.seg_last && j.kind == 0)) continue;
+        const int ab = aseg & 1;
+        ok = mbar_wait(&bars->astat_full[ab], (aseg >> 1) & 1, abort_flag, kWaitBudget);
+        if (!ok) break;
+        const int k = (int)blockIdx.x - sc.first_cta(j.u);
+        // k < maxc always holds (the host sizes maxc from the same partition)
+        if (k >= 0 && k < a.maxc) {
+          float2* slot = a.pstats + ((size_t)j.u * a.maxc + k) * 2 * kRows;
+#pragma unroll
+          for (int t = 0; t < 8; ++t) slot[t * 32 + lane] = astat[ab * 2 * kRows + t * 32 + lane];
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->astat_empty[ab]);
+        __threadfence();
+        __syncwarp();
+        int last = 0;
+        if (lane == 0) last = atomicAdd(&a.unit_cnt[j.u], 1) == sc.writers(j.u) - 1;
+        last = __shfl_sync(0xffffffffu, last, 0);
+        if (last) {
+          __threadfence();
+          const int ns = sc.nslots(j.u), c0 = sc.first_cta(j.u);
+          float Mr[4], Lr[4];
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            Mr[t] = -INFINITY;
+            Lr[t] = 0.f;
+          }
+          // four slots per round trip: 32 independent loads in flight per lane
+          for (int k0 = 0; k0 < ns; k0 += 4) {
+            float2 pr[4][8];
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk) {
+              const bool use = k0 + kk < ns && !sc.empty(j.r, c0 + k0 + kk);
+              const float2* sl = a.pstats + ((size_t)j.u * a.maxc + k0 + kk) * 2 * kRows;
+#pragma unroll
+              for (int t = 0; t < 8; ++t)
+                pr[kk][t] = use ? sl[(t & 1) * kRows + (t >> 1) * 32 + lane]
+                                : make_float2(-INFINITY, 0.f);
+            }
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)
+#pragma unroll
+              for (int t = 0; t < 8; ++t) {
+                const int rr = t >> 1;
+                const float2 v = pr[kk][t];
+                if (v.x == -INFINITY) continue;
+                if (v.x > Mr[rr]) {
+                  Lr[rr] = Lr[rr] * fast_exp2(Mr[rr] - v.x) + v.y;
+                  Mr[rr] = v.x;
+                } else {
+                  Lr[rr] += v.y * fast_exp2(v.x - Mr[rr]);
+                }
+              }
+          }
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            const int r = t * 32 + lane;
+            a.ustats[(size_t)j.u * kRows + r] = make_float2(Mr[t], Lr[t]);
+            if (r < a.m) {
+              a.row_stats[((size_t)j.u * a.m + r) * 2 + 0] = Mr[t] * 0.69314718055994531f;
+              a.row_stats[((size_t)j.u * a.m + r) * 2 + 1] = Lr[t];
+            }
+          }
+          __threadfence();
+          __syncwarp();
+          if (lane == 0) atomicExch(&a.unit_ready[j.u], 1);
+        }
+        ++aseg;
+      }
+    }
+  } else if (warp == 3) {
+    // ------------------------------------------------ statistics fetcher
+    // Ahead of each pass-B segment: wait for the unit's combined statistics
+    // and leave every row's log2 normaliser in shared memory.
+    float* lam_s = (float*)(sm + kOffLam);
+    JobIter it;
+    it.init(&sc, a.n);
+    int bseg = 0;
+    bool ok = true;
+    while (ok && it.next_block()) {
+      for (; ok && it.has_job(); it.advance()) {
+        const Job j = it.job();
+        if (!(j.seg_first && j.kind == 1)) continue;
+        const int lb = bseg & 1;
+        if (bseg >= 2)
+          ok = mbar_wait(&bars->lam_empty[lb], ((bseg >> 1) - 1) & 1, abort_flag, kWaitBudget);
+        if (!ok) break;
+        const long long t0 = clock64();
+        while (ld_acquire(&a.unit_ready[j.u]) == 0) {
+          if (*abort_flag || clock64() - t0 > kWaitBudget) {
+            *abort_flag = 1;
+            ok = false;
+            break;
+          }
+        }
+        if (!ok) break;
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const int r = t * 32 + lane;
+          const float2 st = a.ustats[(size_t)j.u * kRows + r];
+          lam_s[lb * kRows + r] = (r < a.m && st.y > 0.f) ? st.x + __log2f(st.y) : INFINITY;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->lam_full[lb]);
+        ++bseg;
+      }
+    }
+  } else if (warp >= 12) {
+    // ------------------------------------------------------- Y flusher
+    // Each pass-B segment's Y partial (TMEM, one row per lane) is added to
+    // the unit's Y with float4 atomics.
+    const int q = warp & 3, row = q * 32 + lane;
+    const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
+    JobIter it;
+    it.init(&sc, a.n);
+    int bseg = 0;
+    bool ok = true;
+    while (ok && it.next_block()) {
+      for (; ok && it.has_job(); it.advance()) {
+        const Job j = it.job();
+        if (!(j.seg_last && j.kind == 1)) continue;
+        const int yb = bseg & 1;
+        ok = mbar_wait(&bars->y_full[yb], (bseg >> 1) & 1, abort_flag, kWaitBudget);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t ybase = lane_addr + kColY + yb * kD;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          tmem_ld32(ybase + c * 32, v);
+          tmem_ld_wait();
+          if (row < a.m) {
+            float4* dst = (float4*)(a.y + ((size_t)j.u * a.m + row) * kD + c * 32);
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+              atomicAdd(dst + e, make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]));
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(&bars->y_empty[yb]);
+        ++bseg;
+      }
+    }
+    if (!ok && row == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
   } else if (warp >= 4) {
     // ------------------------------------------------------- compute groups
     const int wg = (warp - 4) >> 2, q = warp & 3;
@@ -406,26 +641,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int lim = a.causal ? a.n - a.w + (row_ok ? row % a.w : 0) : a.n - 1;
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
     const uint32_t bar_id = 1 + wg;
+    float2* astat = (float2*)(sm + kOffAstat);
+    const float* lam_s = (const float*)(sm + kOffLam);
     JobIter it;
     it.init(&sc, a.n);
-    int i = 0, bseg = 0, mine = 0;
+    int i = 0, aseg = 0, bseg = 0, mine = 0;
     bool ok = true;
     float M = -INFINITY, L = 0.f;     // pass-A running stats (log2 units)
     float lam = INFINITY;             // pass-B log2 normaliser of this row
-    int yuse[2] = {0, 0};
     while (ok && it.next_block()) {
-      if (it.kind == 1 && a.mode == 2 && it.has_job()) {
-        // every CTA must have finished pass A of this round
-        const long long t0 = clock64();
-        const int target = 2 * (int)gridDim.x;
-        while (ld_acquire(&a.round_done[it.r]) < target) {
-          if (*abort_flag || clock64() - t0 > kWaitBudget) {
-            *abort_flag = 1;
-            ok = false;
-            break;
-          }
-        }
-      }
       for (; ok && it.has_job(); it.advance(), ++i) {
         const Job j = it.job();
         const int b = i & 1;
@@ -434,27 +658,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             M = -INFINITY;
             L = 0.f;
           } else {
-            // combine the pass-A slots of this unit
-            const int ns = sc.nslots(j.u), c0 = sc.first_cta(j.u);
-            float Mr = -INFINITY, Lr = 0.f;
-            for (int k = 0; k < ns; ++k) {
-              if (sc.empty(j.r, c0 + k)) continue;   // that CTA wrote no slot
-              for (int g = 0; g < 2; ++g) {
-                const float2 pr = a.pstats[(((size_t)j.u * a.maxc + k) * 2 + g) * kRows + row];
-                if (pr.x == -INFINITY) continue;
-                if (pr.x > Mr) {
-                  Lr = Lr * fast_exp2(Mr - pr.x) + pr.y;
-                  Mr = pr.x;
-                } else {
-                  Lr += pr.y * fast_exp2(pr.x - Mr);
-                }
-              }
-            }
-            lam = (row_ok && Lr > 0.f) ? Mr + __log2f(Lr) : INFINITY;
-            if (wg == 0 && row_ok && sc.first_cta(j.u) == (int)blockIdx.x) {
-              a.row_stats[((size_t)j.u * a.m + row) * 2 + 0] = Mr * 0.69314718055994531f;
-              a.row_stats[((size_t)j.u * a.m + row) * 2 + 1] = Lr;
-            }
+            const int lb = bseg & 1;
+            ok = mbar_wait(&bars->lam_full[lb], (bseg >> 1) & 1, abort_flag, kWaitBudget);
+            if (!ok) break;
+            lam = lam_s[lb * kRows + row];
+            mbar_arrive(&bars->lam_empty[lb]);
           }
         }
         if (b == wg) {
@@ -462,44 +670,41 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!ok) break;
           tc_fence_after();
           const uint32_t sbase = lane_addr + kColS + b * kTile;
+          // tiles away from the window and the end of the unit need no mask
+          const bool full = row_ok && j.j0 + kTile - 1 <= lim && j.j0 + kTile <= a.n;
+          float va[32], vb[32];
+          tmem_ld32f(sbase, va);
+          tmem_wait32(va);
           if (j.kind == 0) {
-#pragma unroll 1
-            for (int c = 0; c < 4; ++c) {
-              float v[32];
-              tmem_ld32(sbase + c * 32, v);
-              tmem_ld_wait();
-              float vmax = -INFINITY;
-#pragma unroll
-              for (int e = 0; e < 32; ++e) {
-                const int jj = j.j0 + c * 32 + e;
-                if (jj > lim || jj >= a.n || !row_ok) v[e] = -INFINITY;
-                vmax = fmaxf(vmax, v[e]);
-              }
-              if (vmax == -INFINITY) continue;
-              const float cm = vmax * a.sl2;
-              if (cm > M) {
-                L *= fast_exp2(M - cm);
-                M = cm;
-              }
-              float s = 0.f;
-#pragma unroll
-              for (int e = 0; e < 32; ++e) s += fast_exp2(fmaf(v[e], a.sl2, -M));
-              L += s;
-            }
+            tmem_ld32f(sbase + 32, vb);
+            stats_chunk(va, full, j.j0, lim, a.n, row_ok, a.sl2, M, L);
+            tmem_wait32(vb);
+            tmem_ld32f(sbase + 64, va);
+            stats_chunk(vb, full, j.j0 + 32, lim, a.n, row_ok, a.sl2, M, L);
+            tmem_wait32(va);
+            tmem_ld32f(sbase + 96, vb);
+            stats_chunk(va, full, j.j0 + 64, lim, a.n, row_ok, a.sl2, M, L);
+            tmem_wait32(vb);
             tc_fence_before();
-            mbar_arrive(&bars->s_done[b]);
+            mbar_arrive(&bars->s_done[b]);   // S fully read
+            stats_chunk(vb, full, j.j0 + 96, lim, a.n, row_ok, a.sl2, M, L);
           } else {
             float* rb = red + ((wg * 2 + (mine & 1)) * 4) * kTile;
-#pragma unroll 1
-            for (int c = 0; c < 4; ++c) {
-              float v[32];
-              tmem_ld32(sbase + c * 32, v);
-              tmem_ld_wait();
 #pragma unroll
-              for (int e = 0; e < 32; ++e) {
-                const int jj = j.j0 + c * 32 + e;
-                v[e] = (jj > lim || jj >= a.n || !row_ok) ? 0.f
-                                                          : fast_exp2(fmaf(v[e], a.sl2, -lam));
+            for (int c = 0; c < 4; ++c) {
+              float* v = (c & 1) ? vb : va;
+              float* nx = (c & 1) ? va : vb;
+              if (c < 3) tmem_ld32f(sbase + (c + 1) * 32, nx);
+              if (full) {
+#pragma unroll
+                for (int e = 0; e < 32; ++e) v[e] = fast_exp2(fmaf(v[e], a.sl2, -lam));
+              } else {
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                  const int jj = j.j0 + c * 32 + e;
+                  v[e] = (jj > lim || jj >= a.n || !row_ok) ? 0.f
+                                                            : fast_exp2(fmaf(v[e], a.sl2, -lam));
+                }
               }
               uint32_t pk[16];
 #pragma unroll
@@ -517,6 +722,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
               }
               rb[q * kTile + c * 32 + lane] = v[0];
+              if (c < 3) tmem_wait32(nx);
             }
             tmem_st_wait();
             tc_fence_before();
@@ -530,44 +736,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (j.seg_last) {
           if (j.kind == 0) {
-            const int k = (int)blockIdx.x - sc.first_cta(j.u);
-            // k < maxc always holds (the host sizes maxc from the same
-            // partition); the check only keeps a broken launch in bounds.
-            if (k >= 0 && k < a.maxc)
-              a.pstats[(((size_t)j.u * a.maxc + k) * 2 + wg) * kRows + row] = make_float2(M, L);
+            const int ab = aseg & 1;
+            if (aseg >= 2)
+              ok = mbar_wait(&bars->astat_empty[ab], ((aseg >> 1) - 1) & 1, abort_flag,
+                             kWaitBudget);
+            if (!ok) break;
+            astat[(ab * 2 + wg) * kRows + row] = make_float2(M, L);
+            mbar_arrive(&bars->astat_full[ab]);
+            ++aseg;
           } else {
-            const int yb = bseg & 1;
-            if (b == wg) {   // this group ran the segment's last tile: it flushes Y
-              ok = mbar_wait(&bars->y_full[yb], yuse[yb] & 1, abort_flag, kWaitBudget);
-              if (!ok) break;
-              tc_fence_after();
-              const uint32_t ybase = lane_addr + kColY + yb * kD;
-#pragma unroll 1
-              for (int c = 0; c < 4; ++c) {
-                float v[32];
-                tmem_ld32(ybase + c * 32, v);
-                tmem_ld_wait();
-                if (row_ok) {
-                  float4* dst = (float4*)(a.y + ((size_t)j.u * a.m + row) * kD + c * 32);
-#pragma unroll
-                  for (int e = 0; e < 8; ++e)
-                    atomicAdd(dst + e, make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2],
-                                                   v[4 * e + 3]));
-                }
-              }
-              tc_fence_before();
-              mbar_arrive(&bars->y_empty[yb]);
-            }
-            ++yuse[yb];
             ++bseg;
           }
         }
-      }
-      if (ok && it.kind == 0 && a.mode == 2) {
-        // this group's pass-A statistics of the round are in place
-        __threadfence();
-        named_bar(bar_id, 128);
-        if (q == 0 && lane == 0) atomicAdd(&a.round_done[it.r], 1);
       }
     }
     if (!ok && row == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
@@ -637,11 +817,13 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
   a.y = y;
   a.row_stats = row_stats;
   a.pstats = (float2*)(ws + L.pstats_tc);
-  a.round_done = (int*)(ws + L.rounds_tc);
+  a.ustats = (float2*)(ws + L.ustats_tc);
+  a.unit_cnt = (int*)(ws + L.flags_tc);
+  a.unit_ready = a.unit_cnt + s.U;
   a.status = (int*)(ws + L.status);
   cudaError_t e = cudaMemsetAsync(y, 0, (size_t)s.U * s.m * kD * sizeof(float), st);
   if (e != cudaSuccess) return e;
-  e = cudaMemsetAsync(a.round_done, 0, (size_t)rounds * sizeof(int), st);
+  e = cudaMemsetAsync(a.unit_cnt, 0, (size_t)2 * s.U * sizeof(int), st);
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(k_score_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
   if (e != cudaSuccess) return e;
