@@ -131,7 +131,9 @@ WsLayout plan_workspace(const Shape& s) {
     L.ypart = take(U * L.nchunk * m * d * 4);
   }
   L.pooled = take(U * (size_t)s.P * 4);
-  if (!s.tc_merge) {
+  if (s.tc_merge) {
+    L.merge_tc = take(merge_tc_ws_bytes(s));
+  } else {
     L.xbuf = take(U * m * (size_t)s.B * 4);
     L.flags = take(U * (size_t)s.B);
     L.gram = take(U * m * m * 8);

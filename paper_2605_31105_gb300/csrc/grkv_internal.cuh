@@ -46,6 +46,7 @@ struct WsLayout {
   size_t flags;   // uint8 [U][B]      fixed-token flags
   size_t gram;    // acc   [U][m][m]   X_G X_G^T + lambda I, then its Cholesky factor
   size_t rz;      // acc   [U][m][d]   residual R, then Z
+  size_t merge_tc;  // tensor-core merge: R/Z, Gram [U][128][128] fp32, normalisers, fixed bits
   // compress intermediates
   size_t scores;  // float [U][P]
   size_t y;       // float [U][m][d]
@@ -88,6 +89,7 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
 
 // Tensor-core value merge (bf16, m <= 128, B <= 32768).
 bool merge_tc_supported(const Shape& s);
+size_t merge_tc_ws_bytes(const Shape& s);
 cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const void* v,
                             const float* scores, const float* y, const int32_t* idx, void* k_out,
                             void* v_out, char* ws, const WsLayout& L, cudaStream_t st);

@@ -1,22 +1,24 @@
 // GRKV value step on the tensor cores (bf16, d = 128, m <= 128, B <= 32768).
 //
-// One CTA per unit; Algorithm 1's value step in dual form (Sec. 3.4,
-// App. D.1) with the fixed tokens of App. D.3:
-//   phase 1  row max / sum of the retained logits l = s Q K0^T  (K0 gathered
-//            with TMA gather4 from the positions idx);
-//   phase 2  X = softmax over the retained keys; R~ += Xh V0 and the Gram
-//            G += XGh XGh^T + (2 XGl) XGh^T on the tensor cores, where Xh, Xl
-//            are the bf16 high / low parts of X and XG is X with the fixed
-//            columns zeroed (N = (G + G^T) / 2 restores all three cross terms);
-//   phase 3  in shared memory, fp32: N = sym(G) + lambda I, blocked Cholesky,
-//            R = Y - R~, Z = N^-1 R by blocked triangular solves; Z^T (high and
-//            low bf16 parts) goes to TMEM as an MMA operand;
-//   phase 4  per tile D = Zh^T XGh + Zl^T XGh + Zh^T XGl = (dV)^T on the tensor
-//            cores, and V_out = V0 + dV (fixed rows get exactly V0, their XG
-//            columns are zero), K_out = K0.
-// Roles (384 threads): warp 0 TMA, warp 1 MMA issue, warps 4-7 one thread per
-// window row (TMEM lane), warps 8-11 the output epilogue; all warps share the
-// shared-memory solve.
+// Algorithm 1's value step in dual form (Sec. 3.4, App. D.1) with the fixed
+// tokens of App. D.3, one unit per CTA, in three kernels:
+//   k_merge_gram    row max / sum of the retained logits l = s Q K0^T (K0, V0
+//                   gathered with TMA gather4 from the positions idx); then
+//                   X = softmax over the retained keys, R~ += Xh V0 and the Gram
+//                   G += XGh XGh^T + (2 XGl) XGh^T on tcgen05, where Xh, Xl are the
+//                   bf16 high / low parts of X and XG is X with the fixed columns
+//                   zeroed (N = (G + G^T) / 2 restores all three cross terms).
+//                   Writes R = Y - R~, G and the row normalisers to the workspace.
+//   k_merge_solve   fp32 in shared memory: N = sym(G) + lambda I, blocked
+//                   Cholesky, Z = N^-1 R by blocked triangular solves.
+//   k_merge_update  per tile D = Zh^T XGh + Zl^T XGh + Zh^T XGl = dV^T on tcgen05
+//                   with Z^T as a TMEM operand; V_out = V0 + dV (fixed rows get
+//                   exactly V0: their XG columns are zero).
+// K_out = K0 is a plain row gather (k_gather_rows).
+//
+// Both tensor-core kernels rely on the idx contract of grkv.h: ascending, the
+// window n-w..n-1 in the last w slots, so retained slot i is visible to window
+// slot a (causal) exactly when i <= B - w + a.
 #include <cmath>
 
 #include "block_select.cuh"
@@ -36,10 +38,9 @@ constexpr int kThreads = 384;
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KB
 constexpr int kMaxB = 32768;
 constexpr long long kBudget = 1ll << 32;
-
 constexpr int kLD = 129;   // fp32 row stride of N, R/Z and the epilogue stage
 
-// Shared memory (offsets from a 1024-byte aligned base).
+// Shared memory of the tensor-core kernels (offsets from a 1024-byte aligned base).
 constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffRing = kOffQ + kTileBytes;              // 3 x 32 KB gathered tiles
 constexpr uint32_t kOffXG = kOffRing + kRing * kTileBytes;     // 2 x 32 KB
@@ -48,15 +49,13 @@ constexpr uint32_t kOffMask = kOffStage + 32 * kLD * 4;        // fixed-token bi
 constexpr uint32_t kOffMisc = kOffMask + kMaxB / 8;            // hist[256], sh[64]
 constexpr uint32_t kOffBar = kOffMisc + (256 + 64) * 4;
 constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;
-// The solve phase reuses the ring and XG region for N and R/Z.
-constexpr uint32_t kOffN = kOffRing;
-constexpr uint32_t kOffR = kOffN + kRows * kLD * 4;
-static_assert(kOffR + kRows * kLD * 4 <= kOffStage, "solve buffers overlap the stage");
+// k_merge_solve: N and R/Z [128][129] fp32, 1 / L_jj, the failure flag
+constexpr uint32_t kSolveSmem = (2 * kRows * kLD + kRows + 32) * 4;
 
 // TMEM columns.
 constexpr uint32_t kColS = 0;     // two S buffers (128 each)
-constexpr uint32_t kColR = 256;   // phase 2: R~ accumulator; phase 4: Zh^T (64) | Zl^T (64)
-constexpr uint32_t kColG = 384;   // phase 2: Gram accumulator; phase 4: D = dV^T
+constexpr uint32_t kColR = 256;   // gram: R~ accumulator;  update: Zh^T (64) | Zl^T (64)
+constexpr uint32_t kColG = 384;   // gram: Gram accumulator; update: D = dV^T
 
 struct MArgs {
   int U, n, w, m, P, B, causal, n_sink, n_fix;
@@ -65,10 +64,12 @@ struct MArgs {
   const int32_t* idx;        // [U][B]
   const float* scores;       // [U][P]
   const float* y;            // [U][m][128]
-  const __nv_bfloat16* k;    // [U][n][128]
-  const __nv_bfloat16* v;
-  __nv_bfloat16* k_out;      // [U][B][128]
-  __nv_bfloat16* v_out;
+  const __nv_bfloat16* v;    // [U][n][128]
+  __nv_bfloat16* v_out;      // [U][B][128]
+  float* rz;                 // [U][128][128]  R (gram) -> Z (solve)
+  float* gram;               // [U][128][128]  raw Gram
+  float* lam;                // [U][128]       log2 normaliser of each window row
+  uint32_t* mask;            // [U][ceil(B/32)] fixed-token bits
   int* status;
 };
 
@@ -82,40 +83,10 @@ struct MBars {
   uint64_t drain;
   uint32_t tmem;
   int abort;
-  int fail;
 };
 
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&h);
-}
 __device__ __forceinline__ float bf16_round(float x) {
   return __bfloat162float(__float2bfloat16_rn(x));
-}
-__device__ __forceinline__ float fast_exp2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t* r) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
-      "%11, %12, %13, %14, %15, %16};" ::"r"(taddr),
-      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
-      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
-      "r"(r[15])
-      : "memory");
-}
-__device__ __forceinline__ void tmem_st_wait() {
-  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
-                                       uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
 }
 // Four rows (64 columns each) of a 2-D tensor map into consecutive 128-byte rows.
 __device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
@@ -126,36 +97,23 @@ __device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map, u
       "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(r0), "r"(r1), "r"(r2), "r"(r3)
       : "memory");
 }
-
 // Gathers the 128 retained rows of tile t (clamped to the last retained row
-// past B) of one unit's [n][128] matrix into a swizzled 32 KB tile.
+// past B) of one unit's [n][128] matrix into a swizzled 32 KB tile.  Called by
+// a whole warp: lane l fetches rows 4l..4l+3 with one index load each.
 __device__ __forceinline__ void gather_tile(uint8_t* dst, const CUtensorMap* map, uint64_t* bar,
-                                            const int32_t* idx_u, int B, int row0, int t) {
-  mbar_expect_tx(bar, kTileBytes);
-  for (int g = 0; g < kTile / 4; ++g) {
-    int r[4];
+                                            const int32_t* idx_u, int B, int row0, int t,
+                                            int lane) {
+  int r[4];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) r[e] = row0 + __ldg(idx_u + min(t * kTile + 4 * g + e, B - 1));
-    tma_gather4(dst + g * 512, map, bar, 0, r[0], r[1], r[2], r[3]);
-    tma_gather4(dst + kTileBytes / 2 + g * 512, map, bar, 64, r[0], r[1], r[2], r[3]);
-  }
+  for (int e = 0; e < 4; ++e) r[e] = row0 + __ldg(idx_u + min(t * kTile + 4 * lane + e, B - 1));
+  if (lane == 0) mbar_expect_tx(bar, kTileBytes);
+  __syncwarp();
+  tma_gather4(dst + lane * 512, map, bar, 0, r[0], r[1], r[2], r[3]);
+  tma_gather4(dst + kTileBytes / 2 + lane * 512, map, bar, 64, r[0], r[1], r[2], r[3]);
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
-    k_merge_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-               const __grid_constant__ CUtensorMap tmV, MArgs a) {
-  extern __shared__ __align__(1024) uint8_t smraw[];
-  uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
-  MBars* bars = (MBars*)(sm + kOffBar);
-  uint32_t* mask = (uint32_t*)(sm + kOffMask);
-  int* hist = (int*)(sm + kOffMisc);
-  int* sh = hist + 256;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int u = blockIdx.x, B = a.B, T = (B + kTile - 1) / kTile;
-  const int32_t* idx_u = a.idx + (size_t)u * B;
-  const float* sc_u = a.scores + (size_t)u * a.P;
-
-  if (tid == 0) {
+__device__ __forceinline__ void init_common(MBars* bars, int warp) {
+  if (threadIdx.x == 0) {
     for (int i = 0; i < kRing; ++i) {
       mbar_init(&bars->ring_full[i], 1);
       mbar_init(&bars->ring_empty[i], 1);
@@ -172,16 +130,121 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&bars->d_empty, 128);
     mbar_init(&bars->drain, 1);
     bars->abort = 0;
-    bars->fail = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
     tmem_alloc(&bars->tmem, 512);
     tmem_relinquish();
   }
+}
+
+// One 32-column chunk of a gram tile: X, its bf16 high part (TMEM, the R~ MMA
+// operand), XGh (shared memory, the Gram operand) and 2 (X - Xh) on free
+// columns (returned; it goes to TMEM once the S columns it overwrites are read).
+template <int C>
+__device__ __forceinline__ void gram_chunk(const float* v, int t, int vlim, int B, float sl2,
+                                           float lam, const uint32_t* mask, uint32_t sbase,
+                                           uint8_t* xg, int row, uint32_t* lo) {
+  uint32_t hi[16], ghi[16];
+#pragma unroll
+  for (int e = 0; e < 32; e += 2) {
+    float x[2], g[2], l2[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int i = t * kTile + C * 32 + e + h;
+      x[h] = i <= vlim ? fast_exp2(fmaf(v[e + h], sl2, -lam)) : 0.f;
+      const bool fixed = i >= B || ((mask[i >> 5] >> (i & 31)) & 1u);
+      const float xh = bf16_round(x[h]);
+      g[h] = fixed ? 0.f : xh;
+      l2[h] = fixed ? 0.f : 2.f * (x[h] - xh);
+    }
+    hi[e / 2] = pack_bf16(x[0], x[1]);
+    ghi[e / 2] = pack_bf16(g[0], g[1]);
+    lo[e / 2] = pack_bf16(l2[0], l2[1]);
+  }
+  tmem_st16(sbase + C * 16, hi);
+  // XGh row `row`, tokens 32C..32C+31: token block C/2, 16-byte chunks (C&1)*4..+3
+#pragma unroll
+  for (int qq = 0; qq < 4; ++qq)
+    *(uint4*)(xg + (C >> 1) * (kTileBytes / 2) + sw128_offset(row, (C & 1) * 4 + qq)) =
+        make_uint4(ghi[4 * qq], ghi[4 * qq + 1], ghi[4 * qq + 2], ghi[4 * qq + 3]);
+}
+
+// One 32-column chunk of an update tile: XGh and XGl (shared memory, the
+// MN-major B operands of D = Z^T XG).
+template <int C>
+__device__ __forceinline__ void update_chunk(const float* v, int t, int vlim, int B, float sl2,
+                                             float lam, const uint32_t* mask, uint8_t* xh,
+                                             uint8_t* xl, int row) {
+  uint32_t ghi[16], glo[16];
+#pragma unroll
+  for (int e = 0; e < 32; e += 2) {
+    float g[2], l[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int i = t * kTile + C * 32 + e + h;
+      const float x = i <= vlim ? fast_exp2(fmaf(v[e + h], sl2, -lam)) : 0.f;
+      const bool fixed = i >= B || ((mask[i >> 5] >> (i & 31)) & 1u);
+      const float xhv = bf16_round(x);
+      g[h] = fixed ? 0.f : xhv;
+      l[h] = fixed ? 0.f : x - xhv;
+    }
+    ghi[e / 2] = pack_bf16(g[0], g[1]);
+    glo[e / 2] = pack_bf16(l[0], l[1]);
+  }
+#pragma unroll
+  for (int qq = 0; qq < 4; ++qq) {
+    const uint32_t off = (C >> 1) * (kTileBytes / 2) + sw128_offset(row, (C & 1) * 4 + qq);
+    *(uint4*)(xh + off) = make_uint4(ghi[4 * qq], ghi[4 * qq + 1], ghi[4 * qq + 2], ghi[4 * qq + 3]);
+    *(uint4*)(xl + off) = make_uint4(glo[4 * qq], glo[4 * qq + 1], glo[4 * qq + 2], glo[4 * qq + 3]);
+  }
+}
+
+// Online max / sum of exp2 over one 32-column chunk (log2 units).
+__device__ __forceinline__ void stats32(float* v, int i0, int vlim, float sl2, float& M, float& L) {
+#pragma unroll
+  for (int e = 0; e < 32; ++e)
+    if (i0 + e > vlim) v[e] = -INFINITY;
+  float m16[16];
+#pragma unroll
+  for (int e = 0; e < 16; ++e) m16[e] = fmaxf(v[e], v[e + 16]);
+#pragma unroll
+  for (int h = 8; h >= 1; h >>= 1)
+#pragma unroll
+    for (int e = 0; e < h; ++e) m16[e] = fmaxf(m16[e], m16[e + h]);
+  if (m16[0] == -INFINITY) return;
+  const float cm = m16[0] * sl2;
+  if (cm > M) {
+    L *= fast_exp2(M - cm);
+    M = cm;
+  }
+  float s[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int e = 0; e < 32; ++e) s[e & 3] += fast_exp2(fmaf(v[e], sl2, -M));
+  L += (s[0] + s[1]) + (s[2] + s[3]);
+}
+
+// ======================================================== k_merge_gram
+// Roles (384 threads): warp 0 TMA gathers, warp 1 MMA issue, warps 4-7 and
+// 8-11 two compute groups (one thread per window row / TMEM lane) taking
+// alternate tiles.
+__global__ void __launch_bounds__(kThreads, 1)
+    k_merge_gram(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                 const __grid_constant__ CUtensorMap tmV, MArgs a) {
+  extern __shared__ __align__(1024) uint8_t smraw[];
+  uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
+  MBars* bars = (MBars*)(sm + kOffBar);
+  uint32_t* mask = (uint32_t*)(sm + kOffMask);
+  int* hist = (int*)(sm + kOffMisc);
+  int* sh = hist + 256;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int u = blockIdx.x, B = a.B, T = (B + kTile - 1) / kTile, nw = (B + 31) / 32;
+  const int32_t* idx_u = a.idx + (size_t)u * B;
+  const float* sc_u = a.scores + (size_t)u * a.P;
+  init_common(bars, warp);
   // ---- fixed tokens: retained sinks, the window, and the n_fix retained
   // prefix non-sink tokens with the largest scores (ties: smaller position)
-  for (int i = tid; i < (B + 31) / 32; i += kThreads) mask[i] = 0;
+  for (int i = tid; i < nw; i += kThreads) mask[i] = 0;
   __syncthreads();
   auto cand = [&](int i) {
     const int j = __ldg(idx_u + i);
@@ -205,15 +268,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     hist, sh);
   }
   __syncthreads();
+  for (int i = tid; i < nw; i += kThreads) a.mask[(size_t)u * nw + i] = mask[i];
   tc_fence_after();
   const uint32_t tmem = bars->tmem;
   volatile int* abort_flag = &bars->abort;
   const int row0 = u * a.n;   // first row of this unit in the 2-D K / V maps
-  float lam = INFINITY;        // log2 normaliser of the retained softmax (compute rows)
 
-  // Job k: k < T: phase 1 tile k; T <= k < 2T: phase 2 tile k - T;
-  // 2T <= k < 3T: phase 4 tile k - 2T.  S buffer k & 1, ring loads in order.
-  // ================================================= phases 1 and 2
+  // Job k < T: statistics of tile k; T <= k < 2T: Gram and R~ of tile k - T.
+  // S buffer k & 1; gathers in job order (K, then V for the second half).
   if (warp == 0) {
     if (lane == 0) {
       prefetch_tensormap(&tmQ);
@@ -223,24 +285,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t pol = l2_evict_last();
       tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, 0, u, pol);
       tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
-      uint32_t use = 0;
-      bool ok = true;
-      for (int k = 0; k < 2 * T && ok; ++k) {
-        const int t = k < T ? k : k - T;
-        for (int l = 0; l < (k < T ? 1 : 2) && ok; ++l) {
-          const uint32_t slot = use % kRing;
-          if (use >= kRing)
-            ok = mbar_wait(&bars->ring_empty[slot], (use / kRing - 1) & 1, abort_flag, kBudget);
-          if (!ok) break;
-          gather_tile(sm + kOffRing + slot * kTileBytes, l == 0 ? &tmK : &tmV,
-                      &bars->ring_full[slot], idx_u, B, row0, t);
-          ++use;
-        }
-      }
-      // let every issued gather land before the region is reused
-      for (uint32_t i = use > kRing ? use - kRing : 0; i < use; ++i)
-        mbar_wait(&bars->ring_full[i % kRing], (i / kRing) & 1, abort_flag, kBudget);
     }
+    uint32_t use = 0;
+    bool ok = true;
+    for (int k = 0; k < 2 * T && ok; ++k) {
+      const int t = k < T ? k : k - T;
+      for (int l = 0; l < (k < T ? 1 : 2) && ok; ++l) {
+        const uint32_t slot = use % kRing;
+        if (use >= kRing)
+          ok = mbar_wait(&bars->ring_empty[slot], (use / kRing - 1) & 1, abort_flag, kBudget);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) break;
+        gather_tile(sm + kOffRing + slot * kTileBytes, l == 0 ? &tmK : &tmV,
+                    &bars->ring_full[slot], idx_u, B, row0, t, lane);
+        ++use;
+      }
+    }
+    // every issued gather lands before the CTA can exit
+    for (uint32_t i = use > kRing ? use - kRing : 0; i < use; ++i)
+      mbar_wait(&bars->ring_full[i % kRing], (i / kRing) & 1, abort_flag, kBudget);
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t id_s = idesc_bf16(kRows, kTile, 0, 0);
@@ -263,8 +326,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t xa = smem_u32(sm + kOffXG + xb * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < kTile / 16; ++kk)
-          mma_ts(tmem + kColR, tmem + kColS + b * kTile + kk * 8,
-                 sw128_desc(va + kk * 2048, kTileBytes / 2, 1024), id_r, (t > 0 || kk > 0));
+          mma_bf16_ts(tmem + kColR, tmem + kColS + b * kTile + kk * 8,
+                      sw128_desc(va + kk * 2048, kTileBytes / 2, 1024), id_r, (t > 0 || kk > 0));
 #pragma unroll
         for (int kk = 0; kk < kTile / 16; ++kk) {
           const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
@@ -274,8 +337,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int kk = 0; kk < kTile / 16; ++kk) {
           const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
-          mma_ts(tmem + kColG, tmem + kColS + b * kTile + 64 + kk * 8,
-                 sw128_desc(xa + off, 16, 1024), id_g, 1);
+          mma_bf16_ts(tmem + kColG, tmem + kColS + b * kTile + 64 + kk * 8,
+                      sw128_desc(xa + off, 16, 1024), id_g, 1);
         }
         mma_commit(&bars->ring_empty[vuse % kRing]);
         mma_commit(&bars->xg_empty[xb]);
@@ -310,98 +373,84 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (ok && pend >= 0) ok = issue_rg(pend, pend_v);
       mma_commit(&bars->acc_done);
+      mma_commit(&bars->drain);
+      mbar_wait(&bars->drain, 0, abort_flag, kBudget);
     }
-  } else if (warp >= 4 && warp < 8) {
-    const int q = warp & 3, row = q * 32 + lane;
+  } else if (warp >= 4) {
+    const int wg = (warp - 4) >> 2, q = warp & 3, row = q * 32 + lane;
     const bool row_ok = row < a.m;
-    const int lim = a.causal ? a.n - a.w + (row_ok ? row % a.w : 0) : a.n - 1;
+    const int vlim = !row_ok ? -1 : (a.causal ? B - a.w + row % a.w : B - 1);
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
-    float M = -INFINITY, L = 0.f;
+    float M = -INFINITY, L = 0.f, lam = INFINITY;
     bool ok = true;
-    for (int k = 0; k < 2 * T && ok; ++k) {
+    for (int k = 0; k < 2 * T; ++k) {
+      if (k == T) {
+        // both groups combine their statistics (reached even after an abort)
+        float2* comb = (float2*)(sm + kOffStage);
+        comb[wg * kRows + row] = make_float2(M, L);
+        named_bar(4, 256);
+        const float2 o = comb[(wg ^ 1) * kRows + row];
+        if (o.x != -INFINITY) {
+          if (o.x > M) {
+            L = L * fast_exp2(M - o.x) + o.y;
+            M = o.x;
+          } else {
+            L += o.y * fast_exp2(o.x - M);
+          }
+        }
+        lam = (row_ok && L > 0.f) ? M + __log2f(L) : INFINITY;
+        if (wg == 0) a.lam[(size_t)u * kRows + row] = lam;
+      }
+      if (!ok) {
+        if (k < T) continue;
+        break;
+      }
+      if ((k & 1) != wg) continue;
       const int b = k & 1, t = k < T ? k : k - T;
       ok = mbar_wait(&bars->s_full[b], (k >> 1) & 1, abort_flag, kBudget);
-      if (!ok) break;
+      if (!ok) continue;
       tc_fence_after();
       const uint32_t sbase = lane_addr + kColS + b * kTile;
+      float va[32], vb[32];
       if (k < T) {
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          float v[32];
-          tmem_ld32(sbase + c * 32, v);
-          tmem_ld_wait();
-          float vmax = -INFINITY;
-#pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const int i = t * kTile + c * 32 + e;
-            if (i >= B || !row_ok || __ldg(idx_u + i) > lim) v[e] = -INFINITY;
-            vmax = fmaxf(vmax, v[e]);
-          }
-          if (vmax == -INFINITY) continue;
-          const float cm = vmax * a.sl2;
-          if (cm > M) {
-            L *= fast_exp2(M - cm);
-            M = cm;
-          }
-          float s = 0.f;
-#pragma unroll
-          for (int e = 0; e < 32; ++e) s += fast_exp2(fmaf(v[e], a.sl2, -M));
-          L += s;
-        }
+        tmem_ld32f(sbase, va);
+        tmem_wait32(va);
+        tmem_ld32f(sbase + 32, vb);
+        stats32(va, t * kTile, vlim, a.sl2, M, L);
+        tmem_wait32(vb);
+        tmem_ld32f(sbase + 64, va);
+        stats32(vb, t * kTile + 32, vlim, a.sl2, M, L);
+        tmem_wait32(va);
+        tmem_ld32f(sbase + 96, vb);
+        stats32(va, t * kTile + 64, vlim, a.sl2, M, L);
+        tmem_wait32(vb);
         tc_fence_before();
         mbar_arrive(&bars->s_done[b]);
-        if (k == T - 1) lam = (row_ok && L > 0.f) ? M + __log2f(L) : INFINITY;
+        stats32(vb, t * kTile + 96, vlim, a.sl2, M, L);
       } else {
         const int xb = t & 1;
         if (t >= 2) ok = mbar_wait(&bars->xg_empty[xb], ((t >> 1) - 1) & 1, abort_flag, kBudget);
-        if (!ok) break;
+        if (!ok) continue;
         uint8_t* xg = sm + kOffXG + xb * kTileBytes;
         // 2 (X - Xh) goes to TMEM columns 64..127, which hold S chunks 2 and 3:
-        // chunks 0 and 1 are written once chunk 2 is read, chunk 2 once chunk 3 is
-        uint32_t lo2[3][16];
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          float v[32];
-          tmem_ld32(sbase + c * 32, v);
-          tmem_ld_wait();
-          uint32_t hi[16], lo[16], ghi[16];
-#pragma unroll
-          for (int e = 0; e < 32; e += 2) {
-            float x[2], g[2], l2[2];
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              const int i = t * kTile + c * 32 + e + h;
-              const bool vis = i < B && row_ok && __ldg(idx_u + i) <= lim;
-              x[h] = vis ? fast_exp2(fmaf(v[e + h], a.sl2, -lam)) : 0.f;
-              const bool fixed = i >= B || ((mask[i >> 5] >> (i & 31)) & 1u);
-              const float xh = bf16_round(x[h]);
-              g[h] = fixed ? 0.f : xh;
-              l2[h] = fixed ? 0.f : 2.f * (x[h] - xh);
-            }
-            hi[e / 2] = pack_bf16(x[0], x[1]);
-            ghi[e / 2] = pack_bf16(g[0], g[1]);
-            lo[e / 2] = pack_bf16(l2[0], l2[1]);
-          }
-          tmem_st16(sbase + c * 16, hi);
-          // XGh row `row`, tokens 32c..32c+31: token block c/2, 16-byte chunks (c&1)*4..+3
-#pragma unroll
-          for (int qq = 0; qq < 4; ++qq) {
-            const uint4 val = make_uint4(ghi[4 * qq], ghi[4 * qq + 1], ghi[4 * qq + 2],
-                                         ghi[4 * qq + 3]);
-            *(uint4*)(xg + (c >> 1) * (kTileBytes / 2) + sw128_offset(row, (c & 1) * 4 + qq)) = val;
-          }
-          if (c < 3) {
-#pragma unroll
-            for (int e = 0; e < 16; ++e) lo2[c][e] = lo[e];
-          }
-          if (c == 2) {
-            tmem_st16(sbase + 64, lo2[0]);
-            tmem_st16(sbase + 64 + 16, lo2[1]);
-          } else if (c == 3) {
-            tmem_st16(sbase + 64 + 32, lo2[2]);
-            tmem_st16(sbase + 64 + 48, lo);
-          }
-        }
+        // chunks 0 and 1 are written once chunk 2 is read, 2 and 3 after chunk 3
+        uint32_t lo0[16], lo1[16], lo2[16], lo3[16];
+        tmem_ld32f(sbase, va);
+        tmem_wait32(va);
+        tmem_ld32f(sbase + 32, vb);
+        gram_chunk<0>(va, t, vlim, B, a.sl2, lam, mask, sbase, xg, row, lo0);
+        tmem_wait32(vb);
+        tmem_ld32f(sbase + 64, va);
+        gram_chunk<1>(vb, t, vlim, B, a.sl2, lam, mask, sbase, xg, row, lo1);
+        tmem_wait32(va);
+        tmem_ld32f(sbase + 96, vb);
+        gram_chunk<2>(va, t, vlim, B, a.sl2, lam, mask, sbase, xg, row, lo2);
+        tmem_st16(sbase + 64, lo0);
+        tmem_st16(sbase + 80, lo1);
+        tmem_wait32(vb);
+        gram_chunk<3>(vb, t, vlim, B, a.sl2, lam, mask, sbase, xg, row, lo3);
+        tmem_st16(sbase + 96, lo2);
+        tmem_st16(sbase + 112, lo3);
         tmem_st_wait();
         fence_proxy_async_smem();
         tc_fence_before();
@@ -409,27 +458,31 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_arrive(&bars->xg_full[xb]);
       }
     }
-    // R = Y - R~ and the raw Gram rows into shared memory (fp32)
+    // R = Y - R~ and the raw Gram rows to the workspace, half the columns per group
     if (ok) ok = mbar_wait(&bars->acc_done, 0, abort_flag, kBudget);
     tc_fence_after();
-    float* N = (float*)(sm + kOffN);
-    float* R = (float*)(sm + kOffR);
     if (ok) {
+      float* R = a.rz + ((size_t)u * kRows + row) * kD;
+      float* G = a.gram + ((size_t)u * kRows + row) * kRows;
+      const float* yr = a.y + ((size_t)u * a.m + (row_ok ? row : 0)) * kD;
 #pragma unroll 1
-      for (int c = 0; c < 4; ++c) {
+      for (int c = 2 * wg; c < 2 * wg + 2; ++c) {
         float v[32];
-        tmem_ld32(lane_addr + kColR + c * 32, v);
-        tmem_ld_wait();
+        tmem_ld32f(lane_addr + kColR + c * 32, v);
+        tmem_wait32(v);
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const int col = c * 32 + e;
-          R[row * kLD + col] =
-              row_ok ? a.y[((size_t)u * a.m + row) * kD + col] - v[e] : 0.f;
+        for (int e = 0; e < 32; e += 4) {
+          const float4 yv = row_ok ? __ldg((const float4*)(yr + c * 32 + e))
+                                   : make_float4(0.f, 0.f, 0.f, 0.f);
+          *(float4*)(R + c * 32 + e) =
+              row_ok ? make_float4(yv.x - v[e], yv.y - v[e + 1], yv.z - v[e + 2], yv.w - v[e + 3])
+                     : make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        tmem_ld32(lane_addr + kColG + c * 32, v);
-        tmem_ld_wait();
+        tmem_ld32f(lane_addr + kColG + c * 32, v);
+        tmem_wait32(v);
 #pragma unroll
-        for (int e = 0; e < 32; ++e) N[row * kLD + c * 32 + e] = v[e];
+        for (int e = 0; e < 32; e += 4)
+          *(float4*)(G + c * 32 + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
       }
     }
     if (!ok && row == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
@@ -437,311 +490,444 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+}
 
-  // ================================================= phase 3: solve (fp32)
-  float* N = (float*)(sm + kOffN);
-  float* R = (float*)(sm + kOffR);
-  const bool aborted = *abort_flag != 0;
-  if (!aborted) {
-    // N = (G + G^T) / 2 + lambda I on the window rows; identity on padding
-    for (int p = tid; p < kRows * kRows; p += kThreads) {
-      const int i = p / kRows, j = p % kRows;
-      if (j > i) continue;
-      float val;
-      if (i >= a.m || j >= a.m) val = (i == j) ? 1.f : 0.f;
-      else if (i == j) val = N[i * kLD + i] + a.lambda;
-      else val = 0.5f * (N[i * kLD + j] + N[j * kLD + i]);
-      N[i * kLD + j] = val;
+// ======================================================== k_merge_solve
+// The register-resident pieces of the blocked Cholesky and the triangular
+// solves are separate (non-inlined) functions so that their 32-element arrays
+// stay in registers.
+
+// Factors the 32 x 32 diagonal block at k0 (right-looking; lane l holds row
+// k0 + l) and stores 1 / L_jj.  Returns true on a non-positive pivot.
+__device__ __noinline__ bool chol_diag(float* N, float* dinv, int k0, int lane) {
+  float x[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) x[j] = j <= lane ? N[(k0 + lane) * kLD + k0 + j] : 0.f;
+  bool bad = false;
+#pragma unroll
+  for (int k = 0; k < 32; ++k) {
+    const float dkk = __shfl_sync(0xffffffffu, x[k], k);
+    bad |= !(dkk > 0.f);
+    const float piv = sqrtf(fmaxf(dkk, 0.f));
+    const float inv = piv > 0.f ? 1.f / piv : 0.f;
+    x[k] = lane == k ? piv : (lane > k ? x[k] * inv : x[k]);
+    const float lk = x[k];
+#pragma unroll
+    for (int j = k + 1; j < 32; ++j) {
+      const float ljk = __shfl_sync(0xffffffffu, x[k], j);
+      x[j] = lane >= j ? x[j] - lk * ljk : x[j];
+    }
+    if (lane == 0) dinv[k0 + k] = inv;
+  }
+#pragma unroll
+  for (int j = 0; j < 32; ++j)
+    if (j <= lane) N[(k0 + lane) * kLD + k0 + j] = x[j];
+  return bad;
+}
+
+// Row i of the panel below the diagonal block at k0: L_i,k0.. = A_i,k0.. L_kk^-T.
+__device__ __noinline__ void chol_panel_row(float* N, const float* dinv, int k0, int i) {
+  float x[32];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) x[j] = N[i * kLD + k0 + j];
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    float s0 = x[j], s1 = 0.f;
+#pragma unroll
+    for (int p = 0; p < j; ++p) {
+      if (p & 1) s1 += x[p] * N[(k0 + j) * kLD + k0 + p];
+      else s0 -= x[p] * N[(k0 + j) * kLD + k0 + p];
+    }
+    x[j] = (s0 - s1) * dinv[k0 + j];
+  }
+#pragma unroll
+  for (int j = 0; j < 32; ++j) N[i * kLD + k0 + j] = x[j];
+}
+
+// Column e of rows i0..i0+31: W = L_bb^-1 W (forward) or L_bb^-T W (backward).
+__device__ __noinline__ void trsv_fwd(const float* N, float* R, const float* dinv, int i0, int e) {
+  float z[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) z[i] = R[(i0 + i) * kLD + e];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    float s0 = z[i], s1 = 0.f;
+#pragma unroll
+    for (int kx = 0; kx < i; ++kx) {
+      if (kx & 1) s1 += N[(i0 + i) * kLD + i0 + kx] * z[kx];
+      else s0 -= N[(i0 + i) * kLD + i0 + kx] * z[kx];
+    }
+    z[i] = (s0 - s1) * dinv[i0 + i];
+  }
+#pragma unroll
+  for (int i = 0; i < 32; ++i) R[(i0 + i) * kLD + e] = z[i];
+}
+__device__ __noinline__ void trsv_bwd(const float* N, float* R, const float* dinv, int i0, int e) {
+  float z[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) z[i] = R[(i0 + i) * kLD + e];
+#pragma unroll
+  for (int i = 31; i >= 0; --i) {
+    float s0 = z[i], s1 = 0.f;
+#pragma unroll
+    for (int kx = i + 1; kx < 32; ++kx) {
+      if (kx & 1) s1 += N[(i0 + kx) * kLD + i0 + i] * z[kx];
+      else s0 -= N[(i0 + kx) * kLD + i0 + i] * z[kx];
+    }
+    z[i] = (s0 - s1) * dinv[i0 + i];
+  }
+#pragma unroll
+  for (int i = 0; i < 32; ++i) R[(i0 + i) * kLD + e] = z[i];
+}
+
+// N = (G + G^T) / 2 + lambda I on the window rows (identity on padding rows),
+// Cholesky N = L L^T in 32-row blocks, then Z = L^-T L^-1 R; fp32 in shared
+// memory.  A non-positive pivot reports GRKV_ERR_NUMERIC and leaves Z = 0
+// (values stay V0); lambda = +inf also gives Z = 0.
+__global__ void __launch_bounds__(256) k_merge_solve(MArgs a) {
+  extern __shared__ __align__(16) float ssm[];
+  float* N = ssm;                   // [128][kLD]
+  float* R = N + kRows * kLD;       // [128][kLD]
+  float* dinv = R + kRows * kLD;    // [128]
+  int* fail = (int*)(dinv + kRows);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, nt = blockDim.x;
+  const int u = blockIdx.x, m = a.m;
+  const float4* G4 = (const float4*)(a.gram + (size_t)u * kRows * kRows);
+  float* RZ = a.rz + (size_t)u * kRows * kD;
+  if (a.lambda_inf) {
+    for (int p = tid; p < kRows * kD / 4; p += nt) ((float4*)RZ)[p] = make_float4(0.f, 0.f, 0.f, 0.f);
+    return;
+  }
+  if (tid == 0) *fail = 0;
+#pragma unroll 4
+  for (int p = tid; p < kRows * kRows / 4; p += nt) {
+    const float4 g = __ldg(G4 + p), r = __ldg((const float4*)RZ + p);
+    float* n = N + (p >> 5) * kLD + (p & 31) * 4;
+    float* rr = R + (p >> 5) * kLD + (p & 31) * 4;
+    n[0] = g.x; n[1] = g.y; n[2] = g.z; n[3] = g.w;
+    rr[0] = r.x; rr[1] = r.y; rr[2] = r.z; rr[3] = r.w;
+  }
+  __syncthreads();
+  // symmetrise into the lower triangle (reads only the untouched upper one)
+  for (int p = tid; p < kRows * kRows; p += nt) {
+    const int i = p >> 7, j = p & 127;
+    if (j > i) continue;
+    float val;
+    if (i >= m || j >= m) val = (i == j) ? 1.f : 0.f;
+    else if (i == j) val = N[i * kLD + i] + a.lambda;
+    else val = 0.5f * (N[i * kLD + j] + N[j * kLD + i]);
+    N[i * kLD + j] = val;
+  }
+  __syncthreads();
+  for (int kb = 0; kb < kRows / 32; ++kb) {
+    const int k0 = kb * 32;
+    if (warp == 0 && chol_diag(N, dinv, k0, lane) && lane == 0) *fail = 1;
+    __syncthreads();
+    for (int i = k0 + 32 + tid; i < kRows; i += nt) chol_panel_row(N, dinv, k0, i);
+    __syncthreads();
+    // trailing update of the lower triangle in 4x4 register blocks
+    const int k1 = k0 + 32, t4 = (kRows - k1) / 4, nb = t4 * (t4 + 1) / 2;
+    for (int t = tid; t < nb; t += nt) {
+      int bi = (int)((sqrtf(8.f * t + 1.f) - 1.f) * 0.5f);
+      while ((bi + 1) * (bi + 2) / 2 <= t) ++bi;
+      while (bi * (bi + 1) / 2 > t) --bi;
+      const int i = k1 + 4 * bi, j = k1 + 4 * (t - bi * (bi + 1) / 2);
+      float acc[4][4] = {};
+#pragma unroll 4
+      for (int pp = 0; pp < 32; ++pp) {
+        float li[4], lj[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          li[r] = N[(i + r) * kLD + k0 + pp];
+          lj[r] = N[(j + r) * kLD + k0 + pp];
+        }
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) acc[r][c] += li[r] * lj[c];
+      }
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+          if (j + c <= i + r) N[(i + r) * kLD + j + c] -= acc[r][c];
     }
     __syncthreads();
-    for (int kb = 0; kb < kRows / 32 && !a.lambda_inf; ++kb) {
-      const int k0 = kb * 32;
-      if (warp == 0) {   // diagonal block, one warp
-        for (int k = k0; k < k0 + 32; ++k) {
-          if (lane == 0) {
-            const float dkk = N[k * kLD + k];
-            if (!(dkk > 0.f)) bars->fail = 1;
-            N[k * kLD + k] = sqrtf(fmaxf(dkk, 0.f));
-          }
-          __syncwarp();
-          const int i = k0 + lane;
-          const float piv = N[k * kLD + k];
-          if (i > k) N[i * kLD + k] = piv > 0.f ? N[i * kLD + k] / piv : 0.f;
-          __syncwarp();
-          if (i > k)
-            for (int j = k + 1; j <= i; ++j) N[i * kLD + j] -= N[i * kLD + k] * N[j * kLD + k];
-          __syncwarp();
-        }
-      }
-      __syncthreads();
-      // panel below the diagonal block: L_ij = (N_ij - sum_p L_ip L_jp) / L_jj
-      for (int i = k0 + 32 + tid; i < kRows; i += kThreads) {
-        for (int j = k0; j < k0 + 32; ++j) {
-          float s = N[i * kLD + j];
-          for (int p = k0; p < j; ++p) s -= N[i * kLD + p] * N[j * kLD + p];
-          const float piv = N[j * kLD + j];
-          N[i * kLD + j] = piv > 0.f ? s / piv : 0.f;
-        }
-      }
-      __syncthreads();
-      // trailing update of the lower triangle
-      const int rest = kRows - (k0 + 32);
-      for (int p = tid; p < rest * rest; p += kThreads) {
-        const int i = k0 + 32 + p / rest, j = k0 + 32 + p % rest;
-        if (j > i) continue;
-        float s = N[i * kLD + j];
-#pragma unroll 8
-        for (int pp = k0; pp < k0 + 32; ++pp) s -= N[i * kLD + pp] * N[j * kLD + pp];
-        N[i * kLD + j] = s;
-      }
-      __syncthreads();
-    }
-    const bool fail = bars->fail != 0 || a.lambda_inf;
-    if (bars->fail && !a.lambda_inf && tid == 0) set_status(a.status, GRKV_ERR_NUMERIC);
-    if (fail) {   // values stay V0
-      for (int p = tid; p < kRows * kLD; p += kThreads) R[p] = 0.f;
-      __syncthreads();
-    } else {
-      // forward: L W = R, 32-row blocks
-      for (int ib = 0; ib < kRows / 32; ++ib) {
-        const int i0 = ib * 32;
-        if (tid < kD) {
-          for (int i = i0; i < i0 + 32; ++i) {
-            float s = R[i * kLD + tid];
-            for (int kx = i0; kx < i; ++kx) s -= N[i * kLD + kx] * R[kx * kLD + tid];
-            R[i * kLD + tid] = s / N[i * kLD + i];
-          }
-        }
-        __syncthreads();
-        const int rest = kRows - (i0 + 32);
-        for (int p = tid; p < rest * kD; p += kThreads) {
-          const int i = i0 + 32 + p / kD, e = p % kD;
-          float s = R[i * kLD + e];
-#pragma unroll 8
-          for (int kx = i0; kx < i0 + 32; ++kx) s -= N[i * kLD + kx] * R[kx * kLD + e];
-          R[i * kLD + e] = s;
-        }
-        __syncthreads();
-      }
-      // backward: L^T Z = W
-      for (int ib = kRows / 32 - 1; ib >= 0; --ib) {
-        const int i0 = ib * 32;
-        if (tid < kD) {
-          for (int i = i0 + 31; i >= i0; --i) {
-            float s = R[i * kLD + tid];
-            for (int kx = i + 1; kx < i0 + 32; ++kx) s -= N[kx * kLD + i] * R[kx * kLD + tid];
-            R[i * kLD + tid] = s / N[i * kLD + i];
-          }
-        }
-        __syncthreads();
-        for (int p = tid; p < i0 * kD; p += kThreads) {
-          const int i = p / kD, e = p % kD;
-          float s = R[i * kLD + e];
-#pragma unroll 8
-          for (int kx = i0; kx < i0 + 32; ++kx) s -= N[kx * kLD + i] * R[kx * kLD + e];
-          R[i * kLD + e] = s;
-        }
-        __syncthreads();
-      }
-    }
-    // Z^T into TMEM as MMA operands: lane = column e of Z, packed row pairs
-    if (warp >= 4 && warp < 8) {
-      const int q = warp & 3, e = q * 32 + lane;
-      const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
-#pragma unroll 1
-      for (int rc = 0; rc < 4; ++rc) {
-        uint32_t zh[16], zl[16];
-#pragma unroll
-        for (int p = 0; p < 16; ++p) {
-          const float z0 = R[(rc * 32 + 2 * p) * kLD + e], z1 = R[(rc * 32 + 2 * p + 1) * kLD + e];
-          const float h0 = bf16_round(z0), h1 = bf16_round(z1);
-          zh[p] = pack_bf16(h0, h1);
-          zl[p] = pack_bf16(z0 - h0, z1 - h1);
-        }
-        tmem_st16(lane_addr + kColR + rc * 16, zh);
-        tmem_st16(lane_addr + kColR + 64 + rc * 16, zl);
-      }
-      tmem_st_wait();
-    }
   }
-  fence_proxy_async_smem();   // the solve buffers are TMA destinations again
+  if (*fail) {
+    if (tid == 0) set_status(a.status, GRKV_ERR_NUMERIC);
+    for (int p = tid; p < kRows * kD / 4; p += nt) ((float4*)RZ)[p] = make_float4(0.f, 0.f, 0.f, 0.f);
+    return;
+  }
+  // forward: L W = R in 32-row blocks; one column of R per thread
+  for (int ib = 0; ib < kRows / 32; ++ib) {
+    const int i0 = ib * 32;
+    if (tid < kD) trsv_fwd(N, R, dinv, i0, tid);
+    __syncthreads();
+    // rows below: 4 rows x 4 columns (stride 32) per thread
+    const int i1 = i0 + 32, nb = (kRows - i1) / 4 * 32;
+    for (int t = tid; t < nb; t += nt) {
+      const int i = i1 + 4 * (t >> 5), e = t & 31;
+      float acc[4][4] = {};
+#pragma unroll 4
+      for (int kx = 0; kx < 32; ++kx) {
+        float l[4], z[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) l[r] = N[(i + r) * kLD + i0 + kx];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) z[c] = R[(i0 + kx) * kLD + e + 32 * c];
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) acc[r][c] += l[r] * z[c];
+      }
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) R[(i + r) * kLD + e + 32 * c] -= acc[r][c];
+    }
+    __syncthreads();
+  }
+  // backward: L^T Z = W
+  for (int ib = kRows / 32 - 1; ib >= 0; --ib) {
+    const int i0 = ib * 32;
+    if (tid < kD) trsv_bwd(N, R, dinv, i0, tid);
+    __syncthreads();
+    // rows above: 4 rows x 4 columns (stride 32) per thread
+    const int nb = i0 / 4 * 32;
+    for (int t = tid; t < nb; t += nt) {
+      const int i = 4 * (t >> 5), e = t & 31;
+      float acc[4][4] = {};
+#pragma unroll 4
+      for (int kx = 0; kx < 32; ++kx) {
+        float l[4], z[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) l[r] = N[(i0 + kx) * kLD + i + r];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) z[c] = R[(i0 + kx) * kLD + e + 32 * c];
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) acc[r][c] += l[r] * z[c];
+      }
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) R[(i + r) * kLD + e + 32 * c] -= acc[r][c];
+    }
+    __syncthreads();
+  }
+  for (int p = tid; p < kRows * kD / 4; p += nt) {
+    const float* rr = R + (p >> 5) * kLD + (p & 31) * 4;
+    ((float4*)RZ)[p] = make_float4(rr[0], rr[1], rr[2], rr[3]);
+  }
+}
+
+// ======================================================== k_merge_update
+// Roles (384 threads): warp 0 TMA gathers of K0, warp 1 MMA issue, warps 4-7
+// XG tiles (one thread per window row), warps 8-11 the output epilogue.
+__global__ void __launch_bounds__(kThreads, 1)
+    k_merge_update(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                   MArgs a) {
+  extern __shared__ __align__(1024) uint8_t smraw[];
+  uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
+  MBars* bars = (MBars*)(sm + kOffBar);
+  uint32_t* mask = (uint32_t*)(sm + kOffMask);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int u = blockIdx.x, B = a.B, T = (B + kTile - 1) / kTile, nw = (B + 31) / 32;
+  const int32_t* idx_u = a.idx + (size_t)u * B;
+  init_common(bars, warp);
+  for (int i = tid; i < nw; i += kThreads) mask[i] = a.mask[(size_t)u * nw + i];
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem;
+  volatile int* abort_flag = &bars->abort;
+  const int row0 = u * a.n;
+  // Z^T into TMEM as MMA operands: lane = column e of Z, packed row pairs
+  if (warp >= 4 && warp < 8) {
+    const int q = warp & 3, e = q * 32 + lane;
+    const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
+    const float* Z = a.rz + (size_t)u * kRows * kD;
+#pragma unroll 1
+    for (int rc = 0; rc < 4; ++rc) {
+      uint32_t zh[16], zl[16];
+#pragma unroll
+      for (int p = 0; p < 16; ++p) {
+        const float z0 = Z[(rc * 32 + 2 * p) * kD + e], z1 = Z[(rc * 32 + 2 * p + 1) * kD + e];
+        const float h0 = bf16_round(z0), h1 = bf16_round(z1);
+        zh[p] = pack_bf16(h0, h1);
+        zl[p] = pack_bf16(z0 - h0, z1 - h1);
+      }
+      tmem_st16(lane_addr + kColR + rc * 16, zh);
+      tmem_st16(lane_addr + kColR + 64 + rc * 16, zl);
+    }
+    tmem_st_wait();
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
 
-  // ================================================= phase 4: dV and outputs
-  if (!aborted) {
-    if (warp == 0) {
-      if (lane == 0) {
-        uint32_t use = 3u * T;   // loads of phases 1 and 2
-        bool ok = true;
-        for (int t = 0; t < T && ok; ++t) {
-          const uint32_t slot = use % kRing;
-          if (use >= kRing)
-            ok = mbar_wait(&bars->ring_empty[slot], (use / kRing - 1) & 1, abort_flag, kBudget);
-          if (!ok) break;
-          gather_tile(sm + kOffRing + slot * kTileBytes, &tmK, &bars->ring_full[slot], idx_u, B,
-                      row0, t);
-          ++use;
-        }
-        for (uint32_t i = use > kRing ? use - kRing : 0; i < use; ++i)
-          mbar_wait(&bars->ring_full[i % kRing], (i / kRing) & 1, abort_flag, kBudget);
-      }
-    } else if (warp == 1) {
-      if (lane == 0) {
-        const uint32_t id_s = idesc_bf16(kRows, kTile, 0, 0);
-        const uint32_t id_d = idesc_bf16(kD, kTile, 0, 1);   // D = Z^T XG (XG MN-major)
-        const uint32_t qa = smem_u32(sm + kOffQ);
-        uint32_t use = 3u * T;
-        bool ok = true;
-        auto issue_d = [&](int t) -> bool {
-          const int k = 2 * T + t, b = k & 1;
-          bool w = mbar_wait(&bars->xg_full[0], (t + ((T + 1) >> 1)) & 1, abort_flag, kBudget);
-          if (w && t >= 1) w = mbar_wait(&bars->d_empty, (t - 1) & 1, abort_flag, kBudget);
-          (void)b;
-          if (!w) return false;
-          tc_fence_after();
-          const uint32_t xh = smem_u32(sm + kOffXG), xl = xh + kTileBytes;
-#pragma unroll
-          for (int kk = 0; kk < kRows / 16; ++kk)
-            mma_ts(tmem + kColG, tmem + kColR + kk * 8,
-                   sw128_desc(xh + kk * 2048, kTileBytes / 2, 1024), id_d, kk > 0);
-#pragma unroll
-          for (int kk = 0; kk < kRows / 16; ++kk)
-            mma_ts(tmem + kColG, tmem + kColR + 64 + kk * 8,
-                   sw128_desc(xh + kk * 2048, kTileBytes / 2, 1024), id_d, 1);
-#pragma unroll
-          for (int kk = 0; kk < kRows / 16; ++kk)
-            mma_ts(tmem + kColG, tmem + kColR + kk * 8,
-                   sw128_desc(xl + kk * 2048, kTileBytes / 2, 1024), id_d, 1);
-          mma_commit(&bars->xg_empty[0]);
-          mma_commit(&bars->d_full);
-          return true;
-        };
-        for (int t = 0; t < T && ok; ++t) {
-          const int k = 2 * T + t, b = k & 1;
-          const uint32_t kuse = use++;
-          ok = mbar_wait(&bars->ring_full[kuse % kRing], (kuse / kRing) & 1, abort_flag, kBudget);
-          if (ok) ok = mbar_wait(&bars->s_done[b], ((k >> 1) - 1) & 1, abort_flag, kBudget);
-          if (!ok) break;
-          tc_fence_after();
-          const uint32_t ka = smem_u32(sm + kOffRing + (kuse % kRing) * kTileBytes);
-#pragma unroll
-          for (int kk = 0; kk < kD / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
-            mma_bf16(tmem + kColS + b * kTile, sw128_desc(qa + off, 16, 1024),
-                     sw128_desc(ka + off, 16, 1024), id_s, kk > 0);
-          }
-          mma_commit(&bars->ring_empty[kuse % kRing]);
-          mma_commit(&bars->s_full[b]);
-          if (t >= 1) ok = issue_d(t - 1);
-        }
-        if (ok && T >= 1) ok = issue_d(T - 1);
-        mma_commit(&bars->drain);
-        mbar_wait(&bars->drain, 0, abort_flag, kBudget);
-      }
-    } else if (warp >= 4 && warp < 8) {
-      const int q = warp & 3, row = q * 32 + lane;
-      const bool row_ok = row < a.m;
-      const int lim = a.causal ? a.n - a.w + (row_ok ? row % a.w : 0) : a.n - 1;
-      const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
-      bool ok = true;
-      uint8_t* xh = sm + kOffXG;
-      uint8_t* xl = xh + kTileBytes;
-      // xg_empty[0] / xg_full[0] keep counting from phase 2 (tiles t with t&1 == 0)
-      const int base_uses = (T + 1) >> 1;
-      for (int t = 0; t < T && ok; ++t) {
-        const int k = 2 * T + t, b = k & 1;
-        ok = mbar_wait(&bars->s_full[b], (k >> 1) & 1, abort_flag, kBudget);
-        if (ok && base_uses + t >= 1)
-          ok = mbar_wait(&bars->xg_empty[0], (base_uses + t - 1) & 1, abort_flag, kBudget);
-        if (!ok) break;
-        tc_fence_after();
-        const uint32_t sbase = lane_addr + kColS + b * kTile;
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          float v[32];
-          tmem_ld32(sbase + c * 32, v);
-          tmem_ld_wait();
-          uint32_t ghi[16], glo[16];
-#pragma unroll
-          for (int e = 0; e < 32; e += 2) {
-            float g[2], l[2];
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              const int i = t * kTile + c * 32 + e + h;
-              const bool vis = i < B && row_ok && __ldg(idx_u + i) <= lim;
-              const float x = vis ? fast_exp2(fmaf(v[e + h], a.sl2, -lam)) : 0.f;
-              const bool fixed = i >= B || ((mask[i >> 5] >> (i & 31)) & 1u);
-              const float xhv = bf16_round(x);
-              g[h] = fixed ? 0.f : xhv;
-              l[h] = fixed ? 0.f : x - xhv;
-            }
-            ghi[e / 2] = pack_bf16(g[0], g[1]);
-            glo[e / 2] = pack_bf16(l[0], l[1]);
-          }
-#pragma unroll
-          for (int qq = 0; qq < 4; ++qq) {
-            const uint32_t off = (c >> 1) * (kTileBytes / 2) + sw128_offset(row, (c & 1) * 4 + qq);
-            *(uint4*)(xh + off) = make_uint4(ghi[4 * qq], ghi[4 * qq + 1], ghi[4 * qq + 2],
-                                             ghi[4 * qq + 3]);
-            *(uint4*)(xl + off) = make_uint4(glo[4 * qq], glo[4 * qq + 1], glo[4 * qq + 2],
-                                             glo[4 * qq + 3]);
-          }
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        mbar_arrive(&bars->s_done[b]);
-        mbar_arrive(&bars->xg_full[0]);
-      }
-      if (!ok && row == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
-    } else if (warp >= 8) {
-      // epilogue: D = dV^T, lane = column e of V; staged through shared memory
-      const int q = warp & 3, e = q * 32 + lane, et = tid - 256;
-      const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
-      float* stage = (float*)(sm + kOffStage);
-      bool ok = true;
-      for (int t = 0; t < T && ok; ++t) {
-        ok = mbar_wait(&bars->d_full, t & 1, abort_flag, kBudget);
-        if (!ok) break;
-        tc_fence_after();
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          float v[32];
-          tmem_ld32(lane_addr + kColG + c * 32, v);
-          tmem_ld_wait();
-          if (c == 3) {
-            tc_fence_before();
-            mbar_arrive(&bars->d_empty);
-          }
-#pragma unroll
-          for (int tk = 0; tk < 32; ++tk) stage[tk * kLD + e] = v[tk];
-          named_bar(3, 128);
-          // a warp takes 32 tokens of one 32-column block
-          const int tk = et & 31, c0 = (et >> 5) * 32, i = t * kTile + c * 32 + tk;
-          if (i < B) {
-            const size_t src = ((size_t)u * a.n + __ldg(idx_u + i)) * kD + c0;
-            const size_t dst = ((size_t)u * B + i) * kD + c0;
-#pragma unroll
-            for (int h = 0; h < 4; ++h) {
-              const uint4 v0 = *(const uint4*)(a.v + src + 8 * h);
-              const uint4 k0 = *(const uint4*)(a.k + src + 8 * h);
-              const __nv_bfloat16* pv = (const __nv_bfloat16*)&v0;
-              uint32_t o[4];
-#pragma unroll
-              for (int z = 0; z < 4; ++z)
-                o[z] = pack_bf16(__bfloat162float(pv[2 * z]) + stage[tk * kLD + c0 + 8 * h + 2 * z],
-                                 __bfloat162float(pv[2 * z + 1]) +
-                                     stage[tk * kLD + c0 + 8 * h + 2 * z + 1]);
-              *(uint4*)(a.v_out + dst + 8 * h) = make_uint4(o[0], o[1], o[2], o[3]);
-              *(uint4*)(a.k_out + dst + 8 * h) = k0;
-            }
-          }
-          named_bar(3, 128);
-        }
-      }
-      if (!ok && e == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
+  if (warp == 0) {
+    if (lane == 0) {
+      prefetch_tensormap(&tmQ);
+      prefetch_tensormap(&tmK);
+      mbar_expect_tx(&bars->q_full, kTileBytes);
+      const uint64_t pol = l2_evict_last();
+      tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, 0, u, pol);
+      tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
     }
+    uint32_t use = 0;
+    bool ok = true;
+    for (int t = 0; t < T && ok; ++t) {
+      const uint32_t slot = use % kRing;
+      if (use >= kRing)
+        ok = mbar_wait(&bars->ring_empty[slot], (use / kRing - 1) & 1, abort_flag, kBudget);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) break;
+      gather_tile(sm + kOffRing + slot * kTileBytes, &tmK, &bars->ring_full[slot], idx_u, B, row0,
+                  t, lane);
+      ++use;
+    }
+    for (uint32_t i = use > kRing ? use - kRing : 0; i < use; ++i)
+      mbar_wait(&bars->ring_full[i % kRing], (i / kRing) & 1, abort_flag, kBudget);
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t id_s = idesc_bf16(kRows, kTile, 0, 0);
+      const uint32_t id_d = idesc_bf16(kD, kTile, 0, 1);   // D = Z^T XG (XG MN-major)
+      const uint32_t qa = smem_u32(sm + kOffQ);
+      bool ok = mbar_wait(&bars->q_full, 0, abort_flag, kBudget);
+      auto issue_d = [&](int t) -> bool {
+        bool w = mbar_wait(&bars->xg_full[0], t & 1, abort_flag, kBudget);
+        if (w && t >= 1) w = mbar_wait(&bars->d_empty, (t - 1) & 1, abort_flag, kBudget);
+        if (!w) return false;
+        tc_fence_after();
+        const uint32_t xh = smem_u32(sm + kOffXG), xl = xh + kTileBytes;
+#pragma unroll
+        for (int kk = 0; kk < kRows / 16; ++kk)
+          mma_bf16_ts(tmem + kColG, tmem + kColR + kk * 8,
+                      sw128_desc(xh + kk * 2048, kTileBytes / 2, 1024), id_d, kk > 0);
+#pragma unroll
+        for (int kk = 0; kk < kRows / 16; ++kk)
+          mma_bf16_ts(tmem + kColG, tmem + kColR + 64 + kk * 8,
+                      sw128_desc(xh + kk * 2048, kTileBytes / 2, 1024), id_d, 1);
+#pragma unroll
+        for (int kk = 0; kk < kRows / 16; ++kk)
+          mma_bf16_ts(tmem + kColG, tmem + kColR + kk * 8,
+                      sw128_desc(xl + kk * 2048, kTileBytes / 2, 1024), id_d, 1);
+        mma_commit(&bars->xg_empty[0]);
+        mma_commit(&bars->d_full);
+        return true;
+      };
+      for (int t = 0; t < T && ok; ++t) {
+        const int b = t & 1;
+        ok = mbar_wait(&bars->ring_full[t % kRing], (t / kRing) & 1, abort_flag, kBudget);
+        if (ok && t >= 2) ok = mbar_wait(&bars->s_done[b], ((t >> 1) - 1) & 1, abort_flag, kBudget);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t ka = smem_u32(sm + kOffRing + (t % kRing) * kTileBytes);
+#pragma unroll
+        for (int kk = 0; kk < kD / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
+          mma_bf16(tmem + kColS + b * kTile, sw128_desc(qa + off, 16, 1024),
+                   sw128_desc(ka + off, 16, 1024), id_s, kk > 0);
+        }
+        mma_commit(&bars->ring_empty[t % kRing]);
+        mma_commit(&bars->s_full[b]);
+        if (t >= 1) ok = issue_d(t - 1);
+      }
+      if (ok && T >= 1) ok = issue_d(T - 1);
+      mma_commit(&bars->drain);
+      mbar_wait(&bars->drain, 0, abort_flag, kBudget);
+    }
+  } else if (warp >= 4 && warp < 8) {
+    const int q = warp & 3, row = q * 32 + lane;
+    const bool row_ok = row < a.m;
+    const int vlim = !row_ok ? -1 : (a.causal ? B - a.w + row % a.w : B - 1);
+    const float lam = a.lam[(size_t)u * kRows + row];
+    const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
+    uint8_t* xh = sm + kOffXG;
+    uint8_t* xl = xh + kTileBytes;
+    bool ok = true;
+    for (int t = 0; t < T && ok; ++t) {
+      const int b = t & 1;
+      ok = mbar_wait(&bars->s_full[b], (t >> 1) & 1, abort_flag, kBudget);
+      if (ok && t >= 1) ok = mbar_wait(&bars->xg_empty[0], (t - 1) & 1, abort_flag, kBudget);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t sbase = lane_addr + kColS + b * kTile;
+      float va[32], vb[32];
+      tmem_ld32f(sbase, va);
+      tmem_wait32(va);
+      tmem_ld32f(sbase + 32, vb);
+      update_chunk<0>(va, t, vlim, B, a.sl2, lam, mask, xh, xl, row);
+      tmem_wait32(vb);
+      tmem_ld32f(sbase + 64, va);
+      update_chunk<1>(vb, t, vlim, B, a.sl2, lam, mask, xh, xl, row);
+      tmem_wait32(va);
+      tmem_ld32f(sbase + 96, vb);
+      update_chunk<2>(va, t, vlim, B, a.sl2, lam, mask, xh, xl, row);
+      tmem_wait32(vb);
+      tc_fence_before();
+      mbar_arrive(&bars->s_done[b]);   // S is fully read
+      update_chunk<3>(vb, t, vlim, B, a.sl2, lam, mask, xh, xl, row);
+      fence_proxy_async_smem();
+      mbar_arrive(&bars->xg_full[0]);
+    }
+    if (!ok && row == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
+  } else if (warp >= 8) {
+    // epilogue: D = dV^T, lane = column e of V, staged through shared memory
+    const int q = warp & 3, e = q * 32 + lane, et = tid - 256;
+    const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
+    float* stage = (float*)(sm + kOffStage);
+    bool ok = true;
+    for (int t = 0; t < T && ok; ++t) {
+      // V0 segments of this thread's token (32 columns) in the tile's four
+      // chunks, fetched before D is ready
+      const int tk = et & 31, c0 = (et >> 5) * 32;
+      uint4 v0[4][4];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const int srow = __ldg(idx_u + min(t * kTile + c * 32 + tk, B - 1));
+        const uint4* src = (const uint4*)(a.v + ((size_t)u * a.n + srow) * kD + c0);
+#pragma unroll
+        for (int h = 0; h < 4; ++h) v0[c][h] = __ldg(src + h);
+      }
+      ok = mbar_wait(&bars->d_full, t & 1, abort_flag, kBudget);
+      if (!ok) break;
+      tc_fence_after();
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        float v[32];
+        tmem_ld32f(lane_addr + kColG + c * 32, v);
+        tmem_wait32(v);
+        if (c == 3) {
+          tc_fence_before();
+          mbar_arrive(&bars->d_empty);
+        }
+#pragma unroll
+        for (int k2 = 0; k2 < 32; ++k2) stage[k2 * kLD + e] = v[k2];
+        named_bar(3, 128);
+        // a warp takes 32 tokens of one 32-column block
+        const int i = t * kTile + c * 32 + tk;
+        if (i < B) {
+          const size_t dst = ((size_t)u * B + i) * kD + c0;
+#pragma unroll
+          for (int h = 0; h < 4; ++h) {
+            const __nv_bfloat16* pv = (const __nv_bfloat16*)&v0[c][h];
+            uint32_t o[4];
+#pragma unroll
+            for (int z = 0; z < 4; ++z)
+              o[z] = pack_bf16(__bfloat162float(pv[2 * z]) + stage[tk * kLD + c0 + 8 * h + 2 * z],
+                               __bfloat162float(pv[2 * z + 1]) +
+                                   stage[tk * kLD + c0 + 8 * h + 2 * z + 1]);
+            *(uint4*)(a.v_out + dst + 8 * h) = make_uint4(o[0], o[1], o[2], o[3]);
+          }
+        }
+        named_bar(3, 128);
+      }
+    }
+    if (!ok && e == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
   }
   tc_fence_before();
   __syncthreads();
@@ -749,10 +935,26 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) tmem_dealloc(tmem, 512);
 }
 
+// K_out = K0: copies the retained rows, 16 threads per 256-byte row.
+__global__ void __launch_bounds__(256) k_gather_rows(const uint4* __restrict__ k,
+                                                     const int32_t* __restrict__ idx,
+                                                     uint4* __restrict__ k_out, int n, int B) {
+  const int u = blockIdx.y, i = blockIdx.x * 16 + (threadIdx.x >> 4), c = threadIdx.x & 15;
+  if (i >= B) return;
+  const int j = __ldg(idx + (size_t)u * B + i);
+  k_out[((size_t)u * B + i) * 16 + c] = __ldg(k + ((size_t)u * n + j) * 16 + c);
+}
+
 }  // namespace
 
 bool merge_tc_supported(const Shape& s) {
   return s.dtype == GRKV_BF16 && s.m <= kRows && s.B <= kMaxB && s.B >= 1;
+}
+
+size_t merge_tc_ws_bytes(const Shape& s) {
+  const size_t U = (size_t)s.U;
+  return U * kRows * kD * 4 + U * kRows * kRows * 4 + U * kRows * 4 +
+         U * (size_t)((s.B + 31) / 32) * 4;
 }
 
 cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const void* v,
@@ -779,16 +981,28 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
   a.idx = idx;
   a.scores = scores;
   a.y = y;
-  a.k = (const __nv_bfloat16*)k;
   a.v = (const __nv_bfloat16*)v;
-  a.k_out = (__nv_bfloat16*)k_out;
   a.v_out = (__nv_bfloat16*)v_out;
+  const size_t U = (size_t)s.U;
+  a.rz = (float*)(ws + L.merge_tc);
+  a.gram = a.rz + U * kRows * kD;
+  a.lam = a.gram + U * kRows * kRows;
+  a.mask = (uint32_t*)(a.lam + U * kRows);
   a.status = (int*)(ws + L.status);
-  cudaError_t e =
-      cudaFuncSetAttribute(k_merge_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-  if (e != cudaSuccess) return e;
-  k_merge_tc<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, a);
-  count_launches(1);
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(k_merge_gram, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kSmemBytes)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(k_merge_update, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kSmemBytes)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(k_merge_solve, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kSolveSmem)) != cudaSuccess)
+    return e;
+  k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, a);
+  k_merge_solve<<<s.U, 256, kSolveSmem, st>>>(a);
+  k_merge_update<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, a);
+  k_gather_rows<<<dim3((s.B + 15) / 16, s.U), 256, 0, st>>>((const uint4*)k, idx, (uint4*)k_out,
+                                                             s.n, s.B);
+  count_launches(4);
   return cudaGetLastError();
 }
 
