@@ -24,7 +24,9 @@
  *   row_stats[U][m][2] fp32    (M_r, L_r): row max of the logits and
  *                              sum_j exp(l_rj - M_r)
  *   idx      [U][B]    int32   retained positions, ascending; the last w are
- *                              the window n-w..n-1
+ *                              the window n-w..n-1.  grkv_merge reports an
+ *                              entry outside [0, n) as GRKV_ERR_INVALID_ARG in
+ *                              the device status (and reads position 0 there)
  *   k_out, v_out [U][B][d]     compressed cache
  *
  * Ownership and ordering: every pointer except `params` and the output

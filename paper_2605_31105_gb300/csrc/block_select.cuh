@@ -52,14 +52,39 @@ __device__ void block_kth_largest(Get get, int count, int k, int* hist, int* sh,
       if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1);
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-      int cum = 0, dg = 255;
-      for (; dg > 0; --dg) {
-        if (cum + hist[dg] >= rem) break;
-        cum += hist[dg];
+    if (threadIdx.x < 32) {
+      // digit search from 255 down: lane l owns bins 8l..8l+7, a suffix sum
+      // over the lanes gives each lane the count above its bins
+      const int lane = threadIdx.x;
+      int c[8], own = 0;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        c[q] = hist[8 * lane + q];
+        own += c[q];
       }
-      sh[0] = dg;
-      sh[1] = rem - cum;
+      int suf = own;   // inclusive suffix sum over lanes >= lane
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_down_sync(0xffffffffu, suf, o);
+        if (lane + o < 32) suf += y;
+      }
+      int above = suf - own, dg = -1, left = 0;
+#pragma unroll
+      for (int q = 7; q >= 0; --q) {
+        if (dg < 0 && (above + c[q] >= rem || (lane == 0 && q == 0))) {
+          dg = 8 * lane + q;
+          left = rem - above;
+        }
+        above += c[q];
+      }
+      // the largest digit whose suffix count reaches rem (digit 0 otherwise)
+      const unsigned found = __ballot_sync(0xffffffffu, dg >= 0);
+      const int src = 31 - __clz(found);
+      const int dsel = __shfl_sync(0xffffffffu, dg, src), lsel = __shfl_sync(0xffffffffu, left, src);
+      if (lane == 0) {
+        sh[0] = dsel;
+        sh[1] = lsel;
+      }
     }
     __syncthreads();
     prefix |= (uint32_t)sh[0] << shift;

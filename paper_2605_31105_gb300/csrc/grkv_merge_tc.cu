@@ -1,24 +1,29 @@
 // GRKV value step on the tensor cores (bf16, d = 128, m <= 128, B <= 32768).
 //
 // Algorithm 1's value step in dual form (Sec. 3.4, App. D.1) with the fixed
-// tokens of App. D.3, one unit per CTA, in three kernels:
-//   k_merge_gram    row max / sum of the retained logits l = s Q K0^T (K0, V0
-//                   gathered with TMA gather4 from the positions idx); then
-//                   X = softmax over the retained keys, R~ += Xh V0 and the Gram
-//                   G += XGh XGh^T + (2 XGl) XGh^T on tcgen05, where Xh, Xl are the
-//                   bf16 high / low parts of X and XG is X with the fixed columns
-//                   zeroed (N = (G + G^T) / 2 restores all three cross terms).
-//                   Writes R = Y - R~, G and the row normalisers to the workspace.
+// tokens of App. D.3, one unit per CTA:
+//   k_merge_fixed   the fixed set (retained sinks, the window, and the n_fix
+//                   retained prefix tokens with the largest scores) and a
+//                   stable partition of the B retained slots into "positions":
+//                   the n_G non-fixed slots first, then the fixed ones, each in
+//                   slot order.  The window stays last, so position p is
+//                   visible to window row r exactly when p <= B - w + r % w.
+//   k_merge_gram    over the retained keys in position order, gathered with
+//                   cp.async: row max / sum of l = s Q K0^T; then X = softmax,
+//                   R~ += Xh V0 and the Gram G += Xh XGh^T + (2 Xl) XGh^T on
+//                   tcgen05 (Xh, Xl the bf16 high / low parts of X; XGh is Xh
+//                   with the fixed columns zeroed, which removes them from both
+//                   terms; N = (G + G^T) / 2 restores the cross terms).  Writes
+//                   R = Y - R~, G and the row normalisers to the workspace.
 //   k_merge_solve   fp32 in shared memory: N = sym(G) + lambda I, blocked
 //                   Cholesky, Z = N^-1 R by blocked triangular solves.
-//   k_merge_update  per tile D = Zh^T XGh + Zl^T XGh + Zh^T XGl = dV^T on tcgen05
-//                   with Z^T as a TMEM operand; V_out = V0 + dV (fixed rows get
-//                   exactly V0: their XG columns are zero).
-// K_out = K0 is a plain row gather (k_gather_rows).
+//   k_merge_update  over the non-fixed positions only: D = Zh^T XGh + Zl^T XGh +
+//                   Zh^T XGl = dV^T on tcgen05 with Z^T as a TMEM operand, and
+//                   V_out = V0 + dV.
+//   k_merge_copy    K_out = K0 for every slot, V_out = V0 for the fixed slots.
 //
-// Both tensor-core kernels rely on the idx contract of grkv.h: ascending, the
-// window n-w..n-1 in the last w slots, so retained slot i is visible to window
-// slot a (causal) exactly when i <= B - w + a.
+// The kernels rely on the idx contract of grkv.h: ascending, with the window
+// n-w..n-1 in the last w slots.
 #include <cmath>
 
 #include "block_select.cuh"
@@ -35,6 +40,7 @@ constexpr int kTile = 128;
 constexpr int kRows = 128;
 constexpr int kRing = 3;
 constexpr int kThreads = 384;
+constexpr int kProducers = 64;                    // gather threads (warps 2 and 3)
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KB
 constexpr int kMaxB = 32768;
 constexpr long long kBudget = 1ll << 32;
@@ -45,9 +51,7 @@ constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffRing = kOffQ + kTileBytes;              // 3 x 32 KB gathered tiles
 constexpr uint32_t kOffXG = kOffRing + kRing * kTileBytes;     // 2 x 32 KB
 constexpr uint32_t kOffStage = kOffXG + 2 * kTileBytes;        // 32 tokens x 129 fp32
-constexpr uint32_t kOffMask = kOffStage + 32 * kLD * 4;        // fixed-token bits
-constexpr uint32_t kOffMisc = kOffMask + kMaxB / 8;            // hist[256], sh[64]
-constexpr uint32_t kOffBar = kOffMisc + (256 + 64) * 4;
+constexpr uint32_t kOffBar = kOffStage + 32 * kLD * 4;
 constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;
 // k_merge_solve: N and R/Z [128][129] fp32, 1 / L_jj, the failure flag
 constexpr uint32_t kSolveSmem = (2 * kRows * kLD + kRows + 32) * 4;
@@ -64,12 +68,16 @@ struct MArgs {
   const int32_t* idx;        // [U][B]
   const float* scores;       // [U][P]
   const float* y;            // [U][m][128]
-  const __nv_bfloat16* v;    // [U][n][128]
-  __nv_bfloat16* v_out;      // [U][B][128]
+  const __nv_bfloat16* k;    // [U][n][128]
+  const __nv_bfloat16* v;
+  __nv_bfloat16* k_out;      // [U][B][128]
+  __nv_bfloat16* v_out;
   float* rz;                 // [U][128][128]  R (gram) -> Z (solve)
   float* gram;               // [U][128][128]  raw Gram
   float* lam;                // [U][128]       log2 normaliser of each window row
-  uint32_t* mask;            // [U][ceil(B/32)] fixed-token bits
+  int32_t* perm;             // [U][B]         slot at each position
+  int32_t* src;              // [U][B]         idx of that slot (the K / V row)
+  int32_t* ng;               // [U]            number of non-fixed slots
   int* status;
 };
 
@@ -85,37 +93,59 @@ struct MBars {
   int abort;
 };
 
-__device__ __forceinline__ float bf16_round(float x) {
-  return __bfloat162float(__float2bfloat16_rn(x));
+__device__ __forceinline__ float lo_half(uint32_t h) { return __uint_as_float(h << 16); }
+__device__ __forceinline__ float hi_half(uint32_t h) { return __uint_as_float(h & 0xFFFF0000u); }
+
+// Gathers the 128 rows at positions t*128 .. t*128+127 (clamped to B-1) of one
+// unit's [n][128] bf16 matrix into a swizzled 32 KB tile with 16-byte cp.async
+// copies, one commit group.  Called by the 64 producer threads: warp pw takes
+// rows pw*64 .. pw*64+63, two rows (256 contiguous bytes each) per instruction.
+__device__ __forceinline__ void gather_tile(uint8_t* dst, const __nv_bfloat16* base,
+                                            const int32_t* src_u, int B, int t, int pw, int lane) {
+  const int r0 = t * kTile + pw * 64 + 2 * lane;
+  const int ra = __ldg(src_u + min(r0, B - 1)), rb = __ldg(src_u + min(r0 + 1, B - 1));
+  const int chunk = lane & 15, half = chunk >> 3, c8 = chunk & 7;
+  const uint32_t sbase = smem_u32(dst) + half * (kTileBytes / 2);
+  const char* gbase = (const char*)base + chunk * 16;
+#pragma unroll 8
+  for (int s = 0; s < 32; ++s) {
+    const int ja = __shfl_sync(0xffffffffu, ra, s), jb = __shfl_sync(0xffffffffu, rb, s);
+    const int r = pw * 64 + 2 * s + (lane >> 4);
+    const int j = lane < 16 ? ja : jb;
+    cp_async16(sbase + r * 128 + ((c8 ^ (r & 7)) << 4), gbase + (size_t)j * (kD * 2));
+  }
+  cp_async_commit();
 }
-// Four rows (64 columns each) of a 2-D tensor map into consecutive 128-byte rows.
-__device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
-                                            int r0, int r1, int r2, int r3) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4, %5, %6, %7}], [%2];" ::"r"(smem_u32(dst)),
-      "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(r0), "r"(r1), "r"(r2), "r"(r3)
-      : "memory");
+
+// Producer side of the gathered-tile ring: issues load number `use` into its
+// slot and publishes the previous load (its copies done, then a proxy fence so
+// the tensor cores see them).  Returns false if a wait gave up.
+__device__ __forceinline__ bool produce(MBars* bars, uint8_t* sm, const __nv_bfloat16* base,
+                                        const int32_t* src_u, int B, int t, int pw, int lane,
+                                        uint32_t use, volatile int* abort_flag) {
+  const uint32_t slot = use % kRing;
+  bool ok = true;
+  if (use >= kRing) ok = mbar_wait(&bars->ring_empty[slot], (use / kRing - 1) & 1, abort_flag, kBudget);
+  ok = __all_sync(0xffffffffu, ok);
+  if (!ok) return false;
+  gather_tile(sm + kOffRing + slot * kTileBytes, base, src_u, B, t, pw, lane);
+  if (use > 0) {
+    cp_async_wait<1>();
+    fence_proxy_async_smem();
+    mbar_arrive(&bars->ring_full[(use - 1) % kRing]);
+  }
+  return true;
 }
-// Gathers the 128 retained rows of tile t (clamped to the last retained row
-// past B) of one unit's [n][128] matrix into a swizzled 32 KB tile.  Called by
-// a whole warp: lane l fetches rows 4l..4l+3 with one index load each.
-__device__ __forceinline__ void gather_tile(uint8_t* dst, const CUtensorMap* map, uint64_t* bar,
-                                            const int32_t* idx_u, int B, int row0, int t,
-                                            int lane) {
-  int r[4];
-#pragma unroll
-  for (int e = 0; e < 4; ++e) r[e] = row0 + __ldg(idx_u + min(t * kTile + 4 * lane + e, B - 1));
-  if (lane == 0) mbar_expect_tx(bar, kTileBytes);
-  __syncwarp();
-  tma_gather4(dst + lane * 512, map, bar, 0, r[0], r[1], r[2], r[3]);
-  tma_gather4(dst + kTileBytes / 2 + lane * 512, map, bar, 64, r[0], r[1], r[2], r[3]);
+__device__ __forceinline__ void produce_drain(MBars* bars, uint32_t use) {
+  cp_async_wait<0>();
+  fence_proxy_async_smem();
+  if (use > 0) mbar_arrive(&bars->ring_full[(use - 1) % kRing]);
 }
 
 __device__ __forceinline__ void init_common(MBars* bars, int warp) {
   if (threadIdx.x == 0) {
     for (int i = 0; i < kRing; ++i) {
-      mbar_init(&bars->ring_full[i], 1);
+      mbar_init(&bars->ring_full[i], kProducers);
       mbar_init(&bars->ring_empty[i], 1);
     }
     mbar_init(&bars->q_full, 1);
@@ -138,73 +168,88 @@ __device__ __forceinline__ void init_common(MBars* bars, int warp) {
   }
 }
 
-// One 32-column chunk of a gram tile: X, its bf16 high part (TMEM, the R~ MMA
-// operand), XGh (shared memory, the Gram operand) and 2 (X - Xh) on free
-// columns (returned; it goes to TMEM once the S columns it overwrites are read).
+__device__ __forceinline__ void store_row_chunk(uint8_t* tile, int row, int C, const uint32_t* w) {
+  // row `row`, tokens 32C..32C+31 of a K-major SW128 tile: token block C/2,
+  // 16-byte chunks (C&1)*4 .. +3
+#pragma unroll
+  for (int qq = 0; qq < 4; ++qq)
+    *(uint4*)(tile + (C >> 1) * (kTileBytes / 2) + sw128_offset(row, (C & 1) * 4 + qq)) =
+        make_uint4(w[4 * qq], w[4 * qq + 1], w[4 * qq + 2], w[4 * qq + 3]);
+}
+
+// One 32-position chunk of a gram tile whose positions are all non-fixed (and
+// so visible): Xh to TMEM (the A operand of R~ and of the Gram's first term),
+// XGh = Xh to shared memory (the Gram's B operand) and 2 (X - Xh) returned (it
+// goes to TMEM once the S columns it overwrites are read).
 template <int C>
-__device__ __forceinline__ void gram_chunk(const float* v, int t, int vlim, int B, float sl2,
-                                           float lam, const uint32_t* mask, uint32_t sbase,
-                                           uint8_t* xg, int row, uint32_t* lo) {
+__device__ __forceinline__ void gram_chunk_fast(const float* v, float sl2, float lam,
+                                                uint32_t sbase, uint8_t* xg, int row,
+                                                uint32_t* lo) {
+  uint32_t hi[16];
+#pragma unroll
+  for (int e = 0; e < 32; e += 2) {
+    const float x0 = fast_exp2(fmaf(v[e], sl2, -lam)), x1 = fast_exp2(fmaf(v[e + 1], sl2, -lam));
+    const uint32_t h = pack_bf16(x0, x1);
+    hi[e / 2] = h;
+    lo[e / 2] = pack_bf16(2.f * (x0 - lo_half(h)), 2.f * (x1 - hi_half(h)));
+  }
+  tmem_st16(sbase + C * 16, hi);
+  store_row_chunk(xg, row, C, hi);
+}
+// The same for a tile with fixed or invisible positions: X = 0 past vlim,
+// XGh = 0 from position ng on; XGh is written only when the tile has
+// non-fixed positions (want_g).
+template <int C>
+__device__ __forceinline__ void gram_chunk_masked(const float* v, int p0, int vlim, int ng,
+                                                  float sl2, float lam, uint32_t sbase,
+                                                  uint8_t* xg, int row, uint32_t* lo,
+                                                  bool want_g) {
   uint32_t hi[16], ghi[16];
 #pragma unroll
   for (int e = 0; e < 32; e += 2) {
-    float x[2], g[2], l2[2];
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int i = t * kTile + C * 32 + e + h;
-      x[h] = i <= vlim ? fast_exp2(fmaf(v[e + h], sl2, -lam)) : 0.f;
-      const bool fixed = i >= B || ((mask[i >> 5] >> (i & 31)) & 1u);
-      const float xh = bf16_round(x[h]);
-      g[h] = fixed ? 0.f : xh;
-      l2[h] = fixed ? 0.f : 2.f * (x[h] - xh);
-    }
-    hi[e / 2] = pack_bf16(x[0], x[1]);
-    ghi[e / 2] = pack_bf16(g[0], g[1]);
-    lo[e / 2] = pack_bf16(l2[0], l2[1]);
+    const int p = p0 + C * 32 + e;
+    const float x0 = p <= vlim ? fast_exp2(fmaf(v[e], sl2, -lam)) : 0.f;
+    const float x1 = p + 1 <= vlim ? fast_exp2(fmaf(v[e + 1], sl2, -lam)) : 0.f;
+    const uint32_t h = pack_bf16(x0, x1);
+    hi[e / 2] = h;
+    lo[e / 2] = pack_bf16(2.f * (x0 - lo_half(h)), 2.f * (x1 - hi_half(h)));
+    ghi[e / 2] = (p < ng ? (h & 0xFFFFu) : 0u) | (p + 1 < ng ? (h & 0xFFFF0000u) : 0u);
   }
   tmem_st16(sbase + C * 16, hi);
-  // XGh row `row`, tokens 32C..32C+31: token block C/2, 16-byte chunks (C&1)*4..+3
-#pragma unroll
-  for (int qq = 0; qq < 4; ++qq)
-    *(uint4*)(xg + (C >> 1) * (kTileBytes / 2) + sw128_offset(row, (C & 1) * 4 + qq)) =
-        make_uint4(ghi[4 * qq], ghi[4 * qq + 1], ghi[4 * qq + 2], ghi[4 * qq + 3]);
+  if (want_g) store_row_chunk(xg, row, C, ghi);
 }
 
-// One 32-column chunk of an update tile: XGh and XGl (shared memory, the
-// MN-major B operands of D = Z^T XG).
-template <int C>
-__device__ __forceinline__ void update_chunk(const float* v, int t, int vlim, int B, float sl2,
-                                             float lam, const uint32_t* mask, uint8_t* xh,
-                                             uint8_t* xl, int row) {
+// One 32-position chunk of an update tile: XGh and XGl (the MN-major B operands
+// of D = Z^T XG); positions from ng on are fixed and get zeros.
+template <int C, bool kMasked>
+__device__ __forceinline__ void update_chunk(const float* v, int p0, int ng, float sl2, float lam,
+                                             uint8_t* xh, uint8_t* xl, int row) {
   uint32_t ghi[16], glo[16];
 #pragma unroll
   for (int e = 0; e < 32; e += 2) {
-    float g[2], l[2];
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int i = t * kTile + C * 32 + e + h;
-      const float x = i <= vlim ? fast_exp2(fmaf(v[e + h], sl2, -lam)) : 0.f;
-      const bool fixed = i >= B || ((mask[i >> 5] >> (i & 31)) & 1u);
-      const float xhv = bf16_round(x);
-      g[h] = fixed ? 0.f : xhv;
-      l[h] = fixed ? 0.f : x - xhv;
+    const int p = p0 + C * 32 + e;
+    float x0 = fast_exp2(fmaf(v[e], sl2, -lam)), x1 = fast_exp2(fmaf(v[e + 1], sl2, -lam));
+    if (kMasked) {
+      x0 = p < ng ? x0 : 0.f;
+      x1 = p + 1 < ng ? x1 : 0.f;
     }
-    ghi[e / 2] = pack_bf16(g[0], g[1]);
-    glo[e / 2] = pack_bf16(l[0], l[1]);
+    const uint32_t h = pack_bf16(x0, x1);
+    ghi[e / 2] = h;
+    glo[e / 2] = pack_bf16(x0 - lo_half(h), x1 - hi_half(h));
   }
-#pragma unroll
-  for (int qq = 0; qq < 4; ++qq) {
-    const uint32_t off = (C >> 1) * (kTileBytes / 2) + sw128_offset(row, (C & 1) * 4 + qq);
-    *(uint4*)(xh + off) = make_uint4(ghi[4 * qq], ghi[4 * qq + 1], ghi[4 * qq + 2], ghi[4 * qq + 3]);
-    *(uint4*)(xl + off) = make_uint4(glo[4 * qq], glo[4 * qq + 1], glo[4 * qq + 2], glo[4 * qq + 3]);
-  }
+  store_row_chunk(xh, row, C, ghi);
+  store_row_chunk(xl, row, C, glo);
 }
 
-// Online max / sum of exp2 over one 32-column chunk (log2 units).
-__device__ __forceinline__ void stats32(float* v, int i0, int vlim, float sl2, float& M, float& L) {
+// Online max / sum of exp2 over one 32-column chunk (log2 units); positions
+// past vlim are skipped when kMasked.
+template <bool kMasked>
+__device__ __forceinline__ void stats32(float* v, int p0, int vlim, float sl2, float& M, float& L) {
+  if (kMasked) {
 #pragma unroll
-  for (int e = 0; e < 32; ++e)
-    if (i0 + e > vlim) v[e] = -INFINITY;
+    for (int e = 0; e < 32; ++e)
+      if (p0 + e > vlim) v[e] = -INFINITY;
+  }
   float m16[16];
 #pragma unroll
   for (int e = 0; e < 16; ++e) m16[e] = fmaxf(v[e], v[e + 16]);
@@ -212,7 +257,7 @@ __device__ __forceinline__ void stats32(float* v, int i0, int vlim, float sl2, f
   for (int h = 8; h >= 1; h >>= 1)
 #pragma unroll
     for (int e = 0; e < h; ++e) m16[e] = fmaxf(m16[e], m16[e + h]);
-  if (m16[0] == -INFINITY) return;
+  if (kMasked && m16[0] == -INFINITY) return;
   const float cm = m16[0] * sl2;
   if (cm > M) {
     L *= fast_exp2(M - cm);
@@ -224,86 +269,109 @@ __device__ __forceinline__ void stats32(float* v, int i0, int vlim, float sl2, f
   L += (s[0] + s[1]) + (s[2] + s[3]);
 }
 
-// ======================================================== k_merge_gram
-// Roles (384 threads): warp 0 TMA gathers, warp 1 MMA issue, warps 4-7 and
-// 8-11 two compute groups (one thread per window row / TMEM lane) taking
-// alternate tiles.
-__global__ void __launch_bounds__(kThreads, 1)
-    k_merge_gram(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                 const __grid_constant__ CUtensorMap tmV, MArgs a) {
-  extern __shared__ __align__(1024) uint8_t smraw[];
-  uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
-  MBars* bars = (MBars*)(sm + kOffBar);
-  uint32_t* mask = (uint32_t*)(sm + kOffMask);
-  int* hist = (int*)(sm + kOffMisc);
-  int* sh = hist + 256;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int u = blockIdx.x, B = a.B, T = (B + kTile - 1) / kTile, nw = (B + 31) / 32;
+// ======================================================== k_merge_fixed
+// One CTA (256 threads) per unit; shared memory holds one key per slot.
+__global__ void __launch_bounds__(256) k_merge_fixed(MArgs a) {
+  extern __shared__ uint32_t fkey[];   // [B] candidate keys, 0 = not a candidate
+  __shared__ int hist[256], sh[64];
+  const int tid = threadIdx.x, nt = blockDim.x;
+  const int u = blockIdx.x, B = a.B;
   const int32_t* idx_u = a.idx + (size_t)u * B;
   const float* sc_u = a.scores + (size_t)u * a.P;
-  init_common(bars, warp);
-  // ---- fixed tokens: retained sinks, the window, and the n_fix retained
-  // prefix non-sink tokens with the largest scores (ties: smaller position)
-  for (int i = tid; i < nw; i += kThreads) mask[i] = 0;
-  __syncthreads();
-  auto cand = [&](int i) {
+  // Candidates for the score-ranked part: retained prefix tokens past the sinks.
+  // Their scores are non-negative, so every key is above 0.
+  // An idx entry outside [0, n) is reported and read as position 0.
+  auto pos = [&](int i) {
     const int j = __ldg(idx_u + i);
-    return j >= a.n_sink && j < a.P;
+    return (unsigned)j < (unsigned)a.n ? j : 0;
   };
   int nc = 0;
-  for (int i = tid; i < B; i += kThreads) {
-    if (!cand(i)) atomicOr(&mask[i >> 5], 1u << (i & 31));
-    else ++nc;
+  for (int i = tid; i < B; i += nt) {
+    if ((unsigned)__ldg(idx_u + i) >= (unsigned)a.n) set_status(a.status, GRKV_ERR_INVALID_ARG);
+    const int j = pos(i);
+    const bool cand = j >= a.n_sink && j < a.P;
+    fkey[i] = cand ? max(order_key(__ldg(sc_u + j)), 1u) : 0u;
+    nc += cand;
   }
+  __syncthreads();
   int ncand;
   (void)block_exclusive_scan(nc, sh + 8, &ncand);
   const int nf = min(a.n_fix, ncand);
+  uint32_t tau = 0xFFFFFFFFu;
+  int need_eq = 0;
   if (nf > 0) {
     auto get = [&](int i, uint32_t* key) {
-      if (!cand(i)) return false;
-      *key = order_key(__ldg(sc_u + __ldg(idx_u + i)));
-      return true;
+      *key = fkey[i];
+      return *key != 0u;
     };
-    block_topk_mark(get, [&](int i, int) { atomicOr(&mask[i >> 5], 1u << (i & 31)); }, B, nf,
-                    hist, sh);
+    block_kth_largest(get, B, nf, hist, sh, &tau, &need_eq);
   }
+  // fixed: not a candidate, above tau, or among the first need_eq ties
+  const int seg = (B + nt - 1) / nt;
+  const int lo = min(B, tid * seg), hi = min(B, lo + seg);
+  int eq = 0;
+  for (int i = lo; i < hi; ++i) eq += (fkey[i] == tau);
+  int tot;
+  int er = block_exclusive_scan(eq, sh + 8, &tot);
+  int keep = 0;
+  for (int i = lo; i < hi; ++i) {
+    const uint32_t kx = fkey[i];
+    bool fixed = kx == 0u || kx > tau;
+    if (kx == tau) fixed = er++ < need_eq;
+    fkey[i] = fixed ? 1u : 0u;   // each thread rewrites only its own segment
+    keep += !fixed;
+  }
+  int ng;
+  const int gpos = block_exclusive_scan(keep, sh + 8, &ng);
+  int g = gpos;
+  for (int i = lo; i < hi; ++i) {
+    const int at = fkey[i] ? ng + (i - g) : g;
+    g += !fkey[i];
+    a.perm[(size_t)u * B + at] = i;
+    a.src[(size_t)u * B + at] = pos(i);
+  }
+  if (tid == 0) a.ng[u] = ng;
+}
+
+// ======================================================== k_merge_gram
+// Roles (384 threads): warp 0 the Q load, warp 1 MMA issue, warps 2-3 the
+// gathers, warps 4-7 and 8-11 two compute groups (one thread per window row /
+// TMEM lane) taking alternate tiles.  Job k < T: statistics of tile k;
+// T <= k < 2T: R~ and Gram of tile k - T.  S buffer k & 1.
+__global__ void __launch_bounds__(kThreads, 1)
+    k_merge_gram(const __grid_constant__ CUtensorMap tmQ, MArgs a) {
+  extern __shared__ __align__(1024) uint8_t smraw[];
+  uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
+  MBars* bars = (MBars*)(sm + kOffBar);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int u = blockIdx.x, B = a.B, T = (B + kTile - 1) / kTile;
+  const int ng = __ldg(a.ng + u);
+  const int32_t* src_u = a.src + (size_t)u * B;
+  init_common(bars, warp);
   __syncthreads();
-  for (int i = tid; i < nw; i += kThreads) a.mask[(size_t)u * nw + i] = mask[i];
   tc_fence_after();
   const uint32_t tmem = bars->tmem;
   volatile int* abort_flag = &bars->abort;
-  const int row0 = u * a.n;   // first row of this unit in the 2-D K / V maps
 
-  // Job k < T: statistics of tile k; T <= k < 2T: Gram and R~ of tile k - T.
-  // S buffer k & 1; gathers in job order (K, then V for the second half).
   if (warp == 0) {
     if (lane == 0) {
       prefetch_tensormap(&tmQ);
-      prefetch_tensormap(&tmK);
-      prefetch_tensormap(&tmV);
       mbar_expect_tx(&bars->q_full, kTileBytes);
       const uint64_t pol = l2_evict_last();
       tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, 0, u, pol);
       tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
     }
+  } else if (warp == 2 || warp == 3) {
+    const __nv_bfloat16* kb = a.k + (size_t)u * a.n * kD;
+    const __nv_bfloat16* vb = a.v + (size_t)u * a.n * kD;
     uint32_t use = 0;
     bool ok = true;
     for (int k = 0; k < 2 * T && ok; ++k) {
       const int t = k < T ? k : k - T;
-      for (int l = 0; l < (k < T ? 1 : 2) && ok; ++l) {
-        const uint32_t slot = use % kRing;
-        if (use >= kRing)
-          ok = mbar_wait(&bars->ring_empty[slot], (use / kRing - 1) & 1, abort_flag, kBudget);
-        ok = __all_sync(0xffffffffu, ok);
-        if (!ok) break;
-        gather_tile(sm + kOffRing + slot * kTileBytes, l == 0 ? &tmK : &tmV,
-                    &bars->ring_full[slot], idx_u, B, row0, t, lane);
-        ++use;
-      }
+      ok = produce(bars, sm, kb, src_u, B, t, warp - 2, lane, use++, abort_flag);
+      if (ok && k >= T) ok = produce(bars, sm, vb, src_u, B, t, warp - 2, lane, use++, abort_flag);
     }
-    // every issued gather lands before the CTA can exit
-    for (uint32_t i = use > kRing ? use - kRing : 0; i < use; ++i)
-      mbar_wait(&bars->ring_full[i % kRing], (i / kRing) & 1, abort_flag, kBudget);
+    produce_drain(bars, ok ? use : 0);
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t id_s = idesc_bf16(kRows, kTile, 0, 0);
@@ -314,6 +382,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t use = 0;
       int pend = -1;
       uint32_t pend_v = 0;
+      bool g_started = false;
       auto issue_rg = [&](int kp, uint32_t vuse) -> bool {
         const int t = kp - T, b = kp & 1, xb = t & 1;
         bool w = mbar_wait(&bars->s_done[b], (kp >> 1) & 1, abort_flag, kBudget);
@@ -324,21 +393,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         const uint32_t va = smem_u32(sm + kOffRing + (vuse % kRing) * kTileBytes);
         const uint32_t xa = smem_u32(sm + kOffXG + xb * kTileBytes);
+        const uint32_t hi = tmem + kColS + b * kTile, lo2 = hi + 64;
 #pragma unroll
         for (int kk = 0; kk < kTile / 16; ++kk)
-          mma_bf16_ts(tmem + kColR, tmem + kColS + b * kTile + kk * 8,
+          mma_bf16_ts(tmem + kColR, hi + kk * 8,
                       sw128_desc(va + kk * 2048, kTileBytes / 2, 1024), id_r, (t > 0 || kk > 0));
+        if (t * kTile < ng) {   // the tile has non-fixed positions
 #pragma unroll
-        for (int kk = 0; kk < kTile / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
-          mma_bf16(tmem + kColG, sw128_desc(xa + off, 16, 1024), sw128_desc(xa + off, 16, 1024),
-                   id_g, (t > 0 || kk > 0));
-        }
+          for (int kk = 0; kk < kTile / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
+            mma_bf16_ts(tmem + kColG, hi + kk * 8, sw128_desc(xa + off, 16, 1024), id_g,
+                        (g_started || kk > 0));
+          }
 #pragma unroll
-        for (int kk = 0; kk < kTile / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
-          mma_bf16_ts(tmem + kColG, tmem + kColS + b * kTile + 64 + kk * 8,
-                      sw128_desc(xa + off, 16, 1024), id_g, 1);
+          for (int kk = 0; kk < kTile / 16; ++kk) {
+            const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
+            mma_bf16_ts(tmem + kColG, lo2 + kk * 8, sw128_desc(xa + off, 16, 1024), id_g, 1);
+          }
+          g_started = true;
         }
         mma_commit(&bars->ring_empty[vuse % kRing]);
         mma_commit(&bars->xg_empty[xb]);
@@ -379,7 +451,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp >= 4) {
     const int wg = (warp - 4) >> 2, q = warp & 3, row = q * 32 + lane;
     const bool row_ok = row < a.m;
+    // positions past vlim are invisible to this row (and so are those >= B)
     const int vlim = !row_ok ? -1 : (a.causal ? B - a.w + row % a.w : B - 1);
+    const int open = B - a.w;   // positions below this are visible to every window row
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
     float M = -INFINITY, L = 0.f, lam = INFINITY;
     bool ok = true;
@@ -406,50 +480,82 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       if ((k & 1) != wg) continue;
-      const int b = k & 1, t = k < T ? k : k - T;
+      const int b = k & 1, t = k < T ? k : k - T, p0 = t * kTile;
       ok = mbar_wait(&bars->s_full[b], (k >> 1) & 1, abort_flag, kBudget);
       if (!ok) continue;
       tc_fence_after();
       const uint32_t sbase = lane_addr + kColS + b * kTile;
       float va[32], vb[32];
       if (k < T) {
+        // warp-uniform: the TMEM loads below are .sync.aligned
+        const bool masked = __any_sync(0xffffffffu, !row_ok) || p0 + kTile > open + 1;
         tmem_ld32f(sbase, va);
         tmem_wait32(va);
         tmem_ld32f(sbase + 32, vb);
-        stats32(va, t * kTile, vlim, a.sl2, M, L);
-        tmem_wait32(vb);
-        tmem_ld32f(sbase + 64, va);
-        stats32(vb, t * kTile + 32, vlim, a.sl2, M, L);
-        tmem_wait32(va);
-        tmem_ld32f(sbase + 96, vb);
-        stats32(va, t * kTile + 64, vlim, a.sl2, M, L);
-        tmem_wait32(vb);
-        tc_fence_before();
-        mbar_arrive(&bars->s_done[b]);
-        stats32(vb, t * kTile + 96, vlim, a.sl2, M, L);
+        if (masked) {
+          stats32<true>(va, p0, vlim, a.sl2, M, L);
+          tmem_wait32(vb);
+          tmem_ld32f(sbase + 64, va);
+          stats32<true>(vb, p0 + 32, vlim, a.sl2, M, L);
+          tmem_wait32(va);
+          tmem_ld32f(sbase + 96, vb);
+          stats32<true>(va, p0 + 64, vlim, a.sl2, M, L);
+          tmem_wait32(vb);
+          tc_fence_before();
+          mbar_arrive(&bars->s_done[b]);
+          stats32<true>(vb, p0 + 96, vlim, a.sl2, M, L);
+        } else {
+          stats32<false>(va, p0, vlim, a.sl2, M, L);
+          tmem_wait32(vb);
+          tmem_ld32f(sbase + 64, va);
+          stats32<false>(vb, p0 + 32, vlim, a.sl2, M, L);
+          tmem_wait32(va);
+          tmem_ld32f(sbase + 96, vb);
+          stats32<false>(va, p0 + 64, vlim, a.sl2, M, L);
+          tmem_wait32(vb);
+          tc_fence_before();
+          mbar_arrive(&bars->s_done[b]);
+          stats32<false>(vb, p0 + 96, vlim, a.sl2, M, L);
+        }
       } else {
         const int xb = t & 1;
         if (t >= 2) ok = mbar_wait(&bars->xg_empty[xb], ((t >> 1) - 1) & 1, abort_flag, kBudget);
         if (!ok) continue;
         uint8_t* xg = sm + kOffXG + xb * kTileBytes;
         // 2 (X - Xh) goes to TMEM columns 64..127, which hold S chunks 2 and 3:
-        // chunks 0 and 1 are written once chunk 2 is read, 2 and 3 after chunk 3
+        // chunks 0 and 1 are written once chunk 2 is read, 2 and 3 once chunk 3 is
         uint32_t lo0[16], lo1[16], lo2[16], lo3[16];
         tmem_ld32f(sbase, va);
         tmem_wait32(va);
         tmem_ld32f(sbase + 32, vb);
-        gram_chunk<0>(va, t, vlim, B, a.sl2, lam, mask, sbase, xg, row, lo0);
-        tmem_wait32(vb);
-        tmem_ld32f(sbase + 64, va);
-        gram_chunk<1>(vb, t, vlim, B, a.sl2, lam, mask, sbase, xg, row, lo1);
-        tmem_wait32(va);
-        tmem_ld32f(sbase + 96, vb);
-        gram_chunk<2>(va, t, vlim, B, a.sl2, lam, mask, sbase, xg, row, lo2);
-        tmem_st16(sbase + 64, lo0);
-        tmem_st16(sbase + 80, lo1);
-        tmem_wait32(vb);
-        gram_chunk<3>(vb, t, vlim, B, a.sl2, lam, mask, sbase, xg, row, lo3);
-        tmem_st16(sbase + 96, lo2);
+        if (__all_sync(0xffffffffu, row_ok) && p0 + kTile <= ng) {
+          gram_chunk_fast<0>(va, a.sl2, lam, sbase, xg, row, lo0);
+          tmem_wait32(vb);
+          tmem_ld32f(sbase + 64, va);
+          gram_chunk_fast<1>(vb, a.sl2, lam, sbase, xg, row, lo1);
+          tmem_wait32(va);
+          tmem_st16(sbase + 64, lo0);
+          tmem_st16(sbase + 80, lo1);
+          tmem_ld32f(sbase + 96, vb);
+          gram_chunk_fast<2>(va, a.sl2, lam, sbase, xg, row, lo2);
+          tmem_wait32(vb);
+          tmem_st16(sbase + 96, lo2);
+          gram_chunk_fast<3>(vb, a.sl2, lam, sbase, xg, row, lo3);
+        } else {
+          const bool want_g = p0 < ng;
+          gram_chunk_masked<0>(va, p0, vlim, ng, a.sl2, lam, sbase, xg, row, lo0, want_g);
+          tmem_wait32(vb);
+          tmem_ld32f(sbase + 64, va);
+          gram_chunk_masked<1>(vb, p0, vlim, ng, a.sl2, lam, sbase, xg, row, lo1, want_g);
+          tmem_wait32(va);
+          tmem_st16(sbase + 64, lo0);
+          tmem_st16(sbase + 80, lo1);
+          tmem_ld32f(sbase + 96, vb);
+          gram_chunk_masked<2>(va, p0, vlim, ng, a.sl2, lam, sbase, xg, row, lo2, want_g);
+          tmem_wait32(vb);
+          tmem_st16(sbase + 96, lo2);
+          gram_chunk_masked<3>(vb, p0, vlim, ng, a.sl2, lam, sbase, xg, row, lo3, want_g);
+        }
         tmem_st16(sbase + 112, lo3);
         tmem_st_wait();
         fence_proxy_async_smem();
@@ -480,6 +586,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tmem_ld32f(lane_addr + kColG + c * 32, v);
         tmem_wait32(v);
+        if (ng == 0) {   // no Gram MMA ran
+#pragma unroll
+          for (int e = 0; e < 32; ++e) v[e] = 0.f;
+        }
 #pragma unroll
         for (int e = 0; e < 32; e += 4)
           *(float4*)(G + c * 32 + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
@@ -725,25 +835,24 @@ __global__ void __launch_bounds__(256) k_merge_solve(MArgs a) {
 }
 
 // ======================================================== k_merge_update
-// Roles (384 threads): warp 0 TMA gathers of K0, warp 1 MMA issue, warps 4-7
-// XG tiles (one thread per window row), warps 8-11 the output epilogue.
+// Roles (384 threads): warp 0 the Q load, warp 1 MMA issue, warps 2-3 the K0
+// gathers, warps 4-7 the XG tiles (one thread per window row), warps 8-11 the
+// output epilogue.  Only the tiles with non-fixed positions are visited.
 __global__ void __launch_bounds__(kThreads, 1)
-    k_merge_update(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                   MArgs a) {
+    k_merge_update(const __grid_constant__ CUtensorMap tmQ, MArgs a) {
   extern __shared__ __align__(1024) uint8_t smraw[];
   uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
   MBars* bars = (MBars*)(sm + kOffBar);
-  uint32_t* mask = (uint32_t*)(sm + kOffMask);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int u = blockIdx.x, B = a.B, T = (B + kTile - 1) / kTile, nw = (B + 31) / 32;
-  const int32_t* idx_u = a.idx + (size_t)u * B;
+  const int u = blockIdx.x, B = a.B;
+  const int ng = __ldg(a.ng + u), T = (ng + kTile - 1) / kTile;
+  const int32_t* src_u = a.src + (size_t)u * B;
+  const int32_t* perm_u = a.perm + (size_t)u * B;
   init_common(bars, warp);
-  for (int i = tid; i < nw; i += kThreads) mask[i] = a.mask[(size_t)u * nw + i];
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars->tmem;
   volatile int* abort_flag = &bars->abort;
-  const int row0 = u * a.n;
   // Z^T into TMEM as MMA operands: lane = column e of Z, packed row pairs
   if (warp >= 4 && warp < 8) {
     const int q = warp & 3, e = q * 32 + lane;
@@ -755,9 +864,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int p = 0; p < 16; ++p) {
         const float z0 = Z[(rc * 32 + 2 * p) * kD + e], z1 = Z[(rc * 32 + 2 * p + 1) * kD + e];
-        const float h0 = bf16_round(z0), h1 = bf16_round(z1);
-        zh[p] = pack_bf16(h0, h1);
-        zl[p] = pack_bf16(z0 - h0, z1 - h1);
+        const uint32_t h = pack_bf16(z0, z1);
+        zh[p] = h;
+        zl[p] = pack_bf16(z0 - lo_half(h), z1 - hi_half(h));
       }
       tmem_st16(lane_addr + kColR + rc * 16, zh);
       tmem_st16(lane_addr + kColR + 64 + rc * 16, zl);
@@ -769,30 +878,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
 
   if (warp == 0) {
-    if (lane == 0) {
+    if (lane == 0 && T > 0) {
       prefetch_tensormap(&tmQ);
-      prefetch_tensormap(&tmK);
       mbar_expect_tx(&bars->q_full, kTileBytes);
       const uint64_t pol = l2_evict_last();
       tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, 0, u, pol);
       tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
     }
+  } else if (warp == 2 || warp == 3) {
+    const __nv_bfloat16* kb = a.k + (size_t)u * a.n * kD;
     uint32_t use = 0;
     bool ok = true;
-    for (int t = 0; t < T && ok; ++t) {
-      const uint32_t slot = use % kRing;
-      if (use >= kRing)
-        ok = mbar_wait(&bars->ring_empty[slot], (use / kRing - 1) & 1, abort_flag, kBudget);
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok) break;
-      gather_tile(sm + kOffRing + slot * kTileBytes, &tmK, &bars->ring_full[slot], idx_u, B, row0,
-                  t, lane);
-      ++use;
-    }
-    for (uint32_t i = use > kRing ? use - kRing : 0; i < use; ++i)
-      mbar_wait(&bars->ring_full[i % kRing], (i / kRing) & 1, abort_flag, kBudget);
+    for (int t = 0; t < T && ok; ++t)
+      ok = produce(bars, sm, kb, src_u, B, t, warp - 2, lane, use++, abort_flag);
+    produce_drain(bars, ok ? use : 0);
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && T > 0) {
       const uint32_t id_s = idesc_bf16(kRows, kTile, 0, 0);
       const uint32_t id_d = idesc_bf16(kD, kTile, 0, 1);   // D = Z^T XG (XG MN-major)
       const uint32_t qa = smem_u32(sm + kOffQ);
@@ -836,21 +937,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         mma_commit(&bars->s_full[b]);
         if (t >= 1) ok = issue_d(t - 1);
       }
-      if (ok && T >= 1) ok = issue_d(T - 1);
+      if (ok) ok = issue_d(T - 1);
       mma_commit(&bars->drain);
       mbar_wait(&bars->drain, 0, abort_flag, kBudget);
     }
   } else if (warp >= 4 && warp < 8) {
     const int q = warp & 3, row = q * 32 + lane;
-    const bool row_ok = row < a.m;
-    const int vlim = !row_ok ? -1 : (a.causal ? B - a.w + row % a.w : B - 1);
+    // rows past m have lam = +inf and give X = 0
     const float lam = a.lam[(size_t)u * kRows + row];
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
     uint8_t* xh = sm + kOffXG;
     uint8_t* xl = xh + kTileBytes;
     bool ok = true;
     for (int t = 0; t < T && ok; ++t) {
-      const int b = t & 1;
+      const int b = t & 1, p0 = t * kTile;
       ok = mbar_wait(&bars->s_full[b], (t >> 1) & 1, abort_flag, kBudget);
       if (ok && t >= 1) ok = mbar_wait(&bars->xg_empty[0], (t - 1) & 1, abort_flag, kBudget);
       if (!ok) break;
@@ -860,38 +960,52 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_ld32f(sbase, va);
       tmem_wait32(va);
       tmem_ld32f(sbase + 32, vb);
-      update_chunk<0>(va, t, vlim, B, a.sl2, lam, mask, xh, xl, row);
-      tmem_wait32(vb);
-      tmem_ld32f(sbase + 64, va);
-      update_chunk<1>(vb, t, vlim, B, a.sl2, lam, mask, xh, xl, row);
-      tmem_wait32(va);
-      tmem_ld32f(sbase + 96, vb);
-      update_chunk<2>(va, t, vlim, B, a.sl2, lam, mask, xh, xl, row);
-      tmem_wait32(vb);
-      tc_fence_before();
-      mbar_arrive(&bars->s_done[b]);   // S is fully read
-      update_chunk<3>(vb, t, vlim, B, a.sl2, lam, mask, xh, xl, row);
+      if (p0 + kTile <= ng) {
+        update_chunk<0, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
+        tmem_wait32(vb);
+        tmem_ld32f(sbase + 64, va);
+        update_chunk<1, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        tmem_wait32(va);
+        tmem_ld32f(sbase + 96, vb);
+        update_chunk<2, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
+        tmem_wait32(vb);
+        tc_fence_before();
+        mbar_arrive(&bars->s_done[b]);   // S is fully read
+        update_chunk<3, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+      } else {
+        update_chunk<0, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
+        tmem_wait32(vb);
+        tmem_ld32f(sbase + 64, va);
+        update_chunk<1, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        tmem_wait32(va);
+        tmem_ld32f(sbase + 96, vb);
+        update_chunk<2, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
+        tmem_wait32(vb);
+        tc_fence_before();
+        mbar_arrive(&bars->s_done[b]);
+        update_chunk<3, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+      }
       fence_proxy_async_smem();
       mbar_arrive(&bars->xg_full[0]);
     }
     if (!ok && row == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
   } else if (warp >= 8) {
-    // epilogue: D = dV^T, lane = column e of V, staged through shared memory
+    // epilogue: D = dV^T, lane = column e of V, staged through shared memory;
+    // thread et then owns position tk of each 32-position block, columns c0..c0+31
     const int q = warp & 3, e = q * 32 + lane, et = tid - 256;
+    const int tk = et & 31, c0 = (et >> 5) * 32;
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
     float* stage = (float*)(sm + kOffStage);
     bool ok = true;
     for (int t = 0; t < T && ok; ++t) {
-      // V0 segments of this thread's token (32 columns) in the tile's four
-      // chunks, fetched before D is ready
-      const int tk = et & 31, c0 = (et >> 5) * 32;
+      // V0 segments of this thread's positions, fetched before D is ready
       uint4 v0[4][4];
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
-        const int srow = __ldg(idx_u + min(t * kTile + c * 32 + tk, B - 1));
-        const uint4* src = (const uint4*)(a.v + ((size_t)u * a.n + srow) * kD + c0);
+        const int srow = __ldg(src_u + min(t * kTile + c * 32 + tk, B - 1));
+        const uint4* gsrc = (const uint4*)(a.v + ((size_t)u * a.n + srow) * kD + c0);
 #pragma unroll
-        for (int h = 0; h < 4; ++h) v0[c][h] = __ldg(src + h);
+        for (int h = 0; h < 4; ++h) v0[c][h] = __ldg(gsrc + h);
       }
       ok = mbar_wait(&bars->d_full, t & 1, abort_flag, kBudget);
       if (!ok) break;
@@ -908,10 +1022,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int k2 = 0; k2 < 32; ++k2) stage[k2 * kLD + e] = v[k2];
         named_bar(3, 128);
-        // a warp takes 32 tokens of one 32-column block
-        const int i = t * kTile + c * 32 + tk;
-        if (i < B) {
-          const size_t dst = ((size_t)u * B + i) * kD + c0;
+        const int p = t * kTile + c * 32 + tk;
+        if (p < ng) {
+          const size_t dst = ((size_t)u * B + __ldg(perm_u + p)) * kD + c0;
 #pragma unroll
           for (int h = 0; h < 4; ++h) {
             const __nv_bfloat16* pv = (const __nv_bfloat16*)&v0[c][h];
@@ -935,14 +1048,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) tmem_dealloc(tmem, 512);
 }
 
-// K_out = K0: copies the retained rows, 16 threads per 256-byte row.
-__global__ void __launch_bounds__(256) k_gather_rows(const uint4* __restrict__ k,
-                                                     const int32_t* __restrict__ idx,
-                                                     uint4* __restrict__ k_out, int n, int B) {
+// K_out = K0 for every slot, V_out = V0 for the fixed slots (positions >= ng);
+// 16 threads per 256-byte row.
+__global__ void __launch_bounds__(256) k_merge_copy(MArgs a) {
   const int u = blockIdx.y, i = blockIdx.x * 16 + (threadIdx.x >> 4), c = threadIdx.x & 15;
-  if (i >= B) return;
-  const int j = __ldg(idx + (size_t)u * B + i);
-  k_out[((size_t)u * B + i) * 16 + c] = __ldg(k + ((size_t)u * n + j) * 16 + c);
+  if (i >= a.B) return;
+  const size_t ub = (size_t)u * a.B;
+  const uint4* k = (const uint4*)a.k + (size_t)u * a.n * 16;
+  const uint4* v = (const uint4*)a.v + (size_t)u * a.n * 16;
+  const int j = __ldg(a.idx + ub + i);
+  ((uint4*)a.k_out)[(ub + i) * 16 + c] =
+      __ldg(k + (size_t)((unsigned)j < (unsigned)a.n ? j : 0) * 16 + c);
+  if (i >= __ldg(a.ng + u))
+    ((uint4*)a.v_out)[(ub + __ldg(a.perm + ub + i)) * 16 + c] =
+        __ldg(v + (size_t)__ldg(a.src + ub + i) * 16 + c);
 }
 
 }  // namespace
@@ -953,18 +1072,15 @@ bool merge_tc_supported(const Shape& s) {
 
 size_t merge_tc_ws_bytes(const Shape& s) {
   const size_t U = (size_t)s.U;
-  return U * kRows * kD * 4 + U * kRows * kRows * 4 + U * kRows * 4 +
-         U * (size_t)((s.B + 31) / 32) * 4;
+  return U * kRows * kD * 4 + U * kRows * kRows * 4 + U * kRows * 4 + 2 * U * (size_t)s.B * 4 +
+         U * 4;
 }
 
 cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const void* v,
                             const float* scores, const float* y, const int32_t* idx, void* k_out,
                             void* v_out, char* ws, const WsLayout& L, cudaStream_t st) {
-  CUtensorMap mq, mk, mv;
-  if (!encode_bf16_3d(&mq, q, kD, s.m, s.U, 64, kRows) ||
-      !encode_bf16_2d_rows(&mk, k, kD, (uint64_t)s.U * s.n) ||
-      !encode_bf16_2d_rows(&mv, v, kD, (uint64_t)s.U * s.n))
-    return cudaErrorInvalidValue;
+  CUtensorMap mq;
+  if (!encode_bf16_3d(&mq, q, kD, s.m, s.U, 64, kRows)) return cudaErrorInvalidValue;
   MArgs a{};
   a.U = s.U;
   a.n = s.n;
@@ -981,13 +1097,17 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
   a.idx = idx;
   a.scores = scores;
   a.y = y;
+  a.k = (const __nv_bfloat16*)k;
   a.v = (const __nv_bfloat16*)v;
+  a.k_out = (__nv_bfloat16*)k_out;
   a.v_out = (__nv_bfloat16*)v_out;
   const size_t U = (size_t)s.U;
   a.rz = (float*)(ws + L.merge_tc);
   a.gram = a.rz + U * kRows * kD;
   a.lam = a.gram + U * kRows * kRows;
-  a.mask = (uint32_t*)(a.lam + U * kRows);
+  a.perm = (int32_t*)(a.lam + U * kRows);
+  a.src = a.perm + U * s.B;
+  a.ng = a.src + U * s.B;
   a.status = (int*)(ws + L.status);
   cudaError_t e;
   if ((e = cudaFuncSetAttribute(k_merge_gram, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -995,14 +1115,16 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
       (e = cudaFuncSetAttribute(k_merge_update, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 kSmemBytes)) != cudaSuccess ||
       (e = cudaFuncSetAttribute(k_merge_solve, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                kSolveSmem)) != cudaSuccess)
+                                kSolveSmem)) != cudaSuccess ||
+      (e = cudaFuncSetAttribute(k_merge_fixed, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                s.B * 4)) != cudaSuccess)
     return e;
-  k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, a);
+  k_merge_fixed<<<s.U, 256, s.B * 4, st>>>(a);
+  k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, a);
   k_merge_solve<<<s.U, 256, kSolveSmem, st>>>(a);
-  k_merge_update<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, a);
-  k_gather_rows<<<dim3((s.B + 15) / 16, s.U), 256, 0, st>>>((const uint4*)k, idx, (uint4*)k_out,
-                                                             s.n, s.B);
-  count_launches(4);
+  k_merge_update<<<s.U, kThreads, kSmemBytes, st>>>(mq, a);
+  k_merge_copy<<<dim3((s.B + 15) / 16, s.U), 256, 0, st>>>(a);
+  count_launches(5);
   return cudaGetLastError();
 }
 

@@ -281,6 +281,13 @@ __global__ void __launch_bounds__(512) k_merge(
   float* tile = qs + m * QP;    // [32][QP]
   float* xt = tile + 32 * QP;   // [m][33]
   const int32_t* id = idx + (size_t)u * B;
+  // retained position of slot i; an entry outside [0, n) is reported and read as 0
+  auto pos = [&](int i) {
+    const int j = id[i];
+    return (unsigned)j < (unsigned)s.n ? j : 0;
+  };
+  for (int i = tid; i < B; i += nthr)
+    if ((unsigned)id[i] >= (unsigned)s.n) set_status(status, GRKV_ERR_INVALID_ARG);
   float* X = xbuf + (size_t)u * m * B;
   uint8_t* F = flags + (size_t)u * B;
   A* N = gram + (size_t)u * m * m;
@@ -295,12 +302,12 @@ __global__ void __launch_bounds__(512) k_merge(
   for (int i = tid; i < m * kD; i += nthr)
     qs[(i / kD) * QP + i % kD] = ldv(q + (size_t)u * m * kD, i);
   // K_out = K0 (the key step is not applied)
-  for (int i = tid; i < B * kD; i += nthr) ko[i] = ku[(size_t)id[i / kD] * kD + i % kD];
+  for (int i = tid; i < B * kD; i += nthr) ko[i] = ku[(size_t)pos(i / kD) * kD + i % kD];
 
   // Fixed set: retained sinks, the window, and the n_fix best-scored
   // retained prefix non-sink tokens.
   auto cand = [&](int i) {
-    const int j = id[i];
+    const int j = pos(i);
     return j >= s.n_sink && j < s.P;
   };
   int nc = 0;
@@ -314,7 +321,7 @@ __global__ void __launch_bounds__(512) k_merge(
   if (nf > 0) {
     auto get = [&](int i, uint32_t* key) {
       if (!cand(i)) return false;
-      *key = order_key(cu[id[i]]);
+      *key = order_key(cu[pos(i)]);
       return true;
     };
     block_topk_mark(get, [&](int i, int) { F[i] = 1; }, B, nf, hist, sh);
@@ -327,13 +334,13 @@ __global__ void __launch_bounds__(512) k_merge(
     __syncthreads();
     for (int i = tid; i < 32 * kD; i += nthr) {
       const int jj = i / kD, t = i % kD;
-      tile[jj * QP + t] = jj < len ? ldv(ku, (size_t)id[base + jj] * kD + t) : 0.f;
+      tile[jj * QP + t] = jj < len ? ldv(ku, (size_t)pos(base + jj) * kD + t) : 0.f;
     }
     __syncthreads();
     for (int pr = tid; pr < m * 32; pr += nthr) {
       const int r = pr >> 5, jj = pr & 31;
       if (jj >= len) continue;
-      const int j = id[base + jj];
+      const int j = pos(base + jj);
       float l = -INFINITY;
       if (visible(s, r, j)) {
         float a = 0.f;
@@ -360,7 +367,7 @@ __global__ void __launch_bounds__(512) k_merge(
   }
   __syncthreads();
   if (s.lambda_inf) {
-    for (int i = tid; i < B * kD; i += nthr) vo[i] = vu[(size_t)id[i / kD] * kD + i % kD];
+    for (int i = tid; i < B * kD; i += nthr) vo[i] = vu[(size_t)pos(i / kD) * kD + i % kD];
     return;
   }
 
@@ -376,7 +383,7 @@ __global__ void __launch_bounds__(512) k_merge(
       __syncthreads();
       for (int i = tid; i < 32 * kD; i += nthr) {
         const int jj = i / kD, t = i % kD;
-        tile[jj * QP + t] = jj < len ? ldv(vu, (size_t)id[base + jj] * kD + t) : 0.f;
+        tile[jj * QP + t] = jj < len ? ldv(vu, (size_t)pos(base + jj) * kD + t) : 0.f;
       }
       for (int i = tid; i < m * 32; i += nthr) {
         const int r = i >> 5, jj = i & 31;
@@ -443,7 +450,7 @@ __global__ void __launch_bounds__(512) k_merge(
     __syncthreads();
     if (sh[0]) {  // singular dual system: report it and leave V0 in place
       if (tid == 0) set_status(status, GRKV_ERR_NUMERIC);
-      for (int i = tid; i < B * kD; i += nthr) vo[i] = vu[(size_t)id[i / kD] * kD + i % kD];
+      for (int i = tid; i < B * kD; i += nthr) vo[i] = vu[(size_t)pos(i / kD) * kD + i % kD];
       return;
     }
     const A piv = N[(size_t)c * m + c];
@@ -482,7 +489,7 @@ __global__ void __launch_bounds__(512) k_merge(
     __syncthreads();
     for (int p = tid; p < len * kD; p += nthr) {
       const int jj = p / kD, c = p % kD, i = base + jj;
-      const size_t src = (size_t)id[i] * kD + c;
+      const size_t src = (size_t)pos(i) * kD + c;
       if (F[i]) {
         vo[(size_t)i * kD + c] = vu[src];
       } else {
