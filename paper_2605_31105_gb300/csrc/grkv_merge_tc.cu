@@ -6,10 +6,12 @@
 //                   retained prefix tokens with the largest scores) and a
 //                   stable partition of the B retained slots into "positions":
 //                   the n_G non-fixed slots first, then the fixed ones, each in
-//                   slot order.  The window stays last, so position p is
-//                   visible to window row r exactly when p <= B - w + r % w.
-//   k_merge_gram    over the retained keys in position order, gathered with
-//                   cp.async: row max / sum of l = s Q K0^T; then X = softmax,
+//                   slot order.  The window stays last in both orders, so slot
+//                   or position p is visible to window row r exactly when
+//                   p <= B - w + r % w.
+//   k_merge_gram    pass 1 over the slots: row max / sum of l = s Q K0^T (K0
+//                   gathered with cp.async) and K_out = K0 by TMA stores of the
+//                   gathered tiles; pass 2 over the positions: X = softmax,
 //                   R~ += Xh V0 and the Gram G += Xh XGh^T + (2 Xl) XGh^T on
 //                   tcgen05 (Xh, Xl the bf16 high / low parts of X; XGh is Xh
 //                   with the fixed columns zeroed, which removes them from both
@@ -17,10 +19,10 @@
 //                   R = Y - R~, G and the row normalisers to the workspace.
 //   k_merge_solve   fp32 in shared memory: N = sym(G) + lambda I, blocked
 //                   Cholesky, Z = N^-1 R by blocked triangular solves.
-//   k_merge_update  over the non-fixed positions only: D = Zh^T XGh + Zl^T XGh +
-//                   Zh^T XGl = dV^T on tcgen05 with Z^T as a TMEM operand, and
+//   k_merge_update  over the non-fixed positions only: dV = XGh^T Zh + XGh^T Zl
+//                   + XGl^T Zh on tcgen05 (one TMEM lane per token), and
 //                   V_out = V0 + dV.
-//   k_merge_copy    K_out = K0 for every slot, V_out = V0 for the fixed slots.
+//   k_merge_copy    V_out = V0 for the fixed slots.
 //
 // The kernels rely on the idx contract of grkv.h: ascending, with the window
 // n-w..n-1 in the last w slots.
@@ -38,28 +40,34 @@ using namespace sm100;
 
 constexpr int kTile = 128;
 constexpr int kRows = 128;
-constexpr int kRing = 3;
 constexpr int kThreads = 384;
 constexpr int kProducers = 64;                    // gather threads (warps 2 and 3)
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KB
 constexpr int kMaxB = 32768;
 constexpr long long kBudget = 1ll << 32;
-constexpr int kLD = 129;   // fp32 row stride of N, R/Z and the epilogue stage
+constexpr int kLD = 129;   // fp32 row stride of N and R/Z in k_merge_solve
 
-// Shared memory of the tensor-core kernels (offsets from a 1024-byte aligned base).
+// Shared memory (offsets from a 1024-byte aligned base).  k_merge_gram: Q, a
+// ring of four gathered tiles, two XGh tiles.  k_merge_update: Q, a ring of
+// two gathered tiles, XGh, XGl, Zh, Zl.  Both end with the barriers.
+constexpr int kRingG = 4, kRingU = 2;
 constexpr uint32_t kOffQ = 0;
-constexpr uint32_t kOffRing = kOffQ + kTileBytes;              // 3 x 32 KB gathered tiles
-constexpr uint32_t kOffXG = kOffRing + kRing * kTileBytes;     // 2 x 32 KB
-constexpr uint32_t kOffStage = kOffXG + 2 * kTileBytes;        // 32 tokens x 129 fp32
-constexpr uint32_t kOffBar = kOffStage + 32 * kLD * 4;
+constexpr uint32_t kOffRing = kTileBytes;
+constexpr uint32_t kOffXG = kOffRing + kRingG * kTileBytes;   // gram: 2 tiles
+constexpr uint32_t kOffXh = kOffRing + kRingU * kTileBytes;   // update: XGh, XGl, Zh, Zl
+constexpr uint32_t kOffBar = 7 * kTileBytes;
+static_assert(kOffXG + 2 * kTileBytes == kOffBar && kOffXh + 4 * kTileBytes == kOffBar,
+              "shared-memory layouts");
 constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;
 // k_merge_solve: N and R/Z [128][129] fp32, 1 / L_jj, the failure flag
 constexpr uint32_t kSolveSmem = (2 * kRows * kLD + kRows + 32) * 4;
 
-// TMEM columns.
-constexpr uint32_t kColS = 0;     // two S buffers (128 each)
-constexpr uint32_t kColR = 256;   // gram: R~ accumulator;  update: Zh^T (64) | Zl^T (64)
-constexpr uint32_t kColG = 384;   // gram: Gram accumulator; update: D = dV^T
+// TMEM columns.  gram: S[2] 0..255, R~ 256..383, Gram 384..511.
+// update: S[2] 0..255, D[2] 256..511.
+constexpr uint32_t kColS = 0;
+constexpr uint32_t kColR = 256;
+constexpr uint32_t kColG = 384;
+constexpr uint32_t kColD = 256;
 
 struct MArgs {
   int U, n, w, m, P, B, causal, n_sink, n_fix;
@@ -70,8 +78,7 @@ struct MArgs {
   const float* y;            // [U][m][128]
   const __nv_bfloat16* k;    // [U][n][128]
   const __nv_bfloat16* v;
-  __nv_bfloat16* k_out;      // [U][B][128]
-  __nv_bfloat16* v_out;
+  __nv_bfloat16* v_out;      // [U][B][128]
   float* rz;                 // [U][128][128]  R (gram) -> Z (solve)
   float* gram;               // [U][128][128]  raw Gram
   float* lam;                // [U][128]       log2 normaliser of each window row
@@ -82,28 +89,33 @@ struct MArgs {
 };
 
 struct MBars {
-  uint64_t ring_full[kRing], ring_empty[kRing];
+  uint64_t ring_full[4], ring_empty[4];
   uint64_t q_full;
   uint64_t s_full[2], s_done[2];
   uint64_t xg_full[2], xg_empty[2];
   uint64_t acc_done;
-  uint64_t d_full, d_empty;
+  uint64_t d_full[2], d_empty[2];
   uint64_t drain;
   uint32_t tmem;
   int abort;
 };
+static_assert(sizeof(MBars) <= 256, "barrier block");
 
 __device__ __forceinline__ float lo_half(uint32_t h) { return __uint_as_float(h << 16); }
 __device__ __forceinline__ float hi_half(uint32_t h) { return __uint_as_float(h & 0xFFFF0000u); }
 
-// Gathers the 128 rows at positions t*128 .. t*128+127 (clamped to B-1) of one
-// unit's [n][128] bf16 matrix into a swizzled 32 KB tile with 16-byte cp.async
-// copies, one commit group.  Called by the 64 producer threads: warp pw takes
-// rows pw*64 .. pw*64+63, two rows (256 contiguous bytes each) per instruction.
+// Gathers rows rows_u[t*128 .. t*128+127] (clamped to slot B-1; a row outside
+// [0, n) reads row 0) of one unit's [n][128] bf16 matrix into a swizzled 32 KB
+// tile with 16-byte cp.async copies, as one commit group.  Called by the 64
+// producer threads: warp pw takes tile rows pw*64 .. pw*64+63, two rows (256
+// contiguous bytes each) per instruction.
 __device__ __forceinline__ void gather_tile(uint8_t* dst, const __nv_bfloat16* base,
-                                            const int32_t* src_u, int B, int t, int pw, int lane) {
+                                            const int32_t* rows_u, int B, int n, int t, int pw,
+                                            int lane) {
   const int r0 = t * kTile + pw * 64 + 2 * lane;
-  const int ra = __ldg(src_u + min(r0, B - 1)), rb = __ldg(src_u + min(r0 + 1, B - 1));
+  int ra = __ldg(rows_u + min(r0, B - 1)), rb = __ldg(rows_u + min(r0 + 1, B - 1));
+  ra = (unsigned)ra < (unsigned)n ? ra : 0;
+  rb = (unsigned)rb < (unsigned)n ? rb : 0;
   const int chunk = lane & 15, half = chunk >> 3, c8 = chunk & 7;
   const uint32_t sbase = smem_u32(dst) + half * (kTileBytes / 2);
   const char* gbase = (const char*)base + chunk * 16;
@@ -117,36 +129,53 @@ __device__ __forceinline__ void gather_tile(uint8_t* dst, const __nv_bfloat16* b
   cp_async_commit();
 }
 
-// Producer side of the gathered-tile ring: issues load number `use` into its
-// slot and publishes the previous load (its copies done, then a proxy fence so
-// the tensor cores see them).  Returns false if a wait gave up.
-__device__ __forceinline__ bool produce(MBars* bars, uint8_t* sm, const __nv_bfloat16* base,
-                                        const int32_t* src_u, int B, int t, int pw, int lane,
-                                        uint32_t use, volatile int* abort_flag) {
-  const uint32_t slot = use % kRing;
-  bool ok = true;
-  if (use >= kRing) ok = mbar_wait(&bars->ring_empty[slot], (use / kRing - 1) & 1, abort_flag, kBudget);
-  ok = __all_sync(0xffffffffu, ok);
-  if (!ok) return false;
-  gather_tile(sm + kOffRing + slot * kTileBytes, base, src_u, B, t, pw, lane);
-  if (use > 0) {
-    cp_async_wait<1>();
+// Producer side of a ring of R gathered tiles.  Each producer thread publishes
+// a load on ring_full once its own copies of it have landed (then a proxy
+// fence, so the tensor cores and TMA see them), at most LAG loads behind the
+// newest, and publishes everything before it blocks on a full ring.
+template <int R, int LAG>
+struct Producer {
+  uint32_t use = 0, pub = 0;
+  __device__ __forceinline__ void publish_one(MBars* bars) {
     fence_proxy_async_smem();
-    mbar_arrive(&bars->ring_full[(use - 1) % kRing]);
+    mbar_arrive(&bars->ring_full[pub % R]);
+    ++pub;
   }
-  return true;
-}
-__device__ __forceinline__ void produce_drain(MBars* bars, uint32_t use) {
-  cp_async_wait<0>();
-  fence_proxy_async_smem();
-  if (use > 0) mbar_arrive(&bars->ring_full[(use - 1) % kRing]);
-}
+  __device__ __forceinline__ bool load(MBars* bars, uint8_t* sm, const __nv_bfloat16* base,
+                                       const int32_t* rows_u, int B, int n, int t, int pw,
+                                       int lane, volatile int* abort_flag) {
+    const uint32_t slot = use % R;
+    bool ok = true;
+    if (use >= R) {
+      const uint32_t par = (use / R - 1) & 1;
+      if (!mbar_try_wait(&bars->ring_empty[slot], par)) {
+        cp_async_wait<0>();
+        while (pub < use) publish_one(bars);
+        ok = mbar_wait(&bars->ring_empty[slot], par, abort_flag, kBudget);
+      }
+    }
+    ok = __all_sync(0xffffffffu, ok);
+    if (!ok) return false;
+    gather_tile(sm + kOffRing + slot * kTileBytes, base, rows_u, B, n, t, pw, lane);
+    ++use;
+    if (use - pub > LAG) {
+      cp_async_wait<LAG>();
+      publish_one(bars);
+    }
+    return true;
+  }
+  __device__ __forceinline__ void drain(MBars* bars, bool ok) {
+    cp_async_wait<0>();
+    if (ok)
+      while (pub < use) publish_one(bars);
+  }
+};
 
-__device__ __forceinline__ void init_common(MBars* bars, int warp) {
+__device__ __forceinline__ void init_common(MBars* bars, int warp, uint32_t ring_empty_count) {
   if (threadIdx.x == 0) {
-    for (int i = 0; i < kRing; ++i) {
+    for (int i = 0; i < 4; ++i) {
       mbar_init(&bars->ring_full[i], kProducers);
-      mbar_init(&bars->ring_empty[i], 1);
+      mbar_init(&bars->ring_empty[i], ring_empty_count);
     }
     mbar_init(&bars->q_full, 1);
     for (int i = 0; i < 2; ++i) {
@@ -154,10 +183,10 @@ __device__ __forceinline__ void init_common(MBars* bars, int warp) {
       mbar_init(&bars->s_done[i], 128);
       mbar_init(&bars->xg_full[i], 128);
       mbar_init(&bars->xg_empty[i], 1);
+      mbar_init(&bars->d_full[i], 1);
+      mbar_init(&bars->d_empty[i], 128);
     }
     mbar_init(&bars->acc_done, 1);
-    mbar_init(&bars->d_full, 1);
-    mbar_init(&bars->d_empty, 128);
     mbar_init(&bars->drain, 1);
     bars->abort = 0;
     fence_mbar_init();
@@ -168,9 +197,19 @@ __device__ __forceinline__ void init_common(MBars* bars, int warp) {
   }
 }
 
+// S = Q K0^T for one gathered tile into TMEM columns s_col (issued by one thread).
+__device__ __forceinline__ void issue_s(uint32_t s_tmem, uint32_t qa, uint32_t ka) {
+  const uint32_t id_s = idesc_bf16(kRows, kTile, 0, 0);
+#pragma unroll
+  for (int kk = 0; kk < kD / 16; ++kk) {
+    const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
+    mma_bf16(s_tmem, sw128_desc(qa + off, 16, 1024), sw128_desc(ka + off, 16, 1024), id_s, kk > 0);
+  }
+}
+
 __device__ __forceinline__ void store_row_chunk(uint8_t* tile, int row, int C, const uint32_t* w) {
-  // row `row`, tokens 32C..32C+31 of a K-major SW128 tile: token block C/2,
-  // 16-byte chunks (C&1)*4 .. +3
+  // row `row`, tokens 32C..32C+31 of a SW128 tile of 128-byte rows: token
+  // block C/2, 16-byte chunks (C&1)*4 .. +3
 #pragma unroll
   for (int qq = 0; qq < 4; ++qq)
     *(uint4*)(tile + (C >> 1) * (kTileBytes / 2) + sw128_offset(row, (C & 1) * 4 + qq)) =
@@ -219,8 +258,8 @@ __device__ __forceinline__ void gram_chunk_masked(const float* v, int p0, int vl
   if (want_g) store_row_chunk(xg, row, C, ghi);
 }
 
-// One 32-position chunk of an update tile: XGh and XGl (the MN-major B operands
-// of D = Z^T XG); positions from ng on are fixed and get zeros.
+// One 32-position chunk of an update tile: XGh and XGl rows (the MN-major A
+// operands of dV = XG^T Z); positions from ng on are fixed and get zeros.
 template <int C, bool kMasked>
 __device__ __forceinline__ void update_chunk(const float* v, int p0, int ng, float sl2, float lam,
                                              uint8_t* xh, uint8_t* xl, int row) {
@@ -334,20 +373,22 @@ __global__ void __launch_bounds__(256) k_merge_fixed(MArgs a) {
 }
 
 // ======================================================== k_merge_gram
-// Roles (384 threads): warp 0 the Q load, warp 1 MMA issue, warps 2-3 the
-// gathers, warps 4-7 and 8-11 two compute groups (one thread per window row /
-// TMEM lane) taking alternate tiles.  Job k < T: statistics of tile k;
-// T <= k < 2T: R~ and Gram of tile k - T.  S buffer k & 1.
+// Roles (384 threads): warp 0 the Q load, then the K_out stores and ring
+// releases; warp 1 MMA issue; warps 2-3 the gathers; warps 4-7 and 8-11 two
+// compute groups (one thread per window row / TMEM lane) taking alternate
+// jobs.  Job k < T: statistics of slot tile k; T <= k < 2T: R~ and Gram of
+// position tile k - T.  S buffer k & 1.  Ring loads: K of each pass-1 job,
+// then K and V of each pass-2 job.
 __global__ void __launch_bounds__(kThreads, 1)
-    k_merge_gram(const __grid_constant__ CUtensorMap tmQ, MArgs a) {
+    k_merge_gram(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKo,
+                 MArgs a) {
   extern __shared__ __align__(1024) uint8_t smraw[];
   uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
   MBars* bars = (MBars*)(sm + kOffBar);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int u = blockIdx.x, B = a.B, T = (B + kTile - 1) / kTile;
   const int ng = __ldg(a.ng + u);
-  const int32_t* src_u = a.src + (size_t)u * B;
-  init_common(bars, warp);
+  init_common(bars, warp, 2);   // ring slots are released by the MMA and by warp 0
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars->tmem;
@@ -356,25 +397,46 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       prefetch_tensormap(&tmQ);
+      prefetch_tensormap(&tmKo);
       mbar_expect_tx(&bars->q_full, kTileBytes);
       const uint64_t pol = l2_evict_last();
       tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, 0, u, pol);
       tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
+      // K_out = K0: the pass-1 tiles are the retained keys in slot order
+      bool ok = true;
+      for (int use = 0; use < 3 * T && ok; ++use) {
+        const int slot = use % kRingG;
+        ok = mbar_wait(&bars->ring_full[slot], (use / kRingG) & 1, abort_flag, kBudget);
+        if (!ok) break;
+        if (use < T) {
+          const uint8_t* tile = sm + kOffRing + slot * kTileBytes;
+          tma_store_3d(&tmKo, tile, 0, use * kTile, u);
+          tma_store_3d(&tmKo, tile + kTileBytes / 2, 64, use * kTile, u);
+          bulk_commit();
+          bulk_wait_read<0>();
+        }
+        mbar_arrive(&bars->ring_empty[slot]);
+      }
+      bulk_wait_all();
     }
   } else if (warp == 2 || warp == 3) {
     const __nv_bfloat16* kb = a.k + (size_t)u * a.n * kD;
     const __nv_bfloat16* vb = a.v + (size_t)u * a.n * kD;
-    uint32_t use = 0;
+    const int32_t* idx_u = a.idx + (size_t)u * B;
+    const int32_t* src_u = a.src + (size_t)u * B;
+    Producer<kRingG, 2> pr;
     bool ok = true;
     for (int k = 0; k < 2 * T && ok; ++k) {
-      const int t = k < T ? k : k - T;
-      ok = produce(bars, sm, kb, src_u, B, t, warp - 2, lane, use++, abort_flag);
-      if (ok && k >= T) ok = produce(bars, sm, vb, src_u, B, t, warp - 2, lane, use++, abort_flag);
+      if (k < T) {
+        ok = pr.load(bars, sm, kb, idx_u, B, a.n, k, warp - 2, lane, abort_flag);
+      } else {
+        ok = pr.load(bars, sm, kb, src_u, B, a.n, k - T, warp - 2, lane, abort_flag);
+        if (ok) ok = pr.load(bars, sm, vb, src_u, B, a.n, k - T, warp - 2, lane, abort_flag);
+      }
     }
-    produce_drain(bars, ok ? use : 0);
+    pr.drain(bars, ok);
   } else if (warp == 1) {
     if (lane == 0) {
-      const uint32_t id_s = idesc_bf16(kRows, kTile, 0, 0);
       const uint32_t id_r = idesc_bf16(kRows, kD, 0, 1);     // R~ += Xh V0 (V0 MN-major)
       const uint32_t id_g = idesc_bf16(kRows, kRows, 0, 0);  // G += A XGh^T
       bool ok = mbar_wait(&bars->q_full, 0, abort_flag, kBudget);
@@ -388,10 +450,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool w = mbar_wait(&bars->s_done[b], (kp >> 1) & 1, abort_flag, kBudget);
         if (w) w = mbar_wait(&bars->xg_full[xb], (t >> 1) & 1, abort_flag, kBudget);
         if (w)
-          w = mbar_wait(&bars->ring_full[vuse % kRing], (vuse / kRing) & 1, abort_flag, kBudget);
+          w = mbar_wait(&bars->ring_full[vuse % kRingG], (vuse / kRingG) & 1, abort_flag, kBudget);
         if (!w) return false;
         tc_fence_after();
-        const uint32_t va = smem_u32(sm + kOffRing + (vuse % kRing) * kTileBytes);
+        const uint32_t va = smem_u32(sm + kOffRing + (vuse % kRingG) * kTileBytes);
         const uint32_t xa = smem_u32(sm + kOffXG + xb * kTileBytes);
         const uint32_t hi = tmem + kColS + b * kTile, lo2 = hi + 64;
 #pragma unroll
@@ -412,25 +474,20 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           g_started = true;
         }
-        mma_commit(&bars->ring_empty[vuse % kRing]);
+        mma_commit(&bars->ring_empty[vuse % kRingG]);
         mma_commit(&bars->xg_empty[xb]);
         return true;
       };
       for (int k = 0; k < 2 * T && ok; ++k) {
         const int b = k & 1;
         const uint32_t kuse = use++;
-        ok = mbar_wait(&bars->ring_full[kuse % kRing], (kuse / kRing) & 1, abort_flag, kBudget);
+        ok = mbar_wait(&bars->ring_full[kuse % kRingG], (kuse / kRingG) & 1, abort_flag, kBudget);
         if (ok && k >= 2) ok = mbar_wait(&bars->s_done[b], ((k >> 1) - 1) & 1, abort_flag, kBudget);
         if (!ok) break;
         tc_fence_after();
-        const uint32_t ka = smem_u32(sm + kOffRing + (kuse % kRing) * kTileBytes);
-#pragma unroll
-        for (int kk = 0; kk < kD / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
-          mma_bf16(tmem + kColS + b * kTile, sw128_desc(qa + off, 16, 1024),
-                   sw128_desc(ka + off, 16, 1024), id_s, kk > 0);
-        }
-        mma_commit(&bars->ring_empty[kuse % kRing]);
+        issue_s(tmem + kColS + b * kTile, qa,
+                smem_u32(sm + kOffRing + (kuse % kRingG) * kTileBytes));
+        mma_commit(&bars->ring_empty[kuse % kRingG]);
         mma_commit(&bars->s_full[b]);
         uint32_t vuse = 0;
         if (k >= T) vuse = use++;
@@ -451,19 +508,21 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp >= 4) {
     const int wg = (warp - 4) >> 2, q = warp & 3, row = q * 32 + lane;
     const bool row_ok = row < a.m;
-    // positions past vlim are invisible to this row (and so are those >= B)
+    // slots / positions past vlim are invisible to this row (and so are those >= B)
     const int vlim = !row_ok ? -1 : (a.causal ? B - a.w + row % a.w : B - 1);
-    const int open = B - a.w;   // positions below this are visible to every window row
+    const int open = B - a.w;   // below this everything is visible to every window row
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
     float M = -INFINITY, L = 0.f, lam = INFINITY;
     bool ok = true;
     for (int k = 0; k < 2 * T; ++k) {
       if (k == T) {
-        // both groups combine their statistics (reached even after an abort)
-        float2* comb = (float2*)(sm + kOffStage);
+        // both groups combine their statistics (reached even after an abort);
+        // the XGh tiles are not in use yet
+        float2* comb = (float2*)(sm + kOffXG);
         comb[wg * kRows + row] = make_float2(M, L);
         named_bar(4, 256);
         const float2 o = comb[(wg ^ 1) * kRows + row];
+        named_bar(4, 256);
         if (o.x != -INFINITY) {
           if (o.x > M) {
             L = L * fast_exp2(M - o.x) + o.y;
@@ -836,46 +895,50 @@ __global__ void __launch_bounds__(256) k_merge_solve(MArgs a) {
 
 // ======================================================== k_merge_update
 // Roles (384 threads): warp 0 the Q load, warp 1 MMA issue, warps 2-3 the K0
-// gathers, warps 4-7 the XG tiles (one thread per window row), warps 8-11 the
-// output epilogue.  Only the tiles with non-fixed positions are visited.
+// gathers, warps 4-7 the XG rows (one thread per window row), warps 8-11 the
+// output epilogue (one thread per token / TMEM lane of D).  Only the tiles
+// with non-fixed positions are visited; the epilogue warps then copy V0 to
+// the fixed slots.
 __global__ void __launch_bounds__(kThreads, 1)
     k_merge_update(const __grid_constant__ CUtensorMap tmQ, MArgs a) {
   extern __shared__ __align__(1024) uint8_t smraw[];
   uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
   MBars* bars = (MBars*)(sm + kOffBar);
+  uint8_t* xh = sm + kOffXh;
+  uint8_t* xl = xh + kTileBytes;
+  uint8_t* zh = xl + kTileBytes;
+  uint8_t* zl = zh + kTileBytes;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int u = blockIdx.x, B = a.B;
   const int ng = __ldg(a.ng + u), T = (ng + kTile - 1) / kTile;
   const int32_t* src_u = a.src + (size_t)u * B;
   const int32_t* perm_u = a.perm + (size_t)u * B;
-  init_common(bars, warp);
+  init_common(bars, warp, 1);
+  // Z (fp32 [row][d]) to the bf16 B operands Zh, Zl: MN-major tiles of
+  // 128-byte rows (d contiguous), two blocks of 64 columns
+  {
+    const float* Z = a.rz + (size_t)u * kRows * kD;
+    for (int i = tid; i < kRows * (kD / 8); i += kThreads) {
+      const int r = i >> 4, d8 = i & 15;
+      const float4 z0 = __ldg((const float4*)(Z + r * kD + d8 * 8));
+      const float4 z1 = __ldg((const float4*)(Z + r * kD + d8 * 8 + 4));
+      const float zz[8] = {z0.x, z0.y, z0.z, z0.w, z1.x, z1.y, z1.z, z1.w};
+      uint32_t h[4], l[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        h[j] = pack_bf16(zz[2 * j], zz[2 * j + 1]);
+        l[j] = pack_bf16(zz[2 * j] - lo_half(h[j]), zz[2 * j + 1] - hi_half(h[j]));
+      }
+      const uint32_t off = (d8 >> 3) * (kTileBytes / 2) + sw128_offset(r, d8 & 7);
+      *(uint4*)(zh + off) = make_uint4(h[0], h[1], h[2], h[3]);
+      *(uint4*)(zl + off) = make_uint4(l[0], l[1], l[2], l[3]);
+    }
+    fence_proxy_async_smem();
+  }
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars->tmem;
   volatile int* abort_flag = &bars->abort;
-  // Z^T into TMEM as MMA operands: lane = column e of Z, packed row pairs
-  if (warp >= 4 && warp < 8) {
-    const int q = warp & 3, e = q * 32 + lane;
-    const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
-    const float* Z = a.rz + (size_t)u * kRows * kD;
-#pragma unroll 1
-    for (int rc = 0; rc < 4; ++rc) {
-      uint32_t zh[16], zl[16];
-#pragma unroll
-      for (int p = 0; p < 16; ++p) {
-        const float z0 = Z[(rc * 32 + 2 * p) * kD + e], z1 = Z[(rc * 32 + 2 * p + 1) * kD + e];
-        const uint32_t h = pack_bf16(z0, z1);
-        zh[p] = h;
-        zl[p] = pack_bf16(z0 - lo_half(h), z1 - hi_half(h));
-      }
-      tmem_st16(lane_addr + kColR + rc * 16, zh);
-      tmem_st16(lane_addr + kColR + 64 + rc * 16, zl);
-    }
-    tmem_st_wait();
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
 
   if (warp == 0) {
     if (lane == 0 && T > 0) {
@@ -887,53 +950,48 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 2 || warp == 3) {
     const __nv_bfloat16* kb = a.k + (size_t)u * a.n * kD;
-    uint32_t use = 0;
+    Producer<kRingU, 1> pr;
     bool ok = true;
     for (int t = 0; t < T && ok; ++t)
-      ok = produce(bars, sm, kb, src_u, B, t, warp - 2, lane, use++, abort_flag);
-    produce_drain(bars, ok ? use : 0);
+      ok = pr.load(bars, sm, kb, src_u, B, a.n, t, warp - 2, lane, abort_flag);
+    pr.drain(bars, ok);
   } else if (warp == 1) {
     if (lane == 0 && T > 0) {
-      const uint32_t id_s = idesc_bf16(kRows, kTile, 0, 0);
-      const uint32_t id_d = idesc_bf16(kD, kTile, 0, 1);   // D = Z^T XG (XG MN-major)
+      const uint32_t id_d = idesc_bf16(kTile, kD, 1, 1);   // dV = XG^T Z, both MN-major
       const uint32_t qa = smem_u32(sm + kOffQ);
+      const uint32_t ah = smem_u32(xh), al = smem_u32(xl), bh = smem_u32(zh), bl = smem_u32(zl);
       bool ok = mbar_wait(&bars->q_full, 0, abort_flag, kBudget);
       auto issue_d = [&](int t) -> bool {
+        const uint32_t d = tmem + kColD + (t & 1) * kD;
         bool w = mbar_wait(&bars->xg_full[0], t & 1, abort_flag, kBudget);
-        if (w && t >= 1) w = mbar_wait(&bars->d_empty, (t - 1) & 1, abort_flag, kBudget);
+        if (w && t >= 2) w = mbar_wait(&bars->d_empty[t & 1], ((t >> 1) - 1) & 1, abort_flag, kBudget);
         if (!w) return false;
         tc_fence_after();
-        const uint32_t xh = smem_u32(sm + kOffXG), xl = xh + kTileBytes;
 #pragma unroll
         for (int kk = 0; kk < kRows / 16; ++kk)
-          mma_bf16_ts(tmem + kColG, tmem + kColR + kk * 8,
-                      sw128_desc(xh + kk * 2048, kTileBytes / 2, 1024), id_d, kk > 0);
+          mma_bf16(d, sw128_desc(ah + kk * 2048, kTileBytes / 2, 1024),
+                   sw128_desc(bh + kk * 2048, kTileBytes / 2, 1024), id_d, kk > 0);
 #pragma unroll
         for (int kk = 0; kk < kRows / 16; ++kk)
-          mma_bf16_ts(tmem + kColG, tmem + kColR + 64 + kk * 8,
-                      sw128_desc(xh + kk * 2048, kTileBytes / 2, 1024), id_d, 1);
+          mma_bf16(d, sw128_desc(ah + kk * 2048, kTileBytes / 2, 1024),
+                   sw128_desc(bl + kk * 2048, kTileBytes / 2, 1024), id_d, 1);
 #pragma unroll
         for (int kk = 0; kk < kRows / 16; ++kk)
-          mma_bf16_ts(tmem + kColG, tmem + kColR + kk * 8,
-                      sw128_desc(xl + kk * 2048, kTileBytes / 2, 1024), id_d, 1);
+          mma_bf16(d, sw128_desc(al + kk * 2048, kTileBytes / 2, 1024),
+                   sw128_desc(bh + kk * 2048, kTileBytes / 2, 1024), id_d, 1);
         mma_commit(&bars->xg_empty[0]);
-        mma_commit(&bars->d_full);
+        mma_commit(&bars->d_full[t & 1]);
         return true;
       };
       for (int t = 0; t < T && ok; ++t) {
         const int b = t & 1;
-        ok = mbar_wait(&bars->ring_full[t % kRing], (t / kRing) & 1, abort_flag, kBudget);
+        ok = mbar_wait(&bars->ring_full[t % kRingU], (t / kRingU) & 1, abort_flag, kBudget);
         if (ok && t >= 2) ok = mbar_wait(&bars->s_done[b], ((t >> 1) - 1) & 1, abort_flag, kBudget);
         if (!ok) break;
         tc_fence_after();
-        const uint32_t ka = smem_u32(sm + kOffRing + (t % kRing) * kTileBytes);
-#pragma unroll
-        for (int kk = 0; kk < kD / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
-          mma_bf16(tmem + kColS + b * kTile, sw128_desc(qa + off, 16, 1024),
-                   sw128_desc(ka + off, 16, 1024), id_s, kk > 0);
-        }
-        mma_commit(&bars->ring_empty[t % kRing]);
+        issue_s(tmem + kColS + b * kTile, qa,
+                smem_u32(sm + kOffRing + (t % kRingU) * kTileBytes));
+        mma_commit(&bars->ring_empty[t % kRingU]);
         mma_commit(&bars->s_full[b]);
         if (t >= 1) ok = issue_d(t - 1);
       }
@@ -946,8 +1004,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     // rows past m have lam = +inf and give X = 0
     const float lam = a.lam[(size_t)u * kRows + row];
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
-    uint8_t* xh = sm + kOffXG;
-    uint8_t* xl = xh + kTileBytes;
     bool ok = true;
     for (int t = 0; t < T && ok; ++t) {
       const int b = t & 1, p0 = t * kTile;
@@ -990,78 +1046,61 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (!ok && row == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
   } else if (warp >= 8) {
-    // epilogue: D = dV^T, lane = column e of V, staged through shared memory;
-    // thread et then owns position tk of each 32-position block, columns c0..c0+31
-    const int q = warp & 3, e = q * 32 + lane, et = tid - 256;
-    const int tk = et & 31, c0 = (et >> 5) * 32;
+    // epilogue: thread = token (TMEM lane) of D = dV, 128 columns of d
+    const int q = warp & 3, tok = q * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
-    float* stage = (float*)(sm + kOffStage);
+    const uint4* v_u = (const uint4*)(a.v + (size_t)u * a.n * kD);
+    uint4* vo_u = (uint4*)(a.v_out + (size_t)u * B * kD);
     bool ok = true;
     for (int t = 0; t < T && ok; ++t) {
-      // V0 segments of this thread's positions, fetched before D is ready
-      uint4 v0[4][4];
+      const int p = t * kTile + tok;
+      const bool live = p < ng;
+      // V0 row of this position, fetched before D is ready
+      uint4 v0[16];
+      const uint4* g = v_u + (size_t)__ldg(src_u + min(p, B - 1)) * 16;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        const int srow = __ldg(src_u + min(t * kTile + c * 32 + tk, B - 1));
-        const uint4* gsrc = (const uint4*)(a.v + ((size_t)u * a.n + srow) * kD + c0);
-#pragma unroll
-        for (int h = 0; h < 4; ++h) v0[c][h] = __ldg(gsrc + h);
-      }
-      ok = mbar_wait(&bars->d_full, t & 1, abort_flag, kBudget);
+      for (int h = 0; h < 16; ++h) v0[h] = __ldg(g + h);
+      const int dst = live ? __ldg(perm_u + p) : 0;
+      ok = mbar_wait(&bars->d_full[t & 1], (t >> 1) & 1, abort_flag, kBudget);
       if (!ok) break;
       tc_fence_after();
+      const uint32_t dcol = lane_addr + kColD + (t & 1) * kD;
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         float v[32];
-        tmem_ld32f(lane_addr + kColG + c * 32, v);
+        tmem_ld32f(dcol + c * 32, v);
         tmem_wait32(v);
         if (c == 3) {
           tc_fence_before();
-          mbar_arrive(&bars->d_empty);
+          mbar_arrive(&bars->d_empty[t & 1]);
         }
-#pragma unroll
-        for (int k2 = 0; k2 < 32; ++k2) stage[k2 * kLD + e] = v[k2];
-        named_bar(3, 128);
-        const int p = t * kTile + c * 32 + tk;
-        if (p < ng) {
-          const size_t dst = ((size_t)u * B + __ldg(perm_u + p)) * kD + c0;
+        if (live) {
 #pragma unroll
           for (int h = 0; h < 4; ++h) {
-            const __nv_bfloat16* pv = (const __nv_bfloat16*)&v0[c][h];
+            const __nv_bfloat16* pv = (const __nv_bfloat16*)&v0[4 * c + h];
             uint32_t o[4];
 #pragma unroll
             for (int z = 0; z < 4; ++z)
-              o[z] = pack_bf16(__bfloat162float(pv[2 * z]) + stage[tk * kLD + c0 + 8 * h + 2 * z],
-                               __bfloat162float(pv[2 * z + 1]) +
-                                   stage[tk * kLD + c0 + 8 * h + 2 * z + 1]);
-            *(uint4*)(a.v_out + dst + 8 * h) = make_uint4(o[0], o[1], o[2], o[3]);
+              o[z] = pack_bf16(__bfloat162float(pv[2 * z]) + v[8 * h + 2 * z],
+                               __bfloat162float(pv[2 * z + 1]) + v[8 * h + 2 * z + 1]);
+            vo_u[(size_t)dst * 16 + 4 * c + h] = make_uint4(o[0], o[1], o[2], o[3]);
           }
         }
-        named_bar(3, 128);
       }
     }
-    if (!ok && e == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
+    if (!ok && tok == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
+    // V_out = V0 for the fixed slots (positions ng .. B-1)
+    for (int p = ng + tok; p < B; p += 128) {
+      const uint4* g = v_u + (size_t)__ldg(src_u + p) * 16;
+      uint4* o = vo_u + (size_t)__ldg(perm_u + p) * 16;
+#pragma unroll
+      for (int h = 0; h < 16; ++h) o[h] = __ldg(g + h);
+    }
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem, 512);
-}
-
-// K_out = K0 for every slot, V_out = V0 for the fixed slots (positions >= ng);
-// 16 threads per 256-byte row.
-__global__ void __launch_bounds__(256) k_merge_copy(MArgs a) {
-  const int u = blockIdx.y, i = blockIdx.x * 16 + (threadIdx.x >> 4), c = threadIdx.x & 15;
-  if (i >= a.B) return;
-  const size_t ub = (size_t)u * a.B;
-  const uint4* k = (const uint4*)a.k + (size_t)u * a.n * 16;
-  const uint4* v = (const uint4*)a.v + (size_t)u * a.n * 16;
-  const int j = __ldg(a.idx + ub + i);
-  ((uint4*)a.k_out)[(ub + i) * 16 + c] =
-      __ldg(k + (size_t)((unsigned)j < (unsigned)a.n ? j : 0) * 16 + c);
-  if (i >= __ldg(a.ng + u))
-    ((uint4*)a.v_out)[(ub + __ldg(a.perm + ub + i)) * 16 + c] =
-        __ldg(v + (size_t)__ldg(a.src + ub + i) * 16 + c);
 }
 
 }  // namespace
@@ -1079,8 +1118,10 @@ size_t merge_tc_ws_bytes(const Shape& s) {
 cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const void* v,
                             const float* scores, const float* y, const int32_t* idx, void* k_out,
                             void* v_out, char* ws, const WsLayout& L, cudaStream_t st) {
-  CUtensorMap mq;
-  if (!encode_bf16_3d(&mq, q, kD, s.m, s.U, 64, kRows)) return cudaErrorInvalidValue;
+  CUtensorMap mq, mko;
+  if (!encode_bf16_3d(&mq, q, kD, s.m, s.U, 64, kRows) ||
+      !encode_bf16_3d(&mko, k_out, kD, s.B, s.U, 64, kTile))
+    return cudaErrorInvalidValue;
   MArgs a{};
   a.U = s.U;
   a.n = s.n;
@@ -1099,7 +1140,6 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
   a.y = y;
   a.k = (const __nv_bfloat16*)k;
   a.v = (const __nv_bfloat16*)v;
-  a.k_out = (__nv_bfloat16*)k_out;
   a.v_out = (__nv_bfloat16*)v_out;
   const size_t U = (size_t)s.U;
   a.rz = (float*)(ws + L.merge_tc);
@@ -1120,11 +1160,10 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
                                 s.B * 4)) != cudaSuccess)
     return e;
   k_merge_fixed<<<s.U, 256, s.B * 4, st>>>(a);
-  k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, a);
+  k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mko, a);
   k_merge_solve<<<s.U, 256, kSolveSmem, st>>>(a);
   k_merge_update<<<s.U, kThreads, kSmemBytes, st>>>(mq, a);
-  k_merge_copy<<<dim3((s.B + 15) / 16, s.U), 256, 0, st>>>(a);
-  count_launches(5);
+  count_launches(4);
   return cudaGetLastError();
 }
 
