@@ -196,6 +196,12 @@ __device__ __forceinline__ int ld_acquire(const int* p) {
   return v;
 }
 
+// TMEM column of the packed bf16 P for tokens 16kk..16kk+15 of a tile: the
+// compute group that owns tokens 0..63 packs them into S columns 0..31, the
+// one that owns 64..127 into S columns 64..95 (each inside the S columns it
+// has already read).
+__device__ __forceinline__ uint32_t p_col(int kk) { return kk < 4 ? kk * 8 : 64 + (kk - 4) * 8; }
+
 struct Bars {
   uint64_t ring_full[kRing], ring_empty[kRing];
   uint64_t q_full[2], q_empty[2];
@@ -228,7 +234,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars->q_full[i], 1);
       mbar_init(&bars->q_empty[i], 1);
       mbar_init(&bars->s_full[i], 1);
-      mbar_init(&bars->s_done[i], 128);
+      mbar_init(&bars->s_done[i], 256);
       mbar_init(&bars->y_full[i], 1);
       mbar_init(&bars->y_empty[i], 128);
       mbar_init(&bars->astat_full[i], 256);
@@ -369,7 +375,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t va = smem_u32(sm + kOffRing + p_vslot * kTileBytes);
 #pragma unroll
             for (int kk = 0; kk < kTile / 16; ++kk)
-              mma_bf16_ts(tmem + kColY + yb * kD, tmem + kColS + pb * kTile + kk * 8,
+              mma_bf16_ts(tmem + kColY + yb * kD, tmem + kColS + pb * kTile + p_col(kk),
                           sw128_desc(va + kk * 2048, kTileBytes / 2, 1024), id_y,
                           (pj.seg_first && kk == 0) ? 0u : 1u);
             mma_commit(&bars->ring_empty[p_vslot]);
@@ -405,7 +411,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t va = smem_u32(sm + kOffRing + p_vslot * kTileBytes);
 #pragma unroll
           for (int kk = 0; kk < kTile / 16; ++kk)
-            mma_bf16_ts(tmem + kColY + yb * kD, tmem + kColS + pb * kTile + kk * 8,
+            mma_bf16_ts(tmem + kColY + yb * kD, tmem + kColS + pb * kTile + p_col(kk),
                         sw128_desc(va + kk * 2048, kTileBytes / 2, 1024), id_y,
                         (pj.seg_first && kk == 0) ? 0u : 1u);
           mma_commit(&bars->ring_empty[p_vslot]);
@@ -584,7 +590,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const float* lam_s = (const float*)(sm + kOffLam);
     JobIter it;
     it.init(&sc, a.n);
-    int i = 0, aseg = 0, bseg = 0, mine = 0;
+    int i = 0, aseg = 0, bseg = 0;
     bool ok = true;
     float M = -INFINITY, L = 0.f;     // pass-A running stats (log2 units)
     float lam = INFINITY;             // pass-B log2 normaliser of this row
@@ -604,43 +610,38 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_arrive(&bars->lam_empty[lb]);
           }
         }
-        if (b == wg) {
+        {
           ok = mbar_wait(&bars->s_full[b], (i >> 1) & 1, abort_flag, kWaitBudget);
           if (!ok) break;
           tc_fence_after();
+          // this group's half of the tile: tokens 64 wg .. 64 wg + 63
+          const int c0 = 2 * wg, t0 = j.j0 + 64 * wg;
           const uint32_t sbase = lane_addr + kColS + b * kTile;
-          // tiles away from the window and the end of the unit need no mask
-          const bool full = row_ok && j.j0 + kTile - 1 <= lim && j.j0 + kTile <= a.n;
+          // halves away from the window and the end of the unit need no mask
+          const bool full = row_ok && t0 + 63 <= lim && t0 + 64 <= a.n;
           float va[32], vb[32];
-          tmem_ld32f(sbase, va);
+          tmem_ld32f(sbase + c0 * 32, va);
           tmem_wait32(va);
+          tmem_ld32f(sbase + c0 * 32 + 32, vb);
           if (j.kind == 0) {
-            tmem_ld32f(sbase + 32, vb);
-            stats_chunk(va, full, j.j0, lim, a.n, row_ok, a.sl2, M, L);
-            tmem_wait32(vb);
-            tmem_ld32f(sbase + 64, va);
-            stats_chunk(vb, full, j.j0 + 32, lim, a.n, row_ok, a.sl2, M, L);
-            tmem_wait32(va);
-            tmem_ld32f(sbase + 96, vb);
-            stats_chunk(va, full, j.j0 + 64, lim, a.n, row_ok, a.sl2, M, L);
+            stats_chunk(va, full, t0, lim, a.n, row_ok, a.sl2, M, L);
             tmem_wait32(vb);
             tc_fence_before();
             mbar_arrive(&bars->s_done[b]);   // S fully read
-            stats_chunk(vb, full, j.j0 + 96, lim, a.n, row_ok, a.sl2, M, L);
+            stats_chunk(vb, full, t0 + 32, lim, a.n, row_ok, a.sl2, M, L);
           } else {
-            float* rb = red + ((wg * 2 + (mine & 1)) * 4) * kTile;
+            float* rb = red + ((wg * 2 + (i & 1)) * 4) * kTile;
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-              float* v = (c & 1) ? vb : va;
-              float* nx = (c & 1) ? va : vb;
-              if (c < 3) tmem_ld32f(sbase + (c + 1) * 32, nx);
+            for (int h = 0; h < 2; ++h) {
+              float* v = h ? vb : va;
+              if (h) tmem_wait32(vb);
               if (full) {
 #pragma unroll
                 for (int e = 0; e < 32; ++e) v[e] = fast_exp2(fmaf(v[e], a.sl2, -lam));
               } else {
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
-                  const int jj = j.j0 + c * 32 + e;
+                  const int jj = t0 + h * 32 + e;
                   v[e] = (jj > lim || jj >= a.n || !row_ok) ? 0.f
                                                             : fast_exp2(fmaf(v[e], a.sl2, -lam));
                 }
@@ -648,29 +649,30 @@ __global__ void __launch_bounds__(kThreads, 1)
               uint32_t pk[16];
 #pragma unroll
               for (int e = 0; e < 16; ++e) pk[e] = pack_bf16(v[2 * e], v[2 * e + 1]);
-              tmem_st16(sbase + c * 16, pk);
-              // transpose-reduce: lane t ends with the warp's sum for token 32c + t
+              // chunk c0 + h packs into the 16 columns at 64 wg + 16 h
+              tmem_st16(sbase + 64 * wg + 16 * h, pk);
+              // transpose-reduce: lane t ends with the warp's sum for token 32h + t
 #pragma unroll
-              for (int h = 16; h >= 1; h >>= 1) {
-                const bool up = (lane & h) != 0;
+              for (int hh = 16; hh >= 1; hh >>= 1) {
+                const bool up = (lane & hh) != 0;
 #pragma unroll
-                for (int e = 0; e < h; ++e) {
-                  const float send = up ? v[e] : v[e + h];
-                  const float keep = up ? v[e + h] : v[e];
-                  v[e] = keep + __shfl_xor_sync(0xffffffffu, send, h);
+                for (int e = 0; e < hh; ++e) {
+                  const float send = up ? v[e] : v[e + hh];
+                  const float keep = up ? v[e + hh] : v[e];
+                  v[e] = keep + __shfl_xor_sync(0xffffffffu, send, hh);
                 }
               }
-              rb[q * kTile + c * 32 + lane] = v[0];
-              if (c < 3) tmem_wait32(nx);
+              rb[q * 64 + h * 32 + lane] = v[0];
             }
             tmem_st_wait();
             tc_fence_before();
             mbar_arrive(&bars->s_done[b]);
             named_bar(bar_id, 128);
-            const int jj = q * 32 + lane;
-            const float cs = ((rb[jj] + rb[kTile + jj]) + rb[2 * kTile + jj]) + rb[3 * kTile + jj];
-            if (j.j0 + jj < a.P && jj < j.len) a.scores[(size_t)j.u * a.P + j.j0 + jj] = cs;
-            ++mine;
+            if (q < 2) {
+              const int jj = q * 32 + lane;
+              const float cs = ((rb[jj] + rb[64 + jj]) + rb[128 + jj]) + rb[192 + jj];
+              if (t0 + jj < a.P && 64 * wg + jj < j.len) a.scores[(size_t)j.u * a.P + t0 + jj] = cs;
+            }
           }
         }
         if (j.seg_last) {
