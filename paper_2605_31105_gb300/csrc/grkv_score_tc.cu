@@ -267,6 +267,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t slot = 0, ring_use = 0;   // ring_use counts loads
       int seg = 0, qissued = 0;
       bool ok = true;
+      bool pend_v = false;
+      int pv_j0 = 0, pv_u = 0;
+      auto load = [&](const CUtensorMap* map, int j0, int u, uint64_t pol) -> bool {
+        if (ring_use >= kRing &&
+            !mbar_wait(&bars->ring_empty[slot], ((ring_use / kRing) - 1) & 1, abort_flag,
+                       kWaitBudget))
+          return false;
+        uint8_t* dst = sm + kOffRing + slot * kTileBytes;
+        mbar_expect_tx(&bars->ring_full[slot], kTileBytes);
+        tma_load_3d(dst, map, &bars->ring_full[slot], 0, j0, u, pol);
+        tma_load_3d(dst + kTileBytes / 2, map, &bars->ring_full[slot], 64, j0, u, pol);
+        ++ring_use;
+        slot = (slot + 1) % kRing;
+        return true;
+      };
       while (ok && it.next_block()) {
         for (; ok && it.has_job(); it.advance()) {
           const Job j = it.job();
@@ -281,24 +296,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_3d(dq, &tmQ, &bars->q_full[qs], 0, 0, j.u, keep);
             tma_load_3d(dq + kTileBytes / 2, &tmQ, &bars->q_full[qs], 64, 0, j.u, keep);
           }
-          const int loads = j.kind == 1 ? 2 : 1;
-          for (int l = 0; l < loads && ok; ++l) {
-            if (ring_use >= kRing)
-              ok = mbar_wait(&bars->ring_empty[slot], ((ring_use / kRing) - 1) & 1, abort_flag,
-                             kWaitBudget);
-            if (!ok) break;
-            const CUtensorMap* map = l == 0 ? &tmK : &tmV;
-            const uint64_t pol = (l == 0 && j.kind == 0 && a.mode == 2) ? keep : stream;
-            uint8_t* dst = sm + kOffRing + slot * kTileBytes;
-            mbar_expect_tx(&bars->ring_full[slot], kTileBytes);
-            tma_load_3d(dst, map, &bars->ring_full[slot], 0, j.j0, j.u, pol);
-            tma_load_3d(dst + kTileBytes / 2, map, &bars->ring_full[slot], 64, j.j0, j.u, pol);
-            ++ring_use;
-            slot = (slot + 1) % kRing;
+          // the job's K, then the V of the previous pass-B job: V waits in the
+          // ring through a tile's compute, so it is fetched one tile later
+          ok = load(&tmK, j.j0, j.u, (j.kind == 0 && a.mode == 2) ? keep : stream);
+          if (ok && pend_v) {
+            ok = load(&tmV, pv_j0, pv_u, stream);
+            pend_v = false;
+          }
+          if (j.kind == 1) {
+            pend_v = true;
+            pv_j0 = j.j0;
+            pv_u = j.u;
           }
           if (j.seg_last) ++seg;
         }
       }
+      if (ok && pend_v) ok = load(&tmV, pv_j0, pv_u, stream);
       // let every issued load land before the CTA can exit
       for (uint32_t i = ring_use > kRing ? ring_use - kRing : 0; i < ring_use; ++i)
         mbar_wait(&bars->ring_full[i % kRing], (i / kRing) & 1, abort_flag, kWaitBudget);
@@ -352,15 +365,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_commit(&bars->q_empty[seg & 1]);
             ++seg;
           }
-          uint32_t vslot = 0, vuse = 0;
-          if (j.kind == 1) {
-            vslot = slot;
-            vuse = ring_use;
+          // Y MMA of the previous pass-B job (its P is ready once s_done fires);
+          // its V is the load after this job's K
+          if (pend) {
+            p_vslot = slot;
+            p_vuse = ring_use;
             ++ring_use;
             slot = (slot + 1) % kRing;
-          }
-          // Y MMA of the previous pass-B job (its P is ready once s_done fires)
-          if (pend) {
             const int pb = p_i & 1, puse = p_i >> 1;
             const int yb = p_yb;
             if (pj.seg_first && ybuf_uses[yb] >= 1)
@@ -389,8 +400,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             pend = true;
             pj = j;
             p_i = i;
-            p_vslot = vslot;
-            p_vuse = vuse;
             if (j.seg_first) p_yb = bseg & 1;
             if (j.seg_last) ++bseg;
           }
@@ -398,6 +407,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (ok && pend) {
+        p_vslot = slot;
+        p_vuse = ring_use;
         const int pb = p_i & 1, puse = p_i >> 1;
         const int yb = p_yb;
         if (pj.seg_first && ybuf_uses[yb] >= 1)
