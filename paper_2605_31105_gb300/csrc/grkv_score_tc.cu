@@ -11,17 +11,20 @@
 // GRKV_FUSED_SCORE).  By default the two passes run as two launches over all
 // units (modes 0 and 1), which reads K twice but needs no cross-CTA waits.
 //
-// Roles (384 threads): warp 0 issues TMA loads (Q per segment, K and V
-// tiles of 128 tokens through a 4-slot ring), warp 1 issues tcgen05 MMAs
-// (S = Q K^T into TMEM; Y += P V with P read from TMEM), warps 4-7 and 8-11
-// are two compute groups that take alternate tiles.  A compute thread owns
-// one window row (one TMEM lane): pass A keeps its running max / sum in
-// registers, pass B writes exp2(l - Lambda_r) back into TMEM as bf16 (the A
-// operand of the Y MMA) and sums probabilities over rows with a warp
-// transpose-reduction plus a 4-way shared-memory sum.  Per-unit statistics of
-// the CTAs that share a unit meet in a global slot array; pass B of round r
-// waits (bounded) on a per-round counter of finished pass-A blocks.  Y
-// partials of the CTAs sharing a unit are added with float4 atomics.
+// Roles (512 threads): warp 0 issues TMA loads (the unit's Q, then K and V
+// tiles of 128 tokens through a 5-slot ring; each V one job after its K, as
+// it stays in the ring through the tile's compute), warp 1 issues tcgen05
+// MMAs (S = Q K^T into TMEM; Y += P V with P read from TMEM), warps 4-7 and
+// 8-11 are two compute groups that share every tile, tokens 0..63 and
+// 64..127.  A compute thread owns one window row (one TMEM lane): pass A
+// keeps its running max / sum in registers, pass B writes exp2(l - Lambda_r)
+// back into TMEM as bf16 (the A operand of the Y MMA) and sums probabilities
+// over rows with a warp transpose-reduction plus a 4-way shared-memory sum.
+// Warp 2 publishes per-segment statistics (the unit's last writer combines
+// them), warp 3 fetches a unit's combined statistics ahead of its pass-B
+// segments, warps 12-15 add each segment's Y partial to the unit's Y with
+// float4 atomics.  Per-unit statistics of the CTAs that share a unit meet in
+// a global slot array; pass B of round r waits (bounded) for them.
 #include <algorithm>
 #include <cmath>
 
@@ -36,14 +39,15 @@ using namespace sm100;
 
 constexpr int kTile = 128;            // tokens per tile
 constexpr int kRows = 128;            // window rows (m padded to 128)
-constexpr int kRing = 4;              // K / V ring slots
+constexpr int kRing = 5;              // K / V ring slots
+constexpr int kQBuf = 1;              // Q buffers (one per unit segment in flight)
 constexpr int kThreads = 512;
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KB
 constexpr long long kWaitBudget = 1ll << 32;      // cycles (~2 s) before a wait gives up
 
 // Shared-memory layout (offsets from a 1024-byte aligned base).
-constexpr uint32_t kOffQ = 0;                                   // 2 x 32 KB
-constexpr uint32_t kOffRing = kOffQ + 2 * kTileBytes;           // 4 x 32 KB
+constexpr uint32_t kOffQ = 0;                                   // kQBuf x 32 KB
+constexpr uint32_t kOffRing = kOffQ + kQBuf * kTileBytes;       // kRing x 32 KB
 constexpr uint32_t kOffRed = kOffRing + kRing * kTileBytes;     // [2 wg][2 buf][4][128] fp32
 constexpr uint32_t kOffAstat = kOffRed + 2 * 2 * 4 * kTile * 4;   // [2 buf][2 wg][128] float2
 constexpr uint32_t kOffLam = kOffAstat + 2 * 2 * kRows * 8;       // [2 buf][128] float
@@ -204,7 +208,7 @@ __device__ __forceinline__ uint32_t p_col(int kk) { return kk < 4 ? kk * 8 : 64 
 
 struct Bars {
   uint64_t ring_full[kRing], ring_empty[kRing];
-  uint64_t q_full[2], q_empty[2];
+  uint64_t q_full[kQBuf], q_empty[kQBuf];
   uint64_t s_full[2], s_done[2];
   uint64_t y_full[2], y_empty[2];
   uint64_t astat_full[2], astat_empty[2];   // compute groups -> statistics publisher
@@ -213,6 +217,7 @@ struct Bars {
   uint32_t tmem;
   int abort;
 };
+static_assert(sizeof(Bars) <= 256, "barrier block");
 
 __global__ void __launch_bounds__(kThreads, 1)
     k_score_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -226,13 +231,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   Sched sc{a.U, a.tpu, (int)gridDim.x, (int)blockIdx.x, a.mode, a.gu, a.rounds};
 
   if (tid == 0) {
+    for (int i = 0; i < kQBuf; ++i) {
+      mbar_init(&bars->q_full[i], 1);
+      mbar_init(&bars->q_empty[i], 1);
+    }
     for (int i = 0; i < kRing; ++i) {
       mbar_init(&bars->ring_full[i], 1);
       mbar_init(&bars->ring_empty[i], 1);
     }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&bars->q_full[i], 1);
-      mbar_init(&bars->q_empty[i], 1);
       mbar_init(&bars->s_full[i], 1);
       mbar_init(&bars->s_done[i], 256);
       mbar_init(&bars->y_full[i], 1);
@@ -286,8 +293,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (; ok && it.has_job(); it.advance()) {
           const Job j = it.job();
           if (j.seg_first) {
-            const int qs = seg & 1;
-            if (seg >= 2) ok = mbar_wait(&bars->q_empty[qs], ((seg >> 1) - 1) & 1, abort_flag,
+            const int qs = seg % kQBuf;
+            if (seg >= kQBuf) ok = mbar_wait(&bars->q_empty[qs], (seg / kQBuf - 1) & 1, abort_flag,
                                          kWaitBudget);
             if (!ok) break;
             ++qissued;
@@ -316,8 +323,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (uint32_t i = ring_use > kRing ? ring_use - kRing : 0; i < ring_use; ++i)
         mbar_wait(&bars->ring_full[i % kRing], (i / kRing) & 1, abort_flag, kWaitBudget);
       const int qloads = qissued;
-      for (int i = qloads > 2 ? qloads - 2 : 0; i < qloads; ++i)
-        mbar_wait(&bars->q_full[i & 1], (i >> 1) & 1, abort_flag, kWaitBudget);
+      for (int i = qloads > kQBuf ? qloads - kQBuf : 0; i < qloads; ++i)
+        mbar_wait(&bars->q_full[i % kQBuf], (i / kQBuf) & 1, abort_flag, kWaitBudget);
     }
   } else if (warp == 1) {
     // ----------------------------------------------------------- MMA issuer
@@ -340,7 +347,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const Job j = it.job();
           const int b = i & 1, use = i >> 1;
           if (j.seg_first) {
-            ok = mbar_wait(&bars->q_full[seg & 1], (seg >> 1) & 1, abort_flag, kWaitBudget);
+            ok = mbar_wait(&bars->q_full[seg % kQBuf], (seg / kQBuf) & 1, abort_flag, kWaitBudget);
             if (!ok) break;
           }
           const uint32_t kslot = slot, kuse = ring_use;
@@ -349,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ok = mbar_wait(&bars->s_done[b], (use - 1) & 1, abort_flag, kWaitBudget);
           if (!ok) break;
           tc_fence_after();
-          const uint32_t qa = smem_u32(sm + kOffQ + (seg & 1) * kTileBytes);
+          const uint32_t qa = smem_u32(sm + kOffQ + (seg % kQBuf) * kTileBytes);
           const uint32_t ka = smem_u32(sm + kOffRing + kslot * kTileBytes);
 #pragma unroll
           for (int kk = 0; kk < kD / 16; ++kk) {
@@ -362,7 +369,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++ring_use;
           slot = (slot + 1) % kRing;
           if (j.seg_last) {
-            mma_commit(&bars->q_empty[seg & 1]);
+            mma_commit(&bars->q_empty[seg % kQBuf]);
             ++seg;
           }
           // Y MMA of the previous pass-B job (its P is ready once s_done fires);
