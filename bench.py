@@ -14,6 +14,7 @@ collective on the data path); rank 0 prints one JSON line.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import math
 import multiprocessing as mp
@@ -69,6 +70,26 @@ def algorithmic_bytes(wl):
     read = 2 * wl.units * wl.n * wl.d * el
     write = 2 * wl.units * wl.budget * wl.d * el
     return read, write
+
+
+# DRAM bytes (read + write) of one grkv_score call, i.e. both k_score_tc launches, from
+# one ncu capture of the full workload (profiles/score_tc_c2_llama_32k.md).  A figure
+# holds only for the kernel source it was taken on, so it is keyed by that file's digest
+# and reported as null once the kernel changes.
+SCORE_TRAFFIC = {
+    "c2_llama_32k_bf16": ("f42aada0f6d0e6e1527fd8437e5aeb097e7d7b76bbc9f498364046f4503822bb",
+                          6501078272),
+}
+
+
+def score_traffic(wl):
+    rec = SCORE_TRAFFIC.get(wl.name)
+    if rec is None:
+        return None
+    src = os.path.join(ROOT, "paper_2605_31105_gb300", "csrc", "grkv_score_tc.cu")
+    with open(src, "rb") as f:
+        digest = hashlib.sha256(f.read()).hexdigest()
+    return rec[1] if digest == rec[0] else None
 
 
 def measured_peaks():
@@ -401,7 +422,8 @@ def run_ours(a):
         "path": a.path,
         "roofline": {"bound": "hbm", "kernel": "grkv_score stage (window scoring + target)",
                      "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "peak_kind": peak_kind, "traffic": None,
+                     "frac": achieved / peak, "peak_kind": peak_kind,
+                     "traffic": score_traffic(wl) if a.path == "default" else None,
                      "algorithmic_bytes_per_launch": score_bytes, "launch_ms": score_ms},
         "path_hbm": {"gbs": path_gbs, "frac_of_measured": path_gbs / peak,
                      "frac_of_8tbs": path_gbs / NOMINAL_HBM_GBS,
