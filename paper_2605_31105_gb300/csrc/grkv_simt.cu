@@ -263,6 +263,162 @@ __global__ void __launch_bounds__(1024) k_select(const float* __restrict__ score
   for (int a = tid; a < s.w; a += blockDim.x) out[s.kk + a] = P + a;
 }
 
+// Selection with the unit's keys resident in shared memory (n - w <= 32768):
+// one 1024-thread CTA per unit.  The scores are staged once, pooled into
+// order-preserving keys (thread t owns positions t + 1024 e, the keys stay in
+// its registers), the (B - w)-th largest key is found by four 8-bit radix
+// passes over per-warp histograms, and the positions are compacted in order
+// from contiguous segments.  Same result as k_select.  Shared-memory words are
+// padded by one per 32 (index j + j / 32) so both the strided and the
+// segmented accesses are free of bank conflicts.
+constexpr int kSelThreads = 1024, kSelPer = 32, kSelMaxP = kSelThreads * kSelPer;
+
+__host__ __device__ __forceinline__ int sel_pad(int j) { return j + (j >> 5); }
+
+size_t select_smem_bytes(int P) {
+  return ((size_t)sel_pad(P) + 4) * 4 + (size_t)32 * 256 * 4;
+}
+
+__global__ void __launch_bounds__(kSelThreads, 1) k_select_smem(const float* __restrict__ scores,
+                                                                Shape s,
+                                                                int32_t* __restrict__ idx) {
+  extern __shared__ uint32_t skey[];   // [sel_pad(P)] scores, then keys
+  __shared__ int hist[256];
+  __shared__ int sh[48];
+  const int u = blockIdx.x, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int P = s.P, h = s.pool_k / 2;
+  int* whist = (int*)(skey + ((sel_pad(P) + 4) & ~3));   // [32][256]
+  const float* c = scores + (size_t)u * P;
+  int32_t* out = idx + (size_t)u * s.B;
+#pragma unroll 8
+  for (int e = 0; e < kSelPer; ++e) {
+    const int j = tid + e * kSelThreads;
+    if (j < P) skey[sel_pad(j)] = __float_as_uint(__ldg(c + j));
+  }
+  __syncthreads();
+  auto cs = [&](int j) { return __uint_as_float(skey[sel_pad(j)]); };
+  uint32_t kr[kSelPer];
+#pragma unroll
+  for (int e = 0; e < kSelPer; ++e) {
+    const int j = tid + e * kSelThreads;
+    kr[e] = 0u;
+    if (j < P) {
+      float pv;
+      if (s.pool_type == GRKV_POOL_MAX) {
+        pv = cs(j);
+        for (int t = 1; t <= h; ++t) {
+          if (j - t >= 0) pv = fmaxf(pv, cs(j - t));
+          if (j + t < P) pv = fmaxf(pv, cs(j + t));
+        }
+      } else {
+        double acc = 0.0;   // left to right, zero padding, divisor k
+        for (int t = -h; t <= h; ++t)
+          if (j + t >= 0 && j + t < P) acc += (double)cs(j + t);
+        pv = (float)(acc / (double)s.pool_k);
+      }
+      kr[e] = order_key(pv);
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int e = 0; e < kSelPer; ++e) {
+    const int j = tid + e * kSelThreads;
+    if (j < P) skey[sel_pad(j)] = kr[e];
+  }
+  __syncthreads();
+  if (s.kk >= P) {
+    for (int j = tid; j < P; j += kSelThreads) out[j] = j;
+  } else if (s.kk > 0) {
+    // (kk)-th largest key: four 8-bit digits, most significant first
+    uint32_t prefix = 0, mask = 0;
+    int rem = s.kk;
+    for (int shift = 24; shift >= 0; shift -= 8) {
+      for (int i = tid; i < 32 * 256; i += kSelThreads) whist[i] = 0;
+      __syncthreads();
+#pragma unroll
+      for (int e = 0; e < kSelPer; ++e) {
+        const int j = tid + e * kSelThreads;
+        if (j < P && (kr[e] & mask) == prefix)
+          atomicAdd(&whist[warp * 256 + ((kr[e] >> shift) & 255u)], 1);
+      }
+      __syncthreads();
+      if (tid < 256) {
+        int a = 0;
+#pragma unroll 8
+        for (int w = 0; w < 32; ++w) a += whist[w * 256 + tid];
+        hist[tid] = a;
+      }
+      __syncthreads();
+      if (warp == 0) {
+        // digit search from 255 down: lane l owns bins 8l..8l+7
+        int cnt[8], own = 0;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          cnt[q] = hist[8 * lane + q];
+          own += cnt[q];
+        }
+        int suf = own;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_down_sync(0xffffffffu, suf, o);
+          if (lane + o < 32) suf += y;
+        }
+        int above = suf - own, dg = -1, left = 0;
+#pragma unroll
+        for (int q = 7; q >= 0; --q) {
+          if (dg < 0 && (above + cnt[q] >= rem || (lane == 0 && q == 0))) {
+            dg = 8 * lane + q;
+            left = rem - above;
+          }
+          above += cnt[q];
+        }
+        const unsigned found = __ballot_sync(0xffffffffu, dg >= 0);
+        const int srcl = 31 - __clz(found);
+        const int dsel = __shfl_sync(0xffffffffu, dg, srcl), lsel = __shfl_sync(0xffffffffu, left, srcl);
+        if (lane == 0) {
+          sh[0] = dsel;
+          sh[1] = lsel;
+        }
+      }
+      __syncthreads();
+      prefix |= (uint32_t)sh[0] << shift;
+      mask |= 255u << shift;
+      rem = sh[1];
+      __syncthreads();
+    }
+    const uint32_t tau = prefix;
+    const int need_eq = rem;
+    // compaction in position order: thread t owns positions 32t .. 32t+31
+    const int lo = min(P, tid * kSelPer), hi = min(P, lo + kSelPer);
+    int eq = 0;
+    for (int i = lo; i < hi; ++i) eq += skey[sel_pad(i)] == tau;
+    int tot;
+    const int er0 = block_exclusive_scan(eq, sh + 8, &tot);
+    int sel = 0, er = er0;
+    for (int i = lo; i < hi; ++i) {
+      const uint32_t key = skey[sel_pad(i)];
+      if (key > tau) {
+        ++sel;
+      } else if (key == tau) {
+        if (er < need_eq) ++sel;
+        ++er;
+      }
+    }
+    int pos = block_exclusive_scan(sel, sh + 8, &tot);
+    er = er0;
+    for (int i = lo; i < hi; ++i) {
+      const uint32_t key = skey[sel_pad(i)];
+      if (key > tau) {
+        out[pos++] = i;
+      } else if (key == tau) {
+        if (er < need_eq) out[pos++] = i;
+        ++er;
+      }
+    }
+  }
+  for (int a = tid; a < s.w; a += kSelThreads) out[s.kk + a] = P + a;
+}
+
 // ------------------------------------------------------------------ merge --
 // One CTA per unit.  A is the accumulation type of the regression (double for
 // fp32 inputs, float for bf16).
@@ -560,18 +716,24 @@ cudaError_t launch_score_simt(const Shape& s, const void* q, const void* k, cons
                                    (const __nv_bfloat16*)v, scores, y, row_stats, ws, L, st);
 }
 
-cudaError_t launch_select(const Shape& s, const float* scores, int32_t* idx, char* ws,
-                          const WsLayout& L, cudaStream_t st) {
-  k_select<<<s.U, 1024, 0, st>>>(scores, s, (float*)(ws + L.pooled), idx);
+cudaError_t launch_select_pooled(const Shape& s, const float* scores, int32_t* idx,
+                                 float* pooled, cudaStream_t st) {
+  if (s.P <= kSelMaxP) {
+    const size_t bytes = select_smem_bytes(s.P);
+    cudaError_t e =
+        cudaFuncSetAttribute(k_select_smem, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (e != cudaSuccess) return e;
+    k_select_smem<<<s.U, kSelThreads, bytes, st>>>(scores, s, idx);
+  } else {
+    k_select<<<s.U, 1024, 0, st>>>(scores, s, pooled, idx);
+  }
   count_launches(1);
   return cudaGetLastError();
 }
 
-cudaError_t launch_select_pooled(const Shape& s, const float* scores, int32_t* idx,
-                                 float* pooled, cudaStream_t st) {
-  k_select<<<s.U, 1024, 0, st>>>(scores, s, pooled, idx);
-  count_launches(1);
-  return cudaGetLastError();
+cudaError_t launch_select(const Shape& s, const float* scores, int32_t* idx, char* ws,
+                          const WsLayout& L, cudaStream_t st) {
+  return launch_select_pooled(s, scores, idx, (float*)(ws + L.pooled), st);
 }
 
 cudaError_t launch_merge_simt(const Shape& s, const void* q, const void* k, const void* v,

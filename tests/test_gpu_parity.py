@@ -154,6 +154,21 @@ def test_select_ties_take_smaller_positions(grkv_lib):
             np.testing.assert_array_equal(idx[i], O.select(O.pool(s[i], op), op))
 
 
+@pytest.mark.parametrize("n", [32768, 32800, 40032])
+@pytest.mark.parametrize("pool", ["max", "avg"])
+def test_select_long_prefixes(grkv_lib, n, pool):
+    """n - w = 32736 and 32768 take the shared-memory selection kernel, 40000
+    the global-memory one; coarse score levels make many ties at the cut."""
+    wl = gi.Workload(f"select_n{n}", 2, 4, n, 128, 32, 2048, 7, 1e-2, "bf16", "lowrank", 4242)
+    p = G.lib_params(wl, 2, pool_type=pool)
+    op = G.oracle_params(wl, pool_type=pool)
+    rng = np.random.default_rng(n)
+    s = rng.integers(0, 64, size=(2, n - 32)).astype(np.float32) / 64.0
+    idx = G.run_select(p, s)
+    for i in range(2):
+        np.testing.assert_array_equal(idx[i], O.select(O.pool(s[i], op), op))
+
+
 def test_zero_units_is_a_no_op(grkv_lib):
     import torch
     p = b.params(0, 4, 1024, 32, 128)
