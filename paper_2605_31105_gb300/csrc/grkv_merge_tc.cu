@@ -59,8 +59,8 @@ constexpr uint32_t kOffBar = 7 * kTileBytes;
 static_assert(kOffXG + 2 * kTileBytes == kOffBar && kOffXh + 4 * kTileBytes == kOffBar,
               "shared-memory layouts");
 constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;
-// k_merge_solve: N and R/Z [128][129] fp32, 1 / L_jj, the failure flag
-constexpr uint32_t kSolveSmem = (2 * kRows * kLD + kRows + 32) * 4;
+// k_merge_solve: packed N (tri(128) + 4 floats), R/Z [128][129] fp32, 1 / L_jj, the failure flag
+constexpr uint32_t kSolveSmem = ((128 * 129) / 2 + 4 + kRows * kLD + kRows + 32) * 4;
 
 // TMEM columns.  gram: S[2] 0..255, R~ 256..383, Gram 384..511.
 // update: S[2] 0..255, D[2] 256..511.
@@ -663,23 +663,27 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ======================================================== k_merge_solve
-// The register-resident pieces of the blocked Cholesky and the triangular
-// solves are separate (non-inlined) functions so that their 32-element arrays
-// stay in registers.
+// N lives in shared memory as a packed lower triangle (row i at tri(i)), so
+// two CTAs fit on an SM.  The register-resident pieces of the blocked
+// Cholesky and of the triangular solves are separate (non-inlined) functions
+// so that their 32-element arrays stay in registers.
+__host__ __device__ constexpr int tri(int i) { return (i * (i + 1)) >> 1; }
+constexpr int kTri = tri(kRows) + 4;   // packed N, padded to 16 bytes
 
 // Factors the 32 x 32 diagonal block at k0 (right-looking; lane l holds row
 // k0 + l) and stores 1 / L_jj.  Returns true on a non-positive pivot.
 __device__ __noinline__ bool chol_diag(float* N, float* dinv, int k0, int lane) {
+  const int rb = tri(k0 + lane) + k0;
   float x[32];
 #pragma unroll
-  for (int j = 0; j < 32; ++j) x[j] = j <= lane ? N[(k0 + lane) * kLD + k0 + j] : 0.f;
+  for (int j = 0; j < 32; ++j) x[j] = j <= lane ? N[rb + j] : 0.f;
   bool bad = false;
 #pragma unroll
   for (int k = 0; k < 32; ++k) {
     const float dkk = __shfl_sync(0xffffffffu, x[k], k);
     bad |= !(dkk > 0.f);
-    const float piv = sqrtf(fmaxf(dkk, 0.f));
-    const float inv = piv > 0.f ? 1.f / piv : 0.f;
+    const float inv = dkk > 0.f ? rsqrtf(dkk) : 0.f;   // 1 / L_kk
+    const float piv = dkk * inv;                         // L_kk
     x[k] = lane == k ? piv : (lane > k ? x[k] * inv : x[k]);
     const float lk = x[k];
 #pragma unroll
@@ -691,27 +695,29 @@ __device__ __noinline__ bool chol_diag(float* N, float* dinv, int k0, int lane) 
   }
 #pragma unroll
   for (int j = 0; j < 32; ++j)
-    if (j <= lane) N[(k0 + lane) * kLD + k0 + j] = x[j];
+    if (j <= lane) N[rb + j] = x[j];
   return bad;
 }
 
 // Row i of the panel below the diagonal block at k0: L_i,k0.. = A_i,k0.. L_kk^-T.
 __device__ __noinline__ void chol_panel_row(float* N, const float* dinv, int k0, int i) {
+  const int rb = tri(i) + k0;
   float x[32];
 #pragma unroll
-  for (int j = 0; j < 32; ++j) x[j] = N[i * kLD + k0 + j];
+  for (int j = 0; j < 32; ++j) x[j] = N[rb + j];
 #pragma unroll
   for (int j = 0; j < 32; ++j) {
+    const float* lj = N + tri(k0 + j) + k0;
     float s0 = x[j], s1 = 0.f;
 #pragma unroll
     for (int p = 0; p < j; ++p) {
-      if (p & 1) s1 += x[p] * N[(k0 + j) * kLD + k0 + p];
-      else s0 -= x[p] * N[(k0 + j) * kLD + k0 + p];
+      if (p & 1) s1 += x[p] * lj[p];
+      else s0 -= x[p] * lj[p];
     }
     x[j] = (s0 - s1) * dinv[k0 + j];
   }
 #pragma unroll
-  for (int j = 0; j < 32; ++j) N[i * kLD + k0 + j] = x[j];
+  for (int j = 0; j < 32; ++j) N[rb + j] = x[j];
 }
 
 // Column e of rows i0..i0+31: W = L_bb^-1 W (forward) or L_bb^-T W (backward).
@@ -721,11 +727,12 @@ __device__ __noinline__ void trsv_fwd(const float* N, float* R, const float* din
   for (int i = 0; i < 32; ++i) z[i] = R[(i0 + i) * kLD + e];
 #pragma unroll
   for (int i = 0; i < 32; ++i) {
+    const float* li = N + tri(i0 + i) + i0;
     float s0 = z[i], s1 = 0.f;
 #pragma unroll
     for (int kx = 0; kx < i; ++kx) {
-      if (kx & 1) s1 += N[(i0 + i) * kLD + i0 + kx] * z[kx];
-      else s0 -= N[(i0 + i) * kLD + i0 + kx] * z[kx];
+      if (kx & 1) s1 += li[kx] * z[kx];
+      else s0 -= li[kx] * z[kx];
     }
     z[i] = (s0 - s1) * dinv[i0 + i];
   }
@@ -741,8 +748,9 @@ __device__ __noinline__ void trsv_bwd(const float* N, float* R, const float* din
     float s0 = z[i], s1 = 0.f;
 #pragma unroll
     for (int kx = i + 1; kx < 32; ++kx) {
-      if (kx & 1) s1 += N[(i0 + kx) * kLD + i0 + i] * z[kx];
-      else s0 -= N[(i0 + kx) * kLD + i0 + i] * z[kx];
+      const float l = N[tri(i0 + kx) + i0 + i];
+      if (kx & 1) s1 += l * z[kx];
+      else s0 -= l * z[kx];
     }
     z[i] = (s0 - s1) * dinv[i0 + i];
   }
@@ -754,10 +762,10 @@ __device__ __noinline__ void trsv_bwd(const float* N, float* R, const float* din
 // Cholesky N = L L^T in 32-row blocks, then Z = L^-T L^-1 R; fp32 in shared
 // memory.  A non-positive pivot reports GRKV_ERR_NUMERIC and leaves Z = 0
 // (values stay V0); lambda = +inf also gives Z = 0.
-__global__ void __launch_bounds__(256) k_merge_solve(MArgs a) {
+__global__ void __launch_bounds__(256, 2) k_merge_solve(MArgs a) {
   extern __shared__ __align__(16) float ssm[];
-  float* N = ssm;                   // [128][kLD]
-  float* R = N + kRows * kLD;       // [128][kLD]
+  float* N = ssm;                   // packed lower triangle
+  float* R = N + kTri;              // [128][kLD]: G first, then R, then Z
   float* dinv = R + kRows * kLD;    // [128]
   int* fail = (int*)(dinv + kRows);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, nt = blockDim.x;
@@ -769,26 +777,29 @@ __global__ void __launch_bounds__(256) k_merge_solve(MArgs a) {
     return;
   }
   if (tid == 0) *fail = 0;
+  // G into the R buffer, then its symmetric part into the packed triangle
 #pragma unroll 4
   for (int p = tid; p < kRows * kRows / 4; p += nt) {
-    const float4 g = __ldg(G4 + p), r = __ldg((const float4*)RZ + p);
-    float* n = N + (p >> 5) * kLD + (p & 31) * 4;
-    float* rr = R + (p >> 5) * kLD + (p & 31) * 4;
-    n[0] = g.x; n[1] = g.y; n[2] = g.z; n[3] = g.w;
-    rr[0] = r.x; rr[1] = r.y; rr[2] = r.z; rr[3] = r.w;
+    const float4 g = __ldg(G4 + p);
+    float* r = R + (p >> 5) * kLD + (p & 31) * 4;
+    r[0] = g.x; r[1] = g.y; r[2] = g.z; r[3] = g.w;
   }
   __syncthreads();
-  // symmetrise into the lower triangle (reads only the untouched upper one)
-  for (int p = tid; p < kRows * kRows; p += nt) {
-    const int i = p >> 7, j = p & 127;
-    if (j > i) continue;
-    float val;
-    if (i >= m || j >= m) val = (i == j) ? 1.f : 0.f;
-    else if (i == j) val = N[i * kLD + i] + a.lambda;
-    else val = 0.5f * (N[i * kLD + j] + N[j * kLD + i]);
-    N[i * kLD + j] = val;
-  }
+  for (int i = warp; i < kRows; i += nt / 32)
+    for (int j = lane; j <= i; j += 32) {
+      float val;
+      if (i >= m || j >= m) val = (i == j) ? 1.f : 0.f;
+      else if (i == j) val = R[i * kLD + i] + a.lambda;
+      else val = 0.5f * (R[i * kLD + j] + R[j * kLD + i]);
+      N[tri(i) + j] = val;
+    }
   __syncthreads();
+#pragma unroll 4
+  for (int p = tid; p < kRows * kD / 4; p += nt) {
+    const float4 r4 = __ldg((const float4*)RZ + p);
+    float* r = R + (p >> 5) * kLD + (p & 31) * 4;
+    r[0] = r4.x; r[1] = r4.y; r[2] = r4.z; r[3] = r4.w;
+  }
   for (int kb = 0; kb < kRows / 32; ++kb) {
     const int k0 = kb * 32;
     if (warp == 0 && chol_diag(N, dinv, k0, lane) && lane == 0) *fail = 1;
@@ -803,24 +814,31 @@ __global__ void __launch_bounds__(256) k_merge_solve(MArgs a) {
       while (bi * (bi + 1) / 2 > t) --bi;
       const int i = k1 + 4 * bi, j = k1 + 4 * (t - bi * (bi + 1) / 2);
       float acc[4][4] = {};
+      const float* li[4];
+      const float* lj[4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        li[r] = N + tri(i + r) + k0;
+        lj[r] = N + tri(j + r) + k0;
+      }
 #pragma unroll 4
       for (int pp = 0; pp < 32; ++pp) {
-        float li[4], lj[4];
+        float vi[4], vj[4];
 #pragma unroll
         for (int r = 0; r < 4; ++r) {
-          li[r] = N[(i + r) * kLD + k0 + pp];
-          lj[r] = N[(j + r) * kLD + k0 + pp];
+          vi[r] = li[r][pp];
+          vj[r] = lj[r][pp];
         }
 #pragma unroll
         for (int r = 0; r < 4; ++r)
 #pragma unroll
-          for (int c = 0; c < 4; ++c) acc[r][c] += li[r] * lj[c];
+          for (int c = 0; c < 4; ++c) acc[r][c] += vi[r] * vj[c];
       }
 #pragma unroll
       for (int r = 0; r < 4; ++r)
 #pragma unroll
         for (int c = 0; c < 4; ++c)
-          if (j + c <= i + r) N[(i + r) * kLD + j + c] -= acc[r][c];
+          if (j + c <= i + r) N[tri(i + r) + j + c] -= acc[r][c];
     }
     __syncthreads();
   }
@@ -839,11 +857,14 @@ __global__ void __launch_bounds__(256) k_merge_solve(MArgs a) {
     for (int t = tid; t < nb; t += nt) {
       const int i = i1 + 4 * (t >> 5), e = t & 31;
       float acc[4][4] = {};
+      const float* li[4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) li[r] = N + tri(i + r) + i0;
 #pragma unroll 4
       for (int kx = 0; kx < 32; ++kx) {
         float l[4], z[4];
 #pragma unroll
-        for (int r = 0; r < 4; ++r) l[r] = N[(i + r) * kLD + i0 + kx];
+        for (int r = 0; r < 4; ++r) l[r] = li[r][kx];
 #pragma unroll
         for (int c = 0; c < 4; ++c) z[c] = R[(i0 + kx) * kLD + e + 32 * c];
 #pragma unroll
@@ -870,9 +891,10 @@ __global__ void __launch_bounds__(256) k_merge_solve(MArgs a) {
       float acc[4][4] = {};
 #pragma unroll 4
       for (int kx = 0; kx < 32; ++kx) {
+        const float* lk = N + tri(i0 + kx) + i;
         float l[4], z[4];
 #pragma unroll
-        for (int r = 0; r < 4; ++r) l[r] = N[(i0 + kx) * kLD + i + r];
+        for (int r = 0; r < 4; ++r) l[r] = lk[r];
 #pragma unroll
         for (int c = 0; c < 4; ++c) z[c] = R[(i0 + kx) * kLD + e + 32 * c];
 #pragma unroll
