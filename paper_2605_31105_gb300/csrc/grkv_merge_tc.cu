@@ -10,7 +10,7 @@
 //                   or position p is visible to window row r exactly when
 //                   p <= B - w + r % w.
 //   k_merge_gram    pass 1 over the slots: row max / sum of l = s Q K0^T (K0
-//                   gathered with cp.async) and K_out = K0 by TMA stores of the
+//                   gathered with TMA gather4) and K_out = K0 by TMA stores of the
 //                   gathered tiles; pass 2 over the positions: X = softmax,
 //                   R~ += Xh V0 and the Gram G += Xh XGh^T + (2 Xl) XGh^T on
 //                   tcgen05 (Xh, Xl the bf16 high / low parts of X; XGh is Xh
@@ -41,7 +41,6 @@ using namespace sm100;
 constexpr int kTile = 128;
 constexpr int kRows = 128;
 constexpr int kThreads = 384;
-constexpr int kProducers = 64;                    // gather threads (warps 2 and 3)
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KB
 constexpr int kMaxB = 32768;
 constexpr long long kBudget = 1ll << 32;
@@ -104,87 +103,74 @@ static_assert(sizeof(MBars) <= 256, "barrier block");
 __device__ __forceinline__ float lo_half(uint32_t h) { return __uint_as_float(h << 16); }
 __device__ __forceinline__ float hi_half(uint32_t h) { return __uint_as_float(h & 0xFFFF0000u); }
 
-// Gathers rows rows_u[t*128 .. t*128+127] (clamped to slot B-1; a row outside
-// [0, n) reads row 0) of one unit's [n][128] bf16 matrix into a swizzled 32 KB
-// tile with 16-byte cp.async copies, as one commit group.  Called by the 64
-// producer threads: warp pw takes tile rows pw*64 .. pw*64+63, two rows (256
-// contiguous bytes each) per instruction.
-__device__ __forceinline__ void gather_tile(uint8_t* dst, const __nv_bfloat16* base,
-                                            const int32_t* rows_u, int B, int n, int t, int pw,
-                                            int lane) {
-  const int r0 = t * kTile + pw * 64 + 2 * lane;
-  int ra = __ldg(rows_u + min(r0, B - 1)), rb = __ldg(rows_u + min(r0 + 1, B - 1));
-  ra = (unsigned)ra < (unsigned)n ? ra : 0;
-  rb = (unsigned)rb < (unsigned)n ? rb : 0;
-  const int chunk = lane & 15, half = chunk >> 3, c8 = chunk & 7;
-  const uint32_t sbase = smem_u32(dst) + half * (kTileBytes / 2);
-  const char* gbase = (const char*)base + chunk * 16;
-#pragma unroll 8
-  for (int s = 0; s < 32; ++s) {
-    const int ja = __shfl_sync(0xffffffffu, ra, s), jb = __shfl_sync(0xffffffffu, rb, s);
-    const int r = pw * 64 + 2 * s + (lane >> 4);
-    const int j = lane < 16 ? ja : jb;
-    cp_async16(sbase + r * 128 + ((c8 ^ (r & 7)) << 4), gbase + (size_t)j * (kD * 2));
-  }
-  cp_async_commit();
+// Four rows (64 columns each) of a 2-D tensor map into consecutive 128-byte rows.
+__device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
+                                            int r0, int r1, int r2, int r3) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5, %6, %7}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(r0), "r"(r1), "r"(r2), "r"(r3)
+      : "memory");
 }
 
-// Producer side of a ring of R gathered tiles.  Each producer thread publishes
-// a load on ring_full once its own copies of it have landed (then a proxy
-// fence, so the tensor cores and TMA see them), at most LAG loads behind the
-// newest, and publishes everything before it blocks on a full ring.
-template <int R, int LAG>
-struct Producer {
-  uint32_t use = 0, pub = 0;
-  __device__ __forceinline__ void publish_one(MBars* bars) {
-    fence_proxy_async_smem();
-    mbar_arrive(&bars->ring_full[pub % R]);
-    ++pub;
-  }
-  __device__ __forceinline__ bool load(MBars* bars, uint8_t* sm, const __nv_bfloat16* base,
-                                       const int32_t* rows_u, int B, int n, int t, int pw,
-                                       int lane, volatile int* abort_flag) {
+// Producer side of a ring of R gathered tiles, run by warps 2 and 3: warp pw
+// gathers tile rows pw*64 .. pw*64+63 (rows_u at positions t*128 + row,
+// clamped to B-1; a row outside [0, n) reads row 0) with TMA gather4 into the
+// 128-byte-swizzled tile and arrives on ring_full with its 16 KB of
+// transaction bytes, so a slot is full once both halves have landed.
+template <int R>
+struct Gatherer {
+  uint32_t use = 0;
+  __device__ __forceinline__ bool load(MBars* bars, uint8_t* sm, const CUtensorMap* map,
+                                       const int32_t* rows_u, int B, int n, int row0, int t,
+                                       int pw, int lane, volatile int* abort_flag) {
     const uint32_t slot = use % R;
     bool ok = true;
-    if (use >= R) {
-      const uint32_t par = (use / R - 1) & 1;
-      if (!mbar_try_wait(&bars->ring_empty[slot], par)) {
-        cp_async_wait<0>();
-        while (pub < use) publish_one(bars);
-        ok = mbar_wait(&bars->ring_empty[slot], par, abort_flag, kBudget);
-      }
-    }
+    if (use >= R) ok = mbar_wait(&bars->ring_empty[slot], (use / R - 1) & 1, abort_flag, kBudget);
     ok = __all_sync(0xffffffffu, ok);
     if (!ok) return false;
-    gather_tile(sm + kOffRing + slot * kTileBytes, base, rows_u, B, n, t, pw, lane);
-    ++use;
-    if (use - pub > LAG) {
-      cp_async_wait<LAG>();
-      publish_one(bars);
+    uint8_t* dst = sm + kOffRing + slot * kTileBytes;
+    uint64_t* bar = &bars->ring_full[slot];
+    if (lane == 0) mbar_expect_tx(bar, kTileBytes / 2);
+    __syncwarp();
+    if (lane < 16) {
+      const int r = pw * 64 + 4 * lane;
+      int j[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int jj = __ldg(rows_u + min(t * kTile + r + e, B - 1));
+        j[e] = row0 + ((unsigned)jj < (unsigned)n ? jj : 0);
+      }
+      tma_gather4(dst + r * 128, map, bar, 0, j[0], j[1], j[2], j[3]);
+      tma_gather4(dst + kTileBytes / 2 + r * 128, map, bar, 64, j[0], j[1], j[2], j[3]);
     }
+    ++use;
     return true;
   }
-  __device__ __forceinline__ void drain(MBars* bars, bool ok) {
-    cp_async_wait<0>();
-    if (ok)
-      while (pub < use) publish_one(bars);
+  // every issued gather lands before the CTA can exit
+  __device__ __forceinline__ void drain(MBars* bars, volatile int* abort_flag) {
+    for (uint32_t i = use > R ? use - R : 0; i < use; ++i)
+      mbar_wait(&bars->ring_full[i % R], (i / R) & 1, abort_flag, kBudget);
   }
 };
 
-__device__ __forceinline__ void init_common(MBars* bars, int warp, uint32_t ring_empty_count) {
+// ring_empty_count: arrivals that release a ring slot; group_count: threads
+// of the compute warps that arrive on s_done, xg_full and d_empty.
+__device__ __forceinline__ void init_common(MBars* bars, int warp, uint32_t ring_empty_count,
+                                            uint32_t group_count) {
   if (threadIdx.x == 0) {
     for (int i = 0; i < 4; ++i) {
-      mbar_init(&bars->ring_full[i], kProducers);
+      mbar_init(&bars->ring_full[i], 2);   // one expect_tx arrival per gathering warp
       mbar_init(&bars->ring_empty[i], ring_empty_count);
     }
     mbar_init(&bars->q_full, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bars->s_full[i], 1);
-      mbar_init(&bars->s_done[i], 128);
-      mbar_init(&bars->xg_full[i], 128);
+      mbar_init(&bars->s_done[i], group_count);
+      mbar_init(&bars->xg_full[i], group_count);
       mbar_init(&bars->xg_empty[i], 1);
       mbar_init(&bars->d_full[i], 1);
-      mbar_init(&bars->d_empty[i], 128);
+      mbar_init(&bars->d_empty[i], group_count);
     }
     mbar_init(&bars->acc_done, 1);
     mbar_init(&bars->drain, 1);
@@ -374,13 +360,14 @@ __global__ void __launch_bounds__(256) k_merge_fixed(MArgs a) {
 
 // ======================================================== k_merge_gram
 // Roles (384 threads): warp 0 the Q load, then the K_out stores and ring
-// releases; warp 1 MMA issue; warps 2-3 the gathers; warps 4-7 and 8-11 two
+// releases; warp 1 MMA issue; warps 2-3 the gathers (half a tile each); warps 4-7 and 8-11 two
 // compute groups (one thread per window row / TMEM lane) taking alternate
 // jobs.  Job k < T: statistics of slot tile k; T <= k < 2T: R~ and Gram of
 // position tile k - T.  S buffer k & 1.  Ring loads: K of each pass-1 job,
 // then K and V of each pass-2 job.
 __global__ void __launch_bounds__(kThreads, 1)
-    k_merge_gram(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKo,
+    k_merge_gram(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmKo,
                  MArgs a) {
   extern __shared__ __align__(1024) uint8_t smraw[];
   uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
@@ -388,7 +375,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int u = blockIdx.x, B = a.B, T = (B + kTile - 1) / kTile;
   const int ng = __ldg(a.ng + u);
-  init_common(bars, warp, 2);   // ring slots are released by the MMA and by warp 0
+  init_common(bars, warp, 2, 128);   // ring slots are released by the MMA and by warp 0
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars->tmem;
@@ -420,21 +407,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       bulk_wait_all();
     }
   } else if (warp == 2 || warp == 3) {
-    const __nv_bfloat16* kb = a.k + (size_t)u * a.n * kD;
-    const __nv_bfloat16* vb = a.v + (size_t)u * a.n * kD;
     const int32_t* idx_u = a.idx + (size_t)u * B;
     const int32_t* src_u = a.src + (size_t)u * B;
-    Producer<kRingG, 2> pr;
+    const int row0 = u * a.n;   // first row of this unit in the 2-D K / V maps
+    Gatherer<kRingG> gt;
     bool ok = true;
     for (int k = 0; k < 2 * T && ok; ++k) {
       if (k < T) {
-        ok = pr.load(bars, sm, kb, idx_u, B, a.n, k, warp - 2, lane, abort_flag);
+        ok = gt.load(bars, sm, &tmK, idx_u, B, a.n, row0, k, warp - 2, lane, abort_flag);
       } else {
-        ok = pr.load(bars, sm, kb, src_u, B, a.n, k - T, warp - 2, lane, abort_flag);
-        if (ok) ok = pr.load(bars, sm, vb, src_u, B, a.n, k - T, warp - 2, lane, abort_flag);
+        ok = gt.load(bars, sm, &tmK, src_u, B, a.n, row0, k - T, warp - 2, lane, abort_flag);
+        if (ok) ok = gt.load(bars, sm, &tmV, src_u, B, a.n, row0, k - T, warp - 2, lane, abort_flag);
       }
     }
-    pr.drain(bars, ok);
+    gt.drain(bars, abort_flag);
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t id_r = idesc_bf16(kRows, kD, 0, 1);     // R~ += Xh V0 (V0 MN-major)
@@ -917,12 +903,12 @@ __global__ void __launch_bounds__(256, 2) k_merge_solve(MArgs a) {
 
 // ======================================================== k_merge_update
 // Roles (384 threads): warp 0 the Q load, warp 1 MMA issue, warps 2-3 the K0
-// gathers, warps 4-7 the XG rows (one thread per window row), warps 8-11 the
-// output epilogue (one thread per token / TMEM lane of D).  Only the tiles
-// with non-fixed positions are visited; the epilogue warps then copy V0 to
-// the fixed slots.
+// gathers, warps 4-11 two groups that share every tile (XG rows, then the
+// output rows of the previous tile).  Only the tiles with non-fixed
+// positions are visited; the groups then copy V0 to the fixed slots.
 __global__ void __launch_bounds__(kThreads, 1)
-    k_merge_update(const __grid_constant__ CUtensorMap tmQ, MArgs a) {
+    k_merge_update(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                   MArgs a) {
   extern __shared__ __align__(1024) uint8_t smraw[];
   uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
   MBars* bars = (MBars*)(sm + kOffBar);
@@ -935,7 +921,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ng = __ldg(a.ng + u), T = (ng + kTile - 1) / kTile;
   const int32_t* src_u = a.src + (size_t)u * B;
   const int32_t* perm_u = a.perm + (size_t)u * B;
-  init_common(bars, warp, 1);
+  init_common(bars, warp, 1, 256);
   // Z (fp32 [row][d]) to the bf16 B operands Zh, Zl: MN-major tiles of
   // 128-byte rows (d contiguous), two blocks of 64 columns
   {
@@ -971,12 +957,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
     }
   } else if (warp == 2 || warp == 3) {
-    const __nv_bfloat16* kb = a.k + (size_t)u * a.n * kD;
-    Producer<kRingU, 1> pr;
+    Gatherer<kRingU> gt;
     bool ok = true;
     for (int t = 0; t < T && ok; ++t)
-      ok = pr.load(bars, sm, kb, src_u, B, a.n, t, warp - 2, lane, abort_flag);
-    pr.drain(bars, ok);
+      ok = gt.load(bars, sm, &tmK, src_u, B, a.n, u * a.n, t, warp - 2, lane, abort_flag);
+    gt.drain(bars, abort_flag);
   } else if (warp == 1) {
     if (lane == 0 && T > 0) {
       const uint32_t id_d = idesc_bf16(kTile, kD, 1, 1);   // dV = XG^T Z, both MN-major
@@ -1021,98 +1006,96 @@ __global__ void __launch_bounds__(kThreads, 1)
       mma_commit(&bars->drain);
       mbar_wait(&bars->drain, 0, abort_flag, kBudget);
     }
-  } else if (warp >= 4 && warp < 8) {
-    const int q = warp & 3, row = q * 32 + lane;
+  } else if (warp >= 4) {
+    // Two groups (warps 4-7, 8-11) share every tile: group wg computes the XG
+    // rows of tokens 64 wg .. 64 wg + 63 (thread = window row), then writes
+    // the outputs of the previous tile's columns 64 wg .. 64 wg + 63 (thread =
+    // token, one TMEM lane of D).
+    const int wg = (warp - 4) >> 2, q = warp & 3, row = q * 32 + lane, tok = row;
     // rows past m have lam = +inf and give X = 0
     const float lam = a.lam[(size_t)u * kRows + row];
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
+    const uint4* v_u = (const uint4*)(a.v + (size_t)u * a.n * kD);
+    uint4* vo_u = (uint4*)(a.v_out + (size_t)u * B * kD);
+    uint4 v0[8];
+    auto fetch_v0 = [&](int t) {
+      const uint4* g = v_u + (size_t)__ldg(src_u + min(t * kTile + tok, B - 1)) * 16 + 8 * wg;
+#pragma unroll
+      for (int h = 0; h < 8; ++h) v0[h] = __ldg(g + h);
+    };
+    auto epilogue = [&](int t) -> bool {
+      if (!mbar_wait(&bars->d_full[t & 1], (t >> 1) & 1, abort_flag, kBudget)) return false;
+      tc_fence_after();
+      const uint32_t dcol = lane_addr + kColD + (t & 1) * kD + 64 * wg;
+      float da[32], db[32];
+      tmem_ld32f(dcol, da);
+      tmem_ld32f(dcol + 32, db);
+      tmem_wait32(da);
+      tmem_wait32(db);
+      tc_fence_before();
+      mbar_arrive(&bars->d_empty[t & 1]);
+      const int p = t * kTile + tok;
+      if (p < ng) {
+        uint4* o = vo_u + (size_t)__ldg(perm_u + p) * 16 + 8 * wg;
+#pragma unroll
+        for (int h = 0; h < 8; ++h) {
+          const float* dv = h < 4 ? da + 8 * h : db + 8 * (h - 4);
+          const __nv_bfloat16* pv = (const __nv_bfloat16*)&v0[h];
+          uint32_t w[4];
+#pragma unroll
+          for (int z = 0; z < 4; ++z)
+            w[z] = pack_bf16(__bfloat162float(pv[2 * z]) + dv[2 * z],
+                             __bfloat162float(pv[2 * z + 1]) + dv[2 * z + 1]);
+          o[h] = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+      }
+      return true;
+    };
     bool ok = true;
     for (int t = 0; t < T && ok; ++t) {
       const int b = t & 1, p0 = t * kTile;
+      if (t >= 1) fetch_v0(t - 1);
       ok = mbar_wait(&bars->s_full[b], (t >> 1) & 1, abort_flag, kBudget);
       if (ok && t >= 1) ok = mbar_wait(&bars->xg_empty[0], (t - 1) & 1, abort_flag, kBudget);
       if (!ok) break;
       tc_fence_after();
-      const uint32_t sbase = lane_addr + kColS + b * kTile;
+      const uint32_t sbase = lane_addr + kColS + b * kTile + 64 * wg;
       float va[32], vb[32];
       tmem_ld32f(sbase, va);
-      tmem_wait32(va);
       tmem_ld32f(sbase + 32, vb);
-      if (p0 + kTile <= ng) {
-        update_chunk<0, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
-        tmem_wait32(vb);
-        tmem_ld32f(sbase + 64, va);
-        update_chunk<1, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
-        tmem_wait32(va);
-        tmem_ld32f(sbase + 96, vb);
-        update_chunk<2, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
-        tmem_wait32(vb);
-        tc_fence_before();
-        mbar_arrive(&bars->s_done[b]);   // S is fully read
-        update_chunk<3, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+      tmem_wait32(va);
+      tmem_wait32(vb);
+      tc_fence_before();
+      mbar_arrive(&bars->s_done[b]);   // S is read
+      const bool masked = p0 + kTile > ng;
+      if (wg == 0) {
+        if (masked) {
+          update_chunk<0, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
+          update_chunk<1, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        } else {
+          update_chunk<0, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
+          update_chunk<1, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        }
       } else {
-        update_chunk<0, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
-        tmem_wait32(vb);
-        tmem_ld32f(sbase + 64, va);
-        update_chunk<1, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
-        tmem_wait32(va);
-        tmem_ld32f(sbase + 96, vb);
-        update_chunk<2, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
-        tmem_wait32(vb);
-        tc_fence_before();
-        mbar_arrive(&bars->s_done[b]);
-        update_chunk<3, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        if (masked) {
+          update_chunk<2, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
+          update_chunk<3, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        } else {
+          update_chunk<2, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
+          update_chunk<3, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        }
       }
       fence_proxy_async_smem();
       mbar_arrive(&bars->xg_full[0]);
+      if (t >= 1) ok = epilogue(t - 1);
+    }
+    if (ok && T >= 1) {
+      fetch_v0(T - 1);
+      ok = epilogue(T - 1);
     }
     if (!ok && row == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
-  } else if (warp >= 8) {
-    // epilogue: thread = token (TMEM lane) of D = dV, 128 columns of d
-    const int q = warp & 3, tok = q * 32 + lane;
-    const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
-    const uint4* v_u = (const uint4*)(a.v + (size_t)u * a.n * kD);
-    uint4* vo_u = (uint4*)(a.v_out + (size_t)u * B * kD);
-    bool ok = true;
-    for (int t = 0; t < T && ok; ++t) {
-      const int p = t * kTile + tok;
-      const bool live = p < ng;
-      // V0 row of this position, fetched before D is ready
-      uint4 v0[16];
-      const uint4* g = v_u + (size_t)__ldg(src_u + min(p, B - 1)) * 16;
-#pragma unroll
-      for (int h = 0; h < 16; ++h) v0[h] = __ldg(g + h);
-      const int dst = live ? __ldg(perm_u + p) : 0;
-      ok = mbar_wait(&bars->d_full[t & 1], (t >> 1) & 1, abort_flag, kBudget);
-      if (!ok) break;
-      tc_fence_after();
-      const uint32_t dcol = lane_addr + kColD + (t & 1) * kD;
-#pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        float v[32];
-        tmem_ld32f(dcol + c * 32, v);
-        tmem_wait32(v);
-        if (c == 3) {
-          tc_fence_before();
-          mbar_arrive(&bars->d_empty[t & 1]);
-        }
-        if (live) {
-#pragma unroll
-          for (int h = 0; h < 4; ++h) {
-            const __nv_bfloat16* pv = (const __nv_bfloat16*)&v0[4 * c + h];
-            uint32_t o[4];
-#pragma unroll
-            for (int z = 0; z < 4; ++z)
-              o[z] = pack_bf16(__bfloat162float(pv[2 * z]) + v[8 * h + 2 * z],
-                               __bfloat162float(pv[2 * z + 1]) + v[8 * h + 2 * z + 1]);
-            vo_u[(size_t)dst * 16 + 4 * c + h] = make_uint4(o[0], o[1], o[2], o[3]);
-          }
-        }
-      }
-    }
-    if (!ok && tok == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
     // V_out = V0 for the fixed slots (positions ng .. B-1)
-    for (int p = ng + tok; p < B; p += 128) {
+    for (int p = ng + (tid - 128); p < B; p += 256) {
       const uint4* g = v_u + (size_t)__ldg(src_u + p) * 16;
       uint4* o = vo_u + (size_t)__ldg(perm_u + p) * 16;
 #pragma unroll
@@ -1140,8 +1123,10 @@ size_t merge_tc_ws_bytes(const Shape& s) {
 cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const void* v,
                             const float* scores, const float* y, const int32_t* idx, void* k_out,
                             void* v_out, char* ws, const WsLayout& L, cudaStream_t st) {
-  CUtensorMap mq, mko;
+  CUtensorMap mq, mk, mv, mko;
   if (!encode_bf16_3d(&mq, q, kD, s.m, s.U, 64, kRows) ||
+      !encode_bf16_2d_rows(&mk, k, kD, (uint64_t)s.U * s.n) ||
+      !encode_bf16_2d_rows(&mv, v, kD, (uint64_t)s.U * s.n) ||
       !encode_bf16_3d(&mko, k_out, kD, s.B, s.U, 64, kTile))
     return cudaErrorInvalidValue;
   MArgs a{};
@@ -1182,9 +1167,9 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
                                 s.B * 4)) != cudaSuccess)
     return e;
   k_merge_fixed<<<s.U, 256, s.B * 4, st>>>(a);
-  k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mko, a);
+  k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, mko, a);
   k_merge_solve<<<s.U, 256, kSolveSmem, st>>>(a);
-  k_merge_update<<<s.U, kThreads, kSmemBytes, st>>>(mq, a);
+  k_merge_update<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, a);
   count_launches(4);
   return cudaGetLastError();
 }
