@@ -125,9 +125,14 @@ int grkv_select(const grkv_params* p, const float* scores, int32_t* idx,
  *   R = Y - X V0,  Z = (X_G X_G^T + lambda_v I_m)^-1 R,
  *   V_out[G] = V0[G] + X_G^T Z,  V_out[F] = V0[F],  K_out = K0
  * (Algorithm 1 value step; App. D.1 dual form; App. D.3 fixed tokens).
- * Outputs are rounded to `dtype` (round to nearest even). */
+ * Outputs are rounded to `dtype` (round to nearest even).
+ * row_stats may be NULL; given (as grkv_score writes it), the tensor-core
+ * path accumulates the retained softmax against the full-cache row maximum
+ * in one pass over K0 instead of two (same results up to rounding; units
+ * whose retained maximum lies more than 2^64 below it are recomputed with
+ * two passes). */
 int grkv_merge(const grkv_params* p, const void* q, const void* k, const void* v,
-               const float* scores, const float* y, const int32_t* idx,
+               const float* scores, const float* y, const float* row_stats, const int32_t* idx,
                void* k_out, void* v_out, void* ws, size_t ws_bytes, void* stream);
 
 /* The whole path: grkv_score, grkv_select and grkv_merge with every

@@ -71,7 +71,7 @@ def load():
     lib.grkv_workspace_size.argtypes = [_P, ctypes.POINTER(ctypes.c_size_t)]
     lib.grkv_score.argtypes = [_P, _vp, _vp, _vp, _vp, _vp, _vp, _vp, ctypes.c_size_t, _vp]
     lib.grkv_select.argtypes = [_P, _vp, _vp, _vp, ctypes.c_size_t, _vp]
-    lib.grkv_merge.argtypes = [_P, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+    lib.grkv_merge.argtypes = [_P, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                ctypes.c_size_t, _vp]
     lib.grkv_compress.argtypes = [_P, _vp, _vp, _vp, _vp, _vp, _vp, _vp, ctypes.c_size_t, _vp]
     lib.grkv_status.argtypes = [_vp, ctypes.POINTER(ctypes.c_int), _vp]
@@ -153,11 +153,11 @@ def grkv_select(p, scores, idx, ws, ws_bytes=None, stream=None, check=True):
 
 
 def grkv_merge(p, q, k, v, scores, y, idx, k_out, v_out, ws, ws_bytes=None, stream=None,
-               check=True):
+               check=True, row_stats=None):
     ws_bytes = ws.numel() * ws.element_size() if ws_bytes is None else ws_bytes
     rc = load().grkv_merge(ctypes.byref(p), _ptr(q), _ptr(k), _ptr(v), _ptr(scores), _ptr(y),
-                           _ptr(idx), _ptr(k_out), _ptr(v_out), _ptr(ws), ws_bytes,
-                           _stream(stream))
+                           _ptr(row_stats), _ptr(idx), _ptr(k_out), _ptr(v_out), _ptr(ws),
+                           ws_bytes, _stream(stream))
     return _check(rc, "grkv_merge", check)
 
 

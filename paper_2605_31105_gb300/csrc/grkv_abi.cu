@@ -31,10 +31,11 @@ int check_ptr(const void* p, size_t elems) {
 int cuda_rc(cudaError_t e) { return e == cudaSuccess ? GRKV_OK : GRKV_ERR_CUDA; }
 
 cudaError_t launch_merge(const Shape& s, const void* q, const void* k, const void* v,
-                         const float* scores, const float* y, const int32_t* idx, void* k_out,
-                         void* v_out, char* ws, const WsLayout& L, cudaStream_t st) {
+                         const float* scores, const float* y, const float* row_stats,
+                         const int32_t* idx, void* k_out, void* v_out, char* ws, const WsLayout& L,
+                         cudaStream_t st) {
   if (s.tc_merge)
-    return launch_merge_tc(s, q, k, v, scores, y, idx, k_out, v_out, ws, L, st);
+    return launch_merge_tc(s, q, k, v, scores, y, row_stats, idx, k_out, v_out, ws, L, st);
   return launch_merge_simt(s, q, k, v, scores, y, idx, k_out, v_out, ws, L, st);
 }
 
@@ -212,8 +213,8 @@ int grkv_select(const grkv_params* p, const float* scores, int32_t* idx, void* w
 }
 
 int grkv_merge(const grkv_params* p, const void* q, const void* k, const void* v,
-               const float* scores, const float* y, const int32_t* idx, void* k_out, void* v_out,
-               void* ws, size_t ws_bytes, void* stream) {
+               const float* scores, const float* y, const float* row_stats, const int32_t* idx,
+               void* k_out, void* v_out, void* ws, size_t ws_bytes, void* stream) {
   Shape s;
   GRKV_TRY(make_shape(p, &s));
   const WsLayout L = plan_workspace(s);
@@ -221,6 +222,7 @@ int grkv_merge(const grkv_params* p, const void* q, const void* k, const void* v
   GRKV_TRY(check_inputs(s, q, k, v));
   GRKV_TRY(check_ptr(scores, (size_t)s.U * s.P));
   GRKV_TRY(check_ptr(y, (size_t)s.U * s.m));
+  if (row_stats) GRKV_TRY(check_ptr(row_stats, (size_t)s.U * s.m));
   GRKV_TRY(check_ptr(idx, (size_t)s.U * s.B));
   GRKV_TRY(check_ptr(k_out, (size_t)s.U * s.B));
   GRKV_TRY(check_ptr(v_out, (size_t)s.U * s.B));
@@ -228,7 +230,7 @@ int grkv_merge(const grkv_params* p, const void* q, const void* k, const void* v
   char* w = (char*)ws;
   GRKV_TRY(cuda_rc(cudaMemsetAsync(w + L.status, 0, 4, st)));
   if (s.U == 0) return GRKV_OK;
-  return cuda_rc(launch_merge(s, q, k, v, scores, y, idx, k_out, v_out, w, L, st));
+  return cuda_rc(launch_merge(s, q, k, v, scores, y, row_stats, idx, k_out, v_out, w, L, st));
 }
 
 int grkv_compress(const grkv_params* p, const void* q, const void* k, const void* v, void* k_out,
@@ -250,7 +252,7 @@ int grkv_compress(const grkv_params* p, const void* q, const void* k, const void
   float* rstats = (float*)(w + L.rstats);
   GRKV_TRY(cuda_rc(launch_score(s, q, k, v, scores, y, rstats, w, L, st)));
   GRKV_TRY(cuda_rc(launch_select(s, scores, idx, w, L, st)));
-  return cuda_rc(launch_merge(s, q, k, v, scores, y, idx, k_out, v_out, w, L, st));
+  return cuda_rc(launch_merge(s, q, k, v, scores, y, rstats, idx, k_out, v_out, w, L, st));
 }
 
 int grkv_status(const void* ws, int* device_status, void* stream) {

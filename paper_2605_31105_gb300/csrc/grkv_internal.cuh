@@ -90,9 +90,12 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
 // Tensor-core value merge (bf16, m <= 128, B <= 32768).
 bool merge_tc_supported(const Shape& s);
 size_t merge_tc_ws_bytes(const Shape& s);
+// row_stats (nullable): the full-cache row statistics; with them the Gram
+// needs one pass over the retained keys.
 cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const void* v,
-                            const float* scores, const float* y, const int32_t* idx, void* k_out,
-                            void* v_out, char* ws, const WsLayout& L, cudaStream_t st);
+                            const float* scores, const float* y, const float* row_stats,
+                            const int32_t* idx, void* k_out, void* v_out, char* ws,
+                            const WsLayout& L, cudaStream_t st);
 
 // Selection with the pooled-score scratch [U][n-w] given directly.
 cudaError_t launch_select_pooled(const Shape& s, const float* scores, int32_t* idx,

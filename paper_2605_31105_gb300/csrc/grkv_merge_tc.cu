@@ -77,13 +77,17 @@ struct MArgs {
   const float* y;            // [U][m][128]
   const __nv_bfloat16* k;    // [U][n][128]
   const __nv_bfloat16* v;
-  __nv_bfloat16* v_out;      // [U][B][128]
+  __nv_bfloat16* k_out;      // [U][B][128]
+  __nv_bfloat16* v_out;
+  const float* rstats;       // [U][m][2] full-cache row max / sum (natural units) or null
   float* rz;                 // [U][128][128]  R (gram) -> Z (solve)
   float* gram;               // [U][128][128]  raw Gram
   float* lam;                // [U][128]       log2 normaliser of each window row
   int32_t* perm;             // [U][B]         slot at each position
   int32_t* src;              // [U][B]         idx of that slot (the K / V row)
   int32_t* ng;               // [U]            number of non-fixed slots
+  int32_t* redo;             // [U]            single-pass result unusable: run two passes
+  int gram_mode;             // 0 two passes; 1 one pass against rstats; 2 two passes for redo units
   int* status;
 };
 
@@ -97,6 +101,7 @@ struct MBars {
   uint64_t drain;
   uint32_t tmem;
   int abort;
+  int bad;
 };
 static_assert(sizeof(MBars) <= 256, "barrier block");
 
@@ -175,6 +180,7 @@ __device__ __forceinline__ void init_common(MBars* bars, int warp, uint32_t ring
     mbar_init(&bars->acc_done, 1);
     mbar_init(&bars->drain, 1);
     bars->abort = 0;
+    bars->bad = 0;
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -209,11 +215,13 @@ __device__ __forceinline__ void store_row_chunk(uint8_t* tile, int row, int C, c
 template <int C>
 __device__ __forceinline__ void gram_chunk_fast(const float* v, float sl2, float lam,
                                                 uint32_t sbase, uint8_t* xg, int row,
-                                                uint32_t* lo) {
+                                                uint32_t* lo, float& vmax, float& xsum) {
   uint32_t hi[16];
 #pragma unroll
   for (int e = 0; e < 32; e += 2) {
     const float x0 = fast_exp2(fmaf(v[e], sl2, -lam)), x1 = fast_exp2(fmaf(v[e + 1], sl2, -lam));
+    vmax = fmaxf(vmax, fmaxf(v[e], v[e + 1]));
+    xsum += x0 + x1;
     const uint32_t h = pack_bf16(x0, x1);
     hi[e / 2] = h;
     lo[e / 2] = pack_bf16(2.f * (x0 - lo_half(h)), 2.f * (x1 - hi_half(h)));
@@ -228,13 +236,15 @@ template <int C>
 __device__ __forceinline__ void gram_chunk_masked(const float* v, int p0, int vlim, int ng,
                                                   float sl2, float lam, uint32_t sbase,
                                                   uint8_t* xg, int row, uint32_t* lo,
-                                                  bool want_g) {
+                                                  bool want_g, float& vmax, float& xsum) {
   uint32_t hi[16], ghi[16];
 #pragma unroll
   for (int e = 0; e < 32; e += 2) {
     const int p = p0 + C * 32 + e;
     const float x0 = p <= vlim ? fast_exp2(fmaf(v[e], sl2, -lam)) : 0.f;
     const float x1 = p + 1 <= vlim ? fast_exp2(fmaf(v[e + 1], sl2, -lam)) : 0.f;
+    vmax = fmaxf(vmax, fmaxf(p <= vlim ? v[e] : -INFINITY, p + 1 <= vlim ? v[e + 1] : -INFINITY));
+    xsum += x0 + x1;
     const uint32_t h = pack_bf16(x0, x1);
     hi[e / 2] = h;
     lo[e / 2] = pack_bf16(2.f * (x0 - lo_half(h)), 2.f * (x1 - hi_half(h)));
@@ -359,12 +369,20 @@ __global__ void __launch_bounds__(256) k_merge_fixed(MArgs a) {
 }
 
 // ======================================================== k_merge_gram
-// Roles (384 threads): warp 0 the Q load, then the K_out stores and ring
-// releases; warp 1 MMA issue; warps 2-3 the gathers (half a tile each); warps 4-7 and 8-11 two
-// compute groups (one thread per window row / TMEM lane) taking alternate
-// jobs.  Job k < T: statistics of slot tile k; T <= k < 2T: R~ and Gram of
-// position tile k - T.  S buffer k & 1.  Ring loads: K of each pass-1 job,
-// then K and V of each pass-2 job.
+// Roles (384 threads): warp 0 the Q load, then the K_out writes and ring
+// releases; warp 1 MMA issue; warps 2-3 the gathers (half a tile each);
+// warps 4-7 and 8-11 two compute groups (one thread per window row / TMEM
+// lane) taking alternate jobs.  Job k < T: statistics of slot tile k;
+// T <= k < 2T: R~ and Gram of position tile k - T.  Ring loads: K of each
+// pass-1 job, then K and V of each pass-2 job.
+//
+// gram_mode 1 (the full-cache row statistics are known) runs only the second
+// pass, with X accumulated against the full row maximum M_r instead of the
+// retained one: X' = exp2(l - M_r) = X L'_r with L'_r = sum of X' over the
+// visible retained keys, so R = Y - R~'/L'_r and G_ij = G'_ij/(L'_i L'_j).  The
+// retained maximum is at most M_r; if it is more than 64 (log2 units) below
+// it for some row, or L' underflows, the unit is flagged and gram_mode 2
+// recomputes it with both passes.
 __global__ void __launch_bounds__(kThreads, 1)
     k_merge_gram(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                  const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmKo,
@@ -374,6 +392,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   MBars* bars = (MBars*)(sm + kOffBar);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int u = blockIdx.x, B = a.B, T = (B + kTile - 1) / kTile;
+  if (a.gram_mode == 2 && __ldg(a.redo + u) == 0) return;   // the single pass was valid
+  const bool single = a.gram_mode == 1;
+  const int k0 = single ? T : 0;   // first job
   const int ng = __ldg(a.ng + u);
   init_common(bars, warp, 2, 128);   // ring slots are released by the MMA and by warp 0
   __syncthreads();
@@ -381,7 +402,46 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = bars->tmem;
   volatile int* abort_flag = &bars->abort;
 
-  if (warp == 0) {
+  if (warp == 0 && single) {
+    if (lane == 0) {
+      prefetch_tensormap(&tmQ);
+      mbar_expect_tx(&bars->q_full, kTileBytes);
+      const uint64_t pol = l2_evict_last();
+      tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, 0, u, pol);
+      tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
+    }
+    __syncwarp();
+    // K_out = K0 from the K tiles of the (only) pass, position p to slot perm[p]:
+    // two 256-byte rows per step, one 16-byte chunk per lane
+    const int32_t* perm_u = a.perm + (size_t)u * B;
+    uint4* ko_u = (uint4*)(a.k_out + (size_t)u * B * kD);
+    const int c = lane & 15, c8 = c & 7;
+    bool ok = true;
+    for (int use = 0; use < 2 * T && ok; ++use) {
+      const int slot = use % kRingG;
+      const int pt = (use >> 1) * kTile;
+      int dst[4];   // output slots of tile rows 32 i + lane, fetched before the tile lands
+      if ((use & 1) == 0) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) dst[i] = __ldg(perm_u + min(pt + 32 * i + lane, B - 1));
+      }
+      ok = mbar_wait(&bars->ring_full[slot], (use / kRingG) & 1, abort_flag, kBudget);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) break;
+      if ((use & 1) == 0) {
+        const uint8_t* tile = sm + kOffRing + slot * kTileBytes + (c >> 3) * (kTileBytes / 2);
+#pragma unroll
+        for (int it = 0; it < kTile / 2; ++it) {
+          const int r = 2 * it + (lane >> 4);
+          const int d = __shfl_sync(0xffffffffu, dst[it >> 4], r & 31);
+          if (pt + r < B)
+            ko_u[(size_t)d * 16 + c] = *(const uint4*)(tile + r * 128 + ((c8 ^ (r & 7)) << 4));
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars->ring_empty[slot]);
+    }
+  } else if (warp == 0) {
     if (lane == 0) {
       prefetch_tensormap(&tmQ);
       prefetch_tensormap(&tmKo);
@@ -412,7 +472,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int row0 = u * a.n;   // first row of this unit in the 2-D K / V maps
     Gatherer<kRingG> gt;
     bool ok = true;
-    for (int k = 0; k < 2 * T && ok; ++k) {
+    for (int k = k0; k < 2 * T && ok; ++k) {
       if (k < T) {
         ok = gt.load(bars, sm, &tmK, idx_u, B, a.n, row0, k, warp - 2, lane, abort_flag);
       } else {
@@ -432,8 +492,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t pend_v = 0;
       bool g_started = false;
       auto issue_rg = [&](int kp, uint32_t vuse) -> bool {
-        const int t = kp - T, b = kp & 1, xb = t & 1;
-        bool w = mbar_wait(&bars->s_done[b], (kp >> 1) & 1, abort_flag, kBudget);
+        const int t = kp - T, b = (kp - k0) & 1, xb = t & 1;
+        bool w = mbar_wait(&bars->s_done[b], ((kp - k0) >> 1) & 1, abort_flag, kBudget);
         if (w) w = mbar_wait(&bars->xg_full[xb], (t >> 1) & 1, abort_flag, kBudget);
         if (w)
           w = mbar_wait(&bars->ring_full[vuse % kRingG], (vuse / kRingG) & 1, abort_flag, kBudget);
@@ -464,11 +524,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         mma_commit(&bars->xg_empty[xb]);
         return true;
       };
-      for (int k = 0; k < 2 * T && ok; ++k) {
-        const int b = k & 1;
+      for (int k = k0; k < 2 * T && ok; ++k) {
+        const int jk = k - k0, b = jk & 1;
         const uint32_t kuse = use++;
         ok = mbar_wait(&bars->ring_full[kuse % kRingG], (kuse / kRingG) & 1, abort_flag, kBudget);
-        if (ok && k >= 2) ok = mbar_wait(&bars->s_done[b], ((k >> 1) - 1) & 1, abort_flag, kBudget);
+        if (ok && jk >= 2) ok = mbar_wait(&bars->s_done[b], ((jk >> 1) - 1) & 1, abort_flag, kBudget);
         if (!ok) break;
         tc_fence_after();
         issue_s(tmem + kColS + b * kTile, qa,
@@ -499,9 +559,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int open = B - a.w;   // below this everything is visible to every window row
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
     float M = -INFINITY, L = 0.f, lam = INFINITY;
+    float vmax = -INFINITY, xsum = 0.f;   // visible retained logits (raw) and sum of X
+    if (single && row_ok) lam = __ldg(a.rstats + ((size_t)u * a.m + row) * 2) * 1.4426950408889634f;
     bool ok = true;
-    for (int k = 0; k < 2 * T; ++k) {
-      if (k == T) {
+    for (int k = k0; k < 2 * T; ++k) {
+      if (k == T && !single) {
         // both groups combine their statistics (reached even after an abort);
         // the XGh tiles are not in use yet
         float2* comb = (float2*)(sm + kOffXG);
@@ -524,9 +586,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (k < T) continue;
         break;
       }
-      if ((k & 1) != wg) continue;
-      const int b = k & 1, t = k < T ? k : k - T, p0 = t * kTile;
-      ok = mbar_wait(&bars->s_full[b], (k >> 1) & 1, abort_flag, kBudget);
+      if (((k - k0) & 1) != wg) continue;
+      const int b = (k - k0) & 1, t = k < T ? k : k - T, p0 = t * kTile;
+      ok = mbar_wait(&bars->s_full[b], ((k - k0) >> 1) & 1, abort_flag, kBudget);
       if (!ok) continue;
       tc_fence_after();
       const uint32_t sbase = lane_addr + kColS + b * kTile;
@@ -574,32 +636,32 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_wait32(va);
         tmem_ld32f(sbase + 32, vb);
         if (__all_sync(0xffffffffu, row_ok) && p0 + kTile <= ng) {
-          gram_chunk_fast<0>(va, a.sl2, lam, sbase, xg, row, lo0);
+          gram_chunk_fast<0>(va, a.sl2, lam, sbase, xg, row, lo0, vmax, xsum);
           tmem_wait32(vb);
           tmem_ld32f(sbase + 64, va);
-          gram_chunk_fast<1>(vb, a.sl2, lam, sbase, xg, row, lo1);
+          gram_chunk_fast<1>(vb, a.sl2, lam, sbase, xg, row, lo1, vmax, xsum);
           tmem_wait32(va);
           tmem_st16(sbase + 64, lo0);
           tmem_st16(sbase + 80, lo1);
           tmem_ld32f(sbase + 96, vb);
-          gram_chunk_fast<2>(va, a.sl2, lam, sbase, xg, row, lo2);
+          gram_chunk_fast<2>(va, a.sl2, lam, sbase, xg, row, lo2, vmax, xsum);
           tmem_wait32(vb);
           tmem_st16(sbase + 96, lo2);
-          gram_chunk_fast<3>(vb, a.sl2, lam, sbase, xg, row, lo3);
+          gram_chunk_fast<3>(vb, a.sl2, lam, sbase, xg, row, lo3, vmax, xsum);
         } else {
           const bool want_g = p0 < ng;
-          gram_chunk_masked<0>(va, p0, vlim, ng, a.sl2, lam, sbase, xg, row, lo0, want_g);
+          gram_chunk_masked<0>(va, p0, vlim, ng, a.sl2, lam, sbase, xg, row, lo0, want_g, vmax, xsum);
           tmem_wait32(vb);
           tmem_ld32f(sbase + 64, va);
-          gram_chunk_masked<1>(vb, p0, vlim, ng, a.sl2, lam, sbase, xg, row, lo1, want_g);
+          gram_chunk_masked<1>(vb, p0, vlim, ng, a.sl2, lam, sbase, xg, row, lo1, want_g, vmax, xsum);
           tmem_wait32(va);
           tmem_st16(sbase + 64, lo0);
           tmem_st16(sbase + 80, lo1);
           tmem_ld32f(sbase + 96, vb);
-          gram_chunk_masked<2>(va, p0, vlim, ng, a.sl2, lam, sbase, xg, row, lo2, want_g);
+          gram_chunk_masked<2>(va, p0, vlim, ng, a.sl2, lam, sbase, xg, row, lo2, want_g, vmax, xsum);
           tmem_wait32(vb);
           tmem_st16(sbase + 96, lo2);
-          gram_chunk_masked<3>(vb, p0, vlim, ng, a.sl2, lam, sbase, xg, row, lo3, want_g);
+          gram_chunk_masked<3>(vb, p0, vlim, ng, a.sl2, lam, sbase, xg, row, lo3, want_g, vmax, xsum);
         }
         tmem_st16(sbase + 112, lo3);
         tmem_st_wait();
@@ -612,6 +674,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     // R = Y - R~ and the raw Gram rows to the workspace, half the columns per group
     if (ok) ok = mbar_wait(&bars->acc_done, 0, abort_flag, kBudget);
     tc_fence_after();
+    float ci = 1.f;   // 1 / L'_row in the single pass
+    float* cs = (float*)(sm + kOffXG) + 2 * 2 * kRows;   // [128] after the float2 pairs
+    if (single) {
+      // combine the groups' sums and maxima (the XGh tiles are free now)
+      float2* comb = (float2*)(sm + kOffXG);
+      comb[wg * kRows + row] = make_float2(vmax, xsum);
+      named_bar(4, 256);
+      const float2 o = comb[(wg ^ 1) * kRows + row];
+      const float lsum = xsum + o.y, vm = fmaxf(vmax, o.x);
+      const bool bad = row_ok && !(lsum > 0.f && lam - vm * a.sl2 <= 64.f);
+      if (bad) bars->bad = 1;
+      ci = (row_ok && lsum > 0.f) ? 1.f / lsum : 0.f;
+      if (wg == 0) {
+        cs[row] = ci;
+        a.lam[(size_t)u * kRows + row] = (row_ok && lsum > 0.f) ? lam + __log2f(lsum) : INFINITY;
+      }
+      named_bar(4, 256);
+      if (tid == 128) a.redo[u] = bars->bad;
+      if (bars->bad) ok = false;   // gram_mode 2 redoes this unit; not a failure
+    }
     if (ok) {
       float* R = a.rz + ((size_t)u * kRows + row) * kD;
       float* G = a.gram + ((size_t)u * kRows + row) * kRows;
@@ -626,7 +708,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float4 yv = row_ok ? __ldg((const float4*)(yr + c * 32 + e))
                                    : make_float4(0.f, 0.f, 0.f, 0.f);
           *(float4*)(R + c * 32 + e) =
-              row_ok ? make_float4(yv.x - v[e], yv.y - v[e + 1], yv.z - v[e + 2], yv.w - v[e + 3])
+              row_ok ? make_float4(yv.x - ci * v[e], yv.y - ci * v[e + 1], yv.z - ci * v[e + 2],
+                                   yv.w - ci * v[e + 3])
                      : make_float4(0.f, 0.f, 0.f, 0.f);
         }
         tmem_ld32f(lane_addr + kColG + c * 32, v);
@@ -635,12 +718,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int e = 0; e < 32; ++e) v[e] = 0.f;
         }
+        if (single) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) v[e] *= ci * cs[c * 32 + e];
+        }
 #pragma unroll
         for (int e = 0; e < 32; e += 4)
           *(float4*)(G + c * 32 + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
       }
     }
-    if (!ok && row == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
+    if (!ok && row == 0 && !bars->bad) set_status(a.status, GRKV_ERR_TIMEOUT);
   }
   tc_fence_before();
   __syncthreads();
@@ -903,9 +990,10 @@ __global__ void __launch_bounds__(256, 2) k_merge_solve(MArgs a) {
 
 // ======================================================== k_merge_update
 // Roles (384 threads): warp 0 the Q load, warp 1 MMA issue, warps 2-3 the K0
-// gathers, warps 4-11 two groups that share every tile (XG rows, then the
-// output rows of the previous tile).  Only the tiles with non-fixed
-// positions are visited; the groups then copy V0 to the fixed slots.
+// gathers, warps 4-7 the XG rows (one thread per window row), warps 8-11 the
+// output epilogue (one thread per token / TMEM lane of D).  Only the tiles
+// with non-fixed positions are visited; the epilogue warps then copy V0 to
+// the fixed slots.
 __global__ void __launch_bounds__(kThreads, 1)
     k_merge_update(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    MArgs a) {
@@ -921,7 +1009,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ng = __ldg(a.ng + u), T = (ng + kTile - 1) / kTile;
   const int32_t* src_u = a.src + (size_t)u * B;
   const int32_t* perm_u = a.perm + (size_t)u * B;
-  init_common(bars, warp, 1, 256);
+  init_common(bars, warp, 1, 128);
   // Z (fp32 [row][d]) to the bf16 B operands Zh, Zl: MN-major tiles of
   // 128-byte rows (d contiguous), two blocks of 64 columns
   {
@@ -1006,96 +1094,98 @@ __global__ void __launch_bounds__(kThreads, 1)
       mma_commit(&bars->drain);
       mbar_wait(&bars->drain, 0, abort_flag, kBudget);
     }
-  } else if (warp >= 4) {
-    // Two groups (warps 4-7, 8-11) share every tile: group wg computes the XG
-    // rows of tokens 64 wg .. 64 wg + 63 (thread = window row), then writes
-    // the outputs of the previous tile's columns 64 wg .. 64 wg + 63 (thread =
-    // token, one TMEM lane of D).
-    const int wg = (warp - 4) >> 2, q = warp & 3, row = q * 32 + lane, tok = row;
+  } else if (warp >= 4 && warp < 8) {
+    const int q = warp & 3, row = q * 32 + lane;
     // rows past m have lam = +inf and give X = 0
     const float lam = a.lam[(size_t)u * kRows + row];
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
-    const uint4* v_u = (const uint4*)(a.v + (size_t)u * a.n * kD);
-    uint4* vo_u = (uint4*)(a.v_out + (size_t)u * B * kD);
-    uint4 v0[8];
-    auto fetch_v0 = [&](int t) {
-      const uint4* g = v_u + (size_t)__ldg(src_u + min(t * kTile + tok, B - 1)) * 16 + 8 * wg;
-#pragma unroll
-      for (int h = 0; h < 8; ++h) v0[h] = __ldg(g + h);
-    };
-    auto epilogue = [&](int t) -> bool {
-      if (!mbar_wait(&bars->d_full[t & 1], (t >> 1) & 1, abort_flag, kBudget)) return false;
-      tc_fence_after();
-      const uint32_t dcol = lane_addr + kColD + (t & 1) * kD + 64 * wg;
-      float da[32], db[32];
-      tmem_ld32f(dcol, da);
-      tmem_ld32f(dcol + 32, db);
-      tmem_wait32(da);
-      tmem_wait32(db);
-      tc_fence_before();
-      mbar_arrive(&bars->d_empty[t & 1]);
-      const int p = t * kTile + tok;
-      if (p < ng) {
-        uint4* o = vo_u + (size_t)__ldg(perm_u + p) * 16 + 8 * wg;
-#pragma unroll
-        for (int h = 0; h < 8; ++h) {
-          const float* dv = h < 4 ? da + 8 * h : db + 8 * (h - 4);
-          const __nv_bfloat16* pv = (const __nv_bfloat16*)&v0[h];
-          uint32_t w[4];
-#pragma unroll
-          for (int z = 0; z < 4; ++z)
-            w[z] = pack_bf16(__bfloat162float(pv[2 * z]) + dv[2 * z],
-                             __bfloat162float(pv[2 * z + 1]) + dv[2 * z + 1]);
-          o[h] = make_uint4(w[0], w[1], w[2], w[3]);
-        }
-      }
-      return true;
-    };
     bool ok = true;
     for (int t = 0; t < T && ok; ++t) {
       const int b = t & 1, p0 = t * kTile;
-      if (t >= 1) fetch_v0(t - 1);
       ok = mbar_wait(&bars->s_full[b], (t >> 1) & 1, abort_flag, kBudget);
       if (ok && t >= 1) ok = mbar_wait(&bars->xg_empty[0], (t - 1) & 1, abort_flag, kBudget);
       if (!ok) break;
       tc_fence_after();
-      const uint32_t sbase = lane_addr + kColS + b * kTile + 64 * wg;
+      const uint32_t sbase = lane_addr + kColS + b * kTile;
       float va[32], vb[32];
       tmem_ld32f(sbase, va);
-      tmem_ld32f(sbase + 32, vb);
       tmem_wait32(va);
-      tmem_wait32(vb);
-      tc_fence_before();
-      mbar_arrive(&bars->s_done[b]);   // S is read
-      const bool masked = p0 + kTile > ng;
-      if (wg == 0) {
-        if (masked) {
-          update_chunk<0, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
-          update_chunk<1, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
-        } else {
-          update_chunk<0, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
-          update_chunk<1, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
-        }
+      tmem_ld32f(sbase + 32, vb);
+      if (p0 + kTile <= ng) {
+        update_chunk<0, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
+        tmem_wait32(vb);
+        tmem_ld32f(sbase + 64, va);
+        update_chunk<1, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        tmem_wait32(va);
+        tmem_ld32f(sbase + 96, vb);
+        update_chunk<2, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
+        tmem_wait32(vb);
+        tc_fence_before();
+        mbar_arrive(&bars->s_done[b]);   // S is fully read
+        update_chunk<3, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
       } else {
-        if (masked) {
-          update_chunk<2, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
-          update_chunk<3, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
-        } else {
-          update_chunk<2, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
-          update_chunk<3, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
-        }
+        update_chunk<0, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
+        tmem_wait32(vb);
+        tmem_ld32f(sbase + 64, va);
+        update_chunk<1, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        tmem_wait32(va);
+        tmem_ld32f(sbase + 96, vb);
+        update_chunk<2, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
+        tmem_wait32(vb);
+        tc_fence_before();
+        mbar_arrive(&bars->s_done[b]);
+        update_chunk<3, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
       }
       fence_proxy_async_smem();
       mbar_arrive(&bars->xg_full[0]);
-      if (t >= 1) ok = epilogue(t - 1);
-    }
-    if (ok && T >= 1) {
-      fetch_v0(T - 1);
-      ok = epilogue(T - 1);
     }
     if (!ok && row == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
+  } else if (warp >= 8) {
+    // epilogue: thread = token (TMEM lane) of D = dV, 128 columns of d
+    const int q = warp & 3, tok = q * 32 + lane;
+    const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
+    const uint4* v_u = (const uint4*)(a.v + (size_t)u * a.n * kD);
+    uint4* vo_u = (uint4*)(a.v_out + (size_t)u * B * kD);
+    bool ok = true;
+    for (int t = 0; t < T && ok; ++t) {
+      const int p = t * kTile + tok;
+      const bool live = p < ng;
+      // V0 row of this position, fetched before D is ready
+      uint4 v0[16];
+      const uint4* g = v_u + (size_t)__ldg(src_u + min(p, B - 1)) * 16;
+#pragma unroll
+      for (int h = 0; h < 16; ++h) v0[h] = __ldg(g + h);
+      const int dst = live ? __ldg(perm_u + p) : 0;
+      ok = mbar_wait(&bars->d_full[t & 1], (t >> 1) & 1, abort_flag, kBudget);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t dcol = lane_addr + kColD + (t & 1) * kD;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        float v[32];
+        tmem_ld32f(dcol + c * 32, v);
+        tmem_wait32(v);
+        if (c == 3) {
+          tc_fence_before();
+          mbar_arrive(&bars->d_empty[t & 1]);
+        }
+        if (live) {
+#pragma unroll
+          for (int h = 0; h < 4; ++h) {
+            const __nv_bfloat16* pv = (const __nv_bfloat16*)&v0[4 * c + h];
+            uint32_t o[4];
+#pragma unroll
+            for (int z = 0; z < 4; ++z)
+              o[z] = pack_bf16(__bfloat162float(pv[2 * z]) + v[8 * h + 2 * z],
+                               __bfloat162float(pv[2 * z + 1]) + v[8 * h + 2 * z + 1]);
+            vo_u[(size_t)dst * 16 + 4 * c + h] = make_uint4(o[0], o[1], o[2], o[3]);
+          }
+        }
+      }
+    }
+    if (!ok && tok == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
     // V_out = V0 for the fixed slots (positions ng .. B-1)
-    for (int p = ng + (tid - 128); p < B; p += 256) {
+    for (int p = ng + tok; p < B; p += 128) {
       const uint4* g = v_u + (size_t)__ldg(src_u + p) * 16;
       uint4* o = vo_u + (size_t)__ldg(perm_u + p) * 16;
 #pragma unroll
@@ -1117,12 +1207,13 @@ bool merge_tc_supported(const Shape& s) {
 size_t merge_tc_ws_bytes(const Shape& s) {
   const size_t U = (size_t)s.U;
   return U * kRows * kD * 4 + U * kRows * kRows * 4 + U * kRows * 4 + 2 * U * (size_t)s.B * 4 +
-         U * 4;
+         2 * U * 4;
 }
 
 cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const void* v,
-                            const float* scores, const float* y, const int32_t* idx, void* k_out,
-                            void* v_out, char* ws, const WsLayout& L, cudaStream_t st) {
+                            const float* scores, const float* y, const float* row_stats,
+                            const int32_t* idx, void* k_out, void* v_out, char* ws,
+                            const WsLayout& L, cudaStream_t st) {
   CUtensorMap mq, mk, mv, mko;
   if (!encode_bf16_3d(&mq, q, kD, s.m, s.U, 64, kRows) ||
       !encode_bf16_2d_rows(&mk, k, kD, (uint64_t)s.U * s.n) ||
@@ -1147,7 +1238,9 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
   a.y = y;
   a.k = (const __nv_bfloat16*)k;
   a.v = (const __nv_bfloat16*)v;
+  a.k_out = (__nv_bfloat16*)k_out;
   a.v_out = (__nv_bfloat16*)v_out;
+  a.rstats = row_stats;
   const size_t U = (size_t)s.U;
   a.rz = (float*)(ws + L.merge_tc);
   a.gram = a.rz + U * kRows * kD;
@@ -1155,6 +1248,7 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
   a.perm = (int32_t*)(a.lam + U * kRows);
   a.src = a.perm + U * s.B;
   a.ng = a.src + U * s.B;
+  a.redo = a.ng + U;
   a.status = (int*)(ws + L.status);
   cudaError_t e;
   if ((e = cudaFuncSetAttribute(k_merge_gram, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1167,10 +1261,18 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
                                 s.B * 4)) != cudaSuccess)
     return e;
   k_merge_fixed<<<s.U, 256, s.B * 4, st>>>(a);
-  k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, mko, a);
+  if (row_stats) {
+    a.gram_mode = 1;
+    k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, mko, a);
+    a.gram_mode = 2;
+    k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, mko, a);
+  } else {
+    a.gram_mode = 0;
+    k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, mko, a);
+  }
   k_merge_solve<<<s.U, 256, kSolveSmem, st>>>(a);
   k_merge_update<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, a);
-  count_launches(4);
+  count_launches(row_stats ? 5 : 4);
   return cudaGetLastError();
 }
 

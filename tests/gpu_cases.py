@@ -117,14 +117,18 @@ def _out_dtype(c: Case):
     return torch.bfloat16 if c.wl.dtype == "bf16" else torch.float32
 
 
-def run_merge(c: Case, p, scores, y, idx, expect_status=b.GRKV_OK):
+def run_merge(c: Case, p, scores, y, idx, expect_status=b.GRKV_OK, row_stats=None):
     ko = torch.empty((c.U, p.budget, 128), dtype=_out_dtype(c), device="cuda")
     vo = torch.empty_like(ko)
     ws = workspace(p)
+    rs = None
+    if row_stats is not None:
+        rs = torch.from_numpy(np.ascontiguousarray(row_stats, np.float32)).cuda()
     b.grkv_merge(p, c.dq, c.dk, c.dv,
                  torch.from_numpy(np.ascontiguousarray(scores, np.float32)).cuda(),
                  torch.from_numpy(np.ascontiguousarray(y, np.float32)).cuda(),
-                 torch.from_numpy(np.ascontiguousarray(idx, np.int32)).cuda(), ko, vo, ws)
+                 torch.from_numpy(np.ascontiguousarray(idx, np.int32)).cuda(), ko, vo, ws,
+                 row_stats=rs)
     assert b.grkv_status(ws) == expect_status
     return to_host(ko), to_host(vo)
 

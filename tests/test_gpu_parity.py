@@ -79,21 +79,63 @@ def test_select_stage_bit_exact(prep):
         np.testing.assert_array_equal(idx[i], ora["idx"])
 
 
+def oracle_row_stats(prep):
+    """[U][m][2] fp32 (M_r, L_r) of the full window attention, as grkv_score writes them."""
+    return np.stack([np.stack([o["row_max"], o["row_sum"]], -1) for o in prep.ora]).astype(np.float32)
+
+
+@pytest.mark.parametrize("stats", [False, True], ids=["two_pass", "row_stats"])
 @pytest.mark.parametrize("path", ["default", "portable"])
-def test_merge_stage(prep, path):
+def test_merge_stage(prep, path, stats):
     c, op = prep.case, prep.op
     scores32 = np.stack([o["scores32"] for o in prep.ora])
     y32 = np.stack([o["y"].astype(np.float32) for o in prep.ora])
     idx = np.stack([o["idx"] for o in prep.ora])
     p = G.lib_params(prep.wl, c.U, **prep.over)
     p.flags = PATHS[path]
-    ko, vo = G.run_merge(c, p, scores32, y32, idx)
+    ko, vo = G.run_merge(c, p, scores32, y32, idx,
+                         row_stats=oracle_row_stats(prep) if stats else None)
     for i in range(c.U):
         ref = O.merge_unit(c.q[i], c.k[i], c.v[i], scores32[i], y32[i], idx[i], op)
         np.testing.assert_array_equal(ko[i], c.k[i][idx[i]])            # K_out = K0
         fixed = ref["fixed"]
         np.testing.assert_array_equal(vo[i][fixed], c.v[i][idx[i]][fixed])  # F rows as V0
         G.assert_values(vo[i], ref["v_out"], c.wl.dtype)
+
+
+def test_merge_row_stats_far_below_full_max_takes_two_passes(grkv_lib):
+    """A key that dominates one window row is left out of the retained set, so
+    the retained maximum of that row lies far (more than 64 in log2 units)
+    below the full-cache maximum given in row_stats: the one-pass Gram would
+    lose that row, and the unit must be recomputed with two passes."""
+    wl = gi.workload(1).replace(units=2, n=2048, budget=256, seed=99)
+    c = G.Case(wl)
+    op = G.oracle_params(wl)
+    row, jstar = 5, 300
+    qr = c.q[0].reshape(op.m, op.d)[row].astype(np.float64)
+    spike = gi.bf16_value(gi.bf16_bits(qr * (3000.0 / float(qr @ qr))))
+    c.k[0][jstar] = spike
+    c.dk = G.to_device(c.k, wl.dtype)
+    ora = [O.compress_unit(c.q[i], c.k[i], c.v[i], op) for i in range(c.U)]
+    idx = np.stack([o["idx"] for o in ora])
+    P = wl.n - wl.window
+    if jstar in idx[0]:
+        keep = [j for j in idx[0][: op.budget - op.window] if j != jstar]
+        extra = next(j for j in range(op.n_sink, P) if j not in set(idx[0]) and j != jstar)
+        idx[0][: op.budget - op.window] = np.sort(np.array(keep + [extra]))
+    assert jstar not in idx[0]
+    lg = O.window_logits(c.q[0], c.k[0], op)
+    gap = (lg[row].max() - lg[row][idx[0]].max()) / math.log(2.0)
+    assert gap > 64.0, gap
+    scores32 = np.stack([o["scores32"] for o in ora])
+    y32 = np.stack([o["y"].astype(np.float32) for o in ora])
+    rs = np.stack([np.stack([o["row_max"], o["row_sum"]], -1) for o in ora]).astype(np.float32)
+    p = G.lib_params(wl, c.U)
+    ko, vo = G.run_merge(c, p, scores32, y32, idx, row_stats=rs)
+    for i in range(c.U):
+        ref = O.merge_unit(c.q[i], c.k[i], c.v[i], scores32[i], y32[i], idx[i], op)
+        np.testing.assert_array_equal(ko[i], c.k[i][idx[i]])
+        G.assert_values(vo[i], ref["v_out"], wl.dtype)
 
 
 def test_compress_end_to_end(prep):
