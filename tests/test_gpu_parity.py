@@ -267,3 +267,45 @@ def test_full_size_c2_sampled_units(grkv_lib):
         np.testing.assert_array_equal(ko[u], ku[idx[u]])
         if swaps == 0:
             G.assert_values(vo[u], ora["v_out"], wl.dtype)
+
+
+def _compress_sampled(wl, units, check_units):
+    """grkv_compress on `units` units of `wl` (full n), sampled units against the oracle."""
+    import torch
+    sub = wl.replace(units=units)
+    q = np.empty((units, sub.group, sub.window, sub.d), np.uint16)
+    k = np.empty((units, sub.n, sub.d), np.uint16)
+    v = np.empty_like(k)
+    gi.fill_units(sub, q, k, v)
+    as_dev = lambda x: torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).cuda()
+    dq, dk, dv = as_dev(q), as_dev(k), as_dev(v)
+    p = G.lib_params(sub, units)
+    ko = torch.empty((units, sub.budget, sub.d), dtype=torch.bfloat16, device="cuda")
+    vo = torch.empty_like(ko)
+    idx = torch.empty((units, sub.budget), dtype=torch.int32, device="cuda")
+    ws = G.workspace(p)
+    b.grkv_compress(p, dq, dk, dv, ko, vo, idx, ws)
+    assert b.grkv_status(ws) == b.GRKV_OK
+    idx, ko, vo = idx.cpu().numpy(), G.to_host(ko), G.to_host(vo)
+    op = G.oracle_params(sub)
+    for u in check_units:
+        qu, ku, vu = gi.unit_arrays(sub, u)
+        ora = O.compress_unit(qu, ku, vu, op)
+        swaps = G.idx_tie_check(idx[u], ora, op, G.score_rel_tol(qu, ku, op))
+        np.testing.assert_array_equal(ko[u], ku[idx[u]])
+        if swaps == 0:
+            G.assert_values(vo[u], ora["v_out"], sub.dtype)
+
+
+def test_full_length_c3_mistral_128k_sampled_units(grkv_lib):
+    """The Mistral-shaped 128K-token workload (m = 256 stacked rows, portable
+    kernels) at its full length on two units."""
+    _compress_sampled(gi.workload(3), 2, (0, 1))
+
+
+@pytest.mark.parametrize("n,budget", [(131072, 2048), (65536, 128)])
+def test_full_length_c4_sweep_points(grkv_lib, n, budget):
+    """Sweep points at 64K and 128K tokens (tensor-core path; the prefix is
+    longer than the shared-memory selection handles) on two units."""
+    wl = next(w for w in gi.sweep_points() if w.n == n and w.budget == budget)
+    _compress_sampled(wl, 2, (0, 1))
