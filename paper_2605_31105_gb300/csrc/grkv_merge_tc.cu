@@ -40,7 +40,8 @@ using namespace sm100;
 
 constexpr int kTile = 128;
 constexpr int kRows = 128;
-constexpr int kThreads = 384;
+constexpr int kThreads = 384;    // k_merge_gram
+constexpr int kThreadsU = 512;   // k_merge_update
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KB
 constexpr int kMaxB = 32768;
 constexpr long long kBudget = 1ll << 32;
@@ -162,7 +163,7 @@ struct Gatherer {
 // ring_empty_count: arrivals that release a ring slot; group_count: threads
 // of the compute warps that arrive on s_done, xg_full and d_empty.
 __device__ __forceinline__ void init_common(MBars* bars, int warp, uint32_t ring_empty_count,
-                                            uint32_t group_count) {
+                                            uint32_t group_count, uint32_t epi_count) {
   if (threadIdx.x == 0) {
     for (int i = 0; i < 4; ++i) {
       mbar_init(&bars->ring_full[i], 2);   // one expect_tx arrival per gathering warp
@@ -175,7 +176,7 @@ __device__ __forceinline__ void init_common(MBars* bars, int warp, uint32_t ring
       mbar_init(&bars->xg_full[i], group_count);
       mbar_init(&bars->xg_empty[i], 1);
       mbar_init(&bars->d_full[i], 1);
-      mbar_init(&bars->d_empty[i], group_count);
+      mbar_init(&bars->d_empty[i], epi_count);
     }
     mbar_init(&bars->acc_done, 1);
     mbar_init(&bars->drain, 1);
@@ -396,7 +397,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const bool single = a.gram_mode == 1;
   const int k0 = single ? T : 0;   // first job
   const int ng = __ldg(a.ng + u);
-  init_common(bars, warp, 2, 128);   // ring slots are released by the MMA and by warp 0
+  init_common(bars, warp, 2, 128, 128);   // ring slots are released by the MMA and by warp 0
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars->tmem;
@@ -989,12 +990,12 @@ __global__ void __launch_bounds__(256, 2) k_merge_solve(MArgs a) {
 }
 
 // ======================================================== k_merge_update
-// Roles (384 threads): warp 0 the Q load, warp 1 MMA issue, warps 2-3 the K0
-// gathers, warps 4-7 the XG rows (one thread per window row), warps 8-11 the
-// output epilogue (one thread per token / TMEM lane of D).  Only the tiles
-// with non-fixed positions are visited; the epilogue warps then copy V0 to
-// the fixed slots.
-__global__ void __launch_bounds__(kThreads, 1)
+// Roles (512 threads): warp 0 the Q load, warp 1 MMA issue, warps 2-3 the K0
+// gathers, warps 4-7 and 12-15 the XG rows (one thread per window row, half
+// of the tile's tokens each), warps 8-11 the output epilogue (one thread per
+// token / TMEM lane of D).  Only the tiles with non-fixed positions are
+// visited; the epilogue warps then copy V0 to the fixed slots.
+__global__ void __launch_bounds__(kThreadsU, 1)
     k_merge_update(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    MArgs a) {
   extern __shared__ __align__(1024) uint8_t smraw[];
@@ -1009,12 +1010,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ng = __ldg(a.ng + u), T = (ng + kTile - 1) / kTile;
   const int32_t* src_u = a.src + (size_t)u * B;
   const int32_t* perm_u = a.perm + (size_t)u * B;
-  init_common(bars, warp, 1, 128);
+  init_common(bars, warp, 1, 256, 128);
   // Z (fp32 [row][d]) to the bf16 B operands Zh, Zl: MN-major tiles of
   // 128-byte rows (d contiguous), two blocks of 64 columns
   {
     const float* Z = a.rz + (size_t)u * kRows * kD;
-    for (int i = tid; i < kRows * (kD / 8); i += kThreads) {
+    for (int i = tid; i < kRows * (kD / 8); i += kThreadsU) {
       const int r = i >> 4, d8 = i & 15;
       const float4 z0 = __ldg((const float4*)(Z + r * kD + d8 * 8));
       const float4 z1 = __ldg((const float4*)(Z + r * kD + d8 * 8 + 4));
@@ -1094,8 +1095,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mma_commit(&bars->drain);
       mbar_wait(&bars->drain, 0, abort_flag, kBudget);
     }
-  } else if (warp >= 4 && warp < 8) {
-    const int q = warp & 3, row = q * 32 + lane;
+  } else if ((warp >= 4 && warp < 8) || warp >= 12) {
+    // two groups (warps 4-7, 12-15) share every tile: group cg computes the
+    // XG rows of tokens 64 cg .. 64 cg + 63 (thread = window row)
+    const int cg = warp >= 12, q = warp & 3, row = q * 32 + lane;
     // rows past m have lam = +inf and give X = 0
     const float lam = a.lam[(size_t)u * kRows + row];
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
@@ -1106,41 +1109,37 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (ok && t >= 1) ok = mbar_wait(&bars->xg_empty[0], (t - 1) & 1, abort_flag, kBudget);
       if (!ok) break;
       tc_fence_after();
-      const uint32_t sbase = lane_addr + kColS + b * kTile;
+      const uint32_t sbase = lane_addr + kColS + b * kTile + 64 * cg;
       float va[32], vb[32];
       tmem_ld32f(sbase, va);
-      tmem_wait32(va);
       tmem_ld32f(sbase + 32, vb);
-      if (p0 + kTile <= ng) {
-        update_chunk<0, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
-        tmem_wait32(vb);
-        tmem_ld32f(sbase + 64, va);
-        update_chunk<1, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
-        tmem_wait32(va);
-        tmem_ld32f(sbase + 96, vb);
-        update_chunk<2, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
-        tmem_wait32(vb);
-        tc_fence_before();
-        mbar_arrive(&bars->s_done[b]);   // S is fully read
-        update_chunk<3, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+      tmem_wait32(va);
+      tmem_wait32(vb);
+      tc_fence_before();
+      mbar_arrive(&bars->s_done[b]);   // S is read
+      const bool masked = p0 + kTile > ng;
+      if (cg == 0) {
+        if (masked) {
+          update_chunk<0, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
+          update_chunk<1, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        } else {
+          update_chunk<0, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
+          update_chunk<1, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        }
       } else {
-        update_chunk<0, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
-        tmem_wait32(vb);
-        tmem_ld32f(sbase + 64, va);
-        update_chunk<1, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
-        tmem_wait32(va);
-        tmem_ld32f(sbase + 96, vb);
-        update_chunk<2, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
-        tmem_wait32(vb);
-        tc_fence_before();
-        mbar_arrive(&bars->s_done[b]);
-        update_chunk<3, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        if (masked) {
+          update_chunk<2, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
+          update_chunk<3, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        } else {
+          update_chunk<2, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
+          update_chunk<3, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+        }
       }
       fence_proxy_async_smem();
       mbar_arrive(&bars->xg_full[0]);
     }
-    if (!ok && row == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
-  } else if (warp >= 8) {
+    if (!ok && row == 0 && cg == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
+  } else if (warp >= 8 && warp < 12) {
     // epilogue: thread = token (TMEM lane) of D = dV, 128 columns of d
     const int q = warp & 3, tok = q * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
@@ -1271,7 +1270,7 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
     k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, mko, a);
   }
   k_merge_solve<<<s.U, 256, kSolveSmem, st>>>(a);
-  k_merge_update<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, a);
+  k_merge_update<<<s.U, kThreadsU, kSmemBytes, st>>>(mq, mk, a);
   count_launches(row_stats ? 5 : 4);
   return cudaGetLastError();
 }
