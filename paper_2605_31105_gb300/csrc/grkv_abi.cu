@@ -125,8 +125,7 @@ WsLayout plan_workspace(const Shape& s) {
   if (s.tc) {
     int maxc, gu, rounds;
     L.pstats_tc = take(score_tc_pstats_bytes(s, &maxc, &gu, &rounds, kMaxScoreCtas));
-    L.ustats_tc = take(U * 128 * sizeof(float2));
-    L.flags_tc = take(2 * U * sizeof(int));
+    L.flags_tc = take(U * sizeof(int));
   } else {
     L.pstats = take(U * L.nchunk * m * 8);
     L.ypart = take(U * L.nchunk * m * d * 4);

@@ -36,9 +36,8 @@ struct WsLayout {
   size_t ypart;   // float  [U][nchunk][m][d]   per-chunk target partials
   int chunk, nchunk;
   // score path (tensor cores)
-  size_t pstats_tc;  // float2 [U][maxc][2][128] pass-A statistics slots
-  size_t ustats_tc;  // float2 [U][128] combined pass-A statistics per unit
-  size_t flags_tc;   // int [2][U] slots written / statistics ready per unit
+  size_t pstats_tc;  // float2 [U][maxc][128] pass-A statistics slots
+  size_t flags_tc;   // int [U] pass-A slots written per unit
   // select
   size_t pooled;  // float [U][P]
   // merge

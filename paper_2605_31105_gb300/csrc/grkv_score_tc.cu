@@ -39,20 +39,27 @@ using namespace sm100;
 
 constexpr int kTile = 128;            // tokens per tile
 constexpr int kRows = 128;            // window rows (m padded to 128)
-constexpr int kRing = 5;              // K / V ring slots
-constexpr int kQBuf = 1;              // Q buffers (one per unit segment in flight)
 constexpr int kThreads = 512;
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KB
 constexpr long long kWaitBudget = 1ll << 32;      // cycles (~2 s) before a wait gives up
 
-// Shared-memory layout (offsets from a 1024-byte aligned base).
-constexpr uint32_t kOffQ = 0;                                   // kQBuf x 32 KB
-constexpr uint32_t kOffRing = kOffQ + kQBuf * kTileBytes;       // kRing x 32 KB
-constexpr uint32_t kOffRed = kOffRing + kRing * kTileBytes;     // [2 wg][2 buf][4][128] fp32
-constexpr uint32_t kOffAstat = kOffRed + 2 * 2 * 4 * kTile * 4;   // [2 buf][2 wg][128] float2
-constexpr uint32_t kOffLam = kOffAstat + 2 * 2 * kRows * 8;       // [2 buf][128] float
-constexpr uint32_t kOffBar = kOffLam + 2 * kRows * 4;
-constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;           // + alignment slack
+// Shared-memory layout (offsets from a 1024-byte aligned base) for kRing K/V
+// ring slots and kQBuf Q tiles.  The two-launch passes use 5 + 1: a CTA
+// switches units two or three times per launch.  The fused rounds use 4 + 2:
+// a CTA switches units every few tiles, and with two Q tiles the next
+// segment's Q is loaded while the current segment finishes.
+template <int kRing, int kQBuf>
+struct Layout {
+  static constexpr uint32_t kOffQ = 0;                                 // kQBuf x 32 KB
+  static constexpr uint32_t kOffRing = kOffQ + kQBuf * kTileBytes;     // kRing x 32 KB
+  static constexpr uint32_t kOffRed = kOffRing + kRing * kTileBytes;   // [2 wg][2 buf][4][128] fp32
+  static constexpr uint32_t kOffAstat = kOffRed + 2 * 2 * 4 * kTile * 4;   // [2 buf][2 wg][128] float2
+  static constexpr uint32_t kOffLam = kOffAstat + 2 * 2 * kRows * 8;       // [2 buf][128] float
+  static constexpr uint32_t kOffBar = kOffLam + 2 * kRows * 4;
+  static constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;         // + alignment slack
+};
+constexpr int kRingTwo = 5, kQBufTwo = 1;       // modes 0 and 1
+constexpr int kRingFused = 4, kQBufFused = 2;   // mode 2
 
 // TMEM columns: two S buffers, two Y accumulators.
 constexpr uint32_t kColS = 0, kColY = 256;
@@ -68,10 +75,8 @@ struct Args {
   float* scores;  // [U][P]
   float* y;       // [U][m][128], zeroed by the host
   float* row_stats;  // [U][m][2]
-  float2* pstats;    // [U][maxc][2][128]  (max in log2 units, sum)
-  float2* ustats;    // [U][128] combined statistics of each unit (log2 units)
+  float2* pstats;    // [U][maxc][128]  (max in log2 units, sum)
   int* unit_cnt;     // [U] pass-A slots written, zeroed by the host
-  int* unit_ready;   // [U] 1 once ustats of the unit is in place, zeroed by the host
   int* status;
 };
 
@@ -111,11 +116,16 @@ struct Sched {
     const int r = u / gu;
     return owner(r, (long long)(u - r * gu) * tpu);
   }
-  // True if CTA c holds no tile of round r (more CTAs than tiles).
-  __device__ bool empty(int r, int c) const { return start(r, c) == start(r, c + 1); }
+  // True if CTA c holds no tile of round r (only when the round has fewer
+  // tiles than there are CTAs).
+  __device__ bool empty(int r, int c) const {
+    return tiles(r) < G && start(r, c) == start(r, c + 1);
+  }
   // Pass-A statistics slots written for unit u (one per CTA that holds its tiles).
   __device__ int writers(int u) const {
-    const int r = u / gu, c0 = first_cta(u), ns = nslots(u);
+    const int r = u / gu, ns = nslots(u);
+    if (tiles(r) >= G) return ns;
+    const int c0 = first_cta(u);
     int w = 0;
     for (int k = 0; k < ns; ++k) w += empty(r, c0 + k) ? 0 : 1;
     return w;
@@ -151,7 +161,8 @@ struct JobIter {
     Job j;
     j.kind = kind;
     j.r = r;
-    const int lu = (int)(t / sc->tpu), ti = (int)(t % sc->tpu);
+    // round-local tile indices stay below U * tiles per unit, well inside int
+    const int lu = (int)t / sc->tpu, ti = (int)t - lu * sc->tpu;
     j.u = r * sc->gu + lu;
     j.j0 = ti * kTile;
     j.len = min(kTile, n - j.j0);
@@ -206,6 +217,7 @@ __device__ __forceinline__ int ld_acquire(const int* p) {
 // has already read).
 __device__ __forceinline__ uint32_t p_col(int kk) { return kk < 4 ? kk * 8 : 64 + (kk - 4) * 8; }
 
+template <int kRing, int kQBuf>
 struct Bars {
   uint64_t ring_full[kRing], ring_empty[kRing];
   uint64_t q_full[kQBuf], q_empty[kQBuf];
@@ -217,14 +229,28 @@ struct Bars {
   uint32_t tmem;
   int abort;
 };
-static_assert(sizeof(Bars) <= 256, "barrier block");
+static_assert(sizeof(Bars<kRingTwo, kQBufTwo>) <= 256 &&
+                  sizeof(Bars<kRingFused, kQBufFused>) <= 256,
+              "barrier block");
 
+// Merges two (max, sum) row statistics in log2 units.
+__device__ __forceinline__ float2 stat_merge(float2 x, float2 y) {
+  if (x.x == -INFINITY) return y;
+  if (y.x == -INFINITY) return x;
+  const float M = fmaxf(x.x, y.x);
+  return make_float2(M, x.y * fast_exp2(x.x - M) + y.y * fast_exp2(y.x - M));
+}
+
+template <int kRing, int kQBuf>
 __global__ void __launch_bounds__(kThreads, 1)
     k_score_tc(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                const __grid_constant__ CUtensorMap tmV, Args a) {
+  using Lay = Layout<kRing, kQBuf>;
+  constexpr uint32_t kOffQ = Lay::kOffQ, kOffRing = Lay::kOffRing, kOffRed = Lay::kOffRed,
+                     kOffAstat = Lay::kOffAstat, kOffLam = Lay::kOffLam, kOffBar = Lay::kOffBar;
   extern __shared__ __align__(1024) uint8_t smraw[];
   uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
-  Bars* bars = (Bars*)(sm + kOffBar);
+  Bars<kRing, kQBuf>* bars = (Bars<kRing, kQBuf>*)(sm + kOffBar);
   float* red = (float*)(sm + kOffRed);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
@@ -442,8 +468,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 2) {
     // ----------------------------------------------- statistics publisher
-    // Copies each pass-A segment's row statistics to its global slot; the
-    // unit's last writer combines all slots once and raises its ready flag.
+    // Merges the two compute groups' row statistics of each pass-A segment
+    // into the segment's global slot, then counts the slot as written.
     float2* astat = (float2*)(sm + kOffAstat);
     JobIter it;
     it.init(&sc, a.n);
@@ -459,73 +485,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int k = (int)blockIdx.x - sc.first_cta(j.u);
         // k < maxc always holds (the host sizes maxc from the same partition)
         if (k >= 0 && k < a.maxc) {
-          float2* slot = a.pstats + ((size_t)j.u * a.maxc + k) * 2 * kRows;
+          float2* slot = a.pstats + ((size_t)j.u * a.maxc + k) * kRows;
 #pragma unroll
-          for (int t = 0; t < 8; ++t) slot[t * 32 + lane] = astat[ab * 2 * kRows + t * 32 + lane];
+          for (int t = 0; t < 4; ++t) {
+            const int r = t * 32 + lane;
+            slot[r] = stat_merge(astat[(ab * 2 + 0) * kRows + r], astat[(ab * 2 + 1) * kRows + r]);
+          }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars->astat_empty[ab]);
         __threadfence();
         __syncwarp();
-        int last = 0;
-        if (lane == 0) last = atomicAdd(&a.unit_cnt[j.u], 1) == sc.writers(j.u) - 1;
-        last = __shfl_sync(0xffffffffu, last, 0);
-        if (last) {
-          __threadfence();
-          const int ns = sc.nslots(j.u), c0 = sc.first_cta(j.u);
-          float Mr[4], Lr[4];
-#pragma unroll
-          for (int t = 0; t < 4; ++t) {
-            Mr[t] = -INFINITY;
-            Lr[t] = 0.f;
-          }
-          // four slots per round trip: 32 independent loads in flight per lane
-          for (int k0 = 0; k0 < ns; k0 += 4) {
-            float2 pr[4][8];
-#pragma unroll
-            for (int kk = 0; kk < 4; ++kk) {
-              const bool use = k0 + kk < ns && !sc.empty(j.r, c0 + k0 + kk);
-              const float2* sl = a.pstats + ((size_t)j.u * a.maxc + k0 + kk) * 2 * kRows;
-#pragma unroll
-              for (int t = 0; t < 8; ++t)
-                pr[kk][t] = use ? sl[(t & 1) * kRows + (t >> 1) * 32 + lane]
-                                : make_float2(-INFINITY, 0.f);
-            }
-#pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-#pragma unroll
-              for (int t = 0; t < 8; ++t) {
-                const int rr = t >> 1;
-                const float2 v = pr[kk][t];
-                if (v.x == -INFINITY) continue;
-                if (v.x > Mr[rr]) {
-                  Lr[rr] = Lr[rr] * fast_exp2(Mr[rr] - v.x) + v.y;
-                  Mr[rr] = v.x;
-                } else {
-                  Lr[rr] += v.y * fast_exp2(v.x - Mr[rr]);
-                }
-              }
-          }
-#pragma unroll
-          for (int t = 0; t < 4; ++t) {
-            const int r = t * 32 + lane;
-            a.ustats[(size_t)j.u * kRows + r] = make_float2(Mr[t], Lr[t]);
-            if (r < a.m) {
-              a.row_stats[((size_t)j.u * a.m + r) * 2 + 0] = Mr[t] * 0.69314718055994531f;
-              a.row_stats[((size_t)j.u * a.m + r) * 2 + 1] = Lr[t];
-            }
-          }
-          __threadfence();
-          __syncwarp();
-          if (lane == 0) atomicExch(&a.unit_ready[j.u], 1);
-        }
+        if (lane == 0) atomicAdd(&a.unit_cnt[j.u], 1);
         ++aseg;
       }
     }
   } else if (warp == 3) {
     // ------------------------------------------------ statistics fetcher
-    // Ahead of each pass-B segment: wait for the unit's combined statistics
-    // and leave every row's log2 normaliser in shared memory.
+    // Ahead of each pass-B segment: wait until every pass-A slot of the unit
+    // is written, combine the slots, and leave every row's log2 normaliser in
+    // shared memory.  The CTA that holds the unit's first tile also writes
+    // the unit's row statistics.
     float* lam_s = (float*)(sm + kOffLam);
     JobIter it;
     it.init(&sc, a.n);
@@ -539,8 +519,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (bseg >= 2)
           ok = mbar_wait(&bars->lam_empty[lb], ((bseg >> 1) - 1) & 1, abort_flag, kWaitBudget);
         if (!ok) break;
+        const int need = sc.writers(j.u);
         const long long t0 = clock64();
-        while (ld_acquire(&a.unit_ready[j.u]) == 0) {
+        while (ld_acquire(&a.unit_cnt[j.u]) < need) {
           if (*abort_flag || clock64() - t0 > kWaitBudget) {
             *abort_flag = 1;
             ok = false;
@@ -548,11 +529,36 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         if (!ok) break;
+        const int ns = sc.nslots(j.u), c0 = sc.first_cta(j.u);
+        const bool dense = sc.tiles(j.r) >= sc.G;   // every CTA holds tiles of the round
+        float2 st[4];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) st[t] = make_float2(-INFINITY, 0.f);
+        // eight slots per round trip: 32 independent loads in flight per lane
+        for (int k0 = 0; k0 < ns; k0 += 8) {
+          float2 pr[8][4];
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) {
+            const bool use = k0 + kk < ns && (dense || !sc.empty(j.r, c0 + k0 + kk));
+            const float2* sl = a.pstats + ((size_t)j.u * a.maxc + k0 + kk) * kRows;
+#pragma unroll
+            for (int t = 0; t < 4; ++t)
+              pr[kk][t] = use ? __ldcg(sl + t * 32 + lane) : make_float2(-INFINITY, 0.f);
+          }
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk)
+#pragma unroll
+            for (int t = 0; t < 4; ++t) st[t] = stat_merge(st[t], pr[kk][t]);
+        }
+        const bool first = (int)blockIdx.x == c0;
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
           const int r = t * 32 + lane;
-          const float2 st = a.ustats[(size_t)j.u * kRows + r];
-          lam_s[lb * kRows + r] = (r < a.m && st.y > 0.f) ? st.x + __log2f(st.y) : INFINITY;
+          lam_s[lb * kRows + r] = (r < a.m && st[t].y > 0.f) ? st[t].x + __log2f(st[t].y) : INFINITY;
+          if (first && r < a.m) {
+            a.row_stats[((size_t)j.u * a.m + r) * 2 + 0] = st[t].x * 0.69314718055994531f;
+            a.row_stats[((size_t)j.u * a.m + r) * 2 + 1] = st[t].y;
+          }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&bars->lam_full[lb]);
@@ -736,7 +742,7 @@ size_t score_tc_pstats_bytes(const Shape& s, int* maxc, int* gu, int* rounds, in
   *maxc = mc;
   *gu = g;
   *rounds = R;
-  return (size_t)s.U * mc * 2 * kRows * sizeof(float2);
+  return (size_t)s.U * mc * kRows * sizeof(float2);
 }
 
 int sm_count() {
@@ -776,15 +782,11 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
   a.y = y;
   a.row_stats = row_stats;
   a.pstats = (float2*)(ws + L.pstats_tc);
-  a.ustats = (float2*)(ws + L.ustats_tc);
   a.unit_cnt = (int*)(ws + L.flags_tc);
-  a.unit_ready = a.unit_cnt + s.U;
   a.status = (int*)(ws + L.status);
   cudaError_t e = cudaMemsetAsync(y, 0, (size_t)s.U * s.m * kD * sizeof(float), st);
   if (e != cudaSuccess) return e;
-  e = cudaMemsetAsync(a.unit_cnt, 0, (size_t)2 * s.U * sizeof(int), st);
-  if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(k_score_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+  e = cudaMemsetAsync(a.unit_cnt, 0, (size_t)s.U * sizeof(int), st);
   if (e != cudaSuccess) return e;
   auto launch = [&](int md) {
     a.mode = md;
@@ -795,10 +797,15 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
       a.gu = gu;
       a.rounds = rounds;
     }
+    auto kern = md == 2 ? k_score_tc<kRingFused, kQBufFused> : k_score_tc<kRingTwo, kQBufTwo>;
+    const uint32_t smem = md == 2 ? Layout<kRingFused, kQBufFused>::kSmemBytes
+                                  : Layout<kRingTwo, kQBufTwo>::kSmemBytes;
+    cudaError_t fe = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (fe != cudaSuccess) return fe;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(G);
     cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = kSmemBytes;
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeCooperative;
@@ -806,7 +813,7 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     count_launches(1);
-    return cudaLaunchKernelEx(&cfg, k_score_tc, mq, mk, mv, a);
+    return cudaLaunchKernelEx(&cfg, kern, mq, mk, mv, a);
   };
   if (mode == 2) return launch(2);
   e = launch(0);

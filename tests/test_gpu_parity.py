@@ -211,6 +211,24 @@ def test_select_long_prefixes(grkv_lib, n, pool):
         np.testing.assert_array_equal(idx[i], O.select(O.pool(s[i], op), op))
 
 
+@pytest.mark.parametrize("path", ["default", "portable"])
+def test_merge_reports_out_of_range_idx(grkv_lib, path):
+    """An idx entry outside [0, n) is reported as GRKV_ERR_INVALID_ARG in the
+    device status and read as position 0 (no out-of-bounds access)."""
+    wl = gi.workload(1).replace(units=2, n=2048, budget=256, seed=7)
+    c = G.Case(wl)
+    op = G.oracle_params(wl)
+    ora = [O.compress_unit(c.q[i], c.k[i], c.v[i], op) for i in range(c.U)]
+    idx = np.stack([o["idx"] for o in ora]).astype(np.int32)
+    idx[0][10] = wl.n + 5
+    idx[1][3] = -1
+    scores32 = np.stack([o["scores32"] for o in ora])
+    y32 = np.stack([o["y"].astype(np.float32) for o in ora])
+    p = G.lib_params(wl, c.U)
+    p.flags = PATHS[path]
+    G.run_merge(c, p, scores32, y32, idx, expect_status=b.GRKV_ERR_INVALID_ARG)
+
+
 def test_zero_units_is_a_no_op(grkv_lib):
     import torch
     p = b.params(0, 4, 1024, 32, 128)
