@@ -12,7 +12,7 @@
 // units (modes 0 and 1), which reads K twice but needs no cross-CTA waits.
 //
 // Roles (512 threads): warp 0 issues TMA loads (the unit's Q, then K and V
-// tiles of 128 tokens through a 5-slot ring; each V one job after its K, as
+// tiles of 128 tokens through the ring; each V one job after its K, as
 // it stays in the ring through the tile's compute), warp 1 issues tcgen05
 // MMAs (S = Q K^T into TMEM; Y += P V with P read from TMEM), warps 4-7 and
 // 8-11 are two compute groups that share every tile, tokens 0..63 and
@@ -20,11 +20,11 @@
 // keeps its running max / sum in registers, pass B writes exp2(l - Lambda_r)
 // back into TMEM as bf16 (the A operand of the Y MMA) and sums probabilities
 // over rows with a warp transpose-reduction plus a 4-way shared-memory sum.
-// Warp 2 publishes per-segment statistics (the unit's last writer combines
-// them), warp 3 fetches a unit's combined statistics ahead of its pass-B
-// segments, warps 12-15 add each segment's Y partial to the unit's Y with
-// float4 atomics.  Per-unit statistics of the CTAs that share a unit meet in
-// a global slot array; pass B of round r waits (bounded) for them.
+// Warp 2 merges the two groups' statistics of each pass-A segment into the
+// segment's global slot and counts it; warp 3, ahead of each pass-B segment,
+// waits (bounded) until all of the unit's slots are counted and combines
+// them; warps 12-15 add each segment's Y partial to the unit's Y with float4
+// atomics.
 #include <algorithm>
 #include <cmath>
 
