@@ -42,7 +42,8 @@ import scipy.linalg
 __all__ = [
     "Params", "effective_scale", "window_logits", "softmax_rows", "window_attention",
     "target", "column_scores", "pool", "select", "fixed_set", "retained_attention",
-    "value_step_dual", "value_step_primal", "merge_unit", "compress_unit",
+    "value_step_dual", "value_step_primal", "key_jvp", "key_vjp", "key_step_dual",
+    "merge_unit", "compress_unit",
 ]
 
 f64 = np.float64
@@ -62,6 +63,9 @@ class Params:
     lambda_v: float = 1e-2
     scale: float = 0.0            # 0 -> fp32(1/sqrt(d))
     causal: bool = True
+    update_k: bool = False        # also run the key step (App. D.2)
+    lambda_k: float = 1e-2
+    cg_iters: int = 16            # conjugate-gradient iterations of the key step
 
     @property
     def m(self) -> int:
@@ -212,11 +216,81 @@ def value_step_primal(X, Y, V0, free, lam: float):
     return out
 
 
+def key_jvp(X, Q, V, dK, s: float):
+    """Directional derivative of f(K) = softmax(s Q K^T) V at the K whose
+    (masked) retained attention is X, in direction dK (App. D.2, the
+    Jacobian-vector product J[dK]):
+        dS = s Q dK^T,  dA = X o (dS - rowsum(X o dS)),  df = dA V.
+    Masked entries have X = 0 and contribute nothing."""
+    X = np.asarray(X, dtype=f64)
+    dS = s * (np.asarray(Q, dtype=f64) @ np.asarray(dK, dtype=f64).T)
+    dA = X * (dS - (X * dS).sum(axis=1, keepdims=True))
+    return dA @ np.asarray(V, dtype=f64)
+
+
+def key_vjp(X, Q, V, W, s: float):
+    """Adjoint of `key_jvp` (App. D.2, the vector-Jacobian product J^T[W]):
+        dA = W V^T,  dS = X o (dA - rowsum(X o dA)),  dK = s dS^T Q."""
+    X = np.asarray(X, dtype=f64)
+    dA = np.asarray(W, dtype=f64) @ np.asarray(V, dtype=f64).T
+    dS = X * (dA - (X * dA).sum(axis=1, keepdims=True))
+    return s * (dS.T @ np.asarray(Q, dtype=f64))
+
+
+def key_step_dual(X, Q, K0, V, Y, free, lam: float, s: float, iters: int):
+    """Key step of Algorithm 1 at t = 0 (K = K0, so G = K - K0 = 0) in its
+    linearised dual form (Sec. 3.4 'Key step', App. D.2):
+        E = Y - f(K0) = Y - X V,  e = vec(E)
+        alpha = (J_G J_G^T + lambda_k I)^-1 e         (conjugate gradients)
+        K*_G = K0_G + unvec(J_G^T alpha),  K*_F = K0_F
+    J_G is the Jacobian of f with respect to the free rows only; the operator
+    alpha -> J_G (J_G^T alpha) + lambda alpha is applied matrix-free (JVP of
+    the VJP), as the paper does.  CG starts from alpha = 0 and runs `iters`
+    iterations (fewer only once the residual or the search direction
+    vanishes); returns K* and the residual norms ||r_t|| of every iteration."""
+    X = np.asarray(X, dtype=f64)
+    V = np.asarray(V, dtype=f64)
+    K0 = np.asarray(K0, dtype=f64)
+    free = np.asarray(free, dtype=bool)
+
+    def jt(W):
+        dK = key_vjp(X, Q, V, W, s)
+        dK[~free] = 0.0
+        return dK
+
+    def op(a):
+        return key_jvp(X, Q, V, jt(a), s) + lam * a
+
+    E = np.asarray(Y, dtype=f64) - X @ V
+    alpha = np.zeros_like(E)
+    r = E.copy()
+    pdir = r.copy()
+    rs = float((r * r).sum())
+    hist = [math.sqrt(rs)]
+    for _ in range(iters):
+        if rs == 0.0:
+            break
+        Ap = op(pdir)
+        pAp = float((pdir * Ap).sum())
+        if not pAp > 0.0:       # the direction has vanished: converged
+            break
+        a = rs / pAp
+        alpha += a * pdir
+        r -= a * Ap
+        rs_new = float((r * r).sum())
+        hist.append(math.sqrt(rs_new))
+        pdir = r + (rs_new / rs) * pdir
+        rs = rs_new
+    K = K0.copy()
+    K[free] = K0[free] + jt(alpha)[free]
+    return K, hist
+
+
 def merge_unit(q, k, v, c32, y, idx, p: Params, mode: str = "dual"):
-    """Algorithm 1 at S = 1 with the value step only (the key step is not
-    applied, so K_out = K_Ret^0): gather, fixed set, retained attention,
-    value step.  Inputs are the fp32 prefix scores c32 and the target y
-    (as the library's grkv_merge receives them) and the retained idx."""
+    """Algorithm 1 at S = 1: gather, fixed set, retained attention, value
+    step, then (p.update_k) the key step against the merged values; without
+    it K_out = K_Ret^0.  Inputs are the fp32 prefix scores c32 and the target
+    y (as the library's grkv_merge receives them) and the retained idx."""
     idx = np.asarray(idx)
     K0 = np.asarray(k, dtype=f64)[idx]
     V0 = np.asarray(v, dtype=f64)[idx]
@@ -227,7 +301,14 @@ def merge_unit(q, k, v, c32, y, idx, p: Params, mode: str = "dual"):
     else:
         step = value_step_dual if mode == "dual" else value_step_primal
         V = step(X, y, V0, ~fixed, f64(np.float32(p.lambda_v)))
-    return {"k_out": K0, "v_out": V, "fixed": fixed, "x": X}
+    out = {"k_out": K0, "v_out": V, "fixed": fixed, "x": X}
+    if p.update_k:
+        Q = np.asarray(q, dtype=f64).reshape(p.m, p.d)
+        K, hist = key_step_dual(X, Q, K0, V, y, ~fixed, f64(np.float32(p.lambda_k)),
+                                effective_scale(p), p.cg_iters)
+        out["k_out"] = K
+        out["cg_residuals"] = hist
+    return out
 
 
 def compress_unit(q, k, v, p: Params, mode: str = "dual", idx=None):

@@ -312,3 +312,126 @@ def test_compress_unit_structure():
     # lambda = inf: values unchanged
     pinf = O.Params(group=g, n=n, d=d, window=w, budget=B, lambda_v=math.inf)
     np.testing.assert_array_equal(O.compress_unit(q, k, v, pinf)["v_out"], v[idx])
+
+
+# ------------------------------------------------------------- key step (NEXT)
+def _key_case(rng, g=2, w=2, n=9, d=3, causal=True):
+    """A tiny unit with its retained attention X at K0 and merged values V."""
+    q, k, v = _rand_unit(rng, g, w, n, d, peaked=False)
+    p = O.Params(group=g, n=n, d=d, window=w, budget=n - 2, causal=causal, update_k=True)
+    idx = np.sort(rng.choice(n - w, size=n - 2 - w, replace=False))
+    idx = np.concatenate([idx, np.arange(n - w, n)])
+    K0 = k[idx]
+    V = rng.standard_normal((idx.size, d))
+    X = O.retained_attention(q, k, idx, p)
+    Y = rng.standard_normal((p.m, d))
+    return p, q.reshape(p.m, d), K0, V, X, Y, idx
+
+
+def _autograd_jacobian(p, Q, K0, V, idx):
+    """d vec(f)/d vec(K) of f(K) = softmax(s Q K^T + causal mask) V, by torch
+    autograd in fp64 (row-major vec); independent of the oracle's JVP/VJP."""
+    s = O.effective_scale(p)
+    a = np.arange(p.m) % p.window
+    mask = np.asarray(idx)[None, :] <= (p.n - p.window + a)[:, None] if p.causal else np.ones((p.m, len(idx)), bool)
+    Qt, Vt = torch.from_numpy(Q), torch.from_numpy(V)
+    bias = torch.from_numpy(np.where(mask, 0.0, -np.inf))
+
+    def f(Kflat):
+        K = Kflat.reshape(K0.shape)
+        return (torch.softmax(s * Qt @ K.T + bias, dim=1) @ Vt).reshape(-1)
+
+    return torch.autograd.functional.jacobian(f, torch.from_numpy(K0.reshape(-1))).numpy()
+
+
+@pytest.mark.parametrize("causal", [True, False])
+def test_key_jvp_vjp_match_autograd(causal):
+    rng = np.random.default_rng(71 + causal)
+    p, Q, K0, V, X, Y, idx = _key_case(rng, causal=causal)
+    J = _autograd_jacobian(p, Q, K0, V, idx)
+    s = O.effective_scale(p)
+    dK = rng.standard_normal(K0.shape)
+    W = rng.standard_normal((p.m, p.d))
+    np.testing.assert_allclose(O.key_jvp(X, Q, V, dK, s).reshape(-1), J @ dK.reshape(-1),
+                               rtol=0, atol=1e-13)
+    np.testing.assert_allclose(O.key_vjp(X, Q, V, W, s).reshape(-1), J.T @ W.reshape(-1),
+                               rtol=0, atol=1e-13)
+
+
+@pytest.mark.parametrize("lam", [1e-2, 1e-1, 3.0])
+def test_key_step_matches_dense_ridge(lam):
+    """Full CG (md iterations) reaches the linearised ridge solution of App.
+    D.2, computed densely in both forms from the autograd Jacobian:
+    primal (J_G^T J_G + lam I) z = J_G^T e and dual J_G^T (J_G J_G^T + lam I)^-1 e."""
+    rng = np.random.default_rng(int(lam * 1000) + 5)
+    p, Q, K0, V, X, Y, idx = _key_case(rng)
+    free = np.ones(idx.size, bool)
+    free[[0, idx.size - 1]] = False
+    J = _autograd_jacobian(p, Q, K0, V, idx)
+    cols = np.repeat(free, p.d)                       # row-major vec(K): row i -> d entries
+    JG = J[:, cols]
+    e = (Y - X @ V).reshape(-1)
+    z_primal = np.linalg.solve(JG.T @ JG + lam * np.eye(JG.shape[1]), JG.T @ e)
+    z_dual = JG.T @ np.linalg.solve(JG @ JG.T + lam * np.eye(JG.shape[0]), e)
+    np.testing.assert_allclose(z_dual, z_primal, rtol=0, atol=1e-10)
+    # CG reaches the solution in md steps in exact arithmetic; in fp64 at small
+    # lambda the lost orthogonality needs a few times more
+    K, hist = O.key_step_dual(X, Q, K0, V, Y, free, lam, O.effective_scale(p), iters=20 * p.m * p.d)
+    want = K0.copy()
+    want[free] = K0[free] + z_primal.reshape(-1, p.d)
+    np.testing.assert_allclose(K, want, rtol=0, atol=1e-9)
+    assert hist[-1] <= 1e-9 * hist[0]
+    assert np.array_equal(K[~free], K0[~free])
+
+
+def test_key_step_large_lambda_leaves_keys():
+    rng = np.random.default_rng(9)
+    p, Q, K0, V, X, Y, idx = _key_case(rng)
+    free = np.ones(idx.size, bool)
+    s = O.effective_scale(p)
+    lam = 1e8
+    K, _ = O.key_step_dual(X, Q, K0, V, Y, free, lam, s, iters=p.m * p.d)
+    bound = np.linalg.norm(O.key_vjp(X, Q, V, Y - X @ V, s)) / lam
+    assert np.linalg.norm(K - K0) <= 1.0001 * bound
+
+
+def test_key_step_stationarity():
+    """z = K* - K0 solves J_G^T (J_G z - e) + lam z = 0 (normal equation of
+    the local ridge problem), with J applied through autograd."""
+    rng = np.random.default_rng(13)
+    p, Q, K0, V, X, Y, idx = _key_case(rng, g=1, w=3, n=10, d=4)
+    free = np.ones(idx.size, bool)
+    free[1] = False
+    lam = 0.05
+    K, _ = O.key_step_dual(X, Q, K0, V, Y, free, lam, O.effective_scale(p), iters=20 * p.m * p.d)
+    J = _autograd_jacobian(p, Q, K0, V, idx)[:, np.repeat(free, p.d)]
+    z = (K - K0)[free].reshape(-1)
+    e = (Y - X @ V).reshape(-1)
+    g = J.T @ (J @ z - e) + lam * z
+    assert np.abs(g).max() <= 1e-10 * max(1.0, np.abs(J.T @ e).max())
+
+
+def test_merge_unit_key_step_uses_merged_values():
+    """With update_k the key step linearises f around K0 with the merged
+    values V* of the value step, and keeps fixed rows (Algorithm 1)."""
+    rng = np.random.default_rng(21)
+    g, w, n, d = 2, 3, 24, 8
+    q, k, v = _rand_unit(rng, g, w, n, d)
+    p = O.Params(group=g, n=n, d=d, window=w, budget=12, n_sink=2, beta=0.2, update_k=True,
+                 lambda_k=0.05, cg_iters=g * w * d)
+    base = O.compress_unit(q, k, v, dataclasses_replace(p, update_k=False))
+    out = O.compress_unit(q, k, v, p)
+    np.testing.assert_array_equal(out["idx"], base["idx"])
+    np.testing.assert_array_equal(out["v_out"], base["v_out"])
+    K0 = np.asarray(k, dtype=np.float64)[out["idx"]]
+    Q = np.asarray(q, dtype=np.float64).reshape(p.m, d)
+    want, _ = O.key_step_dual(out["x"], Q, K0, out["v_out"], out["y"], ~out["fixed"],
+                              np.float64(np.float32(p.lambda_k)), O.effective_scale(p), p.cg_iters)
+    np.testing.assert_array_equal(out["k_out"], want)
+    assert np.array_equal(out["k_out"][out["fixed"]], K0[out["fixed"]])
+    assert np.abs(out["k_out"] - K0).max() > 0
+
+
+def dataclasses_replace(p, **kw):
+    import dataclasses
+    return dataclasses.replace(p, **kw)
