@@ -67,7 +67,15 @@ extern "C" {
 #define GRKV_POOL_MAX 0
 #define GRKV_POOL_AVG 1
 
-#define GRKV_UPDATE_K      0x1u  /* key step (Sec. 3.4, Eq. key_dual_update): not implemented */
+#define GRKV_UPDATE_K      0x1u  /* grkv_merge / grkv_compress also run the key step of
+                                    Algorithm 1 at t = 0 (Sec. 3.4 "Key step", App. D.2):
+                                    with the merged values V* fixed, alpha = (J_G J_G^T +
+                                    lambda_k I)^-1 vec(Y - X V*) by conjugate gradients
+                                    from alpha = 0 (at most cg_iters iterations, until the
+                                    residual is cg_tol of ||e||; matrix-free JVP / VJP,
+                                    fp32 on CUDA cores), K_out = K0 + J_G^T alpha on
+                                    the free slots, K0 on the fixed ones.  V* is v_out as
+                                    written (rounded to dtype).  Without it K_out = K0 */
 #define GRKV_FORCE_SIMT    0x2u  /* use the portable CUDA-core kernels even for bf16 */
 #define GRKV_FUSED_SCORE   0x4u  /* tensor-core scoring in one persistent launch whose
                                     L2-sized rounds let the probability pass re-read K
@@ -87,14 +95,19 @@ typedef struct {
                            tokens stay fixed (0.10)                                 */
   float   lambda_v;     /* >= 0 (may be +inf: values unchanged): ridge weight of
                            the value step, Eq. 6                                    */
-  float   lambda_k;     /* reserved for the key step                               */
+  float   lambda_k;     /* >= 0, finite: ridge weight of the key step (1e-2); read
+                           only under GRKV_UPDATE_K                                 */
   float   scale;        /* logit scale; 0 -> fp32(1/sqrt(d))                        */
   int32_t causal;       /* 1: window slot a sees keys j <= n-w+a; 0: all n keys      */
   int32_t dtype;        /* GRKV_BF16 or GRKV_F32 for q, k, v, k_out, v_out          */
-  uint32_t flags;       /* GRKV_FORCE_SIMT; GRKV_UPDATE_K -> GRKV_ERR_UNSUPPORTED    */
+  uint32_t flags;       /* GRKV_UPDATE_K, GRKV_FORCE_SIMT, GRKV_FUSED_SCORE          */
+  int32_t cg_iters;     /* 0..4096: most conjugate-gradient iterations of the key
+                           step (512); read only under GRKV_UPDATE_K                */
+  float   cg_tol;       /* >= 0, finite: the key step's CG stops once ||r|| <=
+                           cg_tol ||e|| (1e-4); read only under GRKV_UPDATE_K       */
 } grkv_params;
 
-/* Fills `p` with the defaults above for the given sizes (bf16, lambda 1e-2,
+/* Fills `p` with the defaults above for the given sizes (bf16, lambda 1e-2, CG 512 / 1e-4,
  * max pool 7, 4 sinks, beta 0.10, causal). */
 void grkv_params_init(grkv_params* p, int32_t units, int32_t group, int32_t n,
                       int32_t window, int32_t budget);

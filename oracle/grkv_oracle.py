@@ -65,7 +65,8 @@ class Params:
     causal: bool = True
     update_k: bool = False        # also run the key step (App. D.2)
     lambda_k: float = 1e-2
-    cg_iters: int = 16            # conjugate-gradient iterations of the key step
+    cg_iters: int = 512           # most conjugate-gradient iterations of the key step
+    cg_tol: float = 1e-4          # ... stopping once ||r|| <= cg_tol ||e||
 
     @property
     def m(self) -> int:
@@ -237,7 +238,7 @@ def key_vjp(X, Q, V, W, s: float):
     return s * (dS.T @ np.asarray(Q, dtype=f64))
 
 
-def key_step_dual(X, Q, K0, V, Y, free, lam: float, s: float, iters: int):
+def key_step_dual(X, Q, K0, V, Y, free, lam: float, s: float, iters: int, tol: float = 0.0):
     """Key step of Algorithm 1 at t = 0 (K = K0, so G = K - K0 = 0) in its
     linearised dual form (Sec. 3.4 'Key step', App. D.2):
         E = Y - f(K0) = Y - X V,  e = vec(E)
@@ -245,9 +246,10 @@ def key_step_dual(X, Q, K0, V, Y, free, lam: float, s: float, iters: int):
         K*_G = K0_G + unvec(J_G^T alpha),  K*_F = K0_F
     J_G is the Jacobian of f with respect to the free rows only; the operator
     alpha -> J_G (J_G^T alpha) + lambda alpha is applied matrix-free (JVP of
-    the VJP), as the paper does.  CG starts from alpha = 0 and runs `iters`
-    iterations (fewer only once the residual or the search direction
-    vanishes); returns K* and the residual norms ||r_t|| of every iteration."""
+    the VJP), as the paper does.  CG starts from alpha = 0 and runs at most
+    `iters` iterations, stopping once ||r_t|| <= tol ||e|| or the search
+    direction vanishes; returns K* and the residual norms ||r_t|| of every
+    iteration."""
     X = np.asarray(X, dtype=f64)
     V = np.asarray(V, dtype=f64)
     K0 = np.asarray(K0, dtype=f64)
@@ -267,8 +269,9 @@ def key_step_dual(X, Q, K0, V, Y, free, lam: float, s: float, iters: int):
     pdir = r.copy()
     rs = float((r * r).sum())
     hist = [math.sqrt(rs)]
+    stop = (tol * hist[0]) ** 2
     for _ in range(iters):
-        if rs == 0.0:
+        if rs == 0.0 or rs <= stop:
             break
         Ap = op(pdir)
         pAp = float((pdir * Ap).sum())
@@ -305,7 +308,7 @@ def merge_unit(q, k, v, c32, y, idx, p: Params, mode: str = "dual"):
     if p.update_k:
         Q = np.asarray(q, dtype=f64).reshape(p.m, p.d)
         K, hist = key_step_dual(X, Q, K0, V, y, ~fixed, f64(np.float32(p.lambda_k)),
-                                effective_scale(p), p.cg_iters)
+                                effective_scale(p), p.cg_iters, p.cg_tol)
         out["k_out"] = K
         out["cg_residuals"] = hist
     return out

@@ -42,7 +42,8 @@ class grkv_params(ctypes.Structure):
         ("pool_kernel", ctypes.c_int32), ("pool_type", ctypes.c_int32),
         ("n_sink", ctypes.c_int32), ("beta", ctypes.c_float), ("lambda_v", ctypes.c_float),
         ("lambda_k", ctypes.c_float), ("scale", ctypes.c_float), ("causal", ctypes.c_int32),
-        ("dtype", ctypes.c_int32), ("flags", ctypes.c_uint32),
+        ("dtype", ctypes.c_int32), ("flags", ctypes.c_uint32), ("cg_iters", ctypes.c_int32),
+        ("cg_tol", ctypes.c_float),
     ]
 
 

@@ -78,7 +78,11 @@ int make_shape(const grkv_params* p, Shape* s) {
   if (p->dtype != GRKV_F32 && p->dtype != GRKV_BF16) return GRKV_ERR_INVALID_ARG;
   if (p->flags & ~(GRKV_UPDATE_K | GRKV_FORCE_SIMT | GRKV_FUSED_SCORE)) return GRKV_ERR_INVALID_ARG;
   if (p->d < 1) return GRKV_ERR_INVALID_ARG;
-  if (p->flags & GRKV_UPDATE_K) return GRKV_ERR_UNSUPPORTED;
+  if (p->flags & GRKV_UPDATE_K) {
+    if (!(p->lambda_k >= 0.f) || std::isinf(p->lambda_k)) return GRKV_ERR_INVALID_ARG;
+    if (p->cg_iters < 0 || p->cg_iters > kMaxCgIters) return GRKV_ERR_INVALID_ARG;
+    if (!(p->cg_tol >= 0.f) || std::isinf(p->cg_tol)) return GRKV_ERR_INVALID_ARG;
+  }
   if (p->d != kD) return GRKV_ERR_UNSUPPORTED;
   if ((int64_t)p->group * p->window > kMaxM) return GRKV_ERR_UNSUPPORTED;
   if ((int64_t)p->n * kD > (int64_t)1 << 31) return GRKV_ERR_UNSUPPORTED;
@@ -103,6 +107,10 @@ int make_shape(const grkv_params* p, Shape* s) {
   s->tc = (p->flags & GRKV_FORCE_SIMT) ? 0 : (score_tc_supported(*s) ? 1 : 0);
   s->tc_merge = (s->tc && merge_tc_supported(*s)) ? 1 : 0;
   s->fused = (p->flags & GRKV_FUSED_SCORE) ? 1 : 0;
+  s->update_k = (p->flags & GRKV_UPDATE_K) ? 1 : 0;
+  s->cg_iters = p->cg_iters;
+  s->cg_tol = p->cg_tol;
+  s->lambda_k = p->lambda_k;
   return GRKV_OK;
 }
 
@@ -142,6 +150,7 @@ WsLayout plan_workspace(const Shape& s) {
   L.scores = take(U * (size_t)s.P * 4);
   L.y = take(U * m * d * 4);
   L.rstats = take(U * m * 8);
+  if (s.update_k) L.key = take(key_ws_bytes(s));
   L.total = off;
   return L;
 }
@@ -169,6 +178,8 @@ void grkv_params_init(grkv_params* p, int32_t units, int32_t group, int32_t n, i
   p->causal = 1;
   p->dtype = GRKV_BF16;
   p->flags = 0;
+  p->cg_iters = 512;
+  p->cg_tol = 1e-4f;
 }
 
 int grkv_workspace_size(const grkv_params* p, size_t* bytes) {
@@ -229,7 +240,9 @@ int grkv_merge(const grkv_params* p, const void* q, const void* k, const void* v
   char* w = (char*)ws;
   GRKV_TRY(cuda_rc(cudaMemsetAsync(w + L.status, 0, 4, st)));
   if (s.U == 0) return GRKV_OK;
-  return cuda_rc(launch_merge(s, q, k, v, scores, y, row_stats, idx, k_out, v_out, w, L, st));
+  GRKV_TRY(cuda_rc(launch_merge(s, q, k, v, scores, y, row_stats, idx, k_out, v_out, w, L, st)));
+  if (!s.update_k) return GRKV_OK;
+  return cuda_rc(launch_key_step(s, q, y, scores, idx, v_out, k_out, w, L, st));
 }
 
 int grkv_compress(const grkv_params* p, const void* q, const void* k, const void* v, void* k_out,
@@ -251,7 +264,9 @@ int grkv_compress(const grkv_params* p, const void* q, const void* k, const void
   float* rstats = (float*)(w + L.rstats);
   GRKV_TRY(cuda_rc(launch_score(s, q, k, v, scores, y, rstats, w, L, st)));
   GRKV_TRY(cuda_rc(launch_select(s, scores, idx, w, L, st)));
-  return cuda_rc(launch_merge(s, q, k, v, scores, y, rstats, idx, k_out, v_out, w, L, st));
+  GRKV_TRY(cuda_rc(launch_merge(s, q, k, v, scores, y, rstats, idx, k_out, v_out, w, L, st)));
+  if (!s.update_k) return GRKV_OK;
+  return cuda_rc(launch_key_step(s, q, y, scores, idx, v_out, k_out, w, L, st));
 }
 
 int grkv_status(const void* ws, int* device_status, void* stream) {

@@ -14,6 +14,7 @@ namespace grkv {
 constexpr int kD = 128;          // supported head dimension
 constexpr int kMaxM = 256;       // stacked window rows g*w supported
 constexpr int kMaxScoreCtas = 256;  // persistent score grid bound used to size slots
+constexpr int kMaxCgIters = 4096;   // bound on the key step's conjugate-gradient iterations
 
 // Validated problem sizes, derived once on the host.
 struct Shape {
@@ -26,6 +27,10 @@ struct Shape {
   int tc;         // bf16, m <= 128, not forced portable: tensor-core scoring
   int tc_merge;   // ... and B <= 32768: tensor-core value merge
   int fused;      // tensor-core scoring as one launch in L2-sized rounds
+  int update_k;   // key step after the value step (GRKV_UPDATE_K)
+  int cg_iters;   // most conjugate-gradient iterations of the key step
+  float cg_tol;   // ... until ||r|| <= cg_tol ||e||
+  float lambda_k; // ridge weight of the key step
 };
 
 // Byte offsets of the workspace regions (each 256-B aligned).
@@ -50,6 +55,7 @@ struct WsLayout {
   size_t scores;  // float [U][P]
   size_t y;       // float [U][m][d]
   size_t rstats;  // float2 [U][m]
+  size_t key;     // key step: X, T [U][m][B], dK [U][B][d], CG vectors [U][4][m][d], fixed [U][B]
   size_t total;
 };
 
@@ -91,6 +97,10 @@ bool merge_tc_supported(const Shape& s);
 size_t merge_tc_ws_bytes(const Shape& s);
 // row_stats (nullable): the full-cache row statistics; with them the Gram
 // needs one pass over the retained keys.
+size_t key_ws_bytes(const Shape& s);
+cudaError_t launch_key_step(const Shape& s, const void* q, const float* y, const float* scores,
+                            const int32_t* idx, const void* v_out, void* k_out, char* ws,
+                            const WsLayout& L, cudaStream_t st);
 cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const void* v,
                             const float* scores, const float* y, const float* row_stats,
                             const int32_t* idx, void* k_out, void* v_out, char* ws,

@@ -55,7 +55,14 @@ def test_workspace_size_and_validation(lib):
     bad = [dict(budget=16), dict(budget=9000), dict(pool_kernel=6), dict(pool_kernel=0),
            dict(beta=1.0), dict(beta=-0.1), dict(lambda_v=-1.0), dict(lambda_v=float("nan")),
            dict(causal=2), dict(dtype=7), dict(window_zero=True), dict(units=-1),
-           dict(n_sink=-1), dict(flags=0x100), dict(pool_type=3), dict(scale=-1.0)]
+           dict(n_sink=-1), dict(flags=0x100), dict(pool_type=3), dict(scale=-1.0),
+           dict(flags=b.GRKV_UPDATE_K, lambda_k=-1.0),
+           dict(flags=b.GRKV_UPDATE_K, lambda_k=float("inf")),
+           dict(flags=b.GRKV_UPDATE_K, lambda_k=float("nan")),
+           dict(flags=b.GRKV_UPDATE_K, cg_iters=-1),
+           dict(flags=b.GRKV_UPDATE_K, cg_iters=4097),
+           dict(flags=b.GRKV_UPDATE_K, cg_tol=-1.0),
+           dict(flags=b.GRKV_UPDATE_K, cg_tol=float("inf"))]
     for kw in bad:
         q = b.params(8, 4, 8192, 32, 512)
         for key, val in kw.items():
@@ -67,13 +74,20 @@ def test_workspace_size_and_validation(lib):
         with pytest.raises(b.GrkvError) as e:
             b.grkv_workspace_size(q)
         assert e.value.code == b.GRKV_ERR_INVALID_ARG, kw
-    for kw in (dict(d=64), dict(flags=b.GRKV_UPDATE_K), dict(group=9)):
+    for kw in (dict(d=64), dict(group=9)):
         q = b.params(8, 4, 8192, 32, 512)
         for key, val in kw.items():
             setattr(q, key, val)
         with pytest.raises(b.GrkvError) as e:
             b.grkv_workspace_size(q)
         assert e.value.code == b.GRKV_ERR_UNSUPPORTED, kw
+    # the key step adds its workspace; lambda_k and cg_iters are read only with it
+    plain = b.grkv_workspace_size(b.params(8, 4, 8192, 32, 512))
+    keyed = b.grkv_workspace_size(b.params(8, 4, 8192, 32, 512, flags=b.GRKV_UPDATE_K))
+    assert keyed > plain
+    assert b.grkv_workspace_size(b.params(8, 4, 8192, 32, 512, lambda_k=-1.0, cg_iters=-5)) == plain
+    dp = b.params(1, 1, 64, 8, 16)
+    assert dp.cg_iters == 512 and abs(dp.cg_tol - 1e-4) < 1e-9
     # lambda = +inf is valid: the value step leaves V0 unchanged
     assert b.grkv_workspace_size(b.params(8, 4, 8192, 32, 512, lambda_v=float("inf"))) > 0
 

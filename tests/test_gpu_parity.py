@@ -327,3 +327,86 @@ def test_full_length_c4_sweep_points(grkv_lib, n, budget):
     longer than the shared-memory selection handles) on two units."""
     wl = next(w for w in gi.sweep_points() if w.n == n and w.budget == budget)
     _compress_sampled(wl, 2, (0, 1))
+
+
+# --------------------------------------------------------------- key step --
+EDGE_KEY = gi.Workload("edge_n600", 2, 2, 600, 128, 8, 64, 7, 1e-2, "bf16", "lowrank", 4242)
+KEY_CASES = {
+    # workload, path flags, lambda_k (1e-2 Llama default, 1e-1 Mistral default)
+    "c0_f32_portable": (gi.workload(0), 0, 1e-2),
+    "c1_bf16_default": (gi.workload(1).replace(units=2), 0, 1e-1),
+    "c1_bf16_portable": (gi.workload(1).replace(units=2), b.GRKV_FORCE_SIMT, 1e-1),
+    "edge_bf16_default": (EDGE_KEY, 0, 1e-2),
+}
+
+
+@pytest.mark.parametrize("name", list(KEY_CASES))
+def test_key_step(grkv_lib, name):
+    """GRKV_UPDATE_K: the key step of Algorithm 1 at t = 0 (App. D.2) run to a
+    relative CG residual of 1e-6 in fp32 on the GPU, against the converged
+    linearised ridge solution (fp64 CG to 1e-12) of the oracle, on the
+    oracle's retained set.  K_out is held to the method's bar; the update
+    K_out - K0 to 2e-3 of its norm plus the rounding of K_out to its dtype.
+    V_out and the fixed rows of K_out are those of the value step alone."""
+    wl, flags, lam = KEY_CASES[name]
+    c = G.Case(wl)
+    op = G.oracle_params(wl, update_k=True, lambda_k=lam, cg_iters=4000, cg_tol=1e-12)
+    ora = [O.compress_unit(c.q[i], c.k[i], c.v[i], op) for i in range(c.U)]
+    idx = np.stack([o["idx"] for o in ora]).astype(np.int32)
+    scores32 = np.stack([o["scores32"] for o in ora])
+    y32 = np.stack([o["y"].astype(np.float32) for o in ora])
+    p = G.lib_params(wl, c.U)
+    p.flags = flags
+    ko0, vo0 = G.run_merge(c, p, scores32, y32, idx)
+    p.flags = flags | b.GRKV_UPDATE_K
+    p.lambda_k = lam
+    p.cg_iters = 4000
+    p.cg_tol = 1e-6
+    ko, vo = G.run_merge(c, p, scores32, y32, idx)
+    np.testing.assert_array_equal(vo, vo0)
+    rnd = 2.0 ** -8 if wl.dtype == "bf16" else 2.0 ** -23
+    for i, o in enumerate(ora):
+        K0 = c.k[i][idx[i]].astype(np.float64)
+        fixed = o["fixed"]
+        np.testing.assert_array_equal(ko[i][fixed], ko0[i][fixed])
+        G.assert_values(ko[i], o["k_out"], wl.dtype, what="k_out")
+        d_ora = o["k_out"] - K0
+        d_gpu = ko[i].astype(np.float64) - K0
+        assert np.abs(d_ora).max() > 0
+        err = np.linalg.norm(d_gpu - d_ora)
+        lim = 2e-3 * np.linalg.norm(d_ora) + rnd * np.linalg.norm(o["k_out"])
+        assert err <= lim, f"unit {i}: key update error {err:.3e} > {lim:.3e}"
+
+
+def test_key_step_zero_iterations_and_large_lambda(grkv_lib):
+    wl = gi.workload(1).replace(units=1)
+    c = G.Case(wl)
+    op = G.oracle_params(wl)
+    o = O.compress_unit(c.q[0], c.k[0], c.v[0], op)
+    args = (o["scores32"][None], o["y"].astype(np.float32)[None], o["idx"][None].astype(np.int32))
+    p = G.lib_params(wl, 1)
+    ko0, _ = G.run_merge(c, p, *args)
+    p.flags = b.GRKV_UPDATE_K
+    p.cg_iters = 0                      # alpha = 0: K_out = K0 exactly
+    ko, _ = G.run_merge(c, p, *args)
+    np.testing.assert_array_equal(ko, ko0)
+    p.cg_iters = 64
+    p.lambda_k = 1e7                    # the ridge keeps K0 (update far below a bf16 ulp)
+    ko, _ = G.run_merge(c, p, *args)
+    np.testing.assert_array_equal(ko, ko0)
+
+
+def test_key_step_through_compress(grkv_lib):
+    """grkv_compress with GRKV_UPDATE_K runs the key step on its own selection
+    and target: K_out differs from K0 on free slots only."""
+    wl = EDGE_KEY
+    c = G.Case(wl)
+    p = G.lib_params(wl, c.U)
+    idx0, ko0, vo0 = G.run_compress(c, p)
+    p.flags = b.GRKV_UPDATE_K
+    idx, ko, vo = G.run_compress(c, p)
+    np.testing.assert_array_equal(idx, idx0)
+    np.testing.assert_array_equal(vo, vo0)
+    for i in range(c.U):
+        np.testing.assert_array_equal(ko0[i], c.k[i][idx0[i]])
+        assert (ko[i] != ko0[i]).any()

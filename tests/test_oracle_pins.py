@@ -418,7 +418,7 @@ def test_merge_unit_key_step_uses_merged_values():
     g, w, n, d = 2, 3, 24, 8
     q, k, v = _rand_unit(rng, g, w, n, d)
     p = O.Params(group=g, n=n, d=d, window=w, budget=12, n_sink=2, beta=0.2, update_k=True,
-                 lambda_k=0.05, cg_iters=g * w * d)
+                 lambda_k=0.05, cg_iters=g * w * d, cg_tol=1e-8)
     base = O.compress_unit(q, k, v, dataclasses_replace(p, update_k=False))
     out = O.compress_unit(q, k, v, p)
     np.testing.assert_array_equal(out["idx"], base["idx"])
@@ -426,7 +426,8 @@ def test_merge_unit_key_step_uses_merged_values():
     K0 = np.asarray(k, dtype=np.float64)[out["idx"]]
     Q = np.asarray(q, dtype=np.float64).reshape(p.m, d)
     want, _ = O.key_step_dual(out["x"], Q, K0, out["v_out"], out["y"], ~out["fixed"],
-                              np.float64(np.float32(p.lambda_k)), O.effective_scale(p), p.cg_iters)
+                              np.float64(np.float32(p.lambda_k)), O.effective_scale(p), p.cg_iters,
+                              p.cg_tol)
     np.testing.assert_array_equal(out["k_out"], want)
     assert np.array_equal(out["k_out"][out["fixed"]], K0[out["fixed"]])
     assert np.abs(out["k_out"] - K0).max() > 0
@@ -435,3 +436,14 @@ def test_merge_unit_key_step_uses_merged_values():
 def dataclasses_replace(p, **kw):
     import dataclasses
     return dataclasses.replace(p, **kw)
+
+
+def test_key_step_stops_at_the_residual_tolerance():
+    rng = np.random.default_rng(31)
+    p, Q, K0, V, X, Y, idx = _key_case(rng, g=2, w=3, n=14, d=4)
+    free = np.ones(idx.size, bool)
+    s = O.effective_scale(p)
+    _, full = O.key_step_dual(X, Q, K0, V, Y, free, 0.1, s, iters=400)
+    K, hist = O.key_step_dual(X, Q, K0, V, Y, free, 0.1, s, iters=400, tol=1e-3)
+    assert hist[-1] <= 1e-3 * hist[0] and all(h > 1e-3 * hist[0] for h in hist[:-1])
+    assert len(hist) < len(full)
