@@ -1,4 +1,4 @@
-// Window scoring on the 5th-generation tensor cores (bf16, d = 128, m <= 128).
+// Window scoring on the 5th-generation tensor cores (bf16, d = 128, m <= 256).
 //
 // For every unit the path needs, over all n keys, the row statistics of the
 // window logits (pass A: M_r, L_r) and then, with those, the probabilities,
@@ -66,6 +66,8 @@ constexpr uint32_t kColS = 0, kColY = 256;
 
 struct Args {
   int U, n, w, m, P, causal;
+  int row0, mr;   // stacked rows row0 .. row0 + mr - 1 (mr <= 128) in this launch
+  int acc;        // add the prefix scores to those of an earlier launch (rows before row0)
   int tpu;        // tiles per unit
   int mode;       // 0: pass A only, 1: pass B only, 2: both, in rounds
   int gu;         // units per round
@@ -326,8 +328,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             ++qissued;
             mbar_expect_tx(&bars->q_full[qs], kTileBytes);
             uint8_t* dq = sm + kOffQ + qs * kTileBytes;
-            tma_load_3d(dq, &tmQ, &bars->q_full[qs], 0, 0, j.u, keep);
-            tma_load_3d(dq + kTileBytes / 2, &tmQ, &bars->q_full[qs], 64, 0, j.u, keep);
+            tma_load_3d(dq, &tmQ, &bars->q_full[qs], 0, a.row0, j.u, keep);
+            tma_load_3d(dq + kTileBytes / 2, &tmQ, &bars->q_full[qs], 64, a.row0, j.u, keep);
           }
           // the job's K, then the V of the previous pass-B job: V waits in the
           // ring through a tile's compute, so it is fetched one tile later
@@ -554,10 +556,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int t = 0; t < 4; ++t) {
           const int r = t * 32 + lane;
-          lam_s[lb * kRows + r] = (r < a.m && st[t].y > 0.f) ? st[t].x + __log2f(st[t].y) : INFINITY;
-          if (first && r < a.m) {
-            a.row_stats[((size_t)j.u * a.m + r) * 2 + 0] = st[t].x * 0.69314718055994531f;
-            a.row_stats[((size_t)j.u * a.m + r) * 2 + 1] = st[t].y;
+          lam_s[lb * kRows + r] = (r < a.mr && st[t].y > 0.f) ? st[t].x + __log2f(st[t].y) : INFINITY;
+          if (first && r < a.mr) {
+            a.row_stats[((size_t)j.u * a.m + a.row0 + r) * 2 + 0] = st[t].x * 0.69314718055994531f;
+            a.row_stats[((size_t)j.u * a.m + a.row0 + r) * 2 + 1] = st[t].y;
           }
         }
         __syncwarp();
@@ -589,8 +591,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           float v[32];
           tmem_ld32(ybase + c * 32, v);
           tmem_ld_wait();
-          if (row < a.m) {
-            float4* dst = (float4*)(a.y + ((size_t)j.u * a.m + row) * kD + c * 32);
+          if (row < a.mr) {
+            float4* dst = (float4*)(a.y + ((size_t)j.u * a.m + a.row0 + row) * kD + c * 32);
 #pragma unroll
             for (int e = 0; e < 8; ++e)
               atomicAdd(dst + e, make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]));
@@ -606,8 +608,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------- compute groups
     const int wg = (warp - 4) >> 2, q = warp & 3;
     const int row = q * 32 + lane;
-    const bool row_ok = row < a.m;
-    const int lim = a.causal ? a.n - a.w + (row_ok ? row % a.w : 0) : a.n - 1;
+    const bool row_ok = row < a.mr;
+    const int lim = a.causal ? a.n - a.w + (row_ok ? (a.row0 + row) % a.w : 0) : a.n - 1;
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
     const uint32_t bar_id = 1 + wg;
     float2* astat = (float2*)(sm + kOffAstat);
@@ -695,7 +697,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (q < 2) {
               const int jj = q * 32 + lane;
               const float cs = ((rb[jj] + rb[64 + jj]) + rb[128 + jj]) + rb[192 + jj];
-              if (t0 + jj < a.P && 64 * wg + jj < j.len) a.scores[(size_t)j.u * a.P + t0 + jj] = cs;
+              if (t0 + jj < a.P && 64 * wg + jj < j.len) {
+                float* dst = a.scores + (size_t)j.u * a.P + t0 + jj;
+                *dst = a.acc ? *dst + cs : cs;
+              }
             }
           }
         }
@@ -727,7 +732,10 @@ int g_num_sms[64] = {};
 
 }  // namespace
 
-bool score_tc_supported(const Shape& s) { return s.dtype == GRKV_BF16 && s.m <= kRows; }
+// m <= 256: stacked rows past 128 run as a second pair of passes over the
+// keys (row statistics and Y are per row; the prefix scores of the second
+// pair are added to the first's).
+bool score_tc_supported(const Shape& s) { return s.dtype == GRKV_BF16 && s.m <= 2 * kRows; }
 
 size_t score_tc_pstats_bytes(const Shape& s, int* maxc, int* gu, int* rounds, int sms) {
   const int tpu = (s.n + kTile - 1) / kTile;
@@ -786,8 +794,6 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
   a.status = (int*)(ws + L.status);
   cudaError_t e = cudaMemsetAsync(y, 0, (size_t)s.U * s.m * kD * sizeof(float), st);
   if (e != cudaSuccess) return e;
-  e = cudaMemsetAsync(a.unit_cnt, 0, (size_t)s.U * sizeof(int), st);
-  if (e != cudaSuccess) return e;
   auto launch = [&](int md) {
     a.mode = md;
     if (md != 2) {
@@ -815,10 +821,21 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
     count_launches(1);
     return cudaLaunchKernelEx(&cfg, kern, mq, mk, mv, a);
   };
-  if (mode == 2) return launch(2);
-  e = launch(0);
-  if (e != cudaSuccess) return e;
-  return launch(1);
+  for (int row0 = 0; row0 < s.m; row0 += kRows) {
+    a.row0 = row0;
+    a.mr = std::min(kRows, s.m - row0);
+    a.acc = row0 > 0;
+    e = cudaMemsetAsync(a.unit_cnt, 0, (size_t)s.U * sizeof(int), st);
+    if (e != cudaSuccess) return e;
+    if (mode == 2) {
+      e = launch(2);
+    } else {
+      e = launch(0);
+      if (e == cudaSuccess) e = launch(1);
+    }
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 }  // namespace grkv

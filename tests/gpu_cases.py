@@ -34,8 +34,8 @@ def oracle_params(wl: gi.Workload, **over) -> O.Params:
 
 
 def uses_tensor_cores(p) -> bool:
-    """The library scores on the tensor cores for bf16 with m <= 128."""
-    return (p.dtype == b.GRKV_BF16 and p.group * p.window <= 128
+    """The library scores on the tensor cores for bf16 with m <= 256."""
+    return (p.dtype == b.GRKV_BF16 and p.group * p.window <= 256
             and not (p.flags & b.GRKV_FORCE_SIMT))
 
 
