@@ -11,6 +11,8 @@
 //     dA = W V*^T,  dS = X o (dA - rowsum(X o dA)),  dK = s dS^T Q,
 // with the fixed rows of dK zeroed, and J dK (Jacobian-vector product) is
 //     dS = s Q dK^T,  dA = X o (dS - rowsum(X o dS)),  df = dA V*.
+// Inside CG the two meet as s Q dK^T = (s^2 Q Q^T) dS on the free columns,
+// so an iteration is three GEMMs (m x B x d, m x m x B, m x B x d).
 // Conjugate gradients start from alpha = 0 and run at most cg_iters
 // iterations, stopping once ||r|| <= cg_tol ||e|| or the search direction
 // vanishes.  Each product is a small tiled GEMM over the unit's
@@ -42,6 +44,8 @@ struct KArgs {
   float* X;               // [U][m][B]
   float* T;               // [U][m][B]
   float* dK;              // [U][B][d]
+  float* T2;              // [U][m][B]
+  float* GQ;              // [U][m][m]
   float* vec;             // [U][4][m][d]: r, p, Ap, alpha
   uint8_t* fixed;         // [U][B]
 };
@@ -53,7 +57,8 @@ __device__ __forceinline__ float ldv(const void* p, size_t i, int dtype) {
 
 // Shared-memory k slabs of one block_gemm tile.
 struct GemmSmem {
-  float As[kTK][kTM + 4], Bs[kTK][kTN + 4];
+  alignas(16) float As[kTK][kTM + 4];
+  alignas(16) float Bs[kTK][kTN + 4];
 };
 
 // C(i, j) = sum_k a(i, k) b(k, j) for i < M, j < N; store(i, j, value).
@@ -82,12 +87,10 @@ __device__ void block_gemm(GemmSmem& g, int M, int N, int K, FA a, FB b, FS stor
         __syncthreads();
 #pragma unroll
         for (int kk = 0; kk < kTK; ++kk) {
-          float av[4], bv[4];
-#pragma unroll
-          for (int t = 0; t < 4; ++t) {
-            av[t] = As[kk][ty * 4 + t];
-            bv[t] = Bs[kk][tx * 4 + t];
-          }
+          // rows of 68 floats keep every 4-float group 16-byte aligned
+          const float4 a4 = *reinterpret_cast<const float4*>(&As[kk][ty * 4]);
+          const float4 b4 = *reinterpret_cast<const float4*>(&Bs[kk][tx * 4]);
+          const float av[4] = {a4.x, a4.y, a4.z, a4.w}, bv[4] = {b4.x, b4.y, b4.z, b4.w};
 #pragma unroll
           for (int t = 0; t < 4; ++t)
 #pragma unroll
@@ -146,6 +149,8 @@ __global__ void __launch_bounds__(kKT) k_key_step(KArgs a) {
   float* X = a.X + (size_t)u * m * B;
   float* T = a.T + (size_t)u * m * B;
   float* dK = a.dK + kv_off;
+  float* T2 = a.T2 + (size_t)u * m * B;
+  float* GQ = a.GQ + (size_t)u * m * m;
   float* R = a.vec + (size_t)u * 4 * m * kD;
   float* Pd = R + (size_t)m * kD;
   float* AP = Pd + (size_t)m * kD;
@@ -212,6 +217,11 @@ __global__ void __launch_bounds__(kKT) k_key_step(KArgs a) {
   __syncthreads();
 
   const int md = m * kD;
+  // ---- GQ = s^2 Q Q^T (the Gram of the window queries)
+  block_gemm(gs,
+      m, m, kD, [&](int r, int t) { return ldv(q, (size_t)r * kD + t, dt); },
+      [&](int t, int r2) { return ldv(q, (size_t)r2 * kD + t, dt); },
+      [&](int r, int r2, float v) { GQ[(size_t)r * m + r2] = s * s * v; });
   // ---- r = e = Y - X V*, p = r, alpha = 0
   block_gemm(gs,
       m, kD, B, [&](int r, int j) { return X[(size_t)r * B + j]; },
@@ -243,15 +253,21 @@ __global__ void __launch_bounds__(kKT) k_key_step(KArgs a) {
 
   for (int it = 0; it < a.iters; ++it) {
     if (!(rs > stop) || !(rs > 0.f)) break;
-    vjp(Pd);
-    // Ap = J_G dK + lambda p
+    // Ap = J_G (J_G^T p) + lambda p without forming dK: with dS = X o (dA -
+    // rowsum(X o dA)), dA = p V*^T, the JVP of dK = s dS^T Q (free rows) is
+    // s Q dK^T = (s^2 Q Q^T) dS on the free columns and 0 on the fixed ones.
     block_gemm(gs,
-        m, B, kD, [&](int r, int t) { return ldv(q, (size_t)r * kD + t, dt); },
-        [&](int t, int j) { return dK[(size_t)j * kD + t]; },
-        [&](int r, int j, float v) { T[(size_t)r * B + j] = s * v; });
+        m, B, kD, [&](int r, int t) { return Pd[(size_t)r * kD + t]; },
+        [&](int t, int j) { return ldv(a.v_out, kv_off + (size_t)j * kD + t, dt); },
+        [&](int r, int j, float v) { T[(size_t)r * B + j] = v; });
     softmax_jacobian_rows(X, T, m, B);
     block_gemm(gs,
-        m, kD, B, [&](int r, int j) { return T[(size_t)r * B + j]; },
+        m, B, m, [&](int r, int r2) { return GQ[(size_t)r * m + r2]; },
+        [&](int r2, int j) { return T[(size_t)r2 * B + j]; },
+        [&](int r, int j, float v) { T2[(size_t)r * B + j] = fixed[j] ? 0.f : v; });
+    softmax_jacobian_rows(X, T2, m, B);
+    block_gemm(gs,
+        m, kD, B, [&](int r, int j) { return T2[(size_t)r * B + j]; },
         [&](int j, int t) { return ldv(a.v_out, kv_off + (size_t)j * kD + t, dt); },
         [&](int r, int t, float v) {
           const size_t o = (size_t)r * kD + t;
@@ -294,7 +310,7 @@ __global__ void __launch_bounds__(kKT) k_key_step(KArgs a) {
 
 size_t key_ws_bytes(const Shape& s) {
   const size_t U = (size_t)s.U, m = (size_t)s.m, B = (size_t)s.B, d = (size_t)kD;
-  return U * (2 * m * B * 4 + B * d * 4 + 4 * m * d * 4 + B) + 1024;
+  return U * (3 * m * B * 4 + B * d * 4 + 4 * m * d * 4 + m * m * 4 + B) + 1024;
 }
 
 cudaError_t launch_key_step(const Shape& s, const void* q, const float* y, const float* scores,
@@ -326,7 +342,9 @@ cudaError_t launch_key_step(const Shape& s, const void* q, const float* y, const
   a.T = a.X + U * m * B;
   a.dK = a.T + U * m * B;
   a.vec = a.dK + U * B * d;
-  a.fixed = (uint8_t*)(a.vec + U * 4 * m * d);
+  a.T2 = a.vec + U * 4 * m * d;
+  a.GQ = a.T2 + U * m * B;
+  a.fixed = (uint8_t*)(a.GQ + U * m * m);
   count_launches(1);
   k_key_step<<<s.U, kKT, 0, st>>>(a);
   return cudaGetLastError();
