@@ -265,6 +265,30 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------ ours --
+def rank_workload(wl, rank: int, world: int):
+    """Weak scaling: every rank compresses its own batch of units, drawn from
+    a seed of its own (the units of different ranks are independent)."""
+    import grkv_inputs as gi
+    return wl if world <= 1 else wl.replace(seed=gi.seed_for(wl.seed, 7919, rank))
+
+
+def max_over_ranks(values, dist=None, device="cpu"):
+    """The element-wise maximum of `values` over the ranks of the process
+    group (the slowest rank sets the job's time); identity without one."""
+    if dist is None:
+        return [float(x) for x in values]
+    import torch
+    t = torch.tensor([float(x) for x in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t.tolist()]
+
+
+def job_throughput(units: int, n: int, world: int, ms: float) -> float:
+    """Whole-job layer-head tokens/s: every rank processed units x n tokens in
+    at most `ms` milliseconds (the max over ranks)."""
+    return units * n * world / (ms * 1e-3)
+
+
 def run_ours(a):
     import numpy as np
     import torch
@@ -285,9 +309,7 @@ def run_ours(a):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     b.load()
 
-    wl = workload(a)
-    if world > 1:   # every rank compresses its own batch of units
-        wl = wl.replace(seed=gi.seed_for(wl.seed, 7919, rank))
+    wl = rank_workload(workload(a), rank, world)
     U, n, B, d, m = wl.units, wl.n, wl.budget, wl.d, wl.m
     qdt = np.uint16 if wl.dtype == "bf16" else np.float32
     tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
@@ -345,10 +367,7 @@ def run_ours(a):
     ms = e0.elapsed_time(e1) / a.steps
     clk = clocks.stop()
     assert b.grkv_status(ws) == b.GRKV_OK
-    if dist is not None:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms, = max_over_ranks([ms], dist, "cuda")
 
     # ---- dominant kernel: the score stage, timed by itself on the same stream
     P = n - wl.window
@@ -392,10 +411,7 @@ def run_ours(a):
     torch.cuda.synchronize()
     barrier()
     e2e_ms = x0.elapsed_time(x1) / a.e2e_steps
-    if dist is not None:
-        t = torch.tensor([e2e_ms, score_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms, score_ms = (float(x) for x in t.tolist())
+    e2e_ms, score_ms = max_over_ranks([e2e_ms, score_ms], dist, "cuda")
     el = hq.element_size()
     h2d = (hq.numel() + hk.numel() + hv.numel()) * el
     d2h = (hko.numel() + hvo.numel()) * el + hidx.numel() * 4
@@ -406,12 +422,11 @@ def run_ours(a):
         return
     read, write = algorithmic_bytes(wl)
     peak, peak_kind = measured_peaks()
-    tokens = U * n * world
     score_bytes = read                      # K and V, each read once
     achieved = score_bytes / (score_ms * 1e-3) / 1e9
     path_gbs = (read + write) / (ms * 1e-3) / 1e9
     line = {
-        "metric": METRIC, "value": tokens / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
+        "metric": METRIC, "value": job_throughput(U, n, world, ms), "unit": UNIT, "n_gpus": world,
         "steps": a.steps, "warmup": a.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,
         "data": "synthetic (seeded; stands in for LongBench / RULER caches)",
@@ -428,7 +443,7 @@ def run_ours(a):
         "path_hbm": {"gbs": path_gbs, "frac_of_measured": path_gbs / peak,
                      "frac_of_8tbs": path_gbs / NOMINAL_HBM_GBS,
                      "bytes_per_step": read + write},
-        "e2e": {"value": tokens / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+        "e2e": {"value": job_throughput(U, n, world, e2e_ms), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms, "steps": a.e2e_steps},
         "gpu_launches": launches,
         "clocks": clk,
