@@ -43,7 +43,7 @@ __all__ = [
     "Params", "effective_scale", "window_logits", "softmax_rows", "window_attention",
     "target", "column_scores", "pool", "select", "fixed_set", "retained_attention",
     "value_step_dual", "value_step_primal", "key_jvp", "key_vjp", "key_step_dual",
-    "merge_unit", "compress_unit",
+    "alternate", "merge_unit", "compress_unit",
 ]
 
 f64 = np.float64
@@ -238,13 +238,15 @@ def key_vjp(X, Q, V, W, s: float):
     return s * (dS.T @ np.asarray(Q, dtype=f64))
 
 
-def key_step_dual(X, Q, K0, V, Y, free, lam: float, s: float, iters: int, tol: float = 0.0):
-    """Key step of Algorithm 1 at t = 0 (K = K0, so G = K - K0 = 0) in its
-    linearised dual form (Sec. 3.4 'Key step', App. D.2):
-        E = Y - f(K0) = Y - X V,  e = vec(E)
-        alpha = (J_G J_G^T + lambda_k I)^-1 e         (conjugate gradients)
+def key_step_dual(X, Q, K0, V, Y, free, lam: float, s: float, iters: int, tol: float = 0.0,
+                  K=None):
+    """Key step of Algorithm 1 in its linearised dual form (Sec. 3.4 'Key
+    step', App. D.2), linearised at the current keys K (default K0, the
+    t = 0 case, where G = 0) whose retained attention is X:
+        E = Y - f(K) = Y - X V,  e = vec(E),  g = vec(G),  G = K - K0
+        alpha = (J_G J_G^T + lambda_k I)^-1 (e + J_G g)  (conjugate gradients)
         K*_G = K0_G + unvec(J_G^T alpha),  K*_F = K0_F
-    J_G is the Jacobian of f with respect to the free rows only; the operator
+    J_G is the Jacobian of f at K with respect to the free rows only; the operator
     alpha -> J_G (J_G^T alpha) + lambda alpha is applied matrix-free (JVP of
     the VJP), as the paper does.  CG starts from alpha = 0 and runs at most
     `iters` iterations, stopping once ||r_t|| <= tol ||e|| or the search
@@ -264,6 +266,10 @@ def key_step_dual(X, Q, K0, V, Y, free, lam: float, s: float, iters: int, tol: f
         return key_jvp(X, Q, V, jt(a), s) + lam * a
 
     E = np.asarray(Y, dtype=f64) - X @ V
+    if K is not None:
+        G = np.asarray(K, dtype=f64) - K0
+        G[~free] = 0.0
+        E = E + key_jvp(X, Q, V, G, s)
     alpha = np.zeros_like(E)
     r = E.copy()
     pdir = r.copy()
@@ -287,6 +293,34 @@ def key_step_dual(X, Q, K0, V, Y, free, lam: float, s: float, iters: int, tol: f
     K = K0.copy()
     K[free] = K0[free] + jt(alpha)[free]
     return K, hist
+
+
+def alternate(q, k, v, c32, y, idx, p: Params, steps: int, stop: float = 1e-9):
+    """Algorithm 1 with S = `steps` alternating value / key steps (NEXT rows:
+    multi-step alternation), each linearised at the current keys:
+        X = softmax over the retained keys K^(t)
+        V^(t+1) = value step from V0 with that X (fixed rows keep V0)
+        K^(t+1) = key step at K^(t) against V^(t+1), G = K^(t) - K0
+    stopping once max(||K^(t+1) - K^(t)||_inf, ||V^(t+1) - V^(t)||_inf) <= stop.
+    Returns K, V, the fixed mask and the (delta_K, delta_V) of every step."""
+    idx = np.asarray(idx)
+    K0 = np.asarray(k, dtype=f64)[idx]
+    V0 = np.asarray(v, dtype=f64)[idx]
+    fixed = fixed_set(idx, c32, p)
+    Q = np.asarray(q, dtype=f64).reshape(p.m, p.d)
+    s = effective_scale(p)
+    lam_v, lam_k = f64(np.float32(p.lambda_v)), f64(np.float32(p.lambda_k))
+    K, V = K0.copy(), V0.copy()
+    deltas = []
+    for _ in range(steps):
+        X, _, _ = softmax_rows(window_logits(q, K, p, cols=idx))
+        Vn = value_step_dual(X, y, V0, ~fixed, lam_v)
+        Kn, _ = key_step_dual(X, Q, K0, Vn, y, ~fixed, lam_k, s, p.cg_iters, p.cg_tol, K=K)
+        deltas.append((float(np.abs(Kn - K).max()), float(np.abs(Vn - V).max())))
+        K, V = Kn, Vn
+        if max(deltas[-1]) <= stop:
+            break
+    return {"k_out": K, "v_out": V, "fixed": fixed, "deltas": deltas}
 
 
 def merge_unit(q, k, v, c32, y, idx, p: Params, mode: str = "dual"):

@@ -447,3 +447,49 @@ def test_key_step_stops_at_the_residual_tolerance():
     K, hist = O.key_step_dual(X, Q, K0, V, Y, free, 0.1, s, iters=400, tol=1e-3)
     assert hist[-1] <= 1e-3 * hist[0] and all(h > 1e-3 * hist[0] for h in hist[:-1])
     assert len(hist) < len(full)
+
+
+# ------------------------------------------------- multi-step alternation --
+def test_alternation_one_step_is_the_single_step_merge():
+    rng = np.random.default_rng(41)
+    g, w, n, d = 2, 3, 30, 8
+    q, k, v = _rand_unit(rng, g, w, n, d)
+    p = O.Params(group=g, n=n, d=d, window=w, budget=14, n_sink=2, beta=0.2, update_k=True,
+                 lambda_k=0.05, cg_iters=500, cg_tol=1e-12)
+    one = O.compress_unit(q, k, v, p)
+    alt = O.alternate(q, k, v, one["scores32"], one["y"], one["idx"], p, steps=1)
+    np.testing.assert_allclose(alt["v_out"], one["v_out"], rtol=0, atol=1e-13)
+    np.testing.assert_allclose(alt["k_out"], one["k_out"], rtol=0, atol=1e-11)
+
+
+def test_alternation_converges_to_a_stationary_point():
+    """At a fixed point of the alternation, the key step's linearised update
+    reproduces K (G = K - K0), which by the ridge identity means
+    lambda_k (K - K0)_G = J_G^T (Y - f(K)): K is a stationary point of the
+    nonlinear key objective ||Y - f(K)||^2 + lambda_k ||K - K0||^2 with V
+    fixed; V is the exact value step at the final X.  Gradients by autograd."""
+    rng = np.random.default_rng(43)
+    g, w, n, d = 1, 3, 16, 4
+    q, k, v = _rand_unit(rng, g, w, n, d, peaked=False)
+    p = O.Params(group=g, n=n, d=d, window=w, budget=9, n_sink=1, beta=0.2, update_k=True,
+                 lambda_v=0.5, lambda_k=0.5, cg_iters=500, cg_tol=1e-13)
+    base = O.compress_unit(q, k, v, dataclasses_replace(p, update_k=False))
+    out = O.alternate(q, k, v, base["scores32"], base["y"], base["idx"], p, steps=200, stop=1e-11)
+    assert max(out["deltas"][-1]) <= 1e-11, out["deltas"][-3:]
+    idx, K, V, Y = base["idx"], out["k_out"], out["v_out"], base["y"]
+    free = ~out["fixed"]
+    s = O.effective_scale(p)
+    a = np.arange(p.m) % p.window
+    mask = idx[None, :] <= (p.n - p.window + a)[:, None]
+    Qt = torch.from_numpy(np.asarray(q, dtype=np.float64).reshape(p.m, d))
+    Kt = torch.from_numpy(K.copy()).requires_grad_(True)
+    f = torch.softmax(s * Qt @ Kt.T + torch.from_numpy(np.where(mask, 0.0, -np.inf)), dim=1) \
+        @ torch.from_numpy(V)
+    loss = ((torch.from_numpy(Y) - f) ** 2).sum() + p.lambda_k * ((Kt - torch.from_numpy(
+        np.asarray(k, dtype=np.float64)[idx])) ** 2).sum()
+    loss.backward()
+    grad = Kt.grad.numpy()
+    assert np.abs(grad[free]).max() <= 1e-8
+    X, _, _ = O.softmax_rows(O.window_logits(q, K, p, cols=idx))
+    V_want = O.value_step_dual(X, Y, np.asarray(v, dtype=np.float64)[idx], free, 0.5)
+    np.testing.assert_allclose(V, V_want, rtol=0, atol=1e-12)
