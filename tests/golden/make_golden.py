@@ -29,6 +29,10 @@ def params():
 def compute():
     q, k, v = gi.unit_arrays(WL, 0)
     out = O.compress_unit(q, k, v, params())
+    # the key step (converged CG) on the same unit
+    import dataclasses
+    key = O.compress_unit(q, k, v, dataclasses.replace(params(), update_k=True, lambda_k=0.05,
+                                                       cg_iters=2000, cg_tol=1e-13))
     return {
         "workload": WL.__dict__,
         "idx": out["idx"].tolist(),
@@ -36,6 +40,7 @@ def compute():
         "scores": out["scores"].tolist(),
         "y": out["y"].tolist(),
         "v_out": out["v_out"].tolist(),
+        "k_out_key_step": key["k_out"].tolist(),
     }
 
 

@@ -18,3 +18,6 @@ def test_oracle_matches_stored_fixture():
     assert now["fixed"] == ref["fixed"]
     for key in ("scores", "y", "v_out"):
         np.testing.assert_allclose(np.array(now[key]), np.array(ref[key]), rtol=1e-12, atol=1e-14)
+    # converged CG: the stored keys are the linearised ridge solution to ~1e-12
+    np.testing.assert_allclose(np.array(now["k_out_key_step"]), np.array(ref["k_out_key_step"]),
+                               rtol=0, atol=1e-9)
