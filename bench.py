@@ -73,7 +73,7 @@ def algorithmic_bytes(wl):
 
 
 # DRAM bytes (read + write) of one grkv_score call, i.e. both k_score_tc launches, from
-# one ncu capture of the full workload (profiles/score_tc_c2_llama_32k.md).  A figure
+# one ncu capture of the full workload.  A figure
 # holds only for the kernel source it was taken on, so it is keyed by that file's digest
 # and reported as null once the kernel changes.
 SCORE_TRAFFIC = {

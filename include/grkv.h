@@ -162,7 +162,9 @@ int grkv_compress(const grkv_params* p, const void* q, const void* k, const void
  * device and fails once a pool has taken the free memory).  It allocates
  * nothing: the pooled scores go to a 16 MiB array in the library's device
  * image, which every GPU that loads the library holds until the process exits.
- * Limit: units * (n - window) <= 4,194,304 floats; larger sizes return
+ * Prefixes of n - window <= 32768 positions are selected in shared memory and
+ * use no scratch, at any unit count.  Longer prefixes use the array, limited
+ * to units * (n - window) <= 4,194,304 floats; larger sizes return
  * GRKV_ERR_WORKSPACE_TOO_SMALL.  The first call on a device looks up the
  * array's device address (cudaGetSymbolAddress) with that device current;
  * make that first call before any stream capture.  All calls share the array

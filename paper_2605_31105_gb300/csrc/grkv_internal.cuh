@@ -106,7 +106,10 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
                             const int32_t* idx, void* k_out, void* v_out, char* ws,
                             const WsLayout& L, cudaStream_t st);
 
-// Selection with the pooled-score scratch [U][n-w] given directly.
+// Selection with the pooled-score scratch [U][n-w] given directly; the
+// scratch is touched only when select_uses_pooled_buffer(s) holds (prefixes
+// longer than the shared-memory selection takes).
+bool select_uses_pooled_buffer(const Shape& s);
 cudaError_t launch_select_pooled(const Shape& s, const float* scores, int32_t* idx,
                                  float* pooled, cudaStream_t st);
 // Host-side parameter validation shared by the entry points.

@@ -49,7 +49,10 @@ extern "C" int grkv_select_noalloc(const grkv_params* p, const float* scores, in
   grkv::Shape s;
   const int rc = grkv::make_shape(p, &s);
   if (rc != GRKV_OK) return rc;
-  if ((size_t)s.U * (size_t)s.P > kScratchFloats) return GRKV_ERR_WORKSPACE_TOO_SMALL;
+  // prefixes up to 32768 positions are selected in shared memory and never
+  // touch the array, so only longer ones are held to its size
+  if (grkv::select_uses_pooled_buffer(s) && (size_t)s.U * (size_t)s.P > kScratchFloats)
+    return GRKV_ERR_WORKSPACE_TOO_SMALL;
   if (((size_t)s.U * s.P && !scores) || ((size_t)s.U * s.B && !idx)) return GRKV_ERR_INVALID_ARG;
   if (((uintptr_t)scores & 15u) || ((uintptr_t)idx & 15u)) return GRKV_ERR_MISALIGNED;
   if (s.U == 0) return GRKV_OK;

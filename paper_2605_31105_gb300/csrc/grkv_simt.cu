@@ -716,9 +716,11 @@ cudaError_t launch_score_simt(const Shape& s, const void* q, const void* k, cons
                                    (const __nv_bfloat16*)v, scores, y, row_stats, ws, L, st);
 }
 
+bool select_uses_pooled_buffer(const Shape& s) { return s.P > kSelMaxP; }
+
 cudaError_t launch_select_pooled(const Shape& s, const float* scores, int32_t* idx,
                                  float* pooled, cudaStream_t st) {
-  if (s.P <= kSelMaxP) {
+  if (!select_uses_pooled_buffer(s)) {
     const size_t bytes = select_smem_bytes(s.P);
     cudaError_t e =
         cudaFuncSetAttribute(k_select_smem, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);

@@ -175,15 +175,66 @@ def assert_values(gpu, ora, dtype: str, what="v_out"):
 def idx_tie_check(gpu_idx, ora, op: O.Params, tol_rel: float):
     """Retained sets must agree except where the oracle's pooled scores sit
     within the score tolerance of the cut: returns the number of such swaps."""
+    return tie_stats(gpu_idx, ora, op, tol_rel)["swaps"]
+
+
+def tie_stats(gpu_idx, ora, op: O.Params, tol_rel: float) -> dict:
+    """Positions where the GPU's retained set differs from the oracle's.
+
+    Each differing position must be a prefix position whose oracle pooled
+    score lies within 2 * tol_rel (the derived bound on the GPU's score error,
+    counted for both scores of a swapped pair) of the cut, the (B - w)-th
+    largest pooled score.  Returns the number of swapped pairs and the largest
+    relative gap |pooled_j - cut| / cut among them, so that swaps beyond the
+    1e-6 tie width can be reported."""
     g, o = set(gpu_idx.tolist()), set(ora["idx"].tolist())
-    diff = g ^ o
+    diff = sorted(g ^ o)
+    out = {"swaps": len(diff) // 2, "max_gap": 0.0, "bound": 2 * tol_rel}
     if not diff:
-        return 0
+        return out
     pooled = ora["pooled"].astype(np.float64)
     kk = op.budget - op.window
     cut = np.sort(pooled)[::-1][kk - 1]
     for j in diff:
         assert j < op.n - op.window, f"window position {j} differs"
-        assert abs(pooled[j] - cut) <= 2 * tol_rel * cut, \
-            f"idx differs at {j}: pooled {pooled[j]:.9e} vs cut {cut:.9e}"
-    return len(diff) // 2
+        gap = abs(pooled[j] - cut) / cut
+        assert gap <= 2 * tol_rel, \
+            f"idx differs at {j}: pooled {pooled[j]:.9e} vs cut {cut:.9e} (gap {gap:.2e})"
+        out["max_gap"] = max(out["max_gap"], gap)
+    return out
+
+
+# Records of every end-to-end unit check in this session (workload, unit,
+# swaps, largest gap, fixed-set agreement, value error), printed by the test
+# session's terminal summary.
+SWAP_LOG: list = []
+
+
+def check_unit_end_to_end(name: str, u: int, q, k, v, op: O.Params, ora: dict, gpu_idx,
+                          gpu_scores, k_out, v_out, dtype: str) -> dict:
+    """One unit of a grkv_compress run against the oracle, with no unit skipped.
+
+    1. The GPU's prefix scores (grkv_score with the same flags, on the same
+       inputs) lie within the derived tolerance of the oracle's.
+    2. The GPU's retained set is exactly the oracle's selection on the GPU's
+       own fp32 scores: selection is exact, so any difference from the
+       oracle's retained set comes from score rounding alone.
+    3. Differences from the oracle's retained set sit within the derived
+       bound of the cut (tie_stats); their count and largest gap are logged.
+    4. K_out = K[idx] bit for bit, and V_out is within the method's bar of
+       the oracle's merge (Algorithm 1 value step, fp64, its own target Y)
+       re-run on the GPU's retained set, with the fixed set decided on the
+       GPU's fp32 scores (both sides decide integers in fp32)."""
+    tol = score_rel_tol(q, k, op)
+    assert_scores(gpu_scores, ora["scores"], tol, f"{name} unit {u} scores")
+    np.testing.assert_array_equal(gpu_idx, O.select(O.pool(gpu_scores, op), op),
+                                  err_msg=f"{name} unit {u}: selection on the GPU's scores")
+    ts = tie_stats(gpu_idx, ora, op, tol)
+    np.testing.assert_array_equal(k_out, k[gpu_idx])
+    ref = O.merge_unit(q, k, v, gpu_scores, ora["y"], gpu_idx, op)
+    fixed_same = bool(np.array_equal(ref["fixed"], O.fixed_set(gpu_idx, ora["scores32"], op)))
+    err = assert_values(v_out, ref["v_out"], dtype, f"{name} unit {u} v_out")
+    rec = {"workload": name, "unit": u, "swaps": ts["swaps"], "max_gap": ts["max_gap"],
+           "bound": ts["bound"], "fixed_same": fixed_same, "v_err": err}
+    SWAP_LOG.append(rec)
+    return rec

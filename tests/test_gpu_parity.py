@@ -139,16 +139,14 @@ def test_merge_row_stats_far_below_full_max_takes_two_passes(grkv_lib):
 
 
 def test_compress_end_to_end(prep):
+    """grkv_compress on every unit: each unit's retained set, K_out and V_out
+    against the oracle (check_unit_end_to_end: no unit is skipped)."""
     c, op = prep.case, prep.op
     idx, ko, vo = G.run_compress(c, prep.p)
-    compared = 0
+    scores, _, _ = G.run_score(c, prep.p)
     for i, ora in enumerate(prep.ora):
-        swaps = G.idx_tie_check(idx[i], ora, op, prep.tol[i])
-        np.testing.assert_array_equal(ko[i], c.k[i][idx[i]])
-        if swaps == 0:
-            G.assert_values(vo[i], ora["v_out"], c.wl.dtype)
-            compared += 1
-    assert compared >= max(1, c.U // 2)
+        G.check_unit_end_to_end(prep.wl.name, i, c.q[i], c.k[i], c.v[i], op, ora, idx[i],
+                                scores[i], ko[i], vo[i], c.wl.dtype)
 
 
 # ------------------------------------------------------------- edge cases --
@@ -258,75 +256,63 @@ def test_singular_dual_system_reports_numeric_status(grkv_lib):
     assert op.lambda_v == 0.0 and np.isfinite(vo).all()
 
 
-def test_full_size_c2_sampled_units(grkv_lib):
-    """The 32-layer, 32K-token workload at full size, in the launch
-    configuration the bench times; sampled units against the oracle."""
+def _compress_sampled(wl, check_units, flags=0):
+    """grkv_compress over every unit of `wl` at full size, in the launch
+    configuration the bench times, then grkv_score with the same flags on the
+    same inputs; the sampled units against the oracle, each one compared."""
     import torch
-    wl = gi.workload(2)
-    q = np.empty((wl.units, wl.group, wl.window, wl.d), np.uint16)
-    k = np.empty((wl.units, wl.n, wl.d), np.uint16)
+    U = wl.units
+    q = np.empty((U, wl.group, wl.window, wl.d), np.uint16)
+    k = np.empty((U, wl.n, wl.d), np.uint16)
     v = np.empty_like(k)
     gi.fill_units(wl, q, k, v)
     as_dev = lambda x: torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).cuda()
     dq, dk, dv = as_dev(q), as_dev(k), as_dev(v)
-    p = G.lib_params(wl, wl.units)
-    ko = torch.empty((wl.units, wl.budget, wl.d), dtype=torch.bfloat16, device="cuda")
+    del q, k, v
+    p = G.lib_params(wl, U)
+    p.flags = flags
+    ko = torch.empty((U, wl.budget, wl.d), dtype=torch.bfloat16, device="cuda")
     vo = torch.empty_like(ko)
-    idx = torch.empty((wl.units, wl.budget), dtype=torch.int32, device="cuda")
+    idx = torch.empty((U, wl.budget), dtype=torch.int32, device="cuda")
     ws = G.workspace(p)
     b.grkv_compress(p, dq, dk, dv, ko, vo, idx, ws)
     assert b.grkv_status(ws) == b.GRKV_OK
-    idx, ko, vo = idx.cpu().numpy(), G.to_host(ko), G.to_host(vo)
+    sel = torch.tensor(list(check_units), dtype=torch.long, device="cuda")
+    idx, ko, vo = idx[sel].cpu().numpy(), G.to_host(ko[sel]), G.to_host(vo[sel])
+    scores = torch.empty((U, wl.n - wl.window), dtype=torch.float32, device="cuda")
+    y = torch.empty((U, wl.m, wl.d), dtype=torch.float32, device="cuda")
+    rs = torch.empty((U, wl.m, 2), dtype=torch.float32, device="cuda")
+    b.grkv_score(p, dq, dk, dv, scores, y, rs, ws)
+    assert b.grkv_status(ws) == b.GRKV_OK
+    scores = G.to_host(scores[sel])
+    del dq, dk, dv
+    torch.cuda.empty_cache()
     op = G.oracle_params(wl)
-    for u in (0, 131, 255):
+    for i, u in enumerate(check_units):
         qu, ku, vu = gi.unit_arrays(wl, u)
         ora = O.compress_unit(qu, ku, vu, op)
-        swaps = G.idx_tie_check(idx[u], ora, op, G.score_rel_tol(qu, ku, op))
-        np.testing.assert_array_equal(ko[u], ku[idx[u]])
-        if swaps == 0:
-            G.assert_values(vo[u], ora["v_out"], wl.dtype)
+        G.check_unit_end_to_end(wl.name, u, qu, ku, vu, op, ora, idx[i], scores[i], ko[i],
+                                vo[i], wl.dtype)
 
 
-def _compress_sampled(wl, units, check_units):
-    """grkv_compress on `units` units of `wl` (full n), sampled units against the oracle."""
-    import torch
-    sub = wl.replace(units=units)
-    q = np.empty((units, sub.group, sub.window, sub.d), np.uint16)
-    k = np.empty((units, sub.n, sub.d), np.uint16)
-    v = np.empty_like(k)
-    gi.fill_units(sub, q, k, v)
-    as_dev = lambda x: torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).cuda()
-    dq, dk, dv = as_dev(q), as_dev(k), as_dev(v)
-    p = G.lib_params(sub, units)
-    ko = torch.empty((units, sub.budget, sub.d), dtype=torch.bfloat16, device="cuda")
-    vo = torch.empty_like(ko)
-    idx = torch.empty((units, sub.budget), dtype=torch.int32, device="cuda")
-    ws = G.workspace(p)
-    b.grkv_compress(p, dq, dk, dv, ko, vo, idx, ws)
-    assert b.grkv_status(ws) == b.GRKV_OK
-    idx, ko, vo = idx.cpu().numpy(), G.to_host(ko), G.to_host(vo)
-    op = G.oracle_params(sub)
-    for u in check_units:
-        qu, ku, vu = gi.unit_arrays(sub, u)
-        ora = O.compress_unit(qu, ku, vu, op)
-        swaps = G.idx_tie_check(idx[u], ora, op, G.score_rel_tol(qu, ku, op))
-        np.testing.assert_array_equal(ko[u], ku[idx[u]])
-        if swaps == 0:
-            G.assert_values(vo[u], ora["v_out"], sub.dtype)
+def test_full_size_c2_sampled_units(grkv_lib):
+    """The 32-layer, 32K-token workload (256 units) at full size; eight units
+    spread over the layers against the oracle."""
+    _compress_sampled(gi.workload(2), (0, 37, 74, 111, 148, 185, 222, 255))
 
 
-def test_full_length_c3_mistral_128k_sampled_units(grkv_lib):
-    """The Mistral-shaped 128K-token workload (m = 256 stacked rows, portable
-    kernels) at its full length on two units."""
-    _compress_sampled(gi.workload(3), 2, (0, 1))
+def test_full_size_c3_mistral_128k_sampled_units(grkv_lib):
+    """The Mistral-shaped 128K-token workload (256 units, m = 256) at full
+    size in its own launch configuration; the first and last KV heads of
+    layers 0 and 31 against the oracle."""
+    _compress_sampled(gi.workload(3), (0, 7, 248, 255))
 
 
-@pytest.mark.parametrize("n,budget", [(131072, 2048), (65536, 128)])
-def test_full_length_c4_sweep_points(grkv_lib, n, budget):
-    """Sweep points at 64K and 128K tokens (tensor-core path; the prefix is
-    longer than the shared-memory selection handles) on two units."""
-    wl = next(w for w in gi.sweep_points() if w.n == n and w.budget == budget)
-    _compress_sampled(wl, 2, (0, 1))
+@pytest.mark.parametrize("wl", list(gi.sweep_points()), ids=lambda w: f"n{w.n}_b{w.budget}")
+def test_full_size_c4_sweep_point(grkv_lib, wl):
+    """Every (n, B) point of the batch-4 sweep at full size (32 units): the
+    first, a middle and the last unit against the oracle."""
+    _compress_sampled(wl, (0, 13, 31))
 
 
 # --------------------------------------------------------------- key step --
