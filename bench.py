@@ -46,9 +46,9 @@ def args_():
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
-    ap.add_argument("--path", choices=("default", "fused", "portable"), default="default",
-                    help="scoring kernels: default (two tensor-core launches), fused (one launch "
-                         "in L2-sized rounds) or portable (CUDA cores)")
+    ap.add_argument("--path", choices=("default", "two_pass", "portable"), default="default",
+                    help="scoring kernels: default (one tensor-core launch that reads K once), "
+                         "two_pass (two launches, K read twice) or portable (CUDA cores)")
     return ap.parse_args()
 
 
@@ -72,22 +72,19 @@ def algorithmic_bytes(wl):
     return read, write
 
 
-# DRAM bytes (read + write) of one grkv_score call, i.e. both k_score_tc launches, from
-# one ncu capture of the full workload.  A figure
-# holds only for the kernel source it was taken on, so it is keyed by that file's digest
+# DRAM bytes (read + write) of one grkv_score call (the one-read scoring kernel
+# k_score_pipe) from one ncu capture of the full workload.  A figure holds only
+# for the kernel source it was taken on, so it is keyed by that file's digest
 # and reported as null once the kernel changes.
-SCORE_TRAFFIC = {
-    "c2_llama_32k_bf16": ("5b1b37492f22eeec99c75ffe0d9cd2c73d563c3f6643ed9193a728d7518eadc9",
-                          6501435904),
-}
+SCORE_SRC = os.path.join("paper_2605_31105_gb300", "csrc", "grkv_score_pipe.cu")
+SCORE_TRAFFIC = {}
 
 
 def score_traffic(wl):
     rec = SCORE_TRAFFIC.get(wl.name)
     if rec is None:
         return None
-    src = os.path.join(ROOT, "paper_2605_31105_gb300", "csrc", "grkv_score_tc.cu")
-    with open(src, "rb") as f:
+    with open(os.path.join(ROOT, SCORE_SRC), "rb") as f:
         digest = hashlib.sha256(f.read()).hexdigest()
     return rec[1] if digest == rec[0] else None
 
@@ -322,7 +319,7 @@ def run_ours(a):
     dq, dk, dv = hq.cuda(), hk.cuda(), hv.cuda()
     p = b.params(U, wl.group, n, wl.window, B, pool_kernel=wl.pool_kernel,
                  lambda_v=wl.lambda_v, dtype=wl.dtype,
-                 flags={"default": 0, "fused": b.GRKV_FUSED_SCORE,
+                 flags={"default": 0, "two_pass": b.GRKV_TWO_PASS_SCORE,
                         "portable": b.GRKV_FORCE_SIMT}[a.path])
     ws = torch.empty(b.grkv_workspace_size(p), dtype=torch.uint8, device="cuda")
     ko = torch.empty((U, B, d), dtype=tdt, device="cuda")
@@ -435,7 +432,7 @@ def run_ours(a):
                    "pool_kernel": wl.pool_kernel, "l2": "inputs (K+V %.1f GB) exceed L2" %
                    (read / 1e9), "parallelism": f"units sharded, {world} rank(s)"},
         "path": a.path,
-        "roofline": {"bound": "hbm", "kernel": "grkv_score stage (window scoring + target)",
+        "roofline": {"bound": "hbm", "kernel": "grkv_score stage (k_score_pipe: window scoring + target, K read once)",
                      "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "traffic": score_traffic(wl) if a.path == "default" else None,

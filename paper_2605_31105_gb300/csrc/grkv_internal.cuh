@@ -26,7 +26,7 @@ struct Shape {
   int lambda_inf; // lambda_v == +inf: values stay V0
   int tc;         // bf16, m <= 128, not forced portable: tensor-core scoring
   int tc_merge;   // ... and B <= 32768: tensor-core value merge
-  int fused;      // tensor-core scoring as one launch in L2-sized rounds
+  int two_pass;   // tensor-core scoring as two launches that each read K
   int update_k;   // key step after the value step (GRKV_UPDATE_K)
   int cg_iters;   // most conjugate-gradient iterations of the key step
   float cg_tol;   // ... until ||r|| <= cg_tol ||e||
@@ -43,6 +43,7 @@ struct WsLayout {
   // score path (tensor cores)
   size_t pstats_tc;  // float2 [U][maxc][128] pass-A statistics slots
   size_t flags_tc;   // int [U] pass-A slots written per unit
+  size_t lam_tc;     // float [U][128] combined log2 row normalisers (one-read scoring)
   // select
   size_t pooled;  // float [U][P]
   // merge
@@ -83,9 +84,16 @@ cudaError_t launch_score_simt(const Shape& s, const void* q, const void* k, cons
                               const WsLayout& L, cudaStream_t st);
 cudaError_t launch_select(const Shape& s, const float* scores, int32_t* idx, char* ws,
                           const WsLayout& L, cudaStream_t st);
-// Tensor-core window scoring (bf16, m <= 128); mode 2 = fused rounds,
-// otherwise two launches.
+// Tensor-core window scoring (bf16, m <= 256 in blocks of 128 rows).  The
+// default reads K once (launch_score_pipe); launch_score_tc with mode 0 runs
+// two launches per row block that each read K.
 bool score_tc_supported(const Shape& s);
+int score_pipe_groups(const Shape& s);
+int score_pipe_slots(const Shape& s);
+size_t score_pipe_slot_bytes(const Shape& s);
+cudaError_t launch_score_pipe(const Shape& s, const void* q, const void* k, const void* v,
+                              float* scores, float* y, float* row_stats, char* ws,
+                              const WsLayout& L, cudaStream_t st);
 size_t score_tc_pstats_bytes(const Shape& s, int* maxc, int* gu, int* rounds, int sms);
 int sm_count();
 cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const void* v,

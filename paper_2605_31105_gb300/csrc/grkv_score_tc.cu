@@ -1,15 +1,14 @@
-// Window scoring on the 5th-generation tensor cores (bf16, d = 128, m <= 256).
+// Window scoring on the 5th-generation tensor cores in two launches per 128
+// window rows (bf16, d = 128, m <= 256): the comparison path of
+// GRKV_TWO_PASS_SCORE.  The default path (grkv_score_pipe.cu) reads K once.
 //
 // For every unit the path needs, over all n keys, the row statistics of the
 // window logits (pass A: M_r, L_r) and then, with those, the probabilities,
 // the per-key prefix scores c_j = sum_r P_rj and the target Y = P V (pass B);
 // Eq. 4 and Algorithm 1 of the paper.  The row normaliser depends on every
-// key, so the keys are read twice.  This kernel is persistent (one CTA per
-// SM) and processes the units in rounds small enough that a round's keys stay
-// in L2: each CTA runs pass A of round r+1 and then pass B of round r, so the
-// second read of K is served from L2 and only K and V cross HBM once (mode 2,
-// GRKV_FUSED_SCORE).  By default the two passes run as two launches over all
-// units (modes 0 and 1), which reads K twice but needs no cross-CTA waits.
+// key, so this path reads the keys twice: pass A (mode 0) and pass B (mode 1)
+// are two persistent launches over all units (one CTA per SM), each CTA on a
+// contiguous range of the units' tiles.
 //
 // Roles (512 threads): warp 0 issues TMA loads (the unit's Q, then K and V
 // tiles of 128 tokens through the ring; each V one job after its K, as
@@ -44,10 +43,8 @@ constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KB
 constexpr long long kWaitBudget = 1ll << 32;      // cycles (~2 s) before a wait gives up
 
 // Shared-memory layout (offsets from a 1024-byte aligned base) for kRing K/V
-// ring slots and kQBuf Q tiles.  The two-launch passes use 5 + 1: a CTA
-// switches units two or three times per launch.  The fused rounds use 4 + 2:
-// a CTA switches units every few tiles, and with two Q tiles the next
-// segment's Q is loaded while the current segment finishes.
+// ring slots and kQBuf Q tiles: 5 + 1 (a CTA switches units two or three
+// times per launch).
 template <int kRing, int kQBuf>
 struct Layout {
   static constexpr uint32_t kOffQ = 0;                                 // kQBuf x 32 KB
@@ -58,8 +55,7 @@ struct Layout {
   static constexpr uint32_t kOffBar = kOffLam + 2 * kRows * 4;
   static constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;         // + alignment slack
 };
-constexpr int kRingTwo = 5, kQBufTwo = 1;       // modes 0 and 1
-constexpr int kRingFused = 4, kQBufFused = 2;   // mode 2
+constexpr int kRingTwo = 5, kQBufTwo = 1;
 
 // TMEM columns: two S buffers, two Y accumulators.
 constexpr uint32_t kColS = 0, kColY = 256;
@@ -69,9 +65,9 @@ struct Args {
   int row0, mr;   // stacked rows row0 .. row0 + mr - 1 (mr <= 128) in this launch
   int acc;        // add the prefix scores to those of an earlier launch (rows before row0)
   int tpu;        // tiles per unit
-  int mode;       // 0: pass A only, 1: pass B only, 2: both, in rounds
-  int gu;         // units per round
-  int rounds;
+  int mode;       // 0: pass A, 1: pass B
+  int gu;         // units per round (all of them)
+  int rounds;     // 1
   int maxc;       // stats slots per unit
   float sl2;      // scale * log2(e)
   float* scores;  // [U][P]
@@ -90,21 +86,14 @@ struct Job {
   int seg_first, seg_last;
 };
 
-// The CTA's sequence of blocks is A(0), then A(r+1), B(r) for each round r,
-// ending with B(R-1) (mode 2), or a single A or B block over all units.
+// One block of jobs per launch: pass A (mode 0) or pass B (mode 1) over all
+// units, in one round.
 struct Sched {
   int U, tpu, G, cta, mode, gu, rounds;
-  __device__ int nblocks() const { return mode == 2 ? 2 * rounds : 1; }
-  __device__ void block(int p, int* kind, int* r) const {
-    if (mode != 2) {
-      *kind = mode;
-      *r = 0;
-      return;
-    }
-    if (p == 0) { *kind = 0; *r = 0; }
-    else if (p == 2 * rounds - 1) { *kind = 1; *r = rounds - 1; }
-    else if (p & 1) { *kind = 0; *r = (p + 1) / 2; }
-    else { *kind = 1; *r = p / 2 - 1; }
+  __device__ int nblocks() const { return 1; }
+  __device__ void block(int, int* kind, int* r) const {
+    *kind = mode;
+    *r = 0;
   }
   __device__ int round_units(int r) const { return min(gu, U - r * gu); }
   __device__ long long tiles(int r) const { return (long long)round_units(r) * tpu; }
@@ -231,9 +220,7 @@ struct Bars {
   uint32_t tmem;
   int abort;
 };
-static_assert(sizeof(Bars<kRingTwo, kQBufTwo>) <= 256 &&
-                  sizeof(Bars<kRingFused, kQBufFused>) <= 256,
-              "barrier block");
+static_assert(sizeof(Bars<kRingTwo, kQBufTwo>) <= 256, "barrier block");
 
 // Merges two (max, sum) row statistics in log2 units.
 __device__ __forceinline__ float2 stat_merge(float2 x, float2 y) {
@@ -333,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           // the job's K, then the V of the previous pass-B job: V waits in the
           // ring through a tile's compute, so it is fetched one tile later
-          ok = load(&tmK, j.j0, j.u, (j.kind == 0 && a.mode == 2) ? keep : stream);
+          ok = load(&tmK, j.j0, j.u, stream);
           if (ok && pend_v) {
             ok = load(&tmV, pv_j0, pv_u, stream);
             pend_v = false;
@@ -796,16 +783,10 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
   if (e != cudaSuccess) return e;
   auto launch = [&](int md) {
     a.mode = md;
-    if (md != 2) {
-      a.gu = s.U;
-      a.rounds = 1;
-    } else {
-      a.gu = gu;
-      a.rounds = rounds;
-    }
-    auto kern = md == 2 ? k_score_tc<kRingFused, kQBufFused> : k_score_tc<kRingTwo, kQBufTwo>;
-    const uint32_t smem = md == 2 ? Layout<kRingFused, kQBufFused>::kSmemBytes
-                                  : Layout<kRingTwo, kQBufTwo>::kSmemBytes;
+    a.gu = s.U;
+    a.rounds = 1;
+    auto kern = k_score_tc<kRingTwo, kQBufTwo>;
+    const uint32_t smem = Layout<kRingTwo, kQBufTwo>::kSmemBytes;
     cudaError_t fe = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (fe != cudaSuccess) return fe;
     cudaLaunchConfig_t cfg = {};
@@ -813,26 +794,18 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeCooperative;
-    attr[0].val.cooperative = md == 2 ? 1 : 0;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
     count_launches(1);
     return cudaLaunchKernelEx(&cfg, kern, mq, mk, mv, a);
   };
+  (void)mode;
   for (int row0 = 0; row0 < s.m; row0 += kRows) {
     a.row0 = row0;
     a.mr = std::min(kRows, s.m - row0);
     a.acc = row0 > 0;
     e = cudaMemsetAsync(a.unit_cnt, 0, (size_t)s.U * sizeof(int), st);
     if (e != cudaSuccess) return e;
-    if (mode == 2) {
-      e = launch(2);
-    } else {
-      e = launch(0);
-      if (e == cudaSuccess) e = launch(1);
-    }
+    e = launch(0);
+    if (e == cudaSuccess) e = launch(1);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

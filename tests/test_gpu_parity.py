@@ -52,7 +52,7 @@ def prep(request, grkv_lib):
     return Prepared(wl, over)
 
 
-PATHS = {"default": 0, "fused": b.GRKV_FUSED_SCORE, "portable": b.GRKV_FORCE_SIMT}
+PATHS = {"default": 0, "two_pass": b.GRKV_TWO_PASS_SCORE, "portable": b.GRKV_FORCE_SIMT}
 
 
 @pytest.mark.parametrize("path", list(PATHS))
