@@ -46,9 +46,9 @@ def args_():
     ap.add_argument("--cpu-seconds", type=float, default=20.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
-    ap.add_argument("--path", choices=("default", "two_pass", "portable"), default="default",
-                    help="scoring kernels: default (one tensor-core launch that reads K once), "
-                         "two_pass (two launches, K read twice) or portable (CUDA cores)")
+    ap.add_argument("--path", choices=("default", "one_read", "portable"), default="default",
+                    help="scoring kernels: default (two tensor-core launches, K read twice), "
+                         "one_read (one launch that reads K from HBM once) or portable (CUDA cores)")
     return ap.parse_args()
 
 
@@ -72,11 +72,11 @@ def algorithmic_bytes(wl):
     return read, write
 
 
-# DRAM bytes (read + write) of one grkv_score call (the one-read scoring kernel
-# k_score_pipe) from one ncu capture of the full workload.  A figure holds only
+# DRAM bytes (read + write) of one grkv_score call (both k_score_tc launches)
+# from one ncu capture of the full workload.  A figure holds only
 # for the kernel source it was taken on, so it is keyed by that file's digest
 # and reported as null once the kernel changes.
-SCORE_SRC = os.path.join("paper_2605_31105_gb300", "csrc", "grkv_score_pipe.cu")
+SCORE_SRC = os.path.join("paper_2605_31105_gb300", "csrc", "grkv_score_tc.cu")
 SCORE_TRAFFIC = {}
 
 
@@ -319,7 +319,7 @@ def run_ours(a):
     dq, dk, dv = hq.cuda(), hk.cuda(), hv.cuda()
     p = b.params(U, wl.group, n, wl.window, B, pool_kernel=wl.pool_kernel,
                  lambda_v=wl.lambda_v, dtype=wl.dtype,
-                 flags={"default": 0, "two_pass": b.GRKV_TWO_PASS_SCORE,
+                 flags={"default": 0, "one_read": b.GRKV_ONE_READ_SCORE,
                         "portable": b.GRKV_FORCE_SIMT}[a.path])
     ws = torch.empty(b.grkv_workspace_size(p), dtype=torch.uint8, device="cuda")
     ko = torch.empty((U, B, d), dtype=tdt, device="cuda")
@@ -432,7 +432,7 @@ def run_ours(a):
                    "pool_kernel": wl.pool_kernel, "l2": "inputs (K+V %.1f GB) exceed L2" %
                    (read / 1e9), "parallelism": f"units sharded, {world} rank(s)"},
         "path": a.path,
-        "roofline": {"bound": "hbm", "kernel": "grkv_score stage (k_score_pipe: window scoring + target, K read once)",
+        "roofline": {"bound": "hbm", "kernel": "grkv_score stage (k_score_tc: window scoring + target, two launches)",
                      "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "traffic": score_traffic(wl) if a.path == "default" else None,

@@ -77,11 +77,13 @@ extern "C" {
                                     the free slots, K0 on the fixed ones.  V* is v_out as
                                     written (rounded to dtype).  Without it K_out = K0 */
 #define GRKV_FORCE_SIMT    0x2u  /* use the portable CUDA-core kernels even for bf16 */
-#define GRKV_TWO_PASS_SCORE 0x4u /* tensor-core scoring as two launches per 128 window
-                                    rows, the statistics pass and the probability pass,
-                                    each reading K from HBM (a comparison path).  Default:
-                                    one launch per 128 rows that reads K from HBM once and
-                                    re-reads it from L2 */
+#define GRKV_ONE_READ_SCORE 0x4u /* tensor-core scoring in one launch per 128 window rows
+                                    that reads K from HBM once: groups of CTAs interleave
+                                    the statistics pass of one unit with the probability
+                                    pass of the previous one, which re-reads its keys from
+                                    L2.  Default: two launches per 128 rows (statistics,
+                                    then probabilities), each reading K from HBM, which
+                                    measures faster on GB300 */
 
 typedef struct {
   int32_t units;        /* U >= 0: independent (batch x layer x KV head) problems   */
@@ -102,7 +104,7 @@ typedef struct {
   float   scale;        /* logit scale; 0 -> fp32(1/sqrt(d))                        */
   int32_t causal;       /* 1: window slot a sees keys j <= n-w+a; 0: all n keys      */
   int32_t dtype;        /* GRKV_BF16 or GRKV_F32 for q, k, v, k_out, v_out          */
-  uint32_t flags;       /* GRKV_UPDATE_K, GRKV_FORCE_SIMT, GRKV_TWO_PASS_SCORE          */
+  uint32_t flags;       /* GRKV_UPDATE_K, GRKV_FORCE_SIMT, GRKV_ONE_READ_SCORE          */
   int32_t cg_iters;     /* 0..4096: most conjugate-gradient iterations of the key
                            step (512); read only under GRKV_UPDATE_K                */
   float   cg_tol;       /* >= 0, finite: the key step's CG stops once ||r|| <=

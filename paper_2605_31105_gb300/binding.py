@@ -28,7 +28,7 @@ GRKV_POOL_MAX = 0
 GRKV_POOL_AVG = 1
 GRKV_UPDATE_K = 0x1
 GRKV_FORCE_SIMT = 0x2
-GRKV_TWO_PASS_SCORE = 0x4
+GRKV_ONE_READ_SCORE = 0x4
 
 EXPORTS = ("grkv_params_init", "grkv_workspace_size", "grkv_score", "grkv_select", "grkv_merge",
            "grkv_compress", "grkv_status", "grkv_strerror", "grkv_launch_count",

@@ -42,9 +42,8 @@ cudaError_t launch_merge(const Shape& s, const void* q, const void* k, const voi
 cudaError_t launch_score(const Shape& s, const void* q, const void* k, const void* v,
                          float* scores, float* y, float* row_stats, char* ws, const WsLayout& L,
                          cudaStream_t st) {
-  if (s.tc && s.two_pass)
-    return launch_score_tc(s, q, k, v, scores, y, row_stats, ws, L, 0, st);
-  if (s.tc) return launch_score_pipe(s, q, k, v, scores, y, row_stats, ws, L, st);
+  if (s.tc && s.one_read) return launch_score_pipe(s, q, k, v, scores, y, row_stats, ws, L, st);
+  if (s.tc) return launch_score_tc(s, q, k, v, scores, y, row_stats, ws, L, 0, st);
   return launch_score_simt(s, q, k, v, scores, y, row_stats, ws, L, st);
 }
 
@@ -77,7 +76,7 @@ int make_shape(const grkv_params* p, Shape* s) {
   if (!(p->scale >= 0.f) || std::isinf(p->scale)) return GRKV_ERR_INVALID_ARG;
   if (p->causal != 0 && p->causal != 1) return GRKV_ERR_INVALID_ARG;
   if (p->dtype != GRKV_F32 && p->dtype != GRKV_BF16) return GRKV_ERR_INVALID_ARG;
-  if (p->flags & ~(GRKV_UPDATE_K | GRKV_FORCE_SIMT | GRKV_TWO_PASS_SCORE)) return GRKV_ERR_INVALID_ARG;
+  if (p->flags & ~(GRKV_UPDATE_K | GRKV_FORCE_SIMT | GRKV_ONE_READ_SCORE)) return GRKV_ERR_INVALID_ARG;
   if (p->d < 1) return GRKV_ERR_INVALID_ARG;
   if (p->flags & GRKV_UPDATE_K) {
     if (!(p->lambda_k >= 0.f) || std::isinf(p->lambda_k)) return GRKV_ERR_INVALID_ARG;
@@ -107,7 +106,7 @@ int make_shape(const grkv_params* p, Shape* s) {
   s->scale = p->scale != 0.f ? p->scale : (float)(1.0 / std::sqrt((double)p->d));
   s->tc = (p->flags & GRKV_FORCE_SIMT) ? 0 : (score_tc_supported(*s) ? 1 : 0);
   s->tc_merge = (s->tc && merge_tc_supported(*s)) ? 1 : 0;
-  s->two_pass = (p->flags & GRKV_TWO_PASS_SCORE) ? 1 : 0;
+  s->one_read = (p->flags & GRKV_ONE_READ_SCORE) ? 1 : 0;
   s->update_k = (p->flags & GRKV_UPDATE_K) ? 1 : 0;
   s->cg_iters = p->cg_iters;
   s->cg_tol = p->cg_tol;

@@ -26,7 +26,7 @@ struct Shape {
   int lambda_inf; // lambda_v == +inf: values stay V0
   int tc;         // bf16, m <= 128, not forced portable: tensor-core scoring
   int tc_merge;   // ... and B <= 32768: tensor-core value merge
-  int two_pass;   // tensor-core scoring as two launches that each read K
+  int one_read;   // tensor-core scoring in one launch that reads K from HBM once
   int update_k;   // key step after the value step (GRKV_UPDATE_K)
   int cg_iters;   // most conjugate-gradient iterations of the key step
   float cg_tol;   // ... until ||r|| <= cg_tol ||e||
@@ -85,11 +85,13 @@ cudaError_t launch_score_simt(const Shape& s, const void* q, const void* k, cons
 cudaError_t launch_select(const Shape& s, const float* scores, int32_t* idx, char* ws,
                           const WsLayout& L, cudaStream_t st);
 // Tensor-core window scoring (bf16, m <= 256 in blocks of 128 rows).  The
-// default reads K once (launch_score_pipe); launch_score_tc with mode 0 runs
-// two launches per row block that each read K.
+// default, launch_score_tc, runs two launches per row block that each read
+// K; launch_score_pipe (GRKV_ONE_READ_SCORE) reads K once.
 bool score_tc_supported(const Shape& s);
-int score_pipe_groups(const Shape& s);
-int score_pipe_slots(const Shape& s);
+struct PipePlan {
+  int ng, gs;   // CTA groups, CTAs per group
+};
+PipePlan score_pipe_plan(const Shape& s, int sms);
 size_t score_pipe_slot_bytes(const Shape& s);
 cudaError_t launch_score_pipe(const Shape& s, const void* q, const void* k, const void* v,
                               float* scores, float* y, float* row_stats, char* ws,

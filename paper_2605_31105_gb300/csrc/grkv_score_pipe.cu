@@ -22,13 +22,14 @@
 // them once; the lead gives the other CTAs of the group time to catch up.
 //
 // Roles (512 threads): warp 0 issues TMA loads (Q of the pass-B unit, the K
-// tile of every job, each pass-B job's V tile right after its K), warp 1 issues tcgen05 MMAs (each pass-B tile's Y^T MMA after the S
-// MMA of the job two later, so that the next pass-B S MMA does not wait for
-// it), warp 2 publishes pass-A statistics (and combines them in the last
-// CTA), warp 3 fetches a unit's normalisers ahead of its pass-B tiles, warps
-// 4-11 are two compute groups of 128 threads, warps 12-15 add the two
-// groups' halves of every pass-B tile's column scores and flush each pass-B
-// segment's Y partial.
+// tile of every job, each pass-B job's V tile right after its K) and L2
+// prefetches a few jobs ahead; warp 1 issues the S MMAs of every job; warp 2
+// issues the Y^T MMAs of the pass-B tiles (so that no S MMA waits behind a
+// probability tile); warp 3 publishes pass-A statistics (and combines them
+// in the last CTA) and fetches a unit's normalisers ahead of its pass-B
+// tiles; warps 4-11 are two compute groups of 128 threads; warps 12-15 add
+// the two groups' halves of every pass-B tile's column scores and flush each
+// pass-B segment's Y partial.
 //
 // Pass A: S = Q K^T (window rows on TMEM lanes, Q as the A operand in TMEM,
 // filled by the compute threads).  A compute thread owns one row; the two
@@ -58,12 +59,13 @@ constexpr int kTile = 128;      // tokens per tile
 constexpr int kRows = 128;      // window rows per launch (row block)
 constexpr int kThreads = 512;
 constexpr int kRing = 5;        // K / V ring slots
-constexpr int kLead = 4;        // pass-A tiles of a phase ahead of its first pass-B tile
+constexpr int kSBufs = 2;       // S tiles in TMEM
+constexpr int kLead = 8;        // pass-A tiles of a phase ahead of its first pass-B tile
 constexpr int kRedBufs = 4;
 constexpr int kPrefetch = 4;    // jobs whose K / V tiles are prefetched into L2 ahead of their loads     // column-score buffers (pass-B tiles in flight to the summers)
 constexpr uint32_t kTileBytes = kTile * kD * 2;    // 32 KB
 constexpr long long kWaitBudget = 1ll << 32;       // cycles (~2 s) before a wait gives up
-constexpr size_t kL2KeyBudget = (size_t)64 << 20;  // keys of the units in flight
+constexpr size_t kL2KeyBudget = (size_t)72 << 20;  // keys of the units in flight
 
 // Shared memory (offsets from a 1024-byte aligned base).
 constexpr uint32_t kOffQ = 0;                                   // Q of the pass-B unit, 32 KB
@@ -75,8 +77,10 @@ constexpr uint32_t kOffBar = kOffLam + 2 * kRows * 4;
 constexpr uint32_t kSmemBytes = kOffBar + 512 + 1024;           // + alignment slack
 static_assert(kSmemBytes <= 227 * 1024, "shared memory");
 
-// TMEM columns: two S buffers, the Y^T accumulator, two Q buffers (bf16 pairs).
-constexpr uint32_t kColS = 0, kColY = 256, kColQ = 384;
+// TMEM columns: two S buffers, the Y^T accumulator, two Q buffers of the
+// pass-A unit (bf16 pairs, the A operand of S = Q K^T).
+constexpr uint32_t kColS = 0, kColY = kSBufs * kTile, kColQ = kColY + kD;
+static_assert(kColQ + 2 * 64 <= 512, "TMEM columns");
 
 struct Args {
   int U, n, w, m, P, causal;
@@ -157,6 +161,15 @@ struct JobIter {
     return true;
   }
 };
+
+// mbar_wait for all 32 lanes of a warp with one answer: a lane that sees the
+// abort flag makes the whole warp give up, so warp-collective instructions
+// (tcgen05.ld / st, shuffles) that follow a wait are reached by all lanes or
+// by none.
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                               long long budget) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort, budget));
+}
 
 __device__ __forceinline__ int ld_acquire(const int* p) {
   int v;
@@ -251,13 +264,13 @@ struct Bars {
   uint64_t ring_full[kRing], ring_empty[kRing];
   uint64_t q_full, q_empty;          // Q of the pass-B unit (shared memory)
   uint64_t qa_full[2], qa_empty[2];  // Q of the pass-A unit (TMEM)
-  uint64_t s_full[2], s_done[2];
+  uint64_t s_full[kSBufs], s_done[kSBufs];
   uint64_t p_full[4];                // P^T written (pass-B tile nb uses nb % 4)
   uint64_t y_full, y_empty;
   uint64_t astat_full[2], astat_empty[2];
   uint64_t lam_full[2], lam_empty[2];
   uint64_t red_full[kRedBufs], red_empty[kRedBufs];  // column-score halves of a pass-B tile
-  uint64_t drain;
+  uint64_t drain, drain_y;
   uint32_t tmem;
   int abort;
 };
@@ -280,19 +293,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(&bars->q_full, 1);
     mbar_init(&bars->q_empty, 1);
+    for (int i = 0; i < kSBufs; ++i) {
+      mbar_init(&bars->s_full[i], 1);
+      mbar_init(&bars->s_done[i], 256);
+    }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bars->qa_full[i], 256);
       mbar_init(&bars->qa_empty[i], 1);
-      mbar_init(&bars->s_full[i], 1);
-      mbar_init(&bars->s_done[i], 256);
       mbar_init(&bars->astat_full[i], 256);
       mbar_init(&bars->astat_empty[i], 1);
       mbar_init(&bars->lam_full[i], 1);
       mbar_init(&bars->lam_empty[i], 256);
     }
-    // four P^T barriers: a pass-B tile's Y^T MMA waits for its P^T after the
-    // S MMA of the job two later, by which time the compute groups may have
-    // written the P^T of the next two pass-B tiles, never of the fourth
+    // four P^T barriers, one per pass-B tile in flight: the ring holds the K
+    // and V of at most two pass-B tiles whose Y^T MMA has not completed
     for (int i = 0; i < 4; ++i) mbar_init(&bars->p_full[i], 256);
     for (int i = 0; i < kRedBufs; ++i) {
       mbar_init(&bars->red_full[i], 256);
@@ -301,6 +315,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&bars->y_full, 1);
     mbar_init(&bars->y_empty, 128);
     mbar_init(&bars->drain, 1);
+    mbar_init(&bars->drain_y, 1);
     bars->abort = 0;
     fence_mbar_init();
   }
@@ -382,55 +397,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) set_status(a.status, GRKV_ERR_TIMEOUT);
     }
   } else if (warp == 1) {
-    // ----------------------------------------------------------- MMA issuer
+    // ------------------------------------------------------ S MMA issuer
+    // S = Q K^T (pass A, Q in TMEM) or S^T = K Q^T (pass B, Q in shared
+    // memory) of every job, as soon as the K tile has landed and the S
+    // buffer is free; the Y^T MMAs are issued by warp 2, so an S MMA never
+    // waits for a probability tile.
     if (lane == 0) {
       const uint32_t id_a = idesc_bf16(kRows, kTile, 0, 0);   // S = Q K^T
       const uint32_t id_b = idesc_bf16(kTile, kRows, 0, 0);   // S^T = K Q^T
-      const uint32_t id_y = idesc_bf16(kD, kRows, 1, 1);      // Y^T += V^T P^T, both MN-major
       JobIter it;
       it.init(a, gr);
-      uint32_t slot = 0, ring_use = 0;
-      int i = 0, aseg = 0, bseg = 0, nb = 0, y_uses = 0;
+      uint32_t ring_use = 0;
+      int i = 0, aseg = 0, bseg = 0;
       bool ok = true;
-      // pending Y^T MMAs (FIFO of at most two): the one of pass-B job k is
-      // issued after the S MMA of job k + 2, so that the S MMA of the next
-      // pass-B tile does not queue behind it; its P^T sits in its K tile's
-      // slot, its V in the next ring slot
-      struct PendY {
-        Job j;
-        uint32_t kslot, vslot, vuse;
-        int nb, k;
-      };
-      PendY pq[2];
-      int pq_n = 0, pq_h = 0;
-      auto issue_y = [&](const PendY& py) -> bool {
-        const uint32_t vslot = py.vslot, vuse = py.vuse;
-        bool k = true;
-        if (py.j.first && y_uses >= 1)
-          k = mbar_wait(&bars->y_empty, (y_uses - 1) & 1, abort_flag, kWaitBudget);
-        if (k) k = mbar_wait(&bars->p_full[py.nb & 3], (py.nb >> 2) & 1, abort_flag, kWaitBudget);
-        if (k) k = mbar_wait(&bars->ring_full[vslot], (vuse / kRing) & 1, abort_flag, kWaitBudget);
-        if (!k) return false;
-        tc_fence_after();
-        const uint32_t va = smem_u32(sm + kOffRing + vslot * kTileBytes);
-        const uint32_t pa = smem_u32(sm + kOffRing + py.kslot * kTileBytes);
-#pragma unroll
-        for (int kk = 0; kk < kTile / 16; ++kk)
-          mma_bf16(tmem + kColY, sw128_desc(va + kk * 2048, kTileBytes / 2, 1024),
-                   sw128_desc(pa + kk * 2048, kTileBytes / 2, 1024), id_y,
-                   (py.j.first && kk == 0) ? 0u : 1u);
-        mma_commit(&bars->ring_empty[vslot]);
-        mma_commit(&bars->ring_empty[py.kslot]);
-        if (py.j.last) {
-          mma_commit(&bars->y_full);
-          ++y_uses;
-        }
-        return true;
-      };
       Job j;
       while (ok && it.next(&j)) {
-        const int b = i & 1, use = i >> 1;
-        const uint32_t kslot = slot, kuse = ring_use;
+        const int b = i % kSBufs, use = i / kSBufs;
+        const uint32_t kuse = ring_use, kslot = kuse % kRing;
+        ring_use += j.kind == 1 ? 2 : 1;   // a pass-B job's V follows its K
         if (j.first) {
           if (j.kind == 0)
             ok = mbar_wait(&bars->qa_full[aseg & 1], (aseg >> 1) & 1, abort_flag, kWaitBudget);
@@ -465,35 +449,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             mma_bf16(tmem + kColS + b * kTile, sw128_desc(ka + off, 16, 1024),
                      sw128_desc(qa + off, 16, 1024), id_b, kk > 0);
           }
-          mma_commit(&bars->s_full[b]);   // the K slot is released after the Y^T MMA
+          // the K slot then takes the tile's P^T; warp 2 releases it
+          mma_commit(&bars->s_full[b]);
           if (j.last) {
             mma_commit(&bars->q_empty);
             ++bseg;
           }
         }
-        ++ring_use;
-        slot = (slot + 1) % kRing;
-        const uint32_t vslot = slot, vuse = ring_use;
-        if (j.kind == 1) {
-          ++ring_use;
-          slot = (slot + 1) % kRing;
-        }
-        while (ok && pq_n > 0 && pq[pq_h].k <= i - 2) {
-          ok = issue_y(pq[pq_h]);
-          pq_h ^= 1;
-          --pq_n;
-        }
-        if (!ok) break;
-        if (j.kind == 1) {
-          pq[(pq_h + pq_n) & 1] = PendY{j, kslot, vslot, vuse, nb++, i};
-          ++pq_n;
-        }
         ++i;
-      }
-      while (ok && pq_n > 0) {
-        ok = issue_y(pq[pq_h]);
-        pq_h ^= 1;
-        --pq_n;
       }
       // every MMA issued so far completes before TMEM can be released (this
       // wait ignores the abort flag, and is bounded)
@@ -503,108 +466,147 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) set_status(a.status, GRKV_ERR_TIMEOUT);
     }
   } else if (warp == 2) {
-    // ----------------------------------------------- statistics publisher
-    // Merges the two compute groups' statistics of each pass-A segment into
-    // this CTA's slot of the unit and counts it; the CTA whose count
-    // completes the unit combines all slots (in slot order) into the rows'
-    // log2 normalisers and the row statistics, then counts once more.
-    const float2* astat = (const float2*)(sm + kOffAstat);
-    JobIter it;
-    it.init(a, gr);
-    int aseg = 0;
-    bool ok = true;
-    Job j;
-    while (ok && it.next(&j)) {
-      if (!(j.kind == 0 && j.last)) continue;
-      const int ab = aseg & 1;
-      ok = mbar_wait(&bars->astat_full[ab], (aseg >> 1) & 1, abort_flag, kWaitBudget);
-      if (!ok) break;
-      float2* mine = a.pstats + ((size_t)j.u * a.maxgs + gr.i) * kRows;
+    // ---------------------------------------------------- Y^T MMA issuer
+    // Y^T += V^T P^T of every pass-B tile once its P^T is written (into the
+    // tile's K slot) and its V has landed; releases both slots.
+    if (lane == 0) {
+      const uint32_t id_y = idesc_bf16(kD, kRows, 1, 1);   // V^T and P^T both MN-major
+      JobIter it;
+      it.init(a, gr);
+      uint32_t ring_use = 0;
+      int nb = 0, y_uses = 0;
+      bool ok = true;
+      Job j;
+      while (ok && it.next(&j)) {
+        const uint32_t kuse = ring_use;
+        ring_use += j.kind == 1 ? 2 : 1;
+        if (j.kind != 1) continue;
+        const uint32_t kslot = kuse % kRing, vuse = kuse + 1, vslot = vuse % kRing;
+        if (j.first && y_uses >= 1)
+          ok = mbar_wait(&bars->y_empty, (y_uses - 1) & 1, abort_flag, kWaitBudget);
+        if (ok) ok = mbar_wait(&bars->p_full[nb & 3], (nb >> 2) & 1, abort_flag, kWaitBudget);
+        if (ok) ok = mbar_wait(&bars->ring_full[vslot], (vuse / kRing) & 1, abort_flag, kWaitBudget);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t va = smem_u32(sm + kOffRing + vslot * kTileBytes);
+        const uint32_t pa = smem_u32(sm + kOffRing + kslot * kTileBytes);
 #pragma unroll
-      for (int t = 0; t < 4; ++t) {
-        const int r = t * 32 + lane;
-        mine[r] = stat_merge(astat[(ab * 2 + 0) * kRows + r], astat[(ab * 2 + 1) * kRows + r]);
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->astat_empty[ab]);
-      __threadfence();
-      __syncwarp();
-      int old = 0;
-      if (lane == 0) old = atomicAdd(&a.unit_cnt[j.u], 1);
-      old = __shfl_sync(0xffffffffu, old, 0);
-      if (old == writers - 1) {
-        __threadfence();
-        float2 st[4];
-#pragma unroll
-        for (int t = 0; t < 4; ++t) st[t] = make_float2(-INFINITY, 0.f);
-        // eight slots per round trip: 32 independent loads in flight per lane
-        for (int k0 = 0; k0 < gr.size; k0 += 8) {
-          float2 pr[8][4];
-#pragma unroll
-          for (int kk = 0; kk < 8; ++kk) {
-            const int k = k0 + kk;
-            const bool use = k < gr.size && range_begin(a.tpu, k + 1, gr.size) >
-                                                range_begin(a.tpu, k, gr.size);
-            const float2* sl = a.pstats + ((size_t)j.u * a.maxgs + (use ? k : 0)) * kRows;
-#pragma unroll
-            for (int t = 0; t < 4; ++t)
-              pr[kk][t] = use ? __ldcg(sl + t * 32 + lane) : make_float2(-INFINITY, 0.f);
-          }
-#pragma unroll
-          for (int kk = 0; kk < 8; ++kk)
-#pragma unroll
-            for (int t = 0; t < 4; ++t) st[t] = stat_merge(st[t], pr[kk][t]);
+        for (int kk = 0; kk < kTile / 16; ++kk)
+          mma_bf16(tmem + kColY, sw128_desc(va + kk * 2048, kTileBytes / 2, 1024),
+                   sw128_desc(pa + kk * 2048, kTileBytes / 2, 1024), id_y,
+                   (j.first && kk == 0) ? 0u : 1u);
+        mma_commit(&bars->ring_empty[vslot]);
+        mma_commit(&bars->ring_empty[kslot]);
+        if (j.last) {
+          mma_commit(&bars->y_full);
+          ++y_uses;
         }
-#pragma unroll
-        for (int t = 0; t < 4; ++t) {
-          const int r = t * 32 + lane;
-          const bool live = r < a.mr && st[t].y > 0.f;
-          a.lam[(size_t)j.u * kRows + r] = live ? st[t].x + __log2f(st[t].y) : INFINITY;
-          if (r < a.mr) {
-            float* rs = a.row_stats + ((size_t)j.u * a.m + a.row0 + r) * 2;
-            rs[0] = st[t].x * 0.69314718055994531f;
-            rs[1] = st[t].y;
-          }
-        }
-        __threadfence();
-        __syncwarp();
-        if (lane == 0) atomicAdd(&a.unit_cnt[j.u], 1);
+        ++nb;
       }
-      ++aseg;
+      mma_commit(&bars->drain_y);
+      volatile int no_abort = 0;
+      mbar_wait(&bars->drain_y, 0, &no_abort, kWaitBudget);
+      if (!ok) set_status(a.status, GRKV_ERR_TIMEOUT);
     }
-    if (!ok && lane == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
   } else if (warp == 3) {
-    // ------------------------------------------------ statistics fetcher
-    // Ahead of each pass-B segment: wait (bounded) until the unit's
-    // normalisers are published, and leave them in shared memory.
+    // ------------------------------------------------- row statistics
+    // In job order: at the end of each pass-A segment, merges the two
+    // compute groups' statistics into this CTA's slot of the unit and
+    // counts it (the CTA whose count completes the unit combines all slots,
+    // in slot order, into the rows' log2 normalisers and the row statistics,
+    // then counts once more); ahead of each pass-B segment, waits (bounded)
+    // until the unit's normalisers are published and leaves them in shared
+    // memory.  A unit's pass-A segment precedes its pass-B segment in every
+    // CTA's job order, so the two duties share one warp without waiting on
+    // each other.
+    const float2* astat = (const float2*)(sm + kOffAstat);
     float* lam_s = (float*)(sm + kOffLam);
     JobIter it;
     it.init(a, gr);
-    int bseg = 0;
+    int aseg = 0, bseg = 0;
     bool ok = true;
     Job j;
     while (ok && it.next(&j)) {
-      if (!(j.kind == 1 && j.first)) continue;
-      const int lb = bseg & 1;
-      if (bseg >= 2)
-        ok = mbar_wait(&bars->lam_empty[lb], ((bseg >> 1) - 1) & 1, abort_flag, kWaitBudget);
-      if (!ok) break;
-      const long long t0 = clock64();
-      while (ld_acquire(&a.unit_cnt[j.u]) < writers + 1) {
-        if (*abort_flag || clock64() - t0 > kWaitBudget) {
-          *abort_flag = 1;
-          ok = false;
-          break;
-        }
-        __nanosleep(64);
-      }
-      if (!ok) break;
+      if (j.kind == 0 && j.last) {
+        const int ab = aseg & 1;
+        ok = mbar_wait_warp(&bars->astat_full[ab], (aseg >> 1) & 1, abort_flag, kWaitBudget);
+        if (!ok) break;
+        float2* mine = a.pstats + ((size_t)j.u * a.maxgs + gr.i) * kRows;
 #pragma unroll
-      for (int t = 0; t < 4; ++t)
-        lam_s[lb * kRows + t * 32 + lane] = __ldcg(a.lam + (size_t)j.u * kRows + t * 32 + lane);
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->lam_full[lb]);
-      ++bseg;
+        for (int t = 0; t < 4; ++t) {
+          const int r = t * 32 + lane;
+          mine[r] = stat_merge(astat[(ab * 2 + 0) * kRows + r], astat[(ab * 2 + 1) * kRows + r]);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->astat_empty[ab]);
+        __threadfence();
+        __syncwarp();
+        int old = 0;
+        if (lane == 0) old = atomicAdd(&a.unit_cnt[j.u], 1);
+        old = __shfl_sync(0xffffffffu, old, 0);
+        if (old == writers - 1) {
+          __threadfence();
+          float2 st[4];
+#pragma unroll
+          for (int t = 0; t < 4; ++t) st[t] = make_float2(-INFINITY, 0.f);
+          // eight slots per round trip: 32 independent loads in flight per lane
+          for (int k0 = 0; k0 < gr.size; k0 += 8) {
+            float2 pr[8][4];
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+              const int k = k0 + kk;
+              const bool use = k < gr.size && range_begin(a.tpu, k + 1, gr.size) >
+                                                  range_begin(a.tpu, k, gr.size);
+              const float2* sl = a.pstats + ((size_t)j.u * a.maxgs + (use ? k : 0)) * kRows;
+#pragma unroll
+              for (int t = 0; t < 4; ++t)
+                pr[kk][t] = use ? __ldcg(sl + t * 32 + lane) : make_float2(-INFINITY, 0.f);
+            }
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk)
+#pragma unroll
+              for (int t = 0; t < 4; ++t) st[t] = stat_merge(st[t], pr[kk][t]);
+          }
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            const int r = t * 32 + lane;
+            const bool live = r < a.mr && st[t].y > 0.f;
+            a.lam[(size_t)j.u * kRows + r] = live ? st[t].x + __log2f(st[t].y) : INFINITY;
+            if (r < a.mr) {
+              float* rs = a.row_stats + ((size_t)j.u * a.m + a.row0 + r) * 2;
+              rs[0] = st[t].x * 0.69314718055994531f;
+              rs[1] = st[t].y;
+            }
+          }
+          __threadfence();
+          __syncwarp();
+          if (lane == 0) atomicAdd(&a.unit_cnt[j.u], 1);
+        }
+        ++aseg;
+      } else if (j.kind == 1 && j.first) {
+        const int lb = bseg & 1;
+        if (bseg >= 2)
+          ok = mbar_wait_warp(&bars->lam_empty[lb], ((bseg >> 1) - 1) & 1, abort_flag,
+                              kWaitBudget);
+        if (!ok) break;
+        const long long t0 = clock64();
+        while (ld_acquire(&a.unit_cnt[j.u]) < writers + 1) {
+          if (*abort_flag || clock64() - t0 > kWaitBudget) {
+            *abort_flag = 1;
+            ok = false;
+            break;
+          }
+          __nanosleep(64);
+        }
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) break;
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+          lam_s[lb * kRows + t * 32 + lane] = __ldcg(a.lam + (size_t)j.u * kRows + t * 32 + lane);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bars->lam_full[lb]);
+        ++bseg;
+      }
     }
     if (!ok && lane == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
   } else if (warp >= 12) {
@@ -625,7 +627,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     while (ok && it.next(&j)) {
       if (j.kind != 1) continue;
       const int rb = nb % kRedBufs;
-      ok = mbar_wait(&bars->red_full[rb], (nb / kRedBufs) & 1, abort_flag, kWaitBudget);
+      ok = mbar_wait_warp(&bars->red_full[rb], (nb / kRedBufs) & 1, abort_flag, kWaitBudget);
       if (!ok) break;
       const float c2 = red[(rb * 2) * kTile + t] + red[(rb * 2 + 1) * kTile + t];
       mbar_arrive(&bars->red_empty[rb]);
@@ -636,7 +638,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         *dst = a.acc ? *dst + c2 : c2;
       }
       if (!j.last) continue;
-      ok = mbar_wait(&bars->y_full, bseg & 1, abort_flag, kWaitBudget);
+      ok = mbar_wait_warp(&bars->y_full, bseg & 1, abort_flag, kWaitBudget);
       if (!ok) break;
       tc_fence_after();
       float* yu = a.y + ((size_t)j.u * a.m + a.row0) * kD + t;
@@ -672,7 +674,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto fill_q = [&](int s) -> bool {
       const int buf = s & 1;
       if (s >= 2 &&
-          !mbar_wait(&bars->qa_empty[buf], ((s >> 1) - 1) & 1, abort_flag, kWaitBudget))
+          !mbar_wait_warp(&bars->qa_empty[buf], ((s >> 1) - 1) & 1, abort_flag, kWaitBudget))
         return false;
       tc_fence_after();
       const int u = gr.g + a.ng * s;
@@ -709,9 +711,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     float M = -INFINITY, L = 0.f;   // pass-A running stats of this row (log2 units)
     Job j;
     while (ok && it.next(&j)) {
-      const int b = i & 1;
-      // ring slot of this job's K tile (the same count as the producer's: a
-      // pass-B job's V follows its K)
+      const int b = i % kSBufs, sp = (i / kSBufs) & 1;
+      // ring slot of this job's K tile (the producer's count: a pass-B job's V
+      // follows its K); a pass-B tile's P^T goes into its K slot
       const uint32_t kslot = ring_use % kRing;
       ring_use += j.kind == 1 ? 2 : 1;
       if (j.kind == 0) {
@@ -721,7 +723,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           L = 0.f;
           if (aseg + 1 < it.nu && !(ok = fill_q(aseg + 1))) break;
         }
-        ok = mbar_wait(&bars->s_full[b], (i >> 1) & 1, abort_flag, kWaitBudget);
+        ok = mbar_wait_warp(&bars->s_full[b], sp, abort_flag, kWaitBudget);
         if (!ok) break;
         tc_fence_after();
         const int t0 = j.j0 + 64 * wg;
@@ -742,7 +744,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (j.last) {
           const int ab = aseg & 1;
           if (aseg >= 2)
-            ok = mbar_wait(&bars->astat_empty[ab], ((aseg >> 1) - 1) & 1, abort_flag,
+            ok = mbar_wait_warp(&bars->astat_empty[ab], ((aseg >> 1) - 1) & 1, abort_flag,
                            kWaitBudget);
           if (!ok) break;
           astat[(ab * 2 + wg) * kRows + lr] = make_float2(M, L);
@@ -753,10 +755,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---- pass B: this thread's token over the group's 64 rows
         const int lb = bseg & 1;
         if (j.first) {
-          ok = mbar_wait(&bars->lam_full[lb], (bseg >> 1) & 1, abort_flag, kWaitBudget);
+          ok = mbar_wait_warp(&bars->lam_full[lb], (bseg >> 1) & 1, abort_flag, kWaitBudget);
           if (!ok) break;
         }
-        ok = mbar_wait(&bars->s_full[b], (i >> 1) & 1, abort_flag, kWaitBudget);
+        ok = mbar_wait_warp(&bars->s_full[b], sp, abort_flag, kWaitBudget);
         if (!ok) break;
         tc_fence_after();
         const uint32_t sbase = lane_addr + kColS + b * kTile + 64 * wg;
@@ -767,8 +769,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool full = tok && (!a.causal || jt <= a.n - a.w);
         const int thr = a.causal ? jt - (a.n - a.w) : INT_MIN;
         const float* lam = lam_s + lb * kRows + 64 * wg;
-        // P^T row of this token in the K tile's slot (MN-major, 128-byte
-        // swizzle: half wg holds rows 64 wg .. 64 wg + 63)
+        // P^T row of this token (MN-major, 128-byte swizzle: half wg holds
+        // rows 64 wg .. 64 wg + 63)
         const uint32_t pT =
             smem_u32(sm + kOffRing + kslot * kTileBytes) + wg * (kTileBytes / 2) + lr * 128;
         float va[32], vb[32], csum;
@@ -789,7 +791,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // this group's half of the token's column score, for the summers
         const int rb = nb % kRedBufs;
         if (nb >= kRedBufs)
-          ok = mbar_wait(&bars->red_empty[rb], ((nb / kRedBufs) - 1) & 1, abort_flag, kWaitBudget);
+          ok = mbar_wait_warp(&bars->red_empty[rb], ((nb / kRedBufs) - 1) & 1, abort_flag, kWaitBudget);
         if (!ok) break;
         red[(rb * 2 + wg) * kTile + lr] = csum;
         mbar_arrive(&bars->red_full[rb]);
@@ -811,19 +813,36 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-int score_pipe_groups(const Shape& s) {
+// Groups and group size for a grid of at most G CTAs.  At most
+// kL2KeyBudget of keys may be in flight (one unit per group); within that,
+// the plan minimises the modelled time: phases (units per group + 1) x
+// (tiles per CTA and phase + two tiles' worth of statistics exchange), where
+// a group whose CTAs hold unequal tile counts pays 15% (every CTA of a group
+// waits for its slowest one at each phase).
+PipePlan score_pipe_plan(const Shape& s, int G) {
+  const int tpu = (s.n + kTile - 1) / kTile;
   const size_t unit_k = (size_t)s.n * kD * 2;
-  const size_t g = std::max<size_t>(1, kL2KeyBudget / unit_k);
-  return (int)std::min<size_t>(g, (size_t)std::max(1, s.U));
-}
-
-int score_pipe_slots(const Shape& s) {
-  const int ng = score_pipe_groups(s);
-  return (kMaxScoreCtas + ng - 1) / ng;
+  const int ng_max = (int)std::min<size_t>(std::max<size_t>(1, kL2KeyBudget / unit_k),
+                                           (size_t)std::max(1, std::min(s.U, G)));
+  PipePlan best{1, std::max(1, G)};
+  double best_t = 1e300;
+  for (int ng = 1; ng <= ng_max; ++ng) {
+    for (int gs = 1; gs * ng <= G; ++gs) {
+      const double t = (double)((s.U + ng - 1) / ng + 1) *
+                       ((tpu + gs - 1) / gs * (tpu % gs == 0 || tpu < gs ? 1.0 : 1.15) + 2.0);
+      if (t < best_t * (1 - 1e-9) || (t <= best_t * (1 + 1e-9) && ng * gs > best.ng * best.gs)) {
+        best_t = t;
+        best = PipePlan{ng, gs};
+      }
+    }
+  }
+  return best;
 }
 
 size_t score_pipe_slot_bytes(const Shape& s) {
-  return (size_t)s.U * score_pipe_slots(s) * kRows * sizeof(float2);
+  const int G = sm_count();
+  const PipePlan pl = score_pipe_plan(s, G > 0 ? G : kMaxScoreCtas);
+  return (size_t)s.U * pl.gs * kRows * sizeof(float2);
 }
 
 cudaError_t launch_score_pipe(const Shape& s, const void* q, const void* k, const void* v,
@@ -834,8 +853,10 @@ cudaError_t launch_score_pipe(const Shape& s, const void* q, const void* k, cons
       !encode_bf16_3d(&mk, k, kD, s.n, s.U, 64, kTile) ||
       !encode_bf16_3d(&mv, v, kD, s.n, s.U, 64, kTile))
     return cudaErrorInvalidValue;
-  const int G = sm_count();
-  if (G <= 0 || G > kMaxScoreCtas) return cudaErrorInvalidDevice;
+  const int sms = sm_count();
+  if (sms <= 0 || sms > kMaxScoreCtas) return cudaErrorInvalidDevice;
+  const PipePlan pl = score_pipe_plan(s, sms);
+  const int G = pl.ng * pl.gs;   // the grid: ng groups of gs CTAs
   Args a{};
   a.U = s.U;
   a.n = s.n;
@@ -844,8 +865,8 @@ cudaError_t launch_score_pipe(const Shape& s, const void* q, const void* k, cons
   a.P = s.P;
   a.causal = s.causal;
   a.tpu = (s.n + kTile - 1) / kTile;
-  a.ng = std::min(score_pipe_groups(s), G);
-  a.maxgs = score_pipe_slots(s);
+  a.ng = pl.ng;
+  a.maxgs = pl.gs;
   a.sl2 = (float)((double)s.scale * 1.4426950408889634);
   a.q = (const __nv_bfloat16*)q;
   a.scores = scores;

@@ -1,6 +1,6 @@
 // Window scoring on the 5th-generation tensor cores in two launches per 128
-// window rows (bf16, d = 128, m <= 256): the comparison path of
-// GRKV_TWO_PASS_SCORE.  The default path (grkv_score_pipe.cu) reads K once.
+// window rows (bf16, d = 128, m <= 256), the default scoring path.  The
+// one-read path of GRKV_ONE_READ_SCORE is in grkv_score_pipe.cu.
 //
 // For every unit the path needs, over all n keys, the row statistics of the
 // window logits (pass A: M_r, L_r) and then, with those, the probabilities,

@@ -52,7 +52,7 @@ def prep(request, grkv_lib):
     return Prepared(wl, over)
 
 
-PATHS = {"default": 0, "two_pass": b.GRKV_TWO_PASS_SCORE, "portable": b.GRKV_FORCE_SIMT}
+PATHS = {"default": 0, "one_read": b.GRKV_ONE_READ_SCORE, "portable": b.GRKV_FORCE_SIMT}
 
 
 @pytest.mark.parametrize("path", list(PATHS))
@@ -299,6 +299,12 @@ def test_full_size_c2_sampled_units(grkv_lib):
     """The 32-layer, 32K-token workload (256 units) at full size; eight units
     spread over the layers against the oracle."""
     _compress_sampled(gi.workload(2), (0, 37, 74, 111, 148, 185, 222, 255))
+
+
+def test_full_size_c2_one_read_scoring(grkv_lib):
+    """The one-read scoring path (GRKV_ONE_READ_SCORE: groups of CTAs, K re-read
+    from L2) at the full 256-unit size, where every CTA runs many phases."""
+    _compress_sampled(gi.workload(2), (0, 131, 255), flags=b.GRKV_ONE_READ_SCORE)
 
 
 def test_full_size_c3_mistral_128k_sampled_units(grkv_lib):
