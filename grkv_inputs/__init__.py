@@ -38,7 +38,7 @@ import numpy as np
 
 __all__ = [
     "Workload", "workload", "WORKLOADS", "sweep_points", "unit_arrays",
-    "fill_units", "bf16_bits", "bf16_value", "seed_for",
+    "fill_units", "bf16_bits", "bf16_value", "seed_for", "heldout_queries",
 ]
 
 BASE_SEED = 0x47524B56  # "GRKV"
@@ -148,6 +148,26 @@ def _lowrank_keys(g: np.random.Generator, n: int, d: int) -> np.ndarray:
 def unit_arrays(wl: Workload, unit: int):
     """(q [g][w][d], k [n][d], v [n][d]) of one unit as float32 arrays whose
     values are exactly representable in the workload dtype."""
+    return _unit_draw(wl, unit)[:3]
+
+
+def heldout_queries(wl: Workload, unit: int, count: int) -> np.ndarray:
+    """count held-out decoding queries per query head of one unit, [g][count][d]
+    float32 (dtype-exact): drawn like the window queries (noisy copies of
+    random keys, or of the unit's topic direction for the span recipe) from
+    a stream of their own, so that they are not the surrogate window."""
+    _, k, _, topic = _unit_draw(wl, unit)
+    g = np.random.Generator(np.random.Philox(np.random.SeedSequence([wl.seed, unit, 0x484F4C44])))
+    noise = g.standard_normal((wl.group, count, wl.d), dtype=np.float32) * np.float32(0.5)
+    if topic is not None:
+        q = (2.0 * np.sqrt(wl.d) * topic).astype(np.float32)[None, None, :] + noise
+    else:
+        rows = g.integers(0, wl.n, size=(wl.group, count))
+        q = np.float32(2.0) * k[rows] + noise
+    return _round(q, wl.dtype)
+
+
+def _unit_draw(wl: Workload, unit: int):
     g = _rng(wl, unit)
     n, d, w, grp = wl.n, wl.d, wl.window, wl.group
     k = _lowrank_keys(g, n, d)
@@ -177,7 +197,7 @@ def unit_arrays(wl: Workload, unit: int):
         rows = g.integers(0, n, size=(grp, w))
         q = np.float32(2.0) * k[rows] + noise
     q = _round(q, wl.dtype)
-    return q, k, v
+    return q, k, v, topic
 
 
 def _store(dst: np.ndarray, x: np.ndarray, dtype: str):

@@ -85,6 +85,21 @@ extern "C" {
                                     then probabilities), each reading K from HBM, which
                                     measures faster on GB300 */
 
+#define GRKV_DETERMINISTIC  0x8u /* bitwise run-to-run reproducible outputs: the target Y
+                                    is summed from per-CTA partials in a fixed order
+                                    instead of with float atomics (costs a workspace of
+                                    U x slots x m x d floats and one more kernel; selects
+                                    the two-launch scoring even with GRKV_ONE_READ_SCORE).
+                                    Every other step is reproducible in either mode */
+
+#define GRKV_TEST_TIMEOUT 0x80000000u /* tests only: exercises the exit of the bounded device
+                                    waits.  grkv_score / grkv_compress score with the
+                                    one-read kernel (bf16), whose first CTA then withholds
+                                    one arrive, with the waits' budget cut to ~2 ms: the
+                                    kernel gives up, frees its tensor memory, returns, and
+                                    grkv_status reports GRKV_ERR_TIMEOUT; outputs are
+                                    unspecified.  Ignored by the other kernels */
+
 typedef struct {
   int32_t units;        /* U >= 0: independent (batch x layer x KV head) problems   */
   int32_t group;        /* g >= 1: query heads per KV head                          */
@@ -104,7 +119,8 @@ typedef struct {
   float   scale;        /* logit scale; 0 -> fp32(1/sqrt(d))                        */
   int32_t causal;       /* 1: window slot a sees keys j <= n-w+a; 0: all n keys      */
   int32_t dtype;        /* GRKV_BF16 or GRKV_F32 for q, k, v, k_out, v_out          */
-  uint32_t flags;       /* GRKV_UPDATE_K, GRKV_FORCE_SIMT, GRKV_ONE_READ_SCORE          */
+  uint32_t flags;       /* GRKV_UPDATE_K, GRKV_FORCE_SIMT, GRKV_ONE_READ_SCORE,
+                           GRKV_DETERMINISTIC, GRKV_TEST_TIMEOUT          */
   int32_t cg_iters;     /* 0..4096: most conjugate-gradient iterations of the key
                            step (512); read only under GRKV_UPDATE_K                */
   float   cg_tol;       /* >= 0, finite: the key step's CG stops once ||r|| <=
@@ -157,6 +173,54 @@ int grkv_merge(const grkv_params* p, const void* q, const void* k, const void* v
 int grkv_compress(const grkv_params* p, const void* q, const void* k, const void* v,
                   void* k_out, void* v_out, int32_t* idx,
                   void* ws, size_t ws_bytes, void* stream);
+
+/* grkv_compress with a budget per unit (the paper pairs GRKV with layer-wise
+ * (PyramidKV) and head-wise (Ada-KV) budget allocations, Sec. 4.2).
+ * budgets: HOST array [U], window <= budgets[u] <= n; p->budget is ignored.
+ * Outputs are packed: unit u's budgets[u] entries of idx and rows of k_out /
+ * v_out start at row off_u = budgets[0] + ... + budgets[u-1] (idx [sum B_u]
+ * int32, k_out / v_out [sum B_u][d]); each unit's results are those of
+ * grkv_compress with B = budgets[u].  The scoring step runs once over all
+ * units; selection and the value (and key) step run once per run of
+ * consecutive units with equal budgets.  ws must hold
+ * grkv_compress_ragged_workspace_size bytes; device errors of any run go to
+ * its status word (grkv_status). */
+int grkv_compress_ragged_workspace_size(const grkv_params* p, const int32_t* budgets,
+                                        size_t* bytes);
+int grkv_compress_ragged(const grkv_params* p, const int32_t* budgets, const void* q,
+                         const void* k, const void* v, void* k_out, void* v_out, int32_t* idx,
+                         void* ws, size_t ws_bytes, void* stream);
+
+/* Decode-side transfer check (the paper's App. G: the normalised discrepancy
+ * L_common of its loss-performance diagnostic and its held-out-query stress
+ * test).  For every unit it compares the eviction-only cache (K0, V0) =
+ * (K[idx], V[idx]) and the compressed cache (k_out, v_out) with the full
+ * cache, through the attention outputs Y = A V of two query sets:
+ *   q_win  [U][g][w][d]     the surrogate window (the same rule as grkv_score:
+ *                           over a B-slot cache, window row a sees slots
+ *                           j <= B - w + a when causal)
+ *   q_held [U][g][held][d]  held-out decoding queries, which see every slot
+ * and writes report [U][8] fp32:
+ *   [0] e_win(K0,V0)  = ||Y_win_full - Y_win(K0,V0)||_F^2
+ *   [1] e_win(out)    = ||Y_win_full - Y_win(k_out,v_out)||_F^2
+ *   [2] e_held(K0,V0) and [3] e_held(out), the same for the held-out queries
+ *   [4] ||Y_win_full||_F^2, [5] ||Y_held_full||_F^2
+ *   [6] cosine between the mean window output and the mean held-out output
+ *       over the full cache (the surrogate-actual similarity)
+ *   [7] 1 if the compressed cache lowers the window error but raises the
+ *       held-out error (the paper's failure case), else 0.
+ * L_common over a set of units is sum([3]) / sum([5]).  idx, k_out and v_out
+ * are laid out as grkv_compress writes them; held must satisfy 1 <= held <=
+ * budget and group * held <= 256.  Uses the default scoring kernels
+ * (GRKV_FORCE_SIMT and GRKV_DETERMINISTIC apply, the other flags are
+ * ignored); sums in fp64; a tie of the two caches' errors is not a failure.  ws must hold
+ * grkv_transfer_workspace_size bytes; device errors go to its status word,
+ * read with grkv_status. */
+int grkv_transfer_workspace_size(const grkv_params* p, int32_t held, size_t* bytes);
+int grkv_transfer_check(const grkv_params* p, int32_t held, const void* q_win,
+                        const void* q_held, const void* k, const void* v, const int32_t* idx,
+                        const void* k_out, const void* v_out, float* report,
+                        void* ws, size_t ws_bytes, void* stream);
 
 /* grkv_select without a workspace.  The paper has no counterpart: this entry
  * point exists for callers that cannot give the library scratch device

@@ -43,7 +43,7 @@ __all__ = [
     "Params", "effective_scale", "window_logits", "softmax_rows", "window_attention",
     "target", "column_scores", "pool", "select", "fixed_set", "retained_attention",
     "value_step_dual", "value_step_primal", "key_jvp", "key_vjp", "key_step_dual",
-    "alternate", "merge_unit", "compress_unit",
+    "alternate", "merge_unit", "compress_unit", "cache_output", "transfer_check", "l_common",
 ]
 
 f64 = np.float64
@@ -363,3 +363,57 @@ def compress_unit(q, k, v, p: Params, mode: str = "dual", idx=None):
     out.update({"attn": A, "row_max": M, "row_sum": L, "y": Y, "scores": c,
                 "scores32": c32, "pooled": pooled, "idx": np.asarray(idx, dtype=np.int32)})
     return out
+
+
+# --------------------------------------------------- decode-side transfer check
+def cache_output(q, kc, vc, p: Params, window_rule: bool):
+    """Y = A V of the stacked queries q [g][h][d] over a cache of c rows
+    (kc, vc [c][d]): the attention output the paper's diagnostics compare
+    (App. G, "Y = AV").  window_rule: the queries are the surrogate window
+    (h = p.window) and row a sees slots j <= c - w + a, the window occupying
+    the cache's last w slots (the retained-cache rule of Algorithm 1 under
+    the causal reading); otherwise every query sees every slot (decoding
+    queries come after the whole prompt)."""
+    q = np.asarray(q, dtype=f64)
+    g, h = q.shape[0], q.shape[1]
+    kc = np.asarray(kc, dtype=f64)
+    sub = dataclasses.replace(p, group=g, window=h, n=kc.shape[0], budget=kc.shape[0],
+                              causal=bool(window_rule and p.causal))
+    A, _, _ = softmax_rows(window_logits(q, kc, sub))
+    return A @ np.asarray(vc, dtype=f64)
+
+
+def transfer_check(q_win, q_held, k, v, idx, k_out, v_out, p: Params) -> dict:
+    """Decode-side transfer check of one unit (App. G: the normalised
+    discrepancy of the loss-performance diagnostic and the held-out-query
+    stress test), comparing the compressed cache (k_out, v_out) with the
+    eviction-only cache (K0, V0) = (K[idx], V[idx]) against the full cache:
+        e_win(c)  = ||Y_win_full - Y_win(c)||_F^2    (surrogate window queries)
+        e_held(c) = ||Y_held_full - Y_held(c)||_F^2  (held-out queries)
+    A failure is a unit whose compressed cache lowers the window error but
+    raises the held-out error relative to the eviction-only cache.  cos is
+    the cosine between the mean window output and the mean held-out output
+    over the full cache (the surrogate-actual similarity of Sec. 3.2)."""
+    idx = np.asarray(idx)
+    K0 = np.asarray(k, dtype=f64)[idx]
+    V0 = np.asarray(v, dtype=f64)[idx]
+    yw = cache_output(q_win, k, v, p, True)
+    yh = cache_output(q_held, k, v, p, False)
+    out = {"y_win2": float((yw ** 2).sum()), "y_held2": float((yh ** 2).sum())}
+    for name, kc, vc in (("base", K0, V0), ("comp", k_out, v_out)):
+        out["e_win_" + name] = float(((yw - cache_output(q_win, kc, vc, p, True)) ** 2).sum())
+        out["e_held_" + name] = float(((yh - cache_output(q_held, kc, vc, p, False)) ** 2).sum())
+    sw, sh = yw.mean(axis=0), yh.mean(axis=0)
+    out["cos"] = float(sw @ sh / max(np.linalg.norm(sw) * np.linalg.norm(sh), 1e-300))
+    out["fail"] = bool(out["e_win_comp"] < out["e_win_base"] and
+                       out["e_held_comp"] > out["e_held_base"])
+    return out
+
+
+def l_common(reports, which: str = "comp", queries: str = "held") -> float:
+    """L_common = sum over units of ||Y_full - Y_c||_F^2 / sum of ||Y_full||_F^2
+    (App. G, normalised discrepancy), for cache `which` ("comp" or "base")
+    and the held-out or window queries."""
+    num = sum(r[f"e_{queries}_{which}"] for r in reports)
+    den = sum(r["y_held2" if queries == "held" else "y_win2"] for r in reports)
+    return num / den

@@ -29,10 +29,13 @@ GRKV_POOL_AVG = 1
 GRKV_UPDATE_K = 0x1
 GRKV_FORCE_SIMT = 0x2
 GRKV_ONE_READ_SCORE = 0x4
+GRKV_DETERMINISTIC = 0x8
+GRKV_TEST_TIMEOUT = 0x80000000
 
 EXPORTS = ("grkv_params_init", "grkv_workspace_size", "grkv_score", "grkv_select", "grkv_merge",
            "grkv_compress", "grkv_status", "grkv_strerror", "grkv_launch_count",
-           "grkv_select_noalloc")
+           "grkv_select_noalloc", "grkv_transfer_workspace_size", "grkv_transfer_check",
+           "grkv_compress_ragged_workspace_size", "grkv_compress_ragged")
 
 
 class grkv_params(ctypes.Structure):
@@ -82,8 +85,17 @@ def load():
     lib.grkv_select_noalloc.restype = ctypes.c_int
     lib.grkv_launch_count.argtypes = []
     lib.grkv_launch_count.restype = ctypes.c_uint64
+    lib.grkv_transfer_workspace_size.argtypes = [_P, ctypes.c_int32, ctypes.POINTER(ctypes.c_size_t)]
+    lib.grkv_transfer_check.argtypes = [_P, ctypes.c_int32, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                        _vp, _vp, ctypes.c_size_t, _vp]
+    _ip = ctypes.POINTER(ctypes.c_int32)
+    lib.grkv_compress_ragged_workspace_size.argtypes = [_P, _ip, ctypes.POINTER(ctypes.c_size_t)]
+    lib.grkv_compress_ragged.argtypes = [_P, _ip, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                         ctypes.c_size_t, _vp]
     for name in ("grkv_workspace_size", "grkv_score", "grkv_select", "grkv_merge",
-                 "grkv_compress", "grkv_status"):
+                 "grkv_compress", "grkv_status", "grkv_transfer_workspace_size",
+                 "grkv_transfer_check", "grkv_compress_ragged_workspace_size",
+                 "grkv_compress_ragged"):
         getattr(lib, name).restype = ctypes.c_int
     _lib = lib
     return lib
@@ -173,6 +185,46 @@ def grkv_select_noalloc(p, scores, idx, stream=None, check=True):
     """grkv_select with the library's built-in scratch array (no workspace)."""
     rc = load().grkv_select_noalloc(ctypes.byref(p), _ptr(scores), _ptr(idx), _stream(stream))
     return _check(rc, "grkv_select_noalloc", check)
+
+
+def grkv_transfer_workspace_size(p, held: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(load().grkv_transfer_workspace_size(ctypes.byref(p), held, ctypes.byref(n)),
+           "grkv_transfer_workspace_size", True)
+    return n.value
+
+
+def grkv_transfer_check(p, held, q_win, q_held, k, v, idx, k_out, v_out, report, ws,
+                        ws_bytes=None, stream=None, check=True):
+    """Decode-side transfer check: report [U][8] fp32 (see include/grkv.h)."""
+    ws_bytes = ws.numel() * ws.element_size() if ws_bytes is None else ws_bytes
+    rc = load().grkv_transfer_check(ctypes.byref(p), held, _ptr(q_win), _ptr(q_held), _ptr(k),
+                                    _ptr(v), _ptr(idx), _ptr(k_out), _ptr(v_out), _ptr(report),
+                                    _ptr(ws), ws_bytes, _stream(stream))
+    return _check(rc, "grkv_transfer_check", check)
+
+
+def _budgets(budgets):
+    arr = (ctypes.c_int32 * len(budgets))(*[int(x) for x in budgets])
+    return arr
+
+
+def grkv_compress_ragged_workspace_size(p, budgets) -> int:
+    n = ctypes.c_size_t(0)
+    _check(load().grkv_compress_ragged_workspace_size(ctypes.byref(p), _budgets(budgets),
+                                                      ctypes.byref(n)),
+           "grkv_compress_ragged_workspace_size", True)
+    return n.value
+
+
+def grkv_compress_ragged(p, budgets, q, k, v, k_out, v_out, idx, ws, ws_bytes=None,
+                         stream=None, check=True):
+    """grkv_compress with one budget per unit (host list); packed outputs."""
+    ws_bytes = ws.numel() * ws.element_size() if ws_bytes is None else ws_bytes
+    rc = load().grkv_compress_ragged(ctypes.byref(p), _budgets(budgets), _ptr(q), _ptr(k),
+                                     _ptr(v), _ptr(k_out), _ptr(v_out), _ptr(idx), _ptr(ws),
+                                     ws_bytes, _stream(stream))
+    return _check(rc, "grkv_compress_ragged", check)
 
 
 def grkv_launch_count() -> int:

@@ -30,23 +30,6 @@ int check_ptr(const void* p, size_t elems) {
 
 int cuda_rc(cudaError_t e) { return e == cudaSuccess ? GRKV_OK : GRKV_ERR_CUDA; }
 
-cudaError_t launch_merge(const Shape& s, const void* q, const void* k, const void* v,
-                         const float* scores, const float* y, const float* row_stats,
-                         const int32_t* idx, void* k_out, void* v_out, char* ws, const WsLayout& L,
-                         cudaStream_t st) {
-  if (s.tc_merge)
-    return launch_merge_tc(s, q, k, v, scores, y, row_stats, idx, k_out, v_out, ws, L, st);
-  return launch_merge_simt(s, q, k, v, scores, y, idx, k_out, v_out, ws, L, st);
-}
-
-cudaError_t launch_score(const Shape& s, const void* q, const void* k, const void* v,
-                         float* scores, float* y, float* row_stats, char* ws, const WsLayout& L,
-                         cudaStream_t st) {
-  if (s.tc && s.one_read) return launch_score_pipe(s, q, k, v, scores, y, row_stats, ws, L, st);
-  if (s.tc) return launch_score_tc(s, q, k, v, scores, y, row_stats, ws, L, 0, st);
-  return launch_score_simt(s, q, k, v, scores, y, row_stats, ws, L, st);
-}
-
 #define GRKV_TRY(expr)            \
   do {                            \
     const int rc_ = (expr);       \
@@ -64,6 +47,27 @@ int check_inputs(const Shape& s, const void* q, const void* k, const void* v) {
 
 namespace grkv {
 
+// The value step (and gather) on the tensor cores or the portable kernels.
+cudaError_t launch_merge_any(const Shape& s, const void* q, const void* k, const void* v,
+                             const float* scores, const float* y, const float* row_stats,
+                             const int32_t* idx, void* k_out, void* v_out, char* ws,
+                             const WsLayout& L, cudaStream_t st) {
+  if (s.tc_merge)
+    return launch_merge_tc(s, q, k, v, scores, y, row_stats, idx, k_out, v_out, ws, L, st);
+  return launch_merge_simt(s, q, k, v, scores, y, idx, k_out, v_out, ws, L, st);
+}
+
+// Window scoring: the two-launch tensor-core kernel (default), the one-read
+// kernel, or the portable kernels.
+cudaError_t launch_score_any(const Shape& s, const void* q, const void* k, const void* v,
+                             float* scores, float* y, float* row_stats, char* ws,
+                             const WsLayout& L, cudaStream_t st) {
+  if (s.tc && (s.one_read || s.test_timeout) && !s.deterministic)
+    return launch_score_pipe(s, q, k, v, scores, y, row_stats, ws, L, st);
+  if (s.tc) return launch_score_tc(s, q, k, v, scores, y, row_stats, ws, L, 0, st);
+  return launch_score_simt(s, q, k, v, scores, y, row_stats, ws, L, st);
+}
+
 int make_shape(const grkv_params* p, Shape* s) {
   if (!p) return GRKV_ERR_INVALID_ARG;
   if (p->units < 0 || p->group < 1 || p->window < 1 || p->n < p->window) return GRKV_ERR_INVALID_ARG;
@@ -76,7 +80,8 @@ int make_shape(const grkv_params* p, Shape* s) {
   if (!(p->scale >= 0.f) || std::isinf(p->scale)) return GRKV_ERR_INVALID_ARG;
   if (p->causal != 0 && p->causal != 1) return GRKV_ERR_INVALID_ARG;
   if (p->dtype != GRKV_F32 && p->dtype != GRKV_BF16) return GRKV_ERR_INVALID_ARG;
-  if (p->flags & ~(GRKV_UPDATE_K | GRKV_FORCE_SIMT | GRKV_ONE_READ_SCORE)) return GRKV_ERR_INVALID_ARG;
+  if (p->flags & ~(GRKV_UPDATE_K | GRKV_FORCE_SIMT | GRKV_ONE_READ_SCORE | GRKV_DETERMINISTIC |
+                   GRKV_TEST_TIMEOUT)) return GRKV_ERR_INVALID_ARG;
   if (p->d < 1) return GRKV_ERR_INVALID_ARG;
   if (p->flags & GRKV_UPDATE_K) {
     if (!(p->lambda_k >= 0.f) || std::isinf(p->lambda_k)) return GRKV_ERR_INVALID_ARG;
@@ -107,6 +112,8 @@ int make_shape(const grkv_params* p, Shape* s) {
   s->tc = (p->flags & GRKV_FORCE_SIMT) ? 0 : (score_tc_supported(*s) ? 1 : 0);
   s->tc_merge = (s->tc && merge_tc_supported(*s)) ? 1 : 0;
   s->one_read = (p->flags & GRKV_ONE_READ_SCORE) ? 1 : 0;
+  s->deterministic = (p->flags & GRKV_DETERMINISTIC) ? 1 : 0;
+  s->test_timeout = (p->flags & GRKV_TEST_TIMEOUT) ? 1 : 0;
   s->update_k = (p->flags & GRKV_UPDATE_K) ? 1 : 0;
   s->cg_iters = p->cg_iters;
   s->cg_tol = p->cg_tol;
@@ -136,6 +143,7 @@ WsLayout plan_workspace(const Shape& s) {
                                 score_pipe_slot_bytes(s)));
     L.flags_tc = take(U * sizeof(int));
     L.lam_tc = take(U * 128 * sizeof(float));
+    if (s.deterministic) L.ypart_tc = take(U * (size_t)maxc * m * d * sizeof(float));
   } else {
     L.pstats = take(U * L.nchunk * m * 8);
     L.ypart = take(U * L.nchunk * m * d * 4);
@@ -206,7 +214,7 @@ int grkv_score(const grkv_params* p, const void* q, const void* k, const void* v
   char* w = (char*)ws;
   GRKV_TRY(cuda_rc(cudaMemsetAsync(w + L.status, 0, 4, st)));
   if (s.U == 0) return GRKV_OK;
-  return cuda_rc(launch_score(s, q, k, v, scores, y, row_stats, w, L, st));
+  return cuda_rc(launch_score_any(s, q, k, v, scores, y, row_stats, w, L, st));
 }
 
 int grkv_select(const grkv_params* p, const float* scores, int32_t* idx, void* ws,
@@ -242,7 +250,7 @@ int grkv_merge(const grkv_params* p, const void* q, const void* k, const void* v
   char* w = (char*)ws;
   GRKV_TRY(cuda_rc(cudaMemsetAsync(w + L.status, 0, 4, st)));
   if (s.U == 0) return GRKV_OK;
-  GRKV_TRY(cuda_rc(launch_merge(s, q, k, v, scores, y, row_stats, idx, k_out, v_out, w, L, st)));
+  GRKV_TRY(cuda_rc(launch_merge_any(s, q, k, v, scores, y, row_stats, idx, k_out, v_out, w, L, st)));
   if (!s.update_k) return GRKV_OK;
   return cuda_rc(launch_key_step(s, q, y, scores, idx, v_out, k_out, w, L, st));
 }
@@ -264,9 +272,9 @@ int grkv_compress(const grkv_params* p, const void* q, const void* k, const void
   float* scores = (float*)(w + L.scores);
   float* y = (float*)(w + L.y);
   float* rstats = (float*)(w + L.rstats);
-  GRKV_TRY(cuda_rc(launch_score(s, q, k, v, scores, y, rstats, w, L, st)));
+  GRKV_TRY(cuda_rc(launch_score_any(s, q, k, v, scores, y, rstats, w, L, st)));
   GRKV_TRY(cuda_rc(launch_select(s, scores, idx, w, L, st)));
-  GRKV_TRY(cuda_rc(launch_merge(s, q, k, v, scores, y, rstats, idx, k_out, v_out, w, L, st)));
+  GRKV_TRY(cuda_rc(launch_merge_any(s, q, k, v, scores, y, rstats, idx, k_out, v_out, w, L, st)));
   if (!s.update_k) return GRKV_OK;
   return cuda_rc(launch_key_step(s, q, y, scores, idx, v_out, k_out, w, L, st));
 }

@@ -27,6 +27,8 @@ struct Shape {
   int tc;         // bf16, m <= 128, not forced portable: tensor-core scoring
   int tc_merge;   // ... and B <= 32768: tensor-core value merge
   int one_read;   // tensor-core scoring in one launch that reads K from HBM once
+  int deterministic;  // Y summed in a fixed order (GRKV_DETERMINISTIC)
+  int test_timeout;   // GRKV_TEST_TIMEOUT (tests of the bounded-wait exit)
   int update_k;   // key step after the value step (GRKV_UPDATE_K)
   int cg_iters;   // most conjugate-gradient iterations of the key step
   float cg_tol;   // ... until ||r|| <= cg_tol ||e||
@@ -44,6 +46,7 @@ struct WsLayout {
   size_t pstats_tc;  // float2 [U][maxc][128] pass-A statistics slots
   size_t flags_tc;   // int [U] pass-A slots written per unit
   size_t lam_tc;     // float [U][128] combined log2 row normalisers (one-read scoring)
+  size_t ypart_tc;   // float [U][maxc][m][128] segment Y partials (deterministic mode)
   // select
   size_t pooled;  // float [U][P]
   // merge
@@ -122,6 +125,15 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
 bool select_uses_pooled_buffer(const Shape& s);
 cudaError_t launch_select_pooled(const Shape& s, const float* scores, int32_t* idx,
                                  float* pooled, cudaStream_t st);
+// Dispatch of the scoring step and of the value step to the kernels the
+// shape selects (as every entry point runs them).
+cudaError_t launch_score_any(const Shape& s, const void* q, const void* k, const void* v,
+                             float* scores, float* y, float* row_stats, char* ws,
+                             const WsLayout& L, cudaStream_t st);
+cudaError_t launch_merge_any(const Shape& s, const void* q, const void* k, const void* v,
+                             const float* scores, const float* y, const float* row_stats,
+                             const int32_t* idx, void* k_out, void* v_out, char* ws,
+                             const WsLayout& L, cudaStream_t st);
 // Host-side parameter validation shared by the entry points.
 int make_shape(const grkv_params* p, Shape* s);
 cudaError_t launch_merge_simt(const Shape& s, const void* q, const void* k, const void* v,

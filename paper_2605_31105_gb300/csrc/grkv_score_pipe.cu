@@ -65,6 +65,7 @@ constexpr int kRedBufs = 4;
 constexpr int kPrefetch = 4;    // jobs whose K / V tiles are prefetched into L2 ahead of their loads     // column-score buffers (pass-B tiles in flight to the summers)
 constexpr uint32_t kTileBytes = kTile * kD * 2;    // 32 KB
 constexpr long long kWaitBudget = 1ll << 32;       // cycles (~2 s) before a wait gives up
+constexpr long long kTestWaitBudget = 1ll << 22;   // ~2 ms: the budget of GRKV_TEST_TIMEOUT
 constexpr size_t kL2KeyBudget = (size_t)72 << 20;  // keys of the units in flight
 
 // Shared memory (offsets from a 1024-byte aligned base).
@@ -98,6 +99,8 @@ struct Args {
   float* lam;        // [U][128]         combined log2 normalisers
   int* unit_cnt;     // [U] slots written (+1 once combined), zeroed by the host
   int* status;
+  long long wait_budget;   // cycles before a bounded wait gives up
+  int test_withhold;       // GRKV_TEST_TIMEOUT: CTA 0 withholds one arrive
 };
 
 // The group of CTA c, its index inside the group and the group's size: group
@@ -346,7 +349,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto load = [&](const CUtensorMap* map, int j0, int u, uint64_t pol) -> bool {
         if (ring_use >= kRing &&
             !mbar_wait(&bars->ring_empty[slot], ((ring_use / kRing) - 1) & 1, abort_flag,
-                       kWaitBudget))
+                       a.wait_budget))
           return false;
         uint8_t* dst = sm + kOffRing + slot * kTileBytes;
         mbar_expect_tx(&bars->ring_full[slot], kTileBytes);
@@ -376,7 +379,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (j.kind == 1 && j.first) {
           // Q of the pass-B unit, once the previous pass-B segment's MMAs are done
           if (q_loads >= 1)
-            ok = mbar_wait(&bars->q_empty, (q_loads - 1) & 1, abort_flag, kWaitBudget);
+            ok = mbar_wait(&bars->q_empty, (q_loads - 1) & 1, abort_flag, a.wait_budget);
           if (!ok) break;
           mbar_expect_tx(&bars->q_full, kTileBytes);
           tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, a.row0, j.u, keep);
@@ -392,8 +395,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       // the abort flag, and are bounded)
       volatile int no_abort = 0;
       for (uint32_t i = ring_use > kRing ? ring_use - kRing : 0; i < ring_use; ++i)
-        mbar_wait(&bars->ring_full[i % kRing], (i / kRing) & 1, &no_abort, kWaitBudget);
-      if (q_loads > 0) mbar_wait(&bars->q_full, (q_loads - 1) & 1, &no_abort, kWaitBudget);
+        mbar_wait(&bars->ring_full[i % kRing], (i / kRing) & 1, &no_abort, a.wait_budget);
+      if (q_loads > 0) mbar_wait(&bars->q_full, (q_loads - 1) & 1, &no_abort, a.wait_budget);
       if (!ok) set_status(a.status, GRKV_ERR_TIMEOUT);
     }
   } else if (warp == 1) {
@@ -417,13 +420,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         ring_use += j.kind == 1 ? 2 : 1;   // a pass-B job's V follows its K
         if (j.first) {
           if (j.kind == 0)
-            ok = mbar_wait(&bars->qa_full[aseg & 1], (aseg >> 1) & 1, abort_flag, kWaitBudget);
+            ok = mbar_wait(&bars->qa_full[aseg & 1], (aseg >> 1) & 1, abort_flag, a.wait_budget);
           else
-            ok = mbar_wait(&bars->q_full, bseg & 1, abort_flag, kWaitBudget);
+            ok = mbar_wait(&bars->q_full, bseg & 1, abort_flag, a.wait_budget);
         }
-        if (ok) ok = mbar_wait(&bars->ring_full[kslot], (kuse / kRing) & 1, abort_flag, kWaitBudget);
+        if (ok) ok = mbar_wait(&bars->ring_full[kslot], (kuse / kRing) & 1, abort_flag, a.wait_budget);
         if (ok && use >= 1)
-          ok = mbar_wait(&bars->s_done[b], (use - 1) & 1, abort_flag, kWaitBudget);
+          ok = mbar_wait(&bars->s_done[b], (use - 1) & 1, abort_flag, a.wait_budget);
         if (!ok) break;
         tc_fence_after();
         const uint32_t ka = smem_u32(sm + kOffRing + kslot * kTileBytes);
@@ -462,7 +465,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // wait ignores the abort flag, and is bounded)
       mma_commit(&bars->drain);
       volatile int no_abort = 0;
-      mbar_wait(&bars->drain, 0, &no_abort, kWaitBudget);
+      mbar_wait(&bars->drain, 0, &no_abort, a.wait_budget);
       if (!ok) set_status(a.status, GRKV_ERR_TIMEOUT);
     }
   } else if (warp == 2) {
@@ -483,9 +486,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (j.kind != 1) continue;
         const uint32_t kslot = kuse % kRing, vuse = kuse + 1, vslot = vuse % kRing;
         if (j.first && y_uses >= 1)
-          ok = mbar_wait(&bars->y_empty, (y_uses - 1) & 1, abort_flag, kWaitBudget);
-        if (ok) ok = mbar_wait(&bars->p_full[nb & 3], (nb >> 2) & 1, abort_flag, kWaitBudget);
-        if (ok) ok = mbar_wait(&bars->ring_full[vslot], (vuse / kRing) & 1, abort_flag, kWaitBudget);
+          ok = mbar_wait(&bars->y_empty, (y_uses - 1) & 1, abort_flag, a.wait_budget);
+        if (ok) ok = mbar_wait(&bars->p_full[nb & 3], (nb >> 2) & 1, abort_flag, a.wait_budget);
+        if (ok) ok = mbar_wait(&bars->ring_full[vslot], (vuse / kRing) & 1, abort_flag, a.wait_budget);
         if (!ok) break;
         tc_fence_after();
         const uint32_t va = smem_u32(sm + kOffRing + vslot * kTileBytes);
@@ -505,7 +508,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       mma_commit(&bars->drain_y);
       volatile int no_abort = 0;
-      mbar_wait(&bars->drain_y, 0, &no_abort, kWaitBudget);
+      mbar_wait(&bars->drain_y, 0, &no_abort, a.wait_budget);
       if (!ok) set_status(a.status, GRKV_ERR_TIMEOUT);
     }
   } else if (warp == 3) {
@@ -529,7 +532,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     while (ok && it.next(&j)) {
       if (j.kind == 0 && j.last) {
         const int ab = aseg & 1;
-        ok = mbar_wait_warp(&bars->astat_full[ab], (aseg >> 1) & 1, abort_flag, kWaitBudget);
+        ok = mbar_wait_warp(&bars->astat_full[ab], (aseg >> 1) & 1, abort_flag, a.wait_budget);
         if (!ok) break;
         float2* mine = a.pstats + ((size_t)j.u * a.maxgs + gr.i) * kRows;
 #pragma unroll
@@ -587,11 +590,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int lb = bseg & 1;
         if (bseg >= 2)
           ok = mbar_wait_warp(&bars->lam_empty[lb], ((bseg >> 1) - 1) & 1, abort_flag,
-                              kWaitBudget);
+                              a.wait_budget);
         if (!ok) break;
         const long long t0 = clock64();
         while (ld_acquire(&a.unit_cnt[j.u]) < writers + 1) {
-          if (*abort_flag || clock64() - t0 > kWaitBudget) {
+          if (*abort_flag || clock64() - t0 > a.wait_budget) {
             *abort_flag = 1;
             ok = false;
             break;
@@ -604,7 +607,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int t = 0; t < 4; ++t)
           lam_s[lb * kRows + t * 32 + lane] = __ldcg(a.lam + (size_t)j.u * kRows + t * 32 + lane);
         __syncwarp();
-        if (lane == 0) mbar_arrive(&bars->lam_full[lb]);
+        // GRKV_TEST_TIMEOUT: CTA 0 never announces its first pass-B
+        // normalisers, so its compute groups' bounded wait expires
+        if (lane == 0 && !(a.test_withhold && blockIdx.x == 0 && bseg == 0))
+          mbar_arrive(&bars->lam_full[lb]);
         ++bseg;
       }
     }
@@ -627,7 +633,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     while (ok && it.next(&j)) {
       if (j.kind != 1) continue;
       const int rb = nb % kRedBufs;
-      ok = mbar_wait_warp(&bars->red_full[rb], (nb / kRedBufs) & 1, abort_flag, kWaitBudget);
+      ok = mbar_wait_warp(&bars->red_full[rb], (nb / kRedBufs) & 1, abort_flag, a.wait_budget);
       if (!ok) break;
       const float c2 = red[(rb * 2) * kTile + t] + red[(rb * 2 + 1) * kTile + t];
       mbar_arrive(&bars->red_empty[rb]);
@@ -638,7 +644,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         *dst = a.acc ? *dst + c2 : c2;
       }
       if (!j.last) continue;
-      ok = mbar_wait_warp(&bars->y_full, bseg & 1, abort_flag, kWaitBudget);
+      ok = mbar_wait_warp(&bars->y_full, bseg & 1, abort_flag, a.wait_budget);
       if (!ok) break;
       tc_fence_after();
       float* yu = a.y + ((size_t)j.u * a.m + a.row0) * kD + t;
@@ -674,7 +680,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto fill_q = [&](int s) -> bool {
       const int buf = s & 1;
       if (s >= 2 &&
-          !mbar_wait_warp(&bars->qa_empty[buf], ((s >> 1) - 1) & 1, abort_flag, kWaitBudget))
+          !mbar_wait_warp(&bars->qa_empty[buf], ((s >> 1) - 1) & 1, abort_flag, a.wait_budget))
         return false;
       tc_fence_after();
       const int u = gr.g + a.ng * s;
@@ -723,7 +729,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           L = 0.f;
           if (aseg + 1 < it.nu && !(ok = fill_q(aseg + 1))) break;
         }
-        ok = mbar_wait_warp(&bars->s_full[b], sp, abort_flag, kWaitBudget);
+        ok = mbar_wait_warp(&bars->s_full[b], sp, abort_flag, a.wait_budget);
         if (!ok) break;
         tc_fence_after();
         const int t0 = j.j0 + 64 * wg;
@@ -745,7 +751,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int ab = aseg & 1;
           if (aseg >= 2)
             ok = mbar_wait_warp(&bars->astat_empty[ab], ((aseg >> 1) - 1) & 1, abort_flag,
-                           kWaitBudget);
+                           a.wait_budget);
           if (!ok) break;
           astat[(ab * 2 + wg) * kRows + lr] = make_float2(M, L);
           mbar_arrive(&bars->astat_full[ab]);
@@ -755,10 +761,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---- pass B: this thread's token over the group's 64 rows
         const int lb = bseg & 1;
         if (j.first) {
-          ok = mbar_wait_warp(&bars->lam_full[lb], (bseg >> 1) & 1, abort_flag, kWaitBudget);
+          ok = mbar_wait_warp(&bars->lam_full[lb], (bseg >> 1) & 1, abort_flag, a.wait_budget);
           if (!ok) break;
         }
-        ok = mbar_wait_warp(&bars->s_full[b], sp, abort_flag, kWaitBudget);
+        ok = mbar_wait_warp(&bars->s_full[b], sp, abort_flag, a.wait_budget);
         if (!ok) break;
         tc_fence_after();
         const uint32_t sbase = lane_addr + kColS + b * kTile + 64 * wg;
@@ -791,7 +797,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // this group's half of the token's column score, for the summers
         const int rb = nb % kRedBufs;
         if (nb >= kRedBufs)
-          ok = mbar_wait_warp(&bars->red_empty[rb], ((nb / kRedBufs) - 1) & 1, abort_flag, kWaitBudget);
+          ok = mbar_wait_warp(&bars->red_empty[rb], ((nb / kRedBufs) - 1) & 1, abort_flag, a.wait_budget);
         if (!ok) break;
         red[(rb * 2 + wg) * kTile + lr] = csum;
         mbar_arrive(&bars->red_full[rb]);
@@ -876,6 +882,8 @@ cudaError_t launch_score_pipe(const Shape& s, const void* q, const void* k, cons
   a.lam = (float*)(ws + L.lam_tc);
   a.unit_cnt = (int*)(ws + L.flags_tc);
   a.status = (int*)(ws + L.status);
+  a.test_withhold = s.test_timeout;
+  a.wait_budget = s.test_timeout ? kTestWaitBudget : kWaitBudget;
   cudaError_t e = cudaMemsetAsync(y, 0, (size_t)s.U * s.m * kD * sizeof(float), st);
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(k_score_pipe, cudaFuncAttributeMaxDynamicSharedMemorySize,

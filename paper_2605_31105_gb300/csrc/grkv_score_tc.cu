@@ -76,6 +76,7 @@ struct Args {
   float2* pstats;    // [U][maxc][128]  (max in log2 units, sum)
   int* unit_cnt;     // [U] pass-A slots written, zeroed by the host
   int* status;
+  float* ypart;      // [U][maxc][m][128] segment Y partials (deterministic mode) or null
 };
 
 // ------------------------------------------------------------ job schedule
@@ -578,7 +579,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           float v[32];
           tmem_ld32(ybase + c * 32, v);
           tmem_ld_wait();
-          if (row < a.mr) {
+          if (row < a.mr && a.ypart) {
+            // the segment's partial into its own slot, summed in slot order later
+            const int k = (int)blockIdx.x - sc.first_cta(j.u);
+            float4* dst = (float4*)(a.ypart + (((size_t)j.u * a.maxc + k) * a.m + a.row0 + row) *
+                                                  kD + c * 32);
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+              dst[e] = make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+          } else if (row < a.mr) {
             float4* dst = (float4*)(a.y + ((size_t)j.u * a.m + a.row0 + row) * kD + c * 32);
 #pragma unroll
             for (int e = 0; e < 8; ++e)
@@ -715,6 +724,26 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) tmem_dealloc(tmem, 512);
 }
 
+// Deterministic mode: Y[u] = sum over the unit's slots k = 0 .. maxc-1 of the
+// segment partials, in slot order (unwritten slots hold zeros).
+__global__ void k_y_sum_slots(const float4* __restrict__ part, float4* __restrict__ y, int U,
+                              int m, int maxc) {
+  const size_t per_unit = (size_t)m * kD / 4;
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < (size_t)U * per_unit;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const size_t u = i / per_unit, r = i - u * per_unit;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int k = 0; k < maxc; ++k) {
+      const float4 x = __ldg(part + (u * maxc + k) * per_unit + r);
+      acc.x += x.x;
+      acc.y += x.y;
+      acc.z += x.z;
+      acc.w += x.w;
+    }
+    y[i] = acc;
+  }
+}
+
 int g_num_sms[64] = {};
 
 }  // namespace
@@ -779,7 +808,10 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
   a.pstats = (float2*)(ws + L.pstats_tc);
   a.unit_cnt = (int*)(ws + L.flags_tc);
   a.status = (int*)(ws + L.status);
-  cudaError_t e = cudaMemsetAsync(y, 0, (size_t)s.U * s.m * kD * sizeof(float), st);
+  a.ypart = s.deterministic ? (float*)(ws + L.ypart_tc) : nullptr;
+  const size_t part_bytes = (size_t)s.U * maxc * s.m * kD * sizeof(float);
+  cudaError_t e = a.ypart ? cudaMemsetAsync(a.ypart, 0, part_bytes, st)
+                          : cudaMemsetAsync(y, 0, (size_t)s.U * s.m * kD * sizeof(float), st);
   if (e != cudaSuccess) return e;
   auto launch = [&](int md) {
     a.mode = md;
@@ -807,6 +839,13 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
     e = launch(0);
     if (e == cudaSuccess) e = launch(1);
     if (e != cudaSuccess) return e;
+  }
+  if (a.ypart) {
+    const size_t n4 = (size_t)s.U * s.m * kD / 4;
+    const int blocks = (int)std::min<size_t>((n4 + 255) / 256, (size_t)G * 8);
+    k_y_sum_slots<<<blocks, 256, 0, st>>>((const float4*)a.ypart, (float4*)y, s.U, s.m, maxc);
+    count_launches(1);
+    e = cudaGetLastError();
   }
   return cudaSuccess;
 }

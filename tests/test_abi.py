@@ -116,3 +116,18 @@ def test_strerror(lib):
     assert b.strerror(0) == "ok"
     assert "Cholesky" in b.strerror(b.GRKV_ERR_NUMERIC)
     assert b.strerror(-99) == "unknown error"
+
+
+def test_transfer_check_validation(lib):
+    import ctypes as C
+    p = b.params(8, 4, 8192, 32, 512)
+    assert b.grkv_transfer_workspace_size(p, 32) > b.grkv_workspace_size(p) // 4
+    n = C.c_size_t(0)
+    L = b.load()
+    assert L.grkv_transfer_workspace_size(C.byref(p), 0, C.byref(n)) == b.GRKV_ERR_INVALID_ARG
+    assert L.grkv_transfer_workspace_size(C.byref(p), 513, C.byref(n)) == b.GRKV_ERR_INVALID_ARG
+    assert L.grkv_transfer_workspace_size(C.byref(p), 65, C.byref(n)) == b.GRKV_ERR_UNSUPPORTED
+    ws = (C.c_uint8 * 64)()
+    z = C.c_void_p(16)
+    rc = L.grkv_transfer_check(C.byref(p), 32, z, z, z, z, z, z, z, z, C.cast(ws, C.c_void_p), 64, None)
+    assert rc in (b.GRKV_ERR_WORKSPACE_TOO_SMALL, b.GRKV_ERR_MISALIGNED)

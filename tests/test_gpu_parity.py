@@ -402,3 +402,63 @@ def test_key_step_through_compress(grkv_lib):
     for i in range(c.U):
         np.testing.assert_array_equal(ko0[i], c.k[i][idx0[i]])
         assert (ko[i] != ko0[i]).any()
+
+
+# ---------------------------------------------------------- deterministic --
+@pytest.mark.parametrize("wl", [gi.workload(1), gi.workload(2).replace(units=3, n=8192, budget=1024),
+                                M256], ids=["c1", "c2_recipe_n8192", "m256_spans"])
+def test_deterministic_mode_is_bitwise_reproducible(grkv_lib, wl):
+    """GRKV_DETERMINISTIC: two calls give bit-identical Y, scores, row
+    statistics and compressed caches, and the results still match the oracle."""
+    c = G.Case(wl)
+    p = G.lib_params(wl, c.U)
+    p.flags = b.GRKV_DETERMINISTIC
+    s1, y1, r1 = G.run_score(c, p)
+    s2, y2, r2 = G.run_score(c, p)
+    np.testing.assert_array_equal(y1, y2)
+    np.testing.assert_array_equal(s1, s2)
+    np.testing.assert_array_equal(r1, r2)
+    i1, k1, v1 = G.run_compress(c, p)
+    i2, k2, v2 = G.run_compress(c, p)
+    np.testing.assert_array_equal(i1, i2)
+    np.testing.assert_array_equal(k1, k2)
+    np.testing.assert_array_equal(v1, v2)
+    op = G.oracle_params(wl)
+    for i in range(c.U):
+        ora = O.compress_unit(c.q[i], c.k[i], c.v[i], op)
+        tol = G.score_rel_tol(c.q[i], c.k[i], op)
+        s_abs = ora["attn"] @ np.abs(c.v[i].astype(np.float64))
+        lim = (tol + op.n * G.U + G.y_tol_extra(p)) * s_abs + 1e-7
+        assert (np.abs(y1[i] - ora["y"]) <= lim).all()
+        G.check_unit_end_to_end(wl.name + "_deterministic", i, c.q[i], c.k[i], c.v[i], op, ora,
+                                i1[i], s1[i], k1[i], v1[i], wl.dtype)
+
+
+# ------------------------------------------------------ bounded-wait exit --
+def test_bounded_wait_timeout_exits_cleanly(grkv_lib):
+    """GRKV_TEST_TIMEOUT makes the one-read scoring kernel's first CTA withhold
+    one arrive with a ~2 ms wait budget: its waits expire, every role of the
+    CTA (and of the CTAs that wait for its statistics) gives up, the kernel
+    frees its tensor memory and returns, and the status word reads
+    GRKV_ERR_TIMEOUT.  The next calls on the same context run normally (they
+    allocate tensor memory on every SM again) and match the oracle."""
+    import torch
+    wl = gi.workload(1)
+    c = G.Case(wl)
+    p = G.lib_params(wl, c.U)
+    p.flags = b.GRKV_TEST_TIMEOUT
+    m, P = wl.m, wl.n - wl.window
+    scores = torch.empty((c.U, P), dtype=torch.float32, device="cuda")
+    y = torch.empty((c.U, m, 128), dtype=torch.float32, device="cuda")
+    rs = torch.empty((c.U, m, 2), dtype=torch.float32, device="cuda")
+    ws = G.workspace(p)
+    b.grkv_score(p, c.dq, c.dk, c.dv, scores, y, rs, ws)
+    assert b.grkv_status(ws) == b.GRKV_ERR_TIMEOUT
+    torch.cuda.synchronize()
+    op = G.oracle_params(wl)
+    for flags in (b.GRKV_ONE_READ_SCORE, 0):
+        p.flags = flags
+        s2, _, _ = G.run_score(c, p)
+        for i in range(c.U):
+            ora = O.compress_unit(c.q[i], c.k[i], c.v[i], op)
+            G.assert_scores(s2[i], ora["scores"], G.score_rel_tol(c.q[i], c.k[i], op))

@@ -493,3 +493,88 @@ def test_alternation_converges_to_a_stationary_point():
     X, _, _ = O.softmax_rows(O.window_logits(q, K, p, cols=idx))
     V_want = O.value_step_dual(X, Y, np.asarray(v, dtype=np.float64)[idx], free, 0.5)
     np.testing.assert_allclose(V, V_want, rtol=0, atol=1e-12)
+
+
+# ----------------------------------------------- decode-side transfer check --
+@pytest.mark.parametrize("window_rule", [True, False])
+def test_cache_output_matches_sdpa(window_rule):
+    """Y = A V over a cache of c slots: SDPA with the bottom-right causal mask
+    on slots (window rule) or with no mask (decoding queries)."""
+    rng = np.random.default_rng(31 + window_rule)
+    g, h, c, d = 2, 5, 17, 8
+    q, kc, vc = rng.standard_normal((g, h, d)), rng.standard_normal((c, d)), rng.standard_normal((c, d))
+    p = O.Params(group=g, n=40, d=d, window=h, budget=c)
+    sub = O.Params(group=g, n=c, d=d, window=h, budget=c)
+    np.testing.assert_allclose(O.cache_output(q, kc, vc, p, window_rule),
+                               _sdpa(q, kc, vc, sub, window_rule), rtol=0, atol=1e-12)
+
+
+def test_cache_output_single_slot_returns_its_value():
+    rng = np.random.default_rng(5)
+    q, kc, vc = rng.standard_normal((3, 4, 8)), rng.standard_normal((1, 8)), rng.standard_normal((1, 8))
+    p = O.Params(group=3, n=10, d=8, window=4, budget=1, causal=False)
+    np.testing.assert_allclose(O.cache_output(q, kc, vc, p, False), np.repeat(vc, 12, 0), atol=1e-15)
+
+
+def _transfer_case(seed=3, g=2, w=4, h=6, n=60, d=8, B=16, lam=1e-2):
+    rng = np.random.default_rng(seed)
+    q, k, v = _rand_unit(rng, g, w, n, d)
+    qh = 1.5 * k[rng.integers(0, n, size=(g, h))] + 0.3 * rng.standard_normal((g, h, d))
+    p = O.Params(group=g, n=n, d=d, window=w, budget=B, lambda_v=lam)
+    return q, qh, k, v, p
+
+
+def test_transfer_check_full_cache_has_no_error():
+    """B = n and lambda = inf keep the whole cache unchanged: every error is 0."""
+    q, qh, k, v, p = _transfer_case(B=60)
+    p = O.Params(**{**p.__dict__, "lambda_v": math.inf})
+    o = O.compress_unit(q, k, v, p)
+    r = O.transfer_check(q, qh, k, v, o["idx"], o["k_out"], o["v_out"], p)
+    for key in ("e_win_base", "e_win_comp", "e_held_base", "e_held_comp"):
+        assert r[key] <= 1e-24 * r["y_win2"], key
+    assert not r["fail"]
+
+
+def test_transfer_window_error_is_the_value_step_data_term():
+    """e_win of the compressed cache is ||Y - X V*||^2 of the value step
+    (Algorithm 1, slot rule on the retained cache = position rule on idx),
+    and the ridge lowers it below the eviction-only cache's."""
+    q, qh, k, v, p = _transfer_case()
+    o = O.compress_unit(q, k, v, p)
+    X = O.retained_attention(q, k, o["idx"], p)
+    r = O.transfer_check(q, qh, k, v, o["idx"], o["k_out"], o["v_out"], p)
+    np.testing.assert_allclose(r["e_win_comp"], ((o["y"] - X @ o["v_out"]) ** 2).sum(), rtol=1e-10)
+    V0 = v[o["idx"]]
+    np.testing.assert_allclose(r["e_win_base"], ((o["y"] - X @ V0) ** 2).sum(), rtol=1e-10)
+    assert r["e_win_comp"] < r["e_win_base"]
+
+
+def test_transfer_window_error_vanishes_as_lambda_goes_to_zero():
+    """lambda -> 0 with X_G of full row rank interpolates the target (the
+    lambda -> 0 limit of Eq. 7): the compressed cache's window error -> 0."""
+    q, qh, k, v, p = _transfer_case(B=40, lam=1e-9)
+    o = O.compress_unit(q, k, v, p)
+    r = O.transfer_check(q, qh, k, v, o["idx"], o["k_out"], o["v_out"], p)
+    assert r["e_win_comp"] <= 1e-10 * r["y_win2"]
+
+
+def test_transfer_similarity_and_l_common():
+    """cos is 1 when the held-out queries are the window queries seen without
+    the window rule, and is invariant to scaling V; L_common is the ratio of
+    summed squared errors to summed squared targets (App. G)."""
+    q, _, k, v, p = _transfer_case()
+    pn = O.Params(**{**p.__dict__, "causal": False})
+    o = O.compress_unit(q, k, v, pn)
+    r = O.transfer_check(q, q, k, v, o["idx"], o["k_out"], o["v_out"], pn)
+    assert abs(r["cos"] - 1.0) < 1e-12
+    q2, qh, k2, v2, p2 = _transfer_case(seed=9)
+    o2 = O.compress_unit(q2, k2, v2, p2)
+    r2 = O.transfer_check(q2, qh, k2, v2, o2["idx"], o2["k_out"], o2["v_out"], p2)
+    o3 = O.compress_unit(q2, k2, 3.0 * v2, p2)
+    r3 = O.transfer_check(q2, qh, k2, 3.0 * v2, o3["idx"], o3["k_out"], o3["v_out"], p2)
+    assert abs(r2["cos"] - r3["cos"]) < 1e-12
+    reps = [r, r2]
+    want = (r["e_held_comp"] + r2["e_held_comp"]) / (r["y_held2"] + r2["y_held2"])
+    assert abs(O.l_common(reps) - want) <= 1e-15 * want
+    assert abs(O.l_common(reps, "base", "win") -
+               (r["e_win_base"] + r2["e_win_base"]) / (r["y_win2"] + r2["y_win2"])) < 1e-14
