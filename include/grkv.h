@@ -125,6 +125,14 @@ typedef struct {
                            step (512); read only under GRKV_UPDATE_K                */
   float   cg_tol;       /* >= 0, finite: the key step's CG stops once ||r|| <=
                            cg_tol ||e|| (1e-4); read only under GRKV_UPDATE_K       */
+  int32_t steps;        /* 1..64: S, the alternating value / key steps of Algorithm 1
+                           (1, the paper's setting); S > 1 needs GRKV_UPDATE_K.  Step
+                           t >= 1 re-runs the value step from V0 with the retained
+                           attention at the current keys K^(t), then the key step
+                           linearised at K^(t) (its right-hand side gains J_G (K^(t) -
+                           K0)); a unit stops early once max |K^(t+1) - K^(t)| and
+                           max |V^(t+1) - V^(t)| are both <= step_tol                 */
+  float   step_tol;     /* >= 0, finite: the alternation's stop test (1e-9)         */
 } grkv_params;
 
 /* Fills `p` with the defaults above for the given sizes (bf16, lambda 1e-2, CG 512 / 1e-4,

@@ -46,7 +46,7 @@ class grkv_params(ctypes.Structure):
         ("n_sink", ctypes.c_int32), ("beta", ctypes.c_float), ("lambda_v", ctypes.c_float),
         ("lambda_k", ctypes.c_float), ("scale", ctypes.c_float), ("causal", ctypes.c_int32),
         ("dtype", ctypes.c_int32), ("flags", ctypes.c_uint32), ("cg_iters", ctypes.c_int32),
-        ("cg_tol", ctypes.c_float),
+        ("cg_tol", ctypes.c_float), ("steps", ctypes.c_int32), ("step_tol", ctypes.c_float),
     ]
 
 

@@ -88,6 +88,9 @@ int make_shape(const grkv_params* p, Shape* s) {
     if (p->cg_iters < 0 || p->cg_iters > kMaxCgIters) return GRKV_ERR_INVALID_ARG;
     if (!(p->cg_tol >= 0.f) || std::isinf(p->cg_tol)) return GRKV_ERR_INVALID_ARG;
   }
+  if (p->steps < 1 || p->steps > kMaxSteps) return GRKV_ERR_INVALID_ARG;
+  if (p->steps > 1 && !(p->flags & GRKV_UPDATE_K)) return GRKV_ERR_INVALID_ARG;
+  if (!(p->step_tol >= 0.f) || std::isinf(p->step_tol)) return GRKV_ERR_INVALID_ARG;
   if (p->d != kD) return GRKV_ERR_UNSUPPORTED;
   if ((int64_t)p->group * p->window > kMaxM) return GRKV_ERR_UNSUPPORTED;
   if ((int64_t)p->n * kD > (int64_t)1 << 31) return GRKV_ERR_UNSUPPORTED;
@@ -117,6 +120,8 @@ int make_shape(const grkv_params* p, Shape* s) {
   s->update_k = (p->flags & GRKV_UPDATE_K) ? 1 : 0;
   s->cg_iters = p->cg_iters;
   s->cg_tol = p->cg_tol;
+  s->steps = p->steps;
+  s->step_tol = p->step_tol;
   s->lambda_k = p->lambda_k;
   return GRKV_OK;
 }
@@ -190,6 +195,8 @@ void grkv_params_init(grkv_params* p, int32_t units, int32_t group, int32_t n, i
   p->flags = 0;
   p->cg_iters = 512;
   p->cg_tol = 1e-4f;
+  p->steps = 1;
+  p->step_tol = 1e-9f;
 }
 
 int grkv_workspace_size(const grkv_params* p, size_t* bytes) {
@@ -252,7 +259,7 @@ int grkv_merge(const grkv_params* p, const void* q, const void* k, const void* v
   if (s.U == 0) return GRKV_OK;
   GRKV_TRY(cuda_rc(launch_merge_any(s, q, k, v, scores, y, row_stats, idx, k_out, v_out, w, L, st)));
   if (!s.update_k) return GRKV_OK;
-  return cuda_rc(launch_key_step(s, q, y, scores, idx, v_out, k_out, w, L, st));
+  return cuda_rc(launch_key_step(s, q, k, v, y, scores, idx, v_out, k_out, w, L, st));
 }
 
 int grkv_compress(const grkv_params* p, const void* q, const void* k, const void* v, void* k_out,
@@ -276,7 +283,7 @@ int grkv_compress(const grkv_params* p, const void* q, const void* k, const void
   GRKV_TRY(cuda_rc(launch_select(s, scores, idx, w, L, st)));
   GRKV_TRY(cuda_rc(launch_merge_any(s, q, k, v, scores, y, rstats, idx, k_out, v_out, w, L, st)));
   if (!s.update_k) return GRKV_OK;
-  return cuda_rc(launch_key_step(s, q, y, scores, idx, v_out, k_out, w, L, st));
+  return cuda_rc(launch_key_step(s, q, k, v, y, scores, idx, v_out, k_out, w, L, st));
 }
 
 int grkv_status(const void* ws, int* device_status, void* stream) {

@@ -15,6 +15,7 @@ constexpr int kD = 128;          // supported head dimension
 constexpr int kMaxM = 256;       // stacked window rows g*w supported
 constexpr int kMaxScoreCtas = 256;  // persistent score grid bound used to size slots
 constexpr int kMaxCgIters = 4096;   // bound on the key step's conjugate-gradient iterations
+constexpr int kMaxSteps = 64;       // bound on the alternating steps S
 
 // Validated problem sizes, derived once on the host.
 struct Shape {
@@ -33,6 +34,8 @@ struct Shape {
   int cg_iters;   // most conjugate-gradient iterations of the key step
   float cg_tol;   // ... until ||r|| <= cg_tol ||e||
   float lambda_k; // ridge weight of the key step
+  int steps;      // S alternating value / key steps (Algorithm 1)
+  float step_tol; // stop once max |K^(t+1) - K^(t)|, max |V^(t+1) - V^(t)| <= step_tol
 };
 
 // Byte offsets of the workspace regions (each 256-B aligned).
@@ -111,9 +114,12 @@ size_t merge_tc_ws_bytes(const Shape& s);
 // row_stats (nullable): the full-cache row statistics; with them the Gram
 // needs one pass over the retained keys.
 size_t key_ws_bytes(const Shape& s);
-cudaError_t launch_key_step(const Shape& s, const void* q, const float* y, const float* scores,
-                            const int32_t* idx, const void* v_out, void* k_out, char* ws,
-                            const WsLayout& L, cudaStream_t st);
+// The key step (GRKV_UPDATE_K) and, for S > 1, the remaining alternating
+// steps; k, v are the full caches (K0 and V0 of steps t >= 1).
+cudaError_t launch_key_step(const Shape& s, const void* q, const void* k, const void* v,
+                            const float* y, const float* scores, const int32_t* idx,
+                            void* v_out, void* k_out, char* ws, const WsLayout& L,
+                            cudaStream_t st);
 cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const void* v,
                             const float* scores, const float* y, const float* row_stats,
                             const int32_t* idx, void* k_out, void* v_out, char* ws,

@@ -21,6 +21,12 @@
 // V* is read from v_out as written by the value step (rounded to the input
 // dtype), K0 from k_out (the value step copies K0 there), and the fixed set is
 // recomputed from the prefix scores exactly as the value step defines it.
+//
+// With S > 1 steps (Algorithm 1's outer loop), k_alternate_step runs steps
+// t = 1 .. S-1: the value step from V0 with X at the current keys K^(t)
+// (dual form, X_G X_G^T + lambda_v I factored by Cholesky in fp32), then the
+// key step linearised at K^(t), whose right-hand side gains J_G (K^(t) - K0);
+// K^(t) and V^(t) are carried in fp32 between steps.
 #include <cmath>
 
 #include "block_select.cuh"
@@ -35,11 +41,22 @@ constexpr int kTM = 64, kTN = 64, kTK = 16;
 struct KArgs {
   int n, w, m, B, P, n_sink, n_fix, causal, dtype, iters;
   float scale, lambda_k, tol;
+  float lambda_v, step_tol;
+  int lambda_inf;
+  int vt_valid;           // Vt holds V^(t) (false at t = 1: V^(1) is only in v_out)
+  const void* k;          // [U][n][d]  full caches (K0, V0 gathers of steps t >= 1)
+  const void* v;
+  float* Kt;              // [U][B][d]  fp32 K^(t) of the alternation, or null
+  float* Vt;              // [U][B][d]  fp32 V^(t) of the alternation (t >= 2)
+  float* G;               // [U][m][m]  value step: X_G X_G^T + lambda_v I, then its factor
+  float* RZ;              // [U][m][d]  value step: R, then Z
+  int* done;              // [U]        the unit met the alternation's stop test
+  int* status;
   const void* q;          // [U][m][d]
   const float* y;         // [U][m][d]
   const float* scores;    // [U][P]
   const int32_t* idx;     // [U][B]
-  const void* v_out;      // [U][B][d]  merged values V*
+  void* v_out;            // [U][B][d]  merged values V* (rewritten by steps t >= 1)
   void* k_out;            // [U][B][d]  holds K0 on entry, K* on exit
   float* X;               // [U][m][B]
   float* T;               // [U][m][B]
@@ -137,40 +154,49 @@ __device__ void softmax_jacobian_rows(const float* X, float* T, int m, int B) {
   __syncthreads();
 }
 
-__global__ void __launch_bounds__(kKT) k_key_step(KArgs a) {
-  __shared__ int hist[256], sh[64];
-  __shared__ float red[kKT / 32];
-  __shared__ GemmSmem gs;
-  const int u = blockIdx.x, m = a.m, B = a.B, dt = a.dtype;
-  const int32_t* idx = a.idx + (size_t)u * B;
-  const void* q = (const char*)a.q + (size_t)u * m * kD * (dt == GRKV_F32 ? 4 : 2);
-  const size_t kv_off = (size_t)u * B * kD;
-  const float* Y = a.y + (size_t)u * m * kD;
-  float* X = a.X + (size_t)u * m * B;
-  float* T = a.T + (size_t)u * m * B;
-  float* dK = a.dK + kv_off;
-  float* T2 = a.T2 + (size_t)u * m * B;
-  float* GQ = a.GQ + (size_t)u * m * m;
-  float* R = a.vec + (size_t)u * 4 * m * kD;
-  float* Pd = R + (size_t)m * kD;
-  float* AP = Pd + (size_t)m * kD;
-  float* AL = AP + (size_t)m * kD;
-  uint8_t* fixed = a.fixed + (size_t)u * B;
-  const float s = a.scale;
-  auto pos = [&](int i) {
-    const int j = idx[i];
-    return (unsigned)j < (unsigned)a.n ? j : 0;
-  };
+// Per-unit working set of the key step and of the alternation.
+struct KUnit {
+  int u, m, B;
+  const int32_t* idx;
+  const void* q;
+  size_t kv_off;          // u * B * d
+  const float* Y;
+  float *X, *T, *dK, *T2, *GQ, *R, *Pd, *AP, *AL;
+  uint8_t* fixed;
+  __device__ KUnit(const KArgs& a, int u_) : u(u_), m(a.m), B(a.B) {
+    idx = a.idx + (size_t)u * B;
+    q = (const char*)a.q + (size_t)u * m * kD * (a.dtype == GRKV_F32 ? 4 : 2);
+    kv_off = (size_t)u * B * kD;
+    Y = a.y + (size_t)u * m * kD;
+    X = a.X + (size_t)u * m * B;
+    T = a.T + (size_t)u * m * B;
+    dK = a.dK + kv_off;
+    T2 = a.T2 + (size_t)u * m * B;
+    GQ = a.GQ + (size_t)u * m * m;
+    R = a.vec + (size_t)u * 4 * m * kD;
+    Pd = R + (size_t)m * kD;
+    AP = Pd + (size_t)m * kD;
+    AL = AP + (size_t)m * kD;
+    fixed = a.fixed + (size_t)u * B;
+  }
+};
 
-  // ---- fixed set: retained sinks, the window, and the n_fix best-scored
-  // remaining retained prefix tokens (ties to the smaller position)
-  uint32_t* key = (uint32_t*)T;   // scratch, B words
+__device__ __forceinline__ int kpos(const KArgs& a, const KUnit& k, int i) {
+  const int j = k.idx[i];
+  return (unsigned)j < (unsigned)a.n ? j : 0;
+}
+
+// Fixed set: retained sinks, the window, and the n_fix best-scored remaining
+// retained prefix tokens (ties to the smaller position); k.T is scratch.
+__device__ void fixed_set(const KArgs& a, const KUnit& k, int* hist, int* sh) {
+  const int B = k.B;
+  uint32_t* key = (uint32_t*)k.T;
   int nc = 0;
   for (int i = threadIdx.x; i < B; i += kKT) {
-    const int j = pos(i);
+    const int j = kpos(a, k, i);
     const bool cand = j >= a.n_sink && j < a.P;
-    key[i] = cand ? max(order_key(a.scores[(size_t)u * a.P + j]), 1u) : 0u;
-    fixed[i] = cand ? 0 : 1;
+    key[i] = cand ? max(order_key(a.scores[(size_t)k.u * a.P + j]), 1u) : 0u;
+    k.fixed[i] = cand ? 0 : 1;
     nc += cand;
   }
   __syncthreads();
@@ -178,131 +204,305 @@ __global__ void __launch_bounds__(kKT) k_key_step(KArgs a) {
   (void)block_exclusive_scan(nc, sh + 8, &ncand);
   const int nf = min(a.n_fix, ncand);
   if (nf > 0) {
-    auto get = [&](int i, uint32_t* k) {
-      *k = key[i];
-      return *k != 0u;
+    auto get = [&](int i, uint32_t* kk) {
+      *kk = key[i];
+      return *kk != 0u;
     };
-    auto mark = [&](int i, int) { fixed[i] = 1; };
+    auto mark = [&](int i, int) { k.fixed[i] = 1; };
     block_topk_mark(get, mark, B, nf, hist, sh);
   }
   __syncthreads();
+}
 
-  // ---- X = softmax over the retained keys of s q_r . k_j (causal rule)
+// X = softmax over the retained keys of s q_r . k_j with the causal rule of
+// the retained positions; kget(j, t) is element t of retained key j.
+template <class FK>
+__device__ void retained_softmax(const KArgs& a, const KUnit& k, GemmSmem& gs, FK kget) {
+  const int m = k.m, B = k.B, dt = a.dtype;
+  const float s = a.scale;
   block_gemm(gs,
-      m, B, kD, [&](int r, int t) { return ldv(q, (size_t)r * kD + t, dt); },
-      [&](int t, int j) { return ldv(a.k_out, kv_off + (size_t)j * kD + t, dt); },
-      [&](int r, int j, float v) { X[(size_t)r * B + j] = s * v; });
-  {
-    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-    for (int r = wid; r < m; r += kKT / 32) {
-      float* x = X + (size_t)r * B;
-      const int lim = a.causal ? a.n - a.w + r % a.w : a.n - 1;
-      float mx = -INFINITY;
-      for (int j = lane; j < B; j += 32)
-        if (pos(j) <= lim) mx = fmaxf(mx, x[j]);
+      m, B, kD, [&](int r, int t) { return ldv(k.q, (size_t)r * kD + t, dt); },
+      [&](int t, int j) { return kget(j, t); },
+      [&](int r, int j, float v) { k.X[(size_t)r * B + j] = s * v; });
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  for (int r = wid; r < m; r += kKT / 32) {
+    float* x = k.X + (size_t)r * B;
+    const int lim = a.causal ? a.n - a.w + r % a.w : a.n - 1;
+    float mx = -INFINITY;
+    for (int j = lane; j < B; j += 32)
+      if (kpos(a, k, j) <= lim) mx = fmaxf(mx, x[j]);
 #pragma unroll
-      for (int o = 16; o >= 1; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-      float sum = 0.f;
-      for (int j = lane; j < B; j += 32) {
-        const float e = pos(j) <= lim ? expf(x[j] - mx) : 0.f;
-        x[j] = e;
-        sum += e;
-      }
-#pragma unroll
-      for (int o = 16; o >= 1; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-      const float inv = sum > 0.f ? 1.f / sum : 0.f;
-      for (int j = lane; j < B; j += 32) x[j] *= inv;
+    for (int o = 16; o >= 1; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    float sum = 0.f;
+    for (int j = lane; j < B; j += 32) {
+      const float e = kpos(a, k, j) <= lim ? expf(x[j] - mx) : 0.f;
+      x[j] = e;
+      sum += e;
     }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    const float inv = sum > 0.f ? 1.f / sum : 0.f;
+    for (int j = lane; j < B; j += 32) x[j] *= inv;
   }
   __syncthreads();
+}
 
-  const int md = m * kD;
-  // ---- GQ = s^2 Q Q^T (the Gram of the window queries)
+// dK <- J_G^T W (fixed rows zero) with the values vget(j, t).
+template <class FV>
+__device__ void key_vjp(const KArgs& a, const KUnit& k, GemmSmem& gs, const float* W, FV vget) {
+  const int m = k.m, B = k.B, dt = a.dtype;
+  const float s = a.scale;
   block_gemm(gs,
-      m, m, kD, [&](int r, int t) { return ldv(q, (size_t)r * kD + t, dt); },
-      [&](int t, int r2) { return ldv(q, (size_t)r2 * kD + t, dt); },
-      [&](int r, int r2, float v) { GQ[(size_t)r * m + r2] = s * s * v; });
-  // ---- r = e = Y - X V*, p = r, alpha = 0
+      m, B, kD, [&](int r, int t) { return W[(size_t)r * kD + t]; },
+      [&](int t, int j) { return vget(j, t); },
+      [&](int r, int j, float v) { k.T[(size_t)r * B + j] = v; });
+  softmax_jacobian_rows(k.X, k.T, m, B);
   block_gemm(gs,
-      m, kD, B, [&](int r, int j) { return X[(size_t)r * B + j]; },
-      [&](int j, int t) { return ldv(a.v_out, kv_off + (size_t)j * kD + t, dt); },
-      [&](int r, int t, float v) {
-        const size_t o = (size_t)r * kD + t;
-        const float e = Y[o] - v;
-        R[o] = e;
-        Pd[o] = e;
-        AL[o] = 0.f;
-      });
+      B, kD, m, [&](int j, int r) { return k.T[(size_t)r * B + j]; },
+      [&](int r, int t) { return ldv(k.q, (size_t)r * kD + t, dt); },
+      [&](int j, int t, float v) { k.dK[(size_t)j * kD + t] = k.fixed[j] ? 0.f : s * v; });
+}
+
+// Conjugate gradients on (J_G J_G^T + lambda_k I) alpha = e from alpha = 0,
+// with e in k.R on entry; alpha ends in k.AL.  The operator is applied as
+// three GEMMs through the query Gram (see the file comment).
+template <class FV>
+__device__ void key_cg(const KArgs& a, const KUnit& k, GemmSmem& gs, float* red, FV vget) {
+  const int m = k.m, B = k.B, dt = a.dtype, md = m * kD;
+  const float s = a.scale;
+  block_gemm(gs,
+      m, m, kD, [&](int r, int t) { return ldv(k.q, (size_t)r * kD + t, dt); },
+      [&](int t, int r2) { return ldv(k.q, (size_t)r2 * kD + t, dt); },
+      [&](int r, int r2, float v) { k.GQ[(size_t)r * m + r2] = s * s * v; });
   float rs = 0.f;
-  for (int i = threadIdx.x; i < md; i += kKT) rs = fmaf(R[i], R[i], rs);
+  for (int i = threadIdx.x; i < md; i += kKT) {
+    k.Pd[i] = k.R[i];
+    k.AL[i] = 0.f;
+    rs = fmaf(k.R[i], k.R[i], rs);
+  }
   rs = block_sum(rs, red);
   const float stop = a.tol * a.tol * rs;
-
-  // dK <- J_G^T W (fixed rows zero)
-  auto vjp = [&](const float* W) {
-    block_gemm(gs,
-        m, B, kD, [&](int r, int t) { return W[(size_t)r * kD + t]; },
-        [&](int t, int j) { return ldv(a.v_out, kv_off + (size_t)j * kD + t, dt); },
-        [&](int r, int j, float v) { T[(size_t)r * B + j] = v; });
-    softmax_jacobian_rows(X, T, m, B);
-    block_gemm(gs,
-        B, kD, m, [&](int j, int r) { return T[(size_t)r * B + j]; },
-        [&](int r, int t) { return ldv(q, (size_t)r * kD + t, dt); },
-        [&](int j, int t, float v) { dK[(size_t)j * kD + t] = fixed[j] ? 0.f : s * v; });
-  };
-
   for (int it = 0; it < a.iters; ++it) {
     if (!(rs > stop) || !(rs > 0.f)) break;
     // Ap = J_G (J_G^T p) + lambda p without forming dK: with dS = X o (dA -
-    // rowsum(X o dA)), dA = p V*^T, the JVP of dK = s dS^T Q (free rows) is
+    // rowsum(X o dA)), dA = p V^T, the JVP of dK = s dS^T Q (free rows) is
     // s Q dK^T = (s^2 Q Q^T) dS on the free columns and 0 on the fixed ones.
     block_gemm(gs,
-        m, B, kD, [&](int r, int t) { return Pd[(size_t)r * kD + t]; },
-        [&](int t, int j) { return ldv(a.v_out, kv_off + (size_t)j * kD + t, dt); },
-        [&](int r, int j, float v) { T[(size_t)r * B + j] = v; });
-    softmax_jacobian_rows(X, T, m, B);
+        m, B, kD, [&](int r, int t) { return k.Pd[(size_t)r * kD + t]; },
+        [&](int t, int j) { return vget(j, t); },
+        [&](int r, int j, float v) { k.T[(size_t)r * B + j] = v; });
+    softmax_jacobian_rows(k.X, k.T, m, B);
     block_gemm(gs,
-        m, B, m, [&](int r, int r2) { return GQ[(size_t)r * m + r2]; },
-        [&](int r2, int j) { return T[(size_t)r2 * B + j]; },
-        [&](int r, int j, float v) { T2[(size_t)r * B + j] = fixed[j] ? 0.f : v; });
-    softmax_jacobian_rows(X, T2, m, B);
+        m, B, m, [&](int r, int r2) { return k.GQ[(size_t)r * m + r2]; },
+        [&](int r2, int j) { return k.T[(size_t)r2 * B + j]; },
+        [&](int r, int j, float v) { k.T2[(size_t)r * B + j] = k.fixed[j] ? 0.f : v; });
+    softmax_jacobian_rows(k.X, k.T2, m, B);
     block_gemm(gs,
-        m, kD, B, [&](int r, int j) { return T2[(size_t)r * B + j]; },
-        [&](int j, int t) { return ldv(a.v_out, kv_off + (size_t)j * kD + t, dt); },
+        m, kD, B, [&](int r, int j) { return k.T2[(size_t)r * B + j]; },
+        [&](int j, int t) { return vget(j, t); },
         [&](int r, int t, float v) {
           const size_t o = (size_t)r * kD + t;
-          AP[o] = v + a.lambda_k * Pd[o];
+          k.AP[o] = v + a.lambda_k * k.Pd[o];
         });
     float pap = 0.f;
-    for (int i = threadIdx.x; i < md; i += kKT) pap = fmaf(Pd[i], AP[i], pap);
+    for (int i = threadIdx.x; i < md; i += kKT) pap = fmaf(k.Pd[i], k.AP[i], pap);
     pap = block_sum(pap, red);
     if (!(pap > 0.f)) break;   // the direction has vanished
     const float al = rs / pap;
     float rn = 0.f;
     for (int i = threadIdx.x; i < md; i += kKT) {
-      AL[i] = fmaf(al, Pd[i], AL[i]);
-      const float r = fmaf(-al, AP[i], R[i]);
-      R[i] = r;
+      k.AL[i] = fmaf(al, k.Pd[i], k.AL[i]);
+      const float r = fmaf(-al, k.AP[i], k.R[i]);
+      k.R[i] = r;
       rn = fmaf(r, r, rn);
     }
     rn = block_sum(rn, red);
     const float beta = rn / rs;
-    for (int i = threadIdx.x; i < md; i += kKT) Pd[i] = fmaf(beta, Pd[i], R[i]);
+    for (int i = threadIdx.x; i < md; i += kKT) k.Pd[i] = fmaf(beta, k.Pd[i], k.R[i]);
     rs = rn;
     __syncthreads();
   }
+}
 
-  // ---- K*_G = K0_G + J_G^T alpha; fixed rows keep K0
-  vjp(AL);
+__device__ __forceinline__ void stv(void* p, size_t i, int dtype, float v) {
+  if (dtype == GRKV_F32)
+    ((float*)p)[i] = v;
+  else
+    ((__nv_bfloat16*)p)[i] = __float2bfloat16_rn(v);
+}
+
+// Key step of Algorithm 1 at t = 0: linearised at K0 (k_out on entry) with
+// V* = v_out; K* to k_out (and, for an alternation, in fp32 to Kt).
+__global__ void __launch_bounds__(kKT) k_key_step(KArgs a) {
+  __shared__ int hist[256], sh[64];
+  __shared__ float red[kKT / 32];
+  __shared__ GemmSmem gs;
+  const KUnit k(a, blockIdx.x);
+  const int B = k.B, dt = a.dtype;
+  fixed_set(a, k, hist, sh);
+  retained_softmax(a, k, gs, [&](int j, int t) { return ldv(a.k_out, k.kv_off + (size_t)j * kD + t, dt); });
+  auto vget = [&](int j, int t) { return ldv(a.v_out, k.kv_off + (size_t)j * kD + t, dt); };
+  // e = Y - X V*
+  block_gemm(gs,
+      k.m, kD, B, [&](int r, int j) { return k.X[(size_t)r * B + j]; }, vget,
+      [&](int r, int t, float v) { k.R[(size_t)r * kD + t] = k.Y[(size_t)r * kD + t] - v; });
+  key_cg(a, k, gs, red, vget);
+  // K*_G = K0_G + J_G^T alpha; fixed rows keep K0
+  key_vjp(a, k, gs, k.AL, vget);
   for (int i = threadIdx.x; i < B * kD; i += kKT) {
     const int j = i / kD;
-    if (fixed[j]) continue;
-    const size_t o = kv_off + i;
-    const float v = ldv(a.k_out, o, dt) + dK[i];
-    if (dt == GRKV_F32)
-      ((float*)a.k_out)[o] = v;
-    else
-      ((__nv_bfloat16*)a.k_out)[o] = __float2bfloat16_rn(v);
+    const size_t o = k.kv_off + i;
+    const float k0 = ldv(a.k_out, o, dt);
+    const float v = k.fixed[j] ? k0 : k0 + k.dK[i];
+    if (a.Kt) a.Kt[o] = v;
+    if (!k.fixed[j]) stv(a.k_out, o, dt, v);
+  }
+}
+
+// In-place Cholesky of the m x m matrix G (row-major, lower triangle used)
+// by one CTA; returns false on a non-positive pivot.
+__device__ bool block_cholesky(float* G, int m, int* flag) {
+  if (threadIdx.x == 0) *flag = 0;
+  __syncthreads();
+  for (int c = 0; c < m; ++c) {
+    if (threadIdx.x == 0) {
+      const float d = G[(size_t)c * m + c];
+      if (!(d > 0.f)) *flag = 1;
+      G[(size_t)c * m + c] = d > 0.f ? sqrtf(d) : 1.f;
+    }
+    __syncthreads();
+    const float inv = 1.f / G[(size_t)c * m + c];
+    for (int i = c + 1 + threadIdx.x; i < m; i += kKT) G[(size_t)i * m + c] *= inv;
+    __syncthreads();
+    const int rem = m - c - 1;
+    for (int e = threadIdx.x; e < rem * rem; e += kKT) {
+      const int i = c + 1 + e / rem, j = c + 1 + e % rem;
+      if (j <= i) G[(size_t)i * m + j] -= G[(size_t)i * m + c] * G[(size_t)j * m + c];
+    }
+    __syncthreads();
+  }
+  return *flag == 0;
+}
+
+// One step t >= 1 of Algorithm 1's alternation for every unit still running:
+// the value step from V0 with X at the current keys K^(t) (Kt), then the key
+// step linearised at K^(t) (right-hand side e + J_G (K^(t) - K0)).  Writes
+// V^(t+1), K^(t+1) to v_out / k_out (rounded) and to Vt / Kt (fp32), and
+// marks the unit done once both changes are <= step_tol.
+__global__ void __launch_bounds__(kKT) k_alternate_step(KArgs a) {
+  __shared__ int hist[256], sh[64];
+  __shared__ float red[kKT / 32];
+  __shared__ GemmSmem gs;
+  __shared__ int flag;
+  const KUnit k(a, blockIdx.x);
+  if (a.done[k.u]) return;
+  const int m = k.m, B = k.B, dt = a.dtype;
+  const size_t un = (size_t)k.u * a.n;
+  auto k0 = [&](int j, int t) { return ldv(a.k, (un + kpos(a, k, j)) * kD + t, dt); };
+  auto v0 = [&](int j, int t) { return ldv(a.v, (un + kpos(a, k, j)) * kD + t, dt); };
+  fixed_set(a, k, hist, sh);
+  retained_softmax(a, k, gs, [&](int j, int t) { return a.Kt[k.kv_off + (size_t)j * kD + t]; });
+
+  // ---- value step: V = V0 + X_G^T (X_G X_G^T + lambda_v I)^-1 (Y - X V0)
+  float* G = a.G + (size_t)k.u * m * m;
+  float* Z = a.RZ + (size_t)k.u * m * kD;
+  bool solved = false;
+  if (!a.lambda_inf) {
+    block_gemm(gs,
+        m, m, B, [&](int r, int j) { return k.fixed[j] ? 0.f : k.X[(size_t)r * B + j]; },
+        [&](int j, int r2) { return k.fixed[j] ? 0.f : k.X[(size_t)r2 * B + j]; },
+        [&](int r, int r2, float v) { G[(size_t)r * m + r2] = v + (r == r2 ? a.lambda_v : 0.f); });
+    block_gemm(gs,
+        m, kD, B, [&](int r, int j) { return k.X[(size_t)r * B + j]; }, v0,
+        [&](int r, int t, float v) { Z[(size_t)r * kD + t] = k.Y[(size_t)r * kD + t] - v; });
+    solved = block_cholesky(G, m, &flag);
+    if (!solved && threadIdx.x == 0) set_status(a.status, GRKV_ERR_NUMERIC);
+    if (solved) {
+      for (int c = 0; c < m; ++c) {   // L W = R
+        const float inv = 1.f / G[(size_t)c * m + c];
+        for (int t = threadIdx.x; t < kD; t += kKT) Z[(size_t)c * kD + t] *= inv;
+        __syncthreads();
+        for (int e = threadIdx.x; e < (m - c - 1) * kD; e += kKT) {
+          const int i = c + 1 + e / kD, t = e % kD;
+          Z[(size_t)i * kD + t] -= G[(size_t)i * m + c] * Z[(size_t)c * kD + t];
+        }
+        __syncthreads();
+      }
+      for (int c = m - 1; c >= 0; --c) {   // L^T Z = W
+        const float inv = 1.f / G[(size_t)c * m + c];
+        for (int t = threadIdx.x; t < kD; t += kKT) Z[(size_t)c * kD + t] *= inv;
+        __syncthreads();
+        for (int e = threadIdx.x; e < c * kD; e += kKT) {
+          const int i = e / kD, t = e % kD;
+          Z[(size_t)i * kD + t] -= G[(size_t)c * m + i] * Z[(size_t)c * kD + t];
+        }
+        __syncthreads();
+      }
+    }
+  }
+  // V^(t+1) (fp32 in dK as scratch), its largest change, then v_out / Vt
+  if (solved) {
+    block_gemm(gs,
+        B, kD, m, [&](int j, int r) { return k.fixed[j] ? 0.f : k.X[(size_t)r * B + j]; },
+        [&](int r, int t) { return Z[(size_t)r * kD + t]; },
+        [&](int j, int t, float v) { k.dK[(size_t)j * kD + t] = v0(j, t) + v; });
+  } else {
+    for (int i = threadIdx.x; i < B * kD; i += kKT) k.dK[i] = v0(i / kD, i % kD);
+    __syncthreads();
+  }
+  float dv = 0.f;
+  for (int i = threadIdx.x; i < B * kD; i += kKT) {
+    const size_t o = k.kv_off + i;
+    const float prev = a.vt_valid ? a.Vt[o] : ldv(a.v_out, o, dt);
+    dv = fmaxf(dv, fabsf(k.dK[i] - prev));
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < B * kD; i += kKT) {
+    const size_t o = k.kv_off + i;
+    a.Vt[o] = k.dK[i];
+    stv(a.v_out, o, dt, k.dK[i]);
+  }
+  __syncthreads();
+
+  // ---- key step at K^(t) against V^(t+1) (fp32, Vt)
+  auto vget = [&](int j, int t) { return a.Vt[k.kv_off + (size_t)j * kD + t]; };
+  // e = Y - X V, then + J_G g with g = K^(t) - K0 on the free rows:
+  // dS = s Q g^T, dA = X o (dS - rowsum(X o dS)), df = dA V
+  block_gemm(gs,
+      m, kD, B, [&](int r, int j) { return k.X[(size_t)r * B + j]; }, vget,
+      [&](int r, int t, float v) { k.R[(size_t)r * kD + t] = k.Y[(size_t)r * kD + t] - v; });
+  block_gemm(gs,
+      m, B, kD, [&](int r, int t) { return ldv(k.q, (size_t)r * kD + t, dt); },
+      [&](int t, int j) {
+        return k.fixed[j] ? 0.f : a.Kt[k.kv_off + (size_t)j * kD + t] - k0(j, t);
+      },
+      [&](int r, int j, float v) { k.T[(size_t)r * B + j] = a.scale * v; });
+  softmax_jacobian_rows(k.X, k.T, m, B);
+  block_gemm(gs,
+      m, kD, B, [&](int r, int j) { return k.T[(size_t)r * B + j]; }, vget,
+      [&](int r, int t, float v) { k.R[(size_t)r * kD + t] += v; });
+  key_cg(a, k, gs, red, vget);
+  key_vjp(a, k, gs, k.AL, vget);
+  float dkmax = 0.f;
+  for (int i = threadIdx.x; i < B * kD; i += kKT) {
+    const int j = i / kD;
+    const size_t o = k.kv_off + i;
+    const float base = k0(j, i % kD);
+    const float v = k.fixed[j] ? base : base + k.dK[i];
+    dkmax = fmaxf(dkmax, fabsf(v - a.Kt[o]));
+    a.Kt[o] = v;
+    stv(a.k_out, o, dt, v);
+  }
+  // the stop test: both changes within step_tol
+  float ch = fmaxf(dkmax, dv);
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) ch = fmaxf(ch, __shfl_xor_sync(0xffffffffu, ch, o));
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ch;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float mx = 0.f;
+    for (int i = 0; i < kKT / 32; ++i) mx = fmaxf(mx, red[i]);
+    if (mx <= a.step_tol) a.done[k.u] = 1;
   }
 }
 
@@ -310,12 +510,15 @@ __global__ void __launch_bounds__(kKT) k_key_step(KArgs a) {
 
 size_t key_ws_bytes(const Shape& s) {
   const size_t U = (size_t)s.U, m = (size_t)s.m, B = (size_t)s.B, d = (size_t)kD;
-  return U * (3 * m * B * 4 + B * d * 4 + 4 * m * d * 4 + m * m * 4 + B) + 1024;
+  size_t bytes = U * (3 * m * B * 4 + B * d * 4 + 4 * m * d * 4 + m * m * 4 + B) + 1024;
+  if (s.steps > 1) bytes += U * (2 * B * d * 4 + m * m * 4 + m * d * 4 + 4) + 1024;
+  return bytes;
 }
 
-cudaError_t launch_key_step(const Shape& s, const void* q, const float* y, const float* scores,
-                            const int32_t* idx, const void* v_out, void* k_out, char* ws,
-                            const WsLayout& L, cudaStream_t st) {
+cudaError_t launch_key_step(const Shape& s, const void* q, const void* k, const void* v,
+                            const float* y, const float* scores, const int32_t* idx,
+                            void* v_out, void* k_out, char* ws, const WsLayout& L,
+                            cudaStream_t st) {
   const size_t U = (size_t)s.U, m = (size_t)s.m, B = (size_t)s.B, d = (size_t)kD;
   char* base = ws + L.key;
   KArgs a{};
@@ -332,12 +535,18 @@ cudaError_t launch_key_step(const Shape& s, const void* q, const float* y, const
   a.scale = s.scale;
   a.lambda_k = s.lambda_k;
   a.tol = s.cg_tol;
+  a.lambda_v = s.lambda;
+  a.lambda_inf = s.lambda_inf;
+  a.step_tol = s.step_tol;
   a.q = q;
+  a.k = k;
+  a.v = v;
   a.y = y;
   a.scores = scores;
   a.idx = idx;
   a.v_out = v_out;
   a.k_out = k_out;
+  a.status = (int*)(ws + L.status);
   a.X = (float*)base;
   a.T = a.X + U * m * B;
   a.dK = a.T + U * m * B;
@@ -345,9 +554,26 @@ cudaError_t launch_key_step(const Shape& s, const void* q, const float* y, const
   a.T2 = a.vec + U * 4 * m * d;
   a.GQ = a.T2 + U * m * B;
   a.fixed = (uint8_t*)(a.GQ + U * m * m);
+  if (s.steps > 1) {
+    char* alt = (char*)(((uintptr_t)(a.fixed + U * B) + 255) & ~(uintptr_t)255);
+    a.Kt = (float*)alt;
+    a.Vt = a.Kt + U * B * d;
+    a.G = a.Vt + U * B * d;
+    a.RZ = a.G + U * m * m;
+    a.done = (int*)(a.RZ + U * m * d);
+    cudaError_t e = cudaMemsetAsync(a.done, 0, U * sizeof(int), st);
+    if (e != cudaSuccess) return e;
+  }
   count_launches(1);
   k_key_step<<<s.U, kKT, 0, st>>>(a);
-  return cudaGetLastError();
+  cudaError_t e = cudaGetLastError();
+  for (int t = 1; t < s.steps && e == cudaSuccess; ++t) {
+    a.vt_valid = t > 1;   // V^(1) exists only as written to v_out (rounded)
+    count_launches(1);
+    k_alternate_step<<<s.U, kKT, 0, st>>>(a);
+    e = cudaGetLastError();
+  }
+  return e;
 }
 
 }  // namespace grkv

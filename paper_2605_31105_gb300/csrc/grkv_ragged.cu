@@ -142,7 +142,7 @@ extern "C" int grkv_compress_ragged(const grkv_params* p, const int32_t* budgets
     cudaError_t e = launch_select(rs, sb, idx_run, rw, RL, st);
     if (e == cudaSuccess) e = launch_merge_any(rs, qb, kb, vb, sb, yb, rb, idx_run, ko, vo, rw, RL, st);
     if (e == cudaSuccess && rs.update_k)
-      e = launch_key_step(rs, qb, yb, sb, idx_run, vo, ko, rw, RL, st);
+      e = launch_key_step(rs, qb, kb, vb, yb, sb, idx_run, vo, ko, rw, RL, st);
     if (e == cudaSuccess)
       e = cudaMemcpyAsync(idx + r.off[u0], idx_run, (size_t)rs.U * rs.B * sizeof(int32_t),
                           cudaMemcpyDeviceToDevice, st);

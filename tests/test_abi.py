@@ -45,6 +45,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 def test_params_init_defaults(lib):
     p = b.params(256, 4, 32768, 32, 2048)
+    assert p.steps == 1 and p.step_tol == pytest.approx(1e-9)
     assert (p.d, p.pool_kernel, p.pool_type, p.n_sink, p.causal, p.dtype) == (128, 7, 0, 4, 1, 1)
     assert p.beta == pytest.approx(0.1) and p.lambda_v == pytest.approx(1e-2)
 
@@ -62,7 +63,9 @@ def test_workspace_size_and_validation(lib):
            dict(flags=b.GRKV_UPDATE_K, cg_iters=-1),
            dict(flags=b.GRKV_UPDATE_K, cg_iters=4097),
            dict(flags=b.GRKV_UPDATE_K, cg_tol=-1.0),
-           dict(flags=b.GRKV_UPDATE_K, cg_tol=float("inf"))]
+           dict(flags=b.GRKV_UPDATE_K, cg_tol=float("inf")),
+           dict(steps=0), dict(steps=2), dict(flags=b.GRKV_UPDATE_K, steps=65),
+           dict(step_tol=-1.0), dict(step_tol=float("inf"))]
     for kw in bad:
         q = b.params(8, 4, 8192, 32, 512)
         for key, val in kw.items():

@@ -370,6 +370,39 @@ def test_key_step(grkv_lib, name):
         assert err <= lim, f"unit {i}: key update error {err:.3e} > {lim:.3e}"
 
 
+@pytest.mark.parametrize("name,steps", [("c0_f32_portable", 2), ("c0_f32_portable", 3),
+                                        ("c1_bf16_default", 2), ("edge_bf16_default", 3)])
+def test_alternation_steps(grkv_lib, name, steps):
+    """S > 1 (Algorithm 1's outer loop): step t re-runs the value step from V0
+    with X at the current keys K^(t), then the key step linearised at K^(t),
+    against the oracle's alternation (fp64, CG to 1e-12) run for the same S
+    with the stop test off.  K_out and V_out are held to the method's bar;
+    fixed rows keep K0 and V0 bit for bit."""
+    wl, flags, lam = KEY_CASES[name]
+    c = G.Case(wl)
+    op = G.oracle_params(wl, update_k=True, lambda_k=lam, cg_iters=4000, cg_tol=1e-12)
+    ora = [O.compress_unit(c.q[i], c.k[i], c.v[i], G.oracle_params(wl)) for i in range(c.U)]
+    idx = np.stack([o["idx"] for o in ora]).astype(np.int32)
+    scores32 = np.stack([o["scores32"] for o in ora])
+    y32 = np.stack([o["y"].astype(np.float32) for o in ora])
+    p = G.lib_params(wl, c.U)
+    p.flags = flags | b.GRKV_UPDATE_K
+    p.lambda_k = lam
+    p.cg_iters = 4000
+    p.cg_tol = 1e-6
+    p.steps = steps
+    p.step_tol = 0.0
+    ko, vo = G.run_merge(c, p, scores32, y32, idx)
+    for i, o in enumerate(ora):
+        alt = O.alternate(c.q[i], c.k[i], c.v[i], scores32[i], o["y"], idx[i], op, steps, stop=0.0)
+        assert len(alt["deltas"]) == steps
+        fixed = alt["fixed"]
+        np.testing.assert_array_equal(ko[i][fixed], c.k[i][idx[i]][fixed])
+        np.testing.assert_array_equal(vo[i][fixed], c.v[i][idx[i]][fixed])
+        G.assert_values(ko[i], alt["k_out"], wl.dtype, what=f"k_out (S = {steps})")
+        G.assert_values(vo[i], alt["v_out"], wl.dtype, what=f"v_out (S = {steps})")
+
+
 def test_key_step_zero_iterations_and_large_lambda(grkv_lib):
     wl = gi.workload(1).replace(units=1)
     c = G.Case(wl)
