@@ -60,6 +60,7 @@ extern "C" {
 #define GRKV_ERR_CUDA                -5  /* a CUDA call or launch failed          */
 #define GRKV_ERR_NUMERIC             -6  /* device: Cholesky pivot <= 0 (lambda ~ 0) */
 #define GRKV_ERR_TIMEOUT             -7  /* device: a bounded wait expired        */
+#define GRKV_ERR_BOUNDS              -8  /* device, GRKV_CHECKS: idx breaks its contract */
 
 #define GRKV_F32  0
 #define GRKV_BF16 1
@@ -92,13 +93,20 @@ extern "C" {
                                     the two-launch scoring even with GRKV_ONE_READ_SCORE).
                                     Every other step is reproducible in either mode */
 
+#define GRKV_CHECKS        0x10u /* device-side argument checks, written to the status word:
+                                    a non-finite q, k or v element -> GRKV_ERR_INVALID_ARG;
+                                    an idx given to grkv_merge outside [0, n), not ascending
+                                    or without the window n-w..n-1 in its last w slots ->
+                                    GRKV_ERR_BOUNDS.  The kernels still run (reading in-range
+                                    rows only); outputs are then unspecified.  Costs one
+                                    read of q, k and v */
 #define GRKV_TEST_TIMEOUT 0x80000000u /* tests only: exercises the exit of the bounded device
-                                    waits.  grkv_score / grkv_compress score with the
-                                    one-read kernel (bf16), whose first CTA then withholds
-                                    one arrive, with the waits' budget cut to ~2 ms: the
-                                    kernel gives up, frees its tensor memory, returns, and
-                                    grkv_status reports GRKV_ERR_TIMEOUT; outputs are
-                                    unspecified.  Ignored by the other kernels */
+                                    waits.  In the tensor-core scoring kernels (either path)
+                                    the first CTA withholds one arrive and the waits' budget
+                                    is cut to ~2 ms: the kernel gives up, frees its tensor
+                                    memory, returns, and grkv_status reports
+                                    GRKV_ERR_TIMEOUT; outputs are unspecified.  Ignored by
+                                    the other kernels */
 
 typedef struct {
   int32_t units;        /* U >= 0: independent (batch x layer x KV head) problems   */
@@ -120,7 +128,7 @@ typedef struct {
   int32_t causal;       /* 1: window slot a sees keys j <= n-w+a; 0: all n keys      */
   int32_t dtype;        /* GRKV_BF16 or GRKV_F32 for q, k, v, k_out, v_out          */
   uint32_t flags;       /* GRKV_UPDATE_K, GRKV_FORCE_SIMT, GRKV_ONE_READ_SCORE,
-                           GRKV_DETERMINISTIC, GRKV_TEST_TIMEOUT          */
+                           GRKV_DETERMINISTIC, GRKV_CHECKS, GRKV_TEST_TIMEOUT */
   int32_t cg_iters;     /* 0..4096: most conjugate-gradient iterations of the key
                            step (512); read only under GRKV_UPDATE_K                */
   float   cg_tol;       /* >= 0, finite: the key step's CG stops once ||r|| <=

@@ -21,6 +21,7 @@ GRKV_ERR_MISALIGNED = -4
 GRKV_ERR_CUDA = -5
 GRKV_ERR_NUMERIC = -6
 GRKV_ERR_TIMEOUT = -7
+GRKV_ERR_BOUNDS = -8
 
 GRKV_F32 = 0
 GRKV_BF16 = 1
@@ -30,6 +31,7 @@ GRKV_UPDATE_K = 0x1
 GRKV_FORCE_SIMT = 0x2
 GRKV_ONE_READ_SCORE = 0x4
 GRKV_DETERMINISTIC = 0x8
+GRKV_CHECKS = 0x10
 GRKV_TEST_TIMEOUT = 0x80000000
 
 EXPORTS = ("grkv_params_init", "grkv_workspace_size", "grkv_score", "grkv_select", "grkv_merge",

@@ -62,7 +62,7 @@ cudaError_t launch_merge_any(const Shape& s, const void* q, const void* k, const
 cudaError_t launch_score_any(const Shape& s, const void* q, const void* k, const void* v,
                              float* scores, float* y, float* row_stats, char* ws,
                              const WsLayout& L, cudaStream_t st) {
-  if (s.tc && (s.one_read || s.test_timeout) && !s.deterministic)
+  if (s.tc && s.one_read && !s.deterministic)
     return launch_score_pipe(s, q, k, v, scores, y, row_stats, ws, L, st);
   if (s.tc) return launch_score_tc(s, q, k, v, scores, y, row_stats, ws, L, 0, st);
   return launch_score_simt(s, q, k, v, scores, y, row_stats, ws, L, st);
@@ -81,7 +81,7 @@ int make_shape(const grkv_params* p, Shape* s) {
   if (p->causal != 0 && p->causal != 1) return GRKV_ERR_INVALID_ARG;
   if (p->dtype != GRKV_F32 && p->dtype != GRKV_BF16) return GRKV_ERR_INVALID_ARG;
   if (p->flags & ~(GRKV_UPDATE_K | GRKV_FORCE_SIMT | GRKV_ONE_READ_SCORE | GRKV_DETERMINISTIC |
-                   GRKV_TEST_TIMEOUT)) return GRKV_ERR_INVALID_ARG;
+                   GRKV_CHECKS | GRKV_TEST_TIMEOUT)) return GRKV_ERR_INVALID_ARG;
   if (p->d < 1) return GRKV_ERR_INVALID_ARG;
   if (p->flags & GRKV_UPDATE_K) {
     if (!(p->lambda_k >= 0.f) || std::isinf(p->lambda_k)) return GRKV_ERR_INVALID_ARG;
@@ -117,6 +117,7 @@ int make_shape(const grkv_params* p, Shape* s) {
   s->one_read = (p->flags & GRKV_ONE_READ_SCORE) ? 1 : 0;
   s->deterministic = (p->flags & GRKV_DETERMINISTIC) ? 1 : 0;
   s->test_timeout = (p->flags & GRKV_TEST_TIMEOUT) ? 1 : 0;
+  s->checks = (p->flags & GRKV_CHECKS) ? 1 : 0;
   s->update_k = (p->flags & GRKV_UPDATE_K) ? 1 : 0;
   s->cg_iters = p->cg_iters;
   s->cg_tol = p->cg_tol;
@@ -133,7 +134,14 @@ void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order
 WsLayout plan_workspace(const Shape& s) {
   WsLayout L{};
   const size_t U = (size_t)s.U, m = (size_t)s.m, d = (size_t)kD;
-  L.chunk = std::max(1024, ((s.n + 15) / 16 + 63) / 64 * 64);
+  // portable scoring: chunks of a multiple of 64 keys, enough of them that
+  // U x chunks fills the GPU a few times over (608 CTAs) without splitting a
+  // unit into chunks of fewer than 64 keys
+  {
+    const int per_unit = std::max(1, std::min((608 + std::max(s.U, 1) - 1) / std::max(s.U, 1),
+                                              (s.n + 63) / 64));
+    L.chunk = std::max(64, ((s.n + per_unit - 1) / per_unit + 63) / 64 * 64);
+  }
   L.nchunk = (s.n + L.chunk - 1) / L.chunk;
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -257,6 +265,10 @@ int grkv_merge(const grkv_params* p, const void* q, const void* k, const void* v
   char* w = (char*)ws;
   GRKV_TRY(cuda_rc(cudaMemsetAsync(w + L.status, 0, 4, st)));
   if (s.U == 0) return GRKV_OK;
+  if (s.checks) {
+    GRKV_TRY(cuda_rc(launch_check_inputs(s, q, k, v, (int*)(w + L.status), st)));
+    GRKV_TRY(cuda_rc(launch_check_idx(s, idx, (int*)(w + L.status), st)));
+  }
   GRKV_TRY(cuda_rc(launch_merge_any(s, q, k, v, scores, y, row_stats, idx, k_out, v_out, w, L, st)));
   if (!s.update_k) return GRKV_OK;
   return cuda_rc(launch_key_step(s, q, k, v, y, scores, idx, v_out, k_out, w, L, st));
@@ -279,6 +291,7 @@ int grkv_compress(const grkv_params* p, const void* q, const void* k, const void
   float* scores = (float*)(w + L.scores);
   float* y = (float*)(w + L.y);
   float* rstats = (float*)(w + L.rstats);
+  if (s.checks) GRKV_TRY(cuda_rc(launch_check_inputs(s, q, k, v, (int*)(w + L.status), st)));
   GRKV_TRY(cuda_rc(launch_score_any(s, q, k, v, scores, y, rstats, w, L, st)));
   GRKV_TRY(cuda_rc(launch_select(s, scores, idx, w, L, st)));
   GRKV_TRY(cuda_rc(launch_merge_any(s, q, k, v, scores, y, rstats, idx, k_out, v_out, w, L, st)));
@@ -307,6 +320,7 @@ const char* grkv_strerror(int code) {
     case GRKV_ERR_CUDA: return "CUDA error";
     case GRKV_ERR_NUMERIC: return "non-positive Cholesky pivot";
     case GRKV_ERR_TIMEOUT: return "bounded device wait expired";
+    case GRKV_ERR_BOUNDS: return "idx breaks its contract (GRKV_CHECKS)";
     default: return "unknown error";
   }
 }

@@ -30,6 +30,7 @@ struct Shape {
   int one_read;   // tensor-core scoring in one launch that reads K from HBM once
   int deterministic;  // Y summed in a fixed order (GRKV_DETERMINISTIC)
   int test_timeout;   // GRKV_TEST_TIMEOUT (tests of the bounded-wait exit)
+  int checks;         // GRKV_CHECKS: device-side argument checks
   int update_k;   // key step after the value step (GRKV_UPDATE_K)
   int cg_iters;   // most conjugate-gradient iterations of the key step
   float cg_tol;   // ... until ||r|| <= cg_tol ||e||
@@ -140,6 +141,11 @@ cudaError_t launch_merge_any(const Shape& s, const void* q, const void* k, const
                              const float* scores, const float* y, const float* row_stats,
                              const int32_t* idx, void* k_out, void* v_out, char* ws,
                              const WsLayout& L, cudaStream_t st);
+// GRKV_CHECKS: finite inputs (GRKV_ERR_INVALID_ARG) and the idx contract
+// (GRKV_ERR_BOUNDS), written to the status word.
+cudaError_t launch_check_inputs(const Shape& s, const void* q, const void* k, const void* v,
+                                int* status, cudaStream_t st);
+cudaError_t launch_check_idx(const Shape& s, const int32_t* idx, int* status, cudaStream_t st);
 // Host-side parameter validation shared by the entry points.
 int make_shape(const grkv_params* p, Shape* s);
 cudaError_t launch_merge_simt(const Shape& s, const void* q, const void* k, const void* v,

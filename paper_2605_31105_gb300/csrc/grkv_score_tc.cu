@@ -41,6 +41,7 @@ constexpr int kRows = 128;            // window rows (m padded to 128)
 constexpr int kThreads = 512;
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KB
 constexpr long long kWaitBudget = 1ll << 32;      // cycles (~2 s) before a wait gives up
+constexpr long long kTestWaitBudget = 1ll << 22;  // ~2 ms: the budget of GRKV_TEST_TIMEOUT
 
 // Shared-memory layout (offsets from a 1024-byte aligned base) for kRing K/V
 // ring slots and kQBuf Q tiles: 5 + 1 (a CTA switches units two or three
@@ -53,7 +54,7 @@ struct Layout {
   static constexpr uint32_t kOffAstat = kOffRed + 2 * 2 * 4 * kTile * 4;   // [2 buf][2 wg][128] float2
   static constexpr uint32_t kOffLam = kOffAstat + 2 * 2 * kRows * 8;       // [2 buf][128] float
   static constexpr uint32_t kOffBar = kOffLam + 2 * kRows * 4;
-  static constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;         // + alignment slack
+  static constexpr uint32_t kSmemBytes = kOffBar + 512 + 1024;         // + alignment slack
 };
 constexpr int kRingTwo = 5, kQBufTwo = 1;
 
@@ -77,6 +78,8 @@ struct Args {
   int* unit_cnt;     // [U] pass-A slots written, zeroed by the host
   int* status;
   float* ypart;      // [U][maxc][m][128] segment Y partials (deterministic mode) or null
+  long long wait_budget;   // cycles before a bounded wait gives up
+  int test_withhold;       // GRKV_TEST_TIMEOUT: CTA 0 withholds one arrive
 };
 
 // ------------------------------------------------------------ job schedule
@@ -197,6 +200,13 @@ __device__ __forceinline__ void stats_chunk(float* v, bool full, int j0, int lim
   L += (s[0] + s[1]) + (s[2] + s[3]);
 }
 
+// mbar_wait for all lanes of a warp with one answer, so that warp-collective
+// instructions after a wait are reached by all lanes or by none.
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                               long long budget) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort, budget));
+}
+
 __device__ __forceinline__ int ld_acquire(const int* p) {
   int v;
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -217,11 +227,12 @@ struct Bars {
   uint64_t y_full[2], y_empty[2];
   uint64_t astat_full[2], astat_empty[2];   // compute groups -> statistics publisher
   uint64_t lam_full[2], lam_empty[2];       // statistics fetcher -> compute groups
+  uint64_t grp[2][2];                       // per compute group, alternating per pass-B tile
   uint64_t drain;
   uint32_t tmem;
   int abort;
 };
-static_assert(sizeof(Bars<kRingTwo, kQBufTwo>) <= 256, "barrier block");
+static_assert(sizeof(Bars<kRingTwo, kQBufTwo>) <= 512, "barrier block");
 
 // Merges two (max, sum) row statistics in log2 units.
 __device__ __forceinline__ float2 stat_merge(float2 x, float2 y) {
@@ -265,6 +276,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars->lam_full[i], 1);
       mbar_init(&bars->lam_empty[i], 256);
     }
+    for (int g = 0; g < 2; ++g)
+      for (int i = 0; i < 2; ++i) mbar_init(&bars->grp[g][i], 4);   // one arrive per warp
     mbar_init(&bars->drain, 1);
     bars->abort = 0;
     fence_mbar_init();
@@ -295,7 +308,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto load = [&](const CUtensorMap* map, int j0, int u, uint64_t pol) -> bool {
         if (ring_use >= kRing &&
             !mbar_wait(&bars->ring_empty[slot], ((ring_use / kRing) - 1) & 1, abort_flag,
-                       kWaitBudget))
+                       a.wait_budget))
           return false;
         uint8_t* dst = sm + kOffRing + slot * kTileBytes;
         mbar_expect_tx(&bars->ring_full[slot], kTileBytes);
@@ -311,7 +324,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (j.seg_first) {
             const int qs = seg % kQBuf;
             if (seg >= kQBuf) ok = mbar_wait(&bars->q_empty[qs], (seg / kQBuf - 1) & 1, abort_flag,
-                                         kWaitBudget);
+                                         a.wait_budget);
             if (!ok) break;
             ++qissued;
             mbar_expect_tx(&bars->q_full[qs], kTileBytes);
@@ -335,12 +348,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (ok && pend_v) ok = load(&tmV, pv_j0, pv_u, stream);
-      // let every issued load land before the CTA can exit
+      // let every issued load land before the CTA can exit (these waits
+      // ignore the abort flag, and are bounded)
+      volatile int no_abort = 0;
       for (uint32_t i = ring_use > kRing ? ring_use - kRing : 0; i < ring_use; ++i)
-        mbar_wait(&bars->ring_full[i % kRing], (i / kRing) & 1, abort_flag, kWaitBudget);
+        mbar_wait(&bars->ring_full[i % kRing], (i / kRing) & 1, &no_abort, a.wait_budget);
       const int qloads = qissued;
       for (int i = qloads > kQBuf ? qloads - kQBuf : 0; i < qloads; ++i)
-        mbar_wait(&bars->q_full[i % kQBuf], (i / kQBuf) & 1, abort_flag, kWaitBudget);
+        mbar_wait(&bars->q_full[i % kQBuf], (i / kQBuf) & 1, &no_abort, a.wait_budget);
     }
   } else if (warp == 1) {
     // ----------------------------------------------------------- MMA issuer
@@ -363,13 +378,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           const Job j = it.job();
           const int b = i & 1, use = i >> 1;
           if (j.seg_first) {
-            ok = mbar_wait(&bars->q_full[seg % kQBuf], (seg / kQBuf) & 1, abort_flag, kWaitBudget);
+            ok = mbar_wait(&bars->q_full[seg % kQBuf], (seg / kQBuf) & 1, abort_flag, a.wait_budget);
             if (!ok) break;
           }
           const uint32_t kslot = slot, kuse = ring_use;
-          ok = mbar_wait(&bars->ring_full[kslot], (kuse / kRing) & 1, abort_flag, kWaitBudget);
+          ok = mbar_wait(&bars->ring_full[kslot], (kuse / kRing) & 1, abort_flag, a.wait_budget);
           if (ok && use >= 1)
-            ok = mbar_wait(&bars->s_done[b], (use - 1) & 1, abort_flag, kWaitBudget);
+            ok = mbar_wait(&bars->s_done[b], (use - 1) & 1, abort_flag, a.wait_budget);
           if (!ok) break;
           tc_fence_after();
           const uint32_t qa = smem_u32(sm + kOffQ + (seg % kQBuf) * kTileBytes);
@@ -399,11 +414,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int yb = p_yb;
             if (pj.seg_first && ybuf_uses[yb] >= 1)
               ok = mbar_wait(&bars->y_empty[yb], (ybuf_uses[yb] - 1) & 1, abort_flag,
-                             kWaitBudget);
-            if (ok) ok = mbar_wait(&bars->s_done[pb], puse & 1, abort_flag, kWaitBudget);
+                             a.wait_budget);
+            if (ok) ok = mbar_wait(&bars->s_done[pb], puse & 1, abort_flag, a.wait_budget);
             if (ok)
               ok = mbar_wait(&bars->ring_full[p_vslot], (p_vuse / kRing) & 1, abort_flag,
-                             kWaitBudget);
+                             a.wait_budget);
             if (!ok) break;
             tc_fence_after();
             const uint32_t va = smem_u32(sm + kOffRing + p_vslot * kTileBytes);
@@ -435,11 +450,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int pb = p_i & 1, puse = p_i >> 1;
         const int yb = p_yb;
         if (pj.seg_first && ybuf_uses[yb] >= 1)
-          ok = mbar_wait(&bars->y_empty[yb], (ybuf_uses[yb] - 1) & 1, abort_flag, kWaitBudget);
-        if (ok) ok = mbar_wait(&bars->s_done[pb], puse & 1, abort_flag, kWaitBudget);
+          ok = mbar_wait(&bars->y_empty[yb], (ybuf_uses[yb] - 1) & 1, abort_flag, a.wait_budget);
+        if (ok) ok = mbar_wait(&bars->s_done[pb], puse & 1, abort_flag, a.wait_budget);
         if (ok)
           ok = mbar_wait(&bars->ring_full[p_vslot], (p_vuse / kRing) & 1, abort_flag,
-                         kWaitBudget);
+                         a.wait_budget);
         if (ok) {
           tc_fence_after();
           const uint32_t va = smem_u32(sm + kOffRing + p_vslot * kTileBytes);
@@ -452,9 +467,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (pj.seg_last) mma_commit(&bars->y_full[yb]);
         }
       }
-      // every MMA issued so far completes before TMEM can be released
+      // every MMA issued so far completes before TMEM can be released (this
+      // wait ignores the abort flag, and is bounded)
       mma_commit(&bars->drain);
-      mbar_wait(&bars->drain, 0, abort_flag, kWaitBudget);
+      volatile int no_abort = 0;
+      mbar_wait(&bars->drain, 0, &no_abort, a.wait_budget);
     }
   } else if (warp == 2) {
     // ----------------------------------------------- statistics publisher
@@ -470,7 +487,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const Job j = it.job();
         if (!(j.seg_last && j.kind == 0)) continue;
         const int ab = aseg & 1;
-        ok = mbar_wait(&bars->astat_full[ab], (aseg >> 1) & 1, abort_flag, kWaitBudget);
+        ok = mbar_wait_warp(&bars->astat_full[ab], (aseg >> 1) & 1, abort_flag, a.wait_budget);
         if (!ok) break;
         const int k = (int)blockIdx.x - sc.first_cta(j.u);
         // k < maxc always holds (the host sizes maxc from the same partition)
@@ -507,17 +524,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!(j.seg_first && j.kind == 1)) continue;
         const int lb = bseg & 1;
         if (bseg >= 2)
-          ok = mbar_wait(&bars->lam_empty[lb], ((bseg >> 1) - 1) & 1, abort_flag, kWaitBudget);
+          ok = mbar_wait_warp(&bars->lam_empty[lb], ((bseg >> 1) - 1) & 1, abort_flag, a.wait_budget);
         if (!ok) break;
         const int need = sc.writers(j.u);
         const long long t0 = clock64();
         while (ld_acquire(&a.unit_cnt[j.u]) < need) {
-          if (*abort_flag || clock64() - t0 > kWaitBudget) {
+          if (*abort_flag || clock64() - t0 > a.wait_budget) {
             *abort_flag = 1;
             ok = false;
             break;
           }
         }
+        ok = __all_sync(0xffffffffu, ok);
         if (!ok) break;
         const int ns = sc.nslots(j.u), c0 = sc.first_cta(j.u);
         const bool dense = sc.tiles(j.r) >= sc.G;   // every CTA holds tiles of the round
@@ -551,7 +569,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive(&bars->lam_full[lb]);
+        // GRKV_TEST_TIMEOUT: CTA 0 never announces its first pass-B
+        // normalisers, so its compute groups' bounded wait expires
+        if (lane == 0 && !(a.test_withhold && blockIdx.x == 0 && bseg == 0))
+          mbar_arrive(&bars->lam_full[lb]);
         ++bseg;
       }
     }
@@ -570,7 +591,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const Job j = it.job();
         if (!(j.seg_last && j.kind == 1)) continue;
         const int yb = bseg & 1;
-        ok = mbar_wait(&bars->y_full[yb], (bseg >> 1) & 1, abort_flag, kWaitBudget);
+        ok = mbar_wait_warp(&bars->y_full[yb], (bseg >> 1) & 1, abort_flag, a.wait_budget);
         if (!ok) break;
         tc_fence_after();
         const uint32_t ybase = lane_addr + kColY + yb * kD;
@@ -607,7 +628,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool row_ok = row < a.mr;
     const int lim = a.causal ? a.n - a.w + (row_ok ? (a.row0 + row) % a.w : 0) : a.n - 1;
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
-    const uint32_t bar_id = 1 + wg;
     float2* astat = (float2*)(sm + kOffAstat);
     const float* lam_s = (const float*)(sm + kOffLam);
     JobIter it;
@@ -626,14 +646,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             L = 0.f;
           } else {
             const int lb = bseg & 1;
-            ok = mbar_wait(&bars->lam_full[lb], (bseg >> 1) & 1, abort_flag, kWaitBudget);
+            ok = mbar_wait_warp(&bars->lam_full[lb], (bseg >> 1) & 1, abort_flag, a.wait_budget);
             if (!ok) break;
             lam = lam_s[lb * kRows + row];
             mbar_arrive(&bars->lam_empty[lb]);
           }
         }
         {
-          ok = mbar_wait(&bars->s_full[b], (i >> 1) & 1, abort_flag, kWaitBudget);
+          ok = mbar_wait_warp(&bars->s_full[b], (i >> 1) & 1, abort_flag, a.wait_budget);
           if (!ok) break;
           tc_fence_after();
           // this group's half of the tile: tokens 64 wg .. 64 wg + 63
@@ -689,7 +709,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_st_wait();
             tc_fence_before();
             mbar_arrive(&bars->s_done[b]);
-            named_bar(bar_id, 128);
+            // the group's four warps have written their sums (a bounded wait
+            // where a barrier instruction could not give up)
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bars->grp[wg][i & 1]);
+            ok = mbar_wait_warp(&bars->grp[wg][i & 1], (i >> 1) & 1, abort_flag, a.wait_budget);
+            if (!ok) break;
             if (q < 2) {
               const int jj = q * 32 + lane;
               const float cs = ((rb[jj] + rb[64 + jj]) + rb[128 + jj]) + rb[192 + jj];
@@ -704,8 +729,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (j.kind == 0) {
             const int ab = aseg & 1;
             if (aseg >= 2)
-              ok = mbar_wait(&bars->astat_empty[ab], ((aseg >> 1) - 1) & 1, abort_flag,
-                             kWaitBudget);
+              ok = mbar_wait_warp(&bars->astat_empty[ab], ((aseg >> 1) - 1) & 1, abort_flag,
+                             a.wait_budget);
             if (!ok) break;
             astat[(ab * 2 + wg) * kRows + row] = make_float2(M, L);
             mbar_arrive(&bars->astat_full[ab]);
@@ -809,6 +834,8 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
   a.unit_cnt = (int*)(ws + L.flags_tc);
   a.status = (int*)(ws + L.status);
   a.ypart = s.deterministic ? (float*)(ws + L.ypart_tc) : nullptr;
+  a.test_withhold = s.test_timeout;
+  a.wait_budget = s.test_timeout ? kTestWaitBudget : kWaitBudget;
   const size_t part_bytes = (size_t)s.U * maxc * s.m * kD * sizeof(float);
   cudaError_t e = a.ypart ? cudaMemsetAsync(a.ypart, 0, part_bytes, st)
                           : cudaMemsetAsync(y, 0, (size_t)s.U * s.m * kD * sizeof(float), st);

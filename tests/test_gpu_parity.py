@@ -468,18 +468,19 @@ def test_deterministic_mode_is_bitwise_reproducible(grkv_lib, wl):
 
 
 # ------------------------------------------------------ bounded-wait exit --
-def test_bounded_wait_timeout_exits_cleanly(grkv_lib):
-    """GRKV_TEST_TIMEOUT makes the one-read scoring kernel's first CTA withhold
-    one arrive with a ~2 ms wait budget: its waits expire, every role of the
-    CTA (and of the CTAs that wait for its statistics) gives up, the kernel
-    frees its tensor memory and returns, and the status word reads
+@pytest.mark.parametrize("path", ["default", "one_read"])
+def test_bounded_wait_timeout_exits_cleanly(grkv_lib, path):
+    """GRKV_TEST_TIMEOUT makes the scoring kernel's first CTA withhold one
+    arrive with a ~2 ms wait budget: its waits expire, every role of the CTA
+    (and of the CTAs that wait for its statistics) gives up, the kernel frees
+    its tensor memory and returns, and the status word reads
     GRKV_ERR_TIMEOUT.  The next calls on the same context run normally (they
     allocate tensor memory on every SM again) and match the oracle."""
     import torch
     wl = gi.workload(1)
     c = G.Case(wl)
     p = G.lib_params(wl, c.U)
-    p.flags = b.GRKV_TEST_TIMEOUT
+    p.flags = b.GRKV_TEST_TIMEOUT | PATHS[path]
     m, P = wl.m, wl.n - wl.window
     scores = torch.empty((c.U, P), dtype=torch.float32, device="cuda")
     y = torch.empty((c.U, m, 128), dtype=torch.float32, device="cuda")
@@ -495,3 +496,37 @@ def test_bounded_wait_timeout_exits_cleanly(grkv_lib):
         for i in range(c.U):
             ora = O.compress_unit(c.q[i], c.k[i], c.v[i], op)
             G.assert_scores(s2[i], ora["scores"], G.score_rel_tol(c.q[i], c.k[i], op))
+
+
+# ---------------------------------------------------------- GRKV_CHECKS --
+def test_checks_flag_reports_bad_arguments(grkv_lib):
+    """GRKV_CHECKS: valid calls report GRKV_OK; an idx that is not ascending or
+    lacks the window in its last w slots reports GRKV_ERR_BOUNDS; a non-finite
+    key reports GRKV_ERR_INVALID_ARG (device-side checks, status word)."""
+    import torch
+    wl = gi.workload(1).replace(units=2, n=2048, budget=256, seed=7)
+    c = G.Case(wl)
+    op = G.oracle_params(wl)
+    ora = [O.compress_unit(c.q[i], c.k[i], c.v[i], op) for i in range(c.U)]
+    idx = np.stack([o["idx"] for o in ora]).astype(np.int32)
+    scores32 = np.stack([o["scores32"] for o in ora])
+    y32 = np.stack([o["y"].astype(np.float32) for o in ora])
+    p = G.lib_params(wl, c.U)
+    p.flags = b.GRKV_CHECKS
+    G.run_compress(c, p)
+    _, vo = G.run_merge(c, p, scores32, y32, idx)
+    for i in range(c.U):
+        G.assert_values(vo[i], ora[i]["v_out"], wl.dtype)
+    swapped = idx.copy()
+    swapped[0][[10, 11]] = swapped[0][[11, 10]]
+    G.run_merge(c, p, scores32, y32, swapped, expect_status=b.GRKV_ERR_BOUNDS)
+    no_window = idx.copy()
+    no_window[1][-1] = wl.n - wl.window - 1
+    G.run_merge(c, p, scores32, y32, no_window, expect_status=b.GRKV_ERR_BOUNDS)
+    c.dk[1, 17, 5] = float("nan")
+    ko = torch.empty((c.U, wl.budget, 128), dtype=torch.bfloat16, device="cuda")
+    vo2 = torch.empty_like(ko)
+    idx_out = torch.empty((c.U, wl.budget), dtype=torch.int32, device="cuda")
+    ws = G.workspace(p)
+    b.grkv_compress(p, c.dq, c.dk, c.dv, ko, vo2, idx_out, ws)
+    assert b.grkv_status(ws) == b.GRKV_ERR_INVALID_ARG
