@@ -77,7 +77,13 @@ def algorithmic_bytes(wl):
 # for the kernel source it was taken on, so it is keyed by that file's digest
 # and reported as null once the kernel changes.
 SCORE_SRC = os.path.join("paper_2605_31105_gb300", "csrc", "grkv_score_tc.cu")
-SCORE_TRAFFIC = {}
+# DRAM read + write bytes of one grkv_score call (both k_score_tc launches), from
+# the ncu capture in profiles/score_tc_c2_llama_32k.md, keyed by the SHA-256 of the
+# kernel source it was taken on.
+SCORE_TRAFFIC = {
+    "c2_llama_32k_bf16": ("b285ec4c7a2aaf6a53dd98481e67f02df845934f655293d94e3d94cd81a65252",
+                          6529984512),
+}
 
 
 def score_traffic(wl):
