@@ -58,7 +58,7 @@ struct WsLayout {
   size_t flags;   // uint8 [U][B]      fixed-token flags
   size_t gram;    // acc   [U][m][m]   X_G X_G^T + lambda I, then its Cholesky factor
   size_t rz;      // acc   [U][m][d]   residual R, then Z
-  size_t merge_tc;  // tensor-core merge: R/Z, Gram [U][128][128] fp32, normalisers, fixed bits
+  size_t merge_tc;  // tensor-core merge: R/Z, Gram [U][128][128] fp32, normalisers, positions, fixed flags
   // compress intermediates
   size_t scores;  // float [U][P]
   size_t y;       // float [U][m][d]

@@ -3,26 +3,28 @@
 // Algorithm 1's value step in dual form (Sec. 3.4, App. D.1) with the fixed
 // tokens of App. D.3, one unit per CTA:
 //   k_merge_fixed   the fixed set (retained sinks, the window, and the n_fix
-//                   retained prefix tokens with the largest scores) and a
-//                   stable partition of the B retained slots into "positions":
-//                   the n_G non-fixed slots first, then the fixed ones, each in
-//                   slot order.  The window stays last in both orders, so slot
-//                   or position p is visible to window row r exactly when
-//                   p <= B - w + r % w.
+//                   retained prefix tokens with the largest scores), a flag per
+//                   slot, and a stable partition of the B retained slots into
+//                   "positions": the n_G non-fixed slots first, then the fixed
+//                   ones, each in slot order.  The window stays last in both
+//                   orders, so slot or position p is visible to window row r
+//                   exactly when p <= B - w + r % w.
 //   k_merge_gram    pass 1 over the slots: row max / sum of l = s Q K0^T (K0
-//                   gathered with TMA gather4) and K_out = K0 by TMA stores of the
-//                   gathered tiles; pass 2 over the positions: X = softmax,
-//                   R~ += Xh V0 and the Gram G += Xh XGh^T + (2 Xl) XGh^T on
-//                   tcgen05 (Xh, Xl the bf16 high / low parts of X; XGh is Xh
-//                   with the fixed columns zeroed, which removes them from both
-//                   terms; N = (G + G^T) / 2 restores the cross terms).  Writes
-//                   R = Y - R~, G and the row normalisers to the workspace.
+//                   gathered with TMA gather4); pass 2 over the positions:
+//                   X = softmax, R~ += Xh V0 and the Gram G += Xh XGh^T +
+//                   (2 Xl) XGh^T on tcgen05 (Xh, Xl the bf16 high / low parts
+//                   of X; XGh is Xh with the fixed columns zeroed, which removes
+//                   them from both terms; N = (G + G^T) / 2 restores the cross
+//                   terms).  Writes R = Y - R~, G and the row normalisers to the
+//                   workspace.  With the full-cache row statistics only pass 2
+//                   runs.
 //   k_merge_solve   fp32 in shared memory: N = sym(G) + lambda I, blocked
 //                   Cholesky, Z = N^-1 R by blocked triangular solves.
-//   k_merge_update  over the non-fixed positions only: dV = XGh^T Zh + XGh^T Zl
-//                   + XGl^T Zh on tcgen05 (one TMEM lane per token), and
-//                   V_out = V0 + dV.
-//   k_merge_copy    V_out = V0 for the fixed slots.
+//   k_merge_update  over the slots: S^T = K0 Q^T (one TMEM lane per token),
+//                   X_G^T (zero for fixed slots) as bf16 high / low parts back
+//                   into TMEM, dV = XGh^T Zh + XGh^T Zl + XGl^T Zh with X_G^T
+//                   as the TMEM A operand, V_out = V0 + dV in the gathered V0
+//                   tile, and K_out = K0, V_out by TMA tile stores.
 //
 // The kernels rely on the idx contract of grkv.h: ascending, with the window
 // n-w..n-1 in the last w slots.
@@ -48,22 +50,20 @@ constexpr long long kBudget = 1ll << 32;
 constexpr int kLD = 129;   // fp32 row stride of N and R/Z in k_merge_solve
 
 // Shared memory (offsets from a 1024-byte aligned base).  k_merge_gram: Q, a
-// ring of four gathered tiles, two XGh tiles.  k_merge_update: Q, a ring of
-// two gathered tiles, XGh, XGl, Zh, Zl.  Both end with the barriers.
-constexpr int kRingG = 4, kRingU = 2;
+// ring of four gathered tiles, two XGh tiles.  k_merge_update: Q, two K0
+// tiles, two V0 / V_out tiles, Zh, Zl.  Both continue with the barriers.
+constexpr int kRingG = 4;
 constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffRing = kTileBytes;
 constexpr uint32_t kOffXG = kOffRing + kRingG * kTileBytes;   // gram: 2 tiles
-constexpr uint32_t kOffXh = kOffRing + kRingU * kTileBytes;   // update: XGh, XGl, Zh, Zl
 constexpr uint32_t kOffBar = 7 * kTileBytes;
-static_assert(kOffXG + 2 * kTileBytes == kOffBar && kOffXh + 4 * kTileBytes == kOffBar,
-              "shared-memory layouts");
+static_assert(kOffXG + 2 * kTileBytes == kOffBar, "shared-memory layout");
 constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;
 // k_merge_solve: packed N (tri(128) + 4 floats), R/Z [128][129] fp32, 1 / L_jj, the failure flag
 constexpr uint32_t kSolveSmem = ((128 * 129) / 2 + 4 + kRows * kLD + kRows + 32) * 4;
 
 // TMEM columns.  gram: S[2] 0..255, R~ 256..383, Gram 384..511.
-// update: S[2] 0..255, D[2] 256..511.
+// update: S^T[2] (then X_G^T) 0..255, D[2] 256..511.
 constexpr uint32_t kColS = 0;
 constexpr uint32_t kColR = 256;
 constexpr uint32_t kColG = 384;
@@ -84,10 +84,10 @@ struct MArgs {
   float* rz;                 // [U][128][128]  R (gram) -> Z (solve)
   float* gram;               // [U][128][128]  raw Gram
   float* lam;                // [U][128]       log2 normaliser of each window row
-  int32_t* perm;             // [U][B]         slot at each position
-  int32_t* src;              // [U][B]         idx of that slot (the K / V row)
+  int32_t* src;              // [U][B]         K / V row of each position
   int32_t* ng;               // [U]            number of non-fixed slots
   int32_t* redo;             // [U]            single-pass result unusable: run two passes
+  uint8_t* fixed;            // [U][B]         1 for a fixed slot
   int gram_mode;             // 0 two passes; 1 one pass against rstats; 2 two passes for redo units
   int* status;
 };
@@ -109,6 +109,12 @@ static_assert(sizeof(MBars) <= 256, "barrier block");
 __device__ __forceinline__ float lo_half(uint32_t h) { return __uint_as_float(h << 16); }
 __device__ __forceinline__ float hi_half(uint32_t h) { return __uint_as_float(h & 0xFFFF0000u); }
 
+// mbar_wait for all lanes of a warp with one answer, so that warp-collective
+// instructions after a wait are reached by all lanes or by none.
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort, kBudget));
+}
+
 // Four rows (64 columns each) of a 2-D tensor map into consecutive 128-byte rows.
 __device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
                                             int r0, int r1, int r2, int r3) {
@@ -120,33 +126,44 @@ __device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map, u
 }
 
 // Producer side of a ring of R gathered tiles, run by warps 2 and 3: warp pw
-// gathers tile rows pw*64 .. pw*64+63 (rows_u at positions t*128 + row,
-// clamped to B-1; a row outside [0, n) reads row 0) with TMA gather4 into the
-// 128-byte-swizzled tile and arrives on ring_full with its 16 KB of
-// transaction bytes, so a slot is full once both halves have landed.
+// gathers tile rows pw*64 .. pw*64+63 (the rows rows_u[t*128 + row], clamped
+// to B-1; a row outside [0, n) reads row 0) with TMA gather4 into the
+// 128-byte-swizzled tile and arrives on the slot's full barrier with its 16 KB
+// of transaction bytes, so a slot is full once both halves have landed.  The
+// row indices are fetched by rows() one tile ahead of load(), so their
+// latency overlaps the wait for a free slot, and one fetch serves the K and V
+// tiles of the same rows.
 template <int R>
 struct Gatherer {
+  uint8_t* ring;
+  uint64_t* full;
+  uint64_t* empty;
   uint32_t use = 0;
-  __device__ __forceinline__ bool load(MBars* bars, uint8_t* sm, const CUtensorMap* map,
-                                       const int32_t* rows_u, int B, int n, int row0, int t,
-                                       int pw, int lane, volatile int* abort_flag) {
-    const uint32_t slot = use % R;
-    bool ok = true;
-    if (use >= R) ok = mbar_wait(&bars->ring_empty[slot], (use / R - 1) & 1, abort_flag, kBudget);
-    ok = __all_sync(0xffffffffu, ok);
-    if (!ok) return false;
-    uint8_t* dst = sm + kOffRing + slot * kTileBytes;
-    uint64_t* bar = &bars->ring_full[slot];
-    if (lane == 0) mbar_expect_tx(bar, kTileBytes / 2);
-    __syncwarp();
+  // lanes 0..15: the four rows pw*64 + 4*lane .. +3 of tile t, as map rows
+  __device__ __forceinline__ void rows(const int32_t* rows_u, int B, int n, int row0, int t,
+                                       int pw, int lane, int* j) const {
     if (lane < 16) {
       const int r = pw * 64 + 4 * lane;
-      int j[4];
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int jj = __ldg(rows_u + min(t * kTile + r + e, B - 1));
         j[e] = row0 + ((unsigned)jj < (unsigned)n ? jj : 0);
       }
+    }
+  }
+  __device__ __forceinline__ bool load(const CUtensorMap* map, const int* j, int pw, int lane,
+                                       volatile int* abort_flag) {
+    const uint32_t slot = use % R;
+    bool ok = true;
+    if (use >= R) ok = mbar_wait(&empty[slot], (use / R - 1) & 1, abort_flag, kBudget);
+    ok = __all_sync(0xffffffffu, ok);
+    if (!ok) return false;
+    uint8_t* dst = ring + slot * kTileBytes;
+    uint64_t* bar = &full[slot];
+    if (lane == 0) mbar_expect_tx(bar, kTileBytes / 2);
+    __syncwarp();
+    if (lane < 16) {
+      const int r = pw * 64 + 4 * lane;
       tma_gather4(dst + r * 128, map, bar, 0, j[0], j[1], j[2], j[3]);
       tma_gather4(dst + kTileBytes / 2 + r * 128, map, bar, 64, j[0], j[1], j[2], j[3]);
     }
@@ -154,9 +171,9 @@ struct Gatherer {
     return true;
   }
   // every issued gather lands before the CTA can exit
-  __device__ __forceinline__ void drain(MBars* bars, volatile int* abort_flag) {
+  __device__ __forceinline__ void drain(volatile int* abort_flag) {
     for (uint32_t i = use > R ? use - R : 0; i < use; ++i)
-      mbar_wait(&bars->ring_full[i % R], (i / R) & 1, abort_flag, kBudget);
+      mbar_wait(&full[i % R], (i / R) & 1, abort_flag, kBudget);
   }
 };
 
@@ -255,28 +272,6 @@ __device__ __forceinline__ void gram_chunk_masked(const float* v, int p0, int vl
   if (want_g) store_row_chunk(xg, row, C, ghi);
 }
 
-// One 32-position chunk of an update tile: XGh and XGl rows (the MN-major A
-// operands of dV = XG^T Z); positions from ng on are fixed and get zeros.
-template <int C, bool kMasked>
-__device__ __forceinline__ void update_chunk(const float* v, int p0, int ng, float sl2, float lam,
-                                             uint8_t* xh, uint8_t* xl, int row) {
-  uint32_t ghi[16], glo[16];
-#pragma unroll
-  for (int e = 0; e < 32; e += 2) {
-    const int p = p0 + C * 32 + e;
-    float x0 = fast_exp2(fmaf(v[e], sl2, -lam)), x1 = fast_exp2(fmaf(v[e + 1], sl2, -lam));
-    if (kMasked) {
-      x0 = p < ng ? x0 : 0.f;
-      x1 = p + 1 < ng ? x1 : 0.f;
-    }
-    const uint32_t h = pack_bf16(x0, x1);
-    ghi[e / 2] = h;
-    glo[e / 2] = pack_bf16(x0 - lo_half(h), x1 - hi_half(h));
-  }
-  store_row_chunk(xh, row, C, ghi);
-  store_row_chunk(xl, row, C, glo);
-}
-
 // Online max / sum of exp2 over one 32-column chunk (log2 units); positions
 // past vlim are skipped when kMasked.
 template <bool kMasked>
@@ -355,6 +350,7 @@ __global__ void __launch_bounds__(256) k_merge_fixed(MArgs a) {
     bool fixed = kx == 0u || kx > tau;
     if (kx == tau) fixed = er++ < need_eq;
     fkey[i] = fixed ? 1u : 0u;   // each thread rewrites only its own segment
+    a.fixed[(size_t)u * B + i] = fixed ? 1 : 0;
     keep += !fixed;
   }
   int ng;
@@ -363,15 +359,13 @@ __global__ void __launch_bounds__(256) k_merge_fixed(MArgs a) {
   for (int i = lo; i < hi; ++i) {
     const int at = fkey[i] ? ng + (i - g) : g;
     g += !fkey[i];
-    a.perm[(size_t)u * B + at] = i;
     a.src[(size_t)u * B + at] = pos(i);
   }
   if (tid == 0) a.ng[u] = ng;
 }
 
 // ======================================================== k_merge_gram
-// Roles (384 threads): warp 0 the Q load, then the K_out writes and ring
-// releases; warp 1 MMA issue; warps 2-3 the gathers (half a tile each);
+// Roles (384 threads): warp 0 the Q load; warp 1 MMA issue; warps 2-3 the gathers (half a tile each);
 // warps 4-7 and 8-11 two compute groups (one thread per window row / TMEM
 // lane) taking alternate jobs.  Job k < T: statistics of slot tile k;
 // T <= k < 2T: R~ and Gram of position tile k - T.  Ring loads: K of each
@@ -386,8 +380,7 @@ __global__ void __launch_bounds__(256) k_merge_fixed(MArgs a) {
 // recomputes it with both passes.
 __global__ void __launch_bounds__(kThreads, 1)
     k_merge_gram(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                 const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmKo,
-                 MArgs a) {
+                 const __grid_constant__ CUtensorMap tmV, MArgs a) {
   extern __shared__ __align__(1024) uint8_t smraw[];
   uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
   MBars* bars = (MBars*)(sm + kOffBar);
@@ -397,91 +390,40 @@ __global__ void __launch_bounds__(kThreads, 1)
   const bool single = a.gram_mode == 1;
   const int k0 = single ? T : 0;   // first job
   const int ng = __ldg(a.ng + u);
-  init_common(bars, warp, 2, 128, 128);   // ring slots are released by the MMA and by warp 0
+  init_common(bars, warp, 1, 128, 128);   // ring slots are released by the MMA
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars->tmem;
   volatile int* abort_flag = &bars->abort;
 
-  if (warp == 0 && single) {
+  if (warp == 0) {
     if (lane == 0) {
       prefetch_tensormap(&tmQ);
       mbar_expect_tx(&bars->q_full, kTileBytes);
       const uint64_t pol = l2_evict_last();
       tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, 0, u, pol);
       tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
-    }
-    __syncwarp();
-    // K_out = K0 from the K tiles of the (only) pass, position p to slot perm[p]:
-    // two 256-byte rows per step, one 16-byte chunk per lane
-    const int32_t* perm_u = a.perm + (size_t)u * B;
-    uint4* ko_u = (uint4*)(a.k_out + (size_t)u * B * kD);
-    const int c = lane & 15, c8 = c & 7;
-    bool ok = true;
-    for (int use = 0; use < 2 * T && ok; ++use) {
-      const int slot = use % kRingG;
-      const int pt = (use >> 1) * kTile;
-      int dst[4];   // output slots of tile rows 32 i + lane, fetched before the tile lands
-      if ((use & 1) == 0) {
-#pragma unroll
-        for (int i = 0; i < 4; ++i) dst[i] = __ldg(perm_u + min(pt + 32 * i + lane, B - 1));
-      }
-      ok = mbar_wait(&bars->ring_full[slot], (use / kRingG) & 1, abort_flag, kBudget);
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok) break;
-      if ((use & 1) == 0) {
-        const uint8_t* tile = sm + kOffRing + slot * kTileBytes + (c >> 3) * (kTileBytes / 2);
-#pragma unroll
-        for (int it = 0; it < kTile / 2; ++it) {
-          const int r = 2 * it + (lane >> 4);
-          const int d = __shfl_sync(0xffffffffu, dst[it >> 4], r & 31);
-          if (pt + r < B)
-            ko_u[(size_t)d * 16 + c] = *(const uint4*)(tile + r * 128 + ((c8 ^ (r & 7)) << 4));
-        }
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bars->ring_empty[slot]);
-    }
-  } else if (warp == 0) {
-    if (lane == 0) {
-      prefetch_tensormap(&tmQ);
-      prefetch_tensormap(&tmKo);
-      mbar_expect_tx(&bars->q_full, kTileBytes);
-      const uint64_t pol = l2_evict_last();
-      tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, 0, u, pol);
-      tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
-      // K_out = K0: the pass-1 tiles are the retained keys in slot order
-      bool ok = true;
-      for (int use = 0; use < 3 * T && ok; ++use) {
-        const int slot = use % kRingG;
-        ok = mbar_wait(&bars->ring_full[slot], (use / kRingG) & 1, abort_flag, kBudget);
-        if (!ok) break;
-        if (use < T) {
-          const uint8_t* tile = sm + kOffRing + slot * kTileBytes;
-          tma_store_3d(&tmKo, tile, 0, use * kTile, u);
-          tma_store_3d(&tmKo, tile + kTileBytes / 2, 64, use * kTile, u);
-          bulk_commit();
-          bulk_wait_read<0>();
-        }
-        mbar_arrive(&bars->ring_empty[slot]);
-      }
-      bulk_wait_all();
     }
   } else if (warp == 2 || warp == 3) {
     const int32_t* idx_u = a.idx + (size_t)u * B;
     const int32_t* src_u = a.src + (size_t)u * B;
     const int row0 = u * a.n;   // first row of this unit in the 2-D K / V maps
-    Gatherer<kRingG> gt;
+    const int pw = warp - 2;
+    Gatherer<kRingG> gt{sm + kOffRing, bars->ring_full, bars->ring_empty};
+    // job k < T reads K at the slots' rows, job k >= T K and V at the positions' rows
+    auto rows_of = [&](int k, int* j) {
+      gt.rows(k < T ? idx_u : src_u, B, a.n, row0, k < T ? k : k - T, pw, lane, j);
+    };
+    int jn[4];
+    if (k0 < 2 * T) rows_of(k0, jn);
     bool ok = true;
     for (int k = k0; k < 2 * T && ok; ++k) {
-      if (k < T) {
-        ok = gt.load(bars, sm, &tmK, idx_u, B, a.n, row0, k, warp - 2, lane, abort_flag);
-      } else {
-        ok = gt.load(bars, sm, &tmK, src_u, B, a.n, row0, k - T, warp - 2, lane, abort_flag);
-        if (ok) ok = gt.load(bars, sm, &tmV, src_u, B, a.n, row0, k - T, warp - 2, lane, abort_flag);
-      }
+      const int j[4] = {jn[0], jn[1], jn[2], jn[3]};
+      if (k + 1 < 2 * T) rows_of(k + 1, jn);
+      ok = gt.load(&tmK, j, pw, lane, abort_flag);
+      if (ok && k >= T) ok = gt.load(&tmV, j, pw, lane, abort_flag);
     }
-    gt.drain(bars, abort_flag);
+    gt.drain(abort_flag);
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t id_r = idesc_bf16(kRows, kD, 0, 1);     // R~ += Xh V0 (V0 MN-major)
@@ -990,27 +932,73 @@ __global__ void __launch_bounds__(256, 2) k_merge_solve(MArgs a) {
 }
 
 // ======================================================== k_merge_update
-// Roles (512 threads): warp 0 the Q load, warp 1 MMA issue, warps 2-3 the K0
-// gathers, warps 4-7 and 12-15 the XG rows (one thread per window row, half
-// of the tile's tokens each), warps 8-11 the output epilogue (one thread per
-// token / TMEM lane of D).  Only the tiles with non-fixed positions are
-// visited; the epilogue warps then copy V0 to the fixed slots.
+// Slot order, one unit per CTA, 512 threads.  Roles: warp 0 the Q load and
+// the K_out / V_out tile stores; warp 1 MMA issue; warps 2-3 the K0 and V0
+// gathers (two-slot rings each); warps 4-7 and 8-11 two compute groups taking
+// alternate tiles (one thread per token = TMEM lane of S^T): X_G^T from S^T,
+// zero for fixed slots, written back over S^T as packed bf16 (rows 32c ..
+// 32c+31 of chunk c: high parts to columns 32c .. 32c+15, low parts to
+// 32c+16 .. 32c+31, each chunk read before it is overwritten); warps 12-15
+// the epilogue (thread = token): V_out = V0 + dV in the V0 tile, which warp 0
+// then stores.  A fixed slot has X = 0 and so dV = 0: its row is left as V0.
+struct UBars {
+  uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
+  uint64_t q_full;
+  uint64_t s_full[2], x_full[2], d_full[2], d_empty[2], vo_full[2];
+  uint64_t drain;
+  uint32_t tmem;
+  int abort;
+};
+static_assert(sizeof(UBars) <= 256, "barrier block");
+constexpr uint32_t kOffKU = kTileBytes;                    // K0 ring, 2 tiles
+constexpr uint32_t kOffVU = kOffKU + 2 * kTileBytes;       // V0 / V_out ring, 2 tiles
+constexpr uint32_t kOffZU = kOffVU + 2 * kTileBytes;       // Zh, Zl
+constexpr uint32_t kOffLamU = kOffBar + 256;               // [128] row normalisers
+static_assert(kOffZU + 2 * kTileBytes == kOffBar, "update shared-memory layout");
+constexpr uint32_t kSmemBytesU = kOffLamU + kRows * 4 + 1024;
+
+// TMEM column of the packed high (lo = 0) or low (lo = 1) parts of rows
+// 16kk .. 16kk+15 of X_G^T.
+__device__ __forceinline__ uint32_t xt_col(int kk, int lo) {
+  return (kk >> 1) * 32 + lo * 16 + (kk & 1) * 8;
+}
+
 __global__ void __launch_bounds__(kThreadsU, 1)
     k_merge_update(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                   MArgs a) {
+                   const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmKo,
+                   const __grid_constant__ CUtensorMap tmVo, MArgs a) {
   extern __shared__ __align__(1024) uint8_t smraw[];
   uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
-  MBars* bars = (MBars*)(sm + kOffBar);
-  uint8_t* xh = sm + kOffXh;
-  uint8_t* xl = xh + kTileBytes;
-  uint8_t* zh = xl + kTileBytes;
+  UBars* bars = (UBars*)(sm + kOffBar);
+  float* lam_s = (float*)(sm + kOffLamU);
+  uint8_t* zh = sm + kOffZU;
   uint8_t* zl = zh + kTileBytes;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int u = blockIdx.x, B = a.B;
-  const int ng = __ldg(a.ng + u), T = (ng + kTile - 1) / kTile;
-  const int32_t* src_u = a.src + (size_t)u * B;
-  const int32_t* perm_u = a.perm + (size_t)u * B;
-  init_common(bars, warp, 1, 256, 128);
+  const int u = blockIdx.x, B = a.B, T = (B + kTile - 1) / kTile;
+  const int32_t* idx_u = a.idx + (size_t)u * B;
+  if (tid == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bars->k_full[i], 2);    // one expect_tx arrival per gathering warp
+      mbar_init(&bars->v_full[i], 2);
+      mbar_init(&bars->k_empty[i], 2);   // the S^T MMA and the K_out store
+      mbar_init(&bars->v_empty[i], 1);   // the V_out store
+      mbar_init(&bars->s_full[i], 1);
+      mbar_init(&bars->x_full[i], 128);
+      mbar_init(&bars->d_full[i], 1);
+      mbar_init(&bars->d_empty[i], 128);
+      mbar_init(&bars->vo_full[i], 128);
+    }
+    mbar_init(&bars->q_full, 1);
+    mbar_init(&bars->drain, 1);
+    bars->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&bars->tmem, 512);
+    tmem_relinquish();
+  }
+  // rows past m have lam = +inf and give X = 0
+  if (tid < kRows) lam_s[tid] = a.lam[(size_t)u * kRows + tid];
   // Z (fp32 [row][d]) to the bf16 B operands Zh, Zl: MN-major tiles of
   // 128-byte rows (d contiguous), two blocks of 64 columns
   {
@@ -1038,158 +1026,181 @@ __global__ void __launch_bounds__(kThreadsU, 1)
   volatile int* abort_flag = &bars->abort;
 
   if (warp == 0) {
-    if (lane == 0 && T > 0) {
+    if (lane == 0) {
       prefetch_tensormap(&tmQ);
+      prefetch_tensormap(&tmKo);
+      prefetch_tensormap(&tmVo);
       mbar_expect_tx(&bars->q_full, kTileBytes);
       const uint64_t pol = l2_evict_last();
       tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, 0, u, pol);
       tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
+      // K_out = K0 and V_out tile by tile (the maps clip the rows past B)
+      bool ok = true;
+      for (int t = 0; t < T && ok; ++t) {
+        const int sl = t & 1;
+        const uint32_t par = (t >> 1) & 1;
+        ok = mbar_wait(&bars->k_full[sl], par, abort_flag, kBudget);
+        if (!ok) break;
+        const uint8_t* kt = sm + kOffKU + sl * kTileBytes;
+        tma_store_3d(&tmKo, kt, 0, t * kTile, u);
+        tma_store_3d(&tmKo, kt + kTileBytes / 2, 64, t * kTile, u);
+        bulk_commit();
+        bulk_wait_read<0>();
+        mbar_arrive(&bars->k_empty[sl]);
+        ok = mbar_wait(&bars->vo_full[sl], par, abort_flag, kBudget);
+        if (!ok) break;
+        const uint8_t* vt = sm + kOffVU + sl * kTileBytes;
+        tma_store_3d(&tmVo, vt, 0, t * kTile, u);
+        tma_store_3d(&tmVo, vt + kTileBytes / 2, 64, t * kTile, u);
+        bulk_commit();
+        bulk_wait_read<0>();
+        mbar_arrive(&bars->v_empty[sl]);
+      }
+      bulk_wait_all();
+      if (!ok) set_status(a.status, GRKV_ERR_TIMEOUT);
     }
   } else if (warp == 2 || warp == 3) {
-    Gatherer<kRingU> gt;
+    const int pw = warp - 2, row0 = u * a.n;
+    Gatherer<2> gk{sm + kOffKU, bars->k_full, bars->k_empty};
+    Gatherer<2> gv{sm + kOffVU, bars->v_full, bars->v_empty};
+    int jn[4];
+    gk.rows(idx_u, B, a.n, row0, 0, pw, lane, jn);
     bool ok = true;
-    for (int t = 0; t < T && ok; ++t)
-      ok = gt.load(bars, sm, &tmK, src_u, B, a.n, u * a.n, t, warp - 2, lane, abort_flag);
-    gt.drain(bars, abort_flag);
+    for (int t = 0; t < T && ok; ++t) {
+      const int j[4] = {jn[0], jn[1], jn[2], jn[3]};
+      if (t + 1 < T) gk.rows(idx_u, B, a.n, row0, t + 1, pw, lane, jn);
+      ok = gk.load(&tmK, j, pw, lane, abort_flag);
+      if (ok) ok = gv.load(&tmV, j, pw, lane, abort_flag);
+    }
+    gk.drain(abort_flag);
+    gv.drain(abort_flag);
   } else if (warp == 1) {
-    if (lane == 0 && T > 0) {
-      const uint32_t id_d = idesc_bf16(kTile, kD, 1, 1);   // dV = XG^T Z, both MN-major
+    if (lane == 0) {
+      const uint32_t id_s = idesc_bf16(kTile, kRows, 0, 0);   // S^T = K0 Q^T
+      const uint32_t id_d = idesc_bf16(kTile, kD, 0, 1);      // dV = X_G^T Z (Z MN-major)
       const uint32_t qa = smem_u32(sm + kOffQ);
-      const uint32_t ah = smem_u32(xh), al = smem_u32(xl), bh = smem_u32(zh), bl = smem_u32(zl);
+      const uint32_t bh = smem_u32(zh), bl = smem_u32(zl);
       bool ok = mbar_wait(&bars->q_full, 0, abort_flag, kBudget);
       auto issue_d = [&](int t) -> bool {
-        const uint32_t d = tmem + kColD + (t & 1) * kD;
-        bool w = mbar_wait(&bars->xg_full[0], t & 1, abort_flag, kBudget);
+        const uint32_t d = tmem + kColD + (t & 1) * kD, x = tmem + kColS + (t & 1) * kTile;
+        bool w = mbar_wait(&bars->x_full[t & 1], (t >> 1) & 1, abort_flag, kBudget);
         if (w && t >= 2) w = mbar_wait(&bars->d_empty[t & 1], ((t >> 1) - 1) & 1, abort_flag, kBudget);
         if (!w) return false;
         tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < kRows / 16; ++kk)
-          mma_bf16(d, sw128_desc(ah + kk * 2048, kTileBytes / 2, 1024),
-                   sw128_desc(bh + kk * 2048, kTileBytes / 2, 1024), id_d, kk > 0);
+          mma_bf16_ts(d, x + xt_col(kk, 0), sw128_desc(bh + kk * 2048, kTileBytes / 2, 1024), id_d,
+                      kk > 0);
 #pragma unroll
         for (int kk = 0; kk < kRows / 16; ++kk)
-          mma_bf16(d, sw128_desc(ah + kk * 2048, kTileBytes / 2, 1024),
-                   sw128_desc(bl + kk * 2048, kTileBytes / 2, 1024), id_d, 1);
+          mma_bf16_ts(d, x + xt_col(kk, 0), sw128_desc(bl + kk * 2048, kTileBytes / 2, 1024), id_d, 1);
 #pragma unroll
         for (int kk = 0; kk < kRows / 16; ++kk)
-          mma_bf16(d, sw128_desc(al + kk * 2048, kTileBytes / 2, 1024),
-                   sw128_desc(bh + kk * 2048, kTileBytes / 2, 1024), id_d, 1);
-        mma_commit(&bars->xg_empty[0]);
+          mma_bf16_ts(d, x + xt_col(kk, 1), sw128_desc(bh + kk * 2048, kTileBytes / 2, 1024), id_d, 1);
         mma_commit(&bars->d_full[t & 1]);
         return true;
       };
       for (int t = 0; t < T && ok; ++t) {
-        const int b = t & 1;
-        ok = mbar_wait(&bars->ring_full[t % kRingU], (t / kRingU) & 1, abort_flag, kBudget);
-        if (ok && t >= 2) ok = mbar_wait(&bars->s_done[b], ((t >> 1) - 1) & 1, abort_flag, kBudget);
+        const int sl = t & 1;
+        ok = mbar_wait(&bars->k_full[sl], (t >> 1) & 1, abort_flag, kBudget);
         if (!ok) break;
         tc_fence_after();
-        issue_s(tmem + kColS + b * kTile, qa,
-                smem_u32(sm + kOffRing + (t % kRingU) * kTileBytes));
-        mma_commit(&bars->ring_empty[t % kRingU]);
-        mma_commit(&bars->s_full[b]);
+        // S^T into buffer sl: its previous contents (X_G^T of tile t - 2) were
+        // read by the dV MMAs issued before this one
+        const uint32_t ka = smem_u32(sm + kOffKU + sl * kTileBytes);
+#pragma unroll
+        for (int kk = 0; kk < kD / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
+          mma_bf16(tmem + kColS + sl * kTile, sw128_desc(ka + off, 16, 1024),
+                   sw128_desc(qa + off, 16, 1024), id_s, kk > 0);
+        }
+        mma_commit(&bars->k_empty[sl]);
+        mma_commit(&bars->s_full[sl]);
         if (t >= 1) ok = issue_d(t - 1);
       }
-      if (ok) ok = issue_d(T - 1);
+      if (ok && T > 0) ok = issue_d(T - 1);
       mma_commit(&bars->drain);
       mbar_wait(&bars->drain, 0, abort_flag, kBudget);
     }
-  } else if ((warp >= 4 && warp < 8) || warp >= 12) {
-    // two groups (warps 4-7, 12-15) share every tile: group cg computes the
-    // XG rows of tokens 64 cg .. 64 cg + 63 (thread = window row)
-    const int cg = warp >= 12, q = warp & 3, row = q * 32 + lane;
-    // rows past m have lam = +inf and give X = 0
-    const float lam = a.lam[(size_t)u * kRows + row];
+  } else if (warp < 12) {
+    // compute groups: group cg takes the tiles t with t % 2 == cg
+    const int cg = (warp - 4) >> 2, q = warp & 3, tok = q * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
     bool ok = true;
-    for (int t = 0; t < T && ok; ++t) {
-      const int b = t & 1, p0 = t * kTile;
-      ok = mbar_wait(&bars->s_full[b], (t >> 1) & 1, abort_flag, kBudget);
-      if (ok && t >= 1) ok = mbar_wait(&bars->xg_empty[0], (t - 1) & 1, abort_flag, kBudget);
+    for (int t = cg; t < T && ok; t += 2) {
+      const int sl = t & 1, slot = t * kTile + tok;
+      const bool zero = slot >= B || __ldg(a.fixed + (size_t)u * B + min(slot, B - 1)) != 0;
+      ok = mbar_wait_warp(&bars->s_full[sl], (t >> 1) & 1, abort_flag);
       if (!ok) break;
       tc_fence_after();
-      const uint32_t sbase = lane_addr + kColS + b * kTile + 64 * cg;
-      float va[32], vb[32];
-      tmem_ld32f(sbase, va);
-      tmem_ld32f(sbase + 32, vb);
-      tmem_wait32(va);
-      tmem_wait32(vb);
-      tc_fence_before();
-      mbar_arrive(&bars->s_done[b]);   // S is read
-      const bool masked = p0 + kTile > ng;
-      if (cg == 0) {
-        if (masked) {
-          update_chunk<0, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
-          update_chunk<1, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
-        } else {
-          update_chunk<0, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
-          update_chunk<1, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
+      const uint32_t sbase = lane_addr + kColS + sl * kTile;
+      float v[32];
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        tmem_ld32f(sbase + 32 * c, v);
+        tmem_wait32(v);
+        uint32_t hi[16], lo[16];
+#pragma unroll
+        for (int e = 0; e < 32; e += 2) {
+          const float4 l4 = *(const float4*)(lam_s + 32 * c + (e & ~3));
+          const float la = (e & 2) ? l4.z : l4.x, lb = (e & 2) ? l4.w : l4.y;
+          float x0 = fast_exp2(fmaf(v[e], a.sl2, -la)), x1 = fast_exp2(fmaf(v[e + 1], a.sl2, -lb));
+          if (zero) x0 = x1 = 0.f;
+          const uint32_t h = pack_bf16(x0, x1);
+          hi[e / 2] = h;
+          lo[e / 2] = pack_bf16(x0 - lo_half(h), x1 - hi_half(h));
         }
-      } else {
-        if (masked) {
-          update_chunk<2, true>(va, p0, ng, a.sl2, lam, xh, xl, row);
-          update_chunk<3, true>(vb, p0, ng, a.sl2, lam, xh, xl, row);
-        } else {
-          update_chunk<2, false>(va, p0, ng, a.sl2, lam, xh, xl, row);
-          update_chunk<3, false>(vb, p0, ng, a.sl2, lam, xh, xl, row);
-        }
+        tmem_st16(sbase + 32 * c, hi);
+        tmem_st16(sbase + 32 * c + 16, lo);
       }
-      fence_proxy_async_smem();
-      mbar_arrive(&bars->xg_full[0]);
+      tmem_st_wait();
+      tc_fence_before();
+      mbar_arrive(&bars->x_full[sl]);
     }
-    if (!ok && row == 0 && cg == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
-  } else if (warp >= 8 && warp < 12) {
-    // epilogue: thread = token (TMEM lane) of D = dV, 128 columns of d
+    if (!ok && tok == 0 && cg == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
+  } else {
+    // epilogue: thread = token (TMEM lane of D), V_out = V0 + dV in the V tile
     const int q = warp & 3, tok = q * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
-    const uint4* v_u = (const uint4*)(a.v + (size_t)u * a.n * kD);
-    uint4* vo_u = (uint4*)(a.v_out + (size_t)u * B * kD);
     bool ok = true;
     for (int t = 0; t < T && ok; ++t) {
-      const int p = t * kTile + tok;
-      const bool live = p < ng;
-      // V0 row of this position, fetched before D is ready
-      uint4 v0[16];
-      const uint4* g = v_u + (size_t)__ldg(src_u + min(p, B - 1)) * 16;
-#pragma unroll
-      for (int h = 0; h < 16; ++h) v0[h] = __ldg(g + h);
-      const int dst = live ? __ldg(perm_u + p) : 0;
-      ok = mbar_wait(&bars->d_full[t & 1], (t >> 1) & 1, abort_flag, kBudget);
+      const int sl = t & 1, slot = t * kTile + tok;
+      const bool live = slot < B && __ldg(a.fixed + (size_t)u * B + min(slot, B - 1)) == 0;
+      ok = mbar_wait_warp(&bars->d_full[sl], (t >> 1) & 1, abort_flag);
+      if (ok) ok = mbar_wait_warp(&bars->v_full[sl], (t >> 1) & 1, abort_flag);
       if (!ok) break;
       tc_fence_after();
-      const uint32_t dcol = lane_addr + kColD + (t & 1) * kD;
-#pragma unroll
+      uint8_t* vt = sm + kOffVU + sl * kTileBytes;
+      const uint32_t dcol = lane_addr + kColD + sl * kD;
+#pragma unroll 1
       for (int c = 0; c < 4; ++c) {
-        float v[32];
-        tmem_ld32f(dcol + c * 32, v);
-        tmem_wait32(v);
+        float dv[32];
+        tmem_ld32f(dcol + c * 32, dv);
+        tmem_wait32(dv);
         if (c == 3) {
           tc_fence_before();
-          mbar_arrive(&bars->d_empty[t & 1]);
+          mbar_arrive(&bars->d_empty[sl]);
         }
         if (live) {
+          // columns 32c .. 32c+31: half c/2, 16-byte chunks (c%2)*4 .. +3
+          uint8_t* row = vt + (c >> 1) * (kTileBytes / 2);
 #pragma unroll
           for (int h = 0; h < 4; ++h) {
-            const __nv_bfloat16* pv = (const __nv_bfloat16*)&v0[4 * c + h];
+            uint4* p = (uint4*)(row + sw128_offset(tok, (c & 1) * 4 + h));
+            const uint4 v0 = *p;
+            const uint32_t w[4] = {v0.x, v0.y, v0.z, v0.w};
             uint32_t o[4];
 #pragma unroll
             for (int z = 0; z < 4; ++z)
-              o[z] = pack_bf16(__bfloat162float(pv[2 * z]) + v[8 * h + 2 * z],
-                               __bfloat162float(pv[2 * z + 1]) + v[8 * h + 2 * z + 1]);
-            vo_u[(size_t)dst * 16 + 4 * c + h] = make_uint4(o[0], o[1], o[2], o[3]);
+              o[z] = pack_bf16(lo_half(w[z]) + dv[8 * h + 2 * z], hi_half(w[z]) + dv[8 * h + 2 * z + 1]);
+            *p = make_uint4(o[0], o[1], o[2], o[3]);
           }
         }
       }
+      fence_proxy_async_smem();
+      mbar_arrive(&bars->vo_full[sl]);
     }
     if (!ok && tok == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
-    // V_out = V0 for the fixed slots (positions ng .. B-1)
-    for (int p = ng + tok; p < B; p += 128) {
-      const uint4* g = v_u + (size_t)__ldg(src_u + p) * 16;
-      uint4* o = vo_u + (size_t)__ldg(perm_u + p) * 16;
-#pragma unroll
-      for (int h = 0; h < 16; ++h) o[h] = __ldg(g + h);
-    }
   }
   tc_fence_before();
   __syncthreads();
@@ -1205,19 +1216,20 @@ bool merge_tc_supported(const Shape& s) {
 
 size_t merge_tc_ws_bytes(const Shape& s) {
   const size_t U = (size_t)s.U;
-  return U * kRows * kD * 4 + U * kRows * kRows * 4 + U * kRows * 4 + 2 * U * (size_t)s.B * 4 +
-         2 * U * 4;
+  return U * kRows * kD * 4 + U * kRows * kRows * 4 + U * kRows * 4 + U * (size_t)s.B * 4 +
+         2 * U * 4 + ((U * (size_t)s.B + 15) & ~(size_t)15);
 }
 
 cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const void* v,
                             const float* scores, const float* y, const float* row_stats,
                             const int32_t* idx, void* k_out, void* v_out, char* ws,
                             const WsLayout& L, cudaStream_t st) {
-  CUtensorMap mq, mk, mv, mko;
+  CUtensorMap mq, mk, mv, mko, mvo;
   if (!encode_bf16_3d(&mq, q, kD, s.m, s.U, 64, kRows) ||
       !encode_bf16_2d_rows(&mk, k, kD, (uint64_t)s.U * s.n) ||
       !encode_bf16_2d_rows(&mv, v, kD, (uint64_t)s.U * s.n) ||
-      !encode_bf16_3d(&mko, k_out, kD, s.B, s.U, 64, kTile))
+      !encode_bf16_3d(&mko, k_out, kD, s.B, s.U, 64, kTile) ||
+      !encode_bf16_3d(&mvo, v_out, kD, s.B, s.U, 64, kTile))
     return cudaErrorInvalidValue;
   MArgs a{};
   a.U = s.U;
@@ -1244,16 +1256,16 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
   a.rz = (float*)(ws + L.merge_tc);
   a.gram = a.rz + U * kRows * kD;
   a.lam = a.gram + U * kRows * kRows;
-  a.perm = (int32_t*)(a.lam + U * kRows);
-  a.src = a.perm + U * s.B;
+  a.src = (int32_t*)(a.lam + U * kRows);
   a.ng = a.src + U * s.B;
   a.redo = a.ng + U;
+  a.fixed = (uint8_t*)(a.redo + U);
   a.status = (int*)(ws + L.status);
   cudaError_t e;
   if ((e = cudaFuncSetAttribute(k_merge_gram, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 kSmemBytes)) != cudaSuccess ||
       (e = cudaFuncSetAttribute(k_merge_update, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                kSmemBytes)) != cudaSuccess ||
+                                kSmemBytesU)) != cudaSuccess ||
       (e = cudaFuncSetAttribute(k_merge_solve, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 kSolveSmem)) != cudaSuccess ||
       (e = cudaFuncSetAttribute(k_merge_fixed, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1262,15 +1274,15 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
   k_merge_fixed<<<s.U, 256, s.B * 4, st>>>(a);
   if (row_stats) {
     a.gram_mode = 1;
-    k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, mko, a);
+    k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, a);
     a.gram_mode = 2;
-    k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, mko, a);
+    k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, a);
   } else {
     a.gram_mode = 0;
-    k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, mko, a);
+    k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, a);
   }
   k_merge_solve<<<s.U, 256, kSolveSmem, st>>>(a);
-  k_merge_update<<<s.U, kThreadsU, kSmemBytes, st>>>(mq, mk, a);
+  k_merge_update<<<s.U, kThreadsU, kSmemBytesU, st>>>(mq, mk, mv, mko, mvo, a);
   count_launches(row_stats ? 5 : 4);
   return cudaGetLastError();
 }
