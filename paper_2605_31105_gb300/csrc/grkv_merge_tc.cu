@@ -43,7 +43,7 @@ using namespace sm100;
 constexpr int kTile = 128;
 constexpr int kRows = 128;
 constexpr int kThreads = 384;    // k_merge_gram
-constexpr int kThreadsU = 512;   // k_merge_update
+constexpr int kThreadsU = 736;   // k_merge_update
 constexpr uint32_t kTileBytes = kTile * kD * 2;   // 32 KB
 constexpr int kMaxB = 32768;
 constexpr long long kBudget = 1ll << 32;
@@ -125,25 +125,30 @@ __device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map, u
       : "memory");
 }
 
-// Producer side of a ring of R gathered tiles, run by warps 2 and 3: warp pw
-// gathers tile rows pw*64 .. pw*64+63 (the rows rows_u[t*128 + row], clamped
-// to B-1; a row outside [0, n) reads row 0) with TMA gather4 into the
-// 128-byte-swizzled tile and arrives on the slot's full barrier with its 16 KB
-// of transaction bytes, so a slot is full once both halves have landed.  The
+// Producer side of a ring of R gathered tiles, run by W warps: warp pw
+// (0 <= pw < W) gathers tile rows pw*128/W .. (pw+1)*128/W - 1 (the rows
+// rows_u[t*128 + row], clamped to B-1; a row outside [0, n) reads row 0) with
+// TMA gather4 into the 128-byte-swizzled tile and arrives on the slot's full
+// barrier (initialised with W arrivals) with its share of the transaction
+// bytes, so a slot is full once every share has landed.  The issue cost of
+// gather4 is paid by the issuing warp, so more warps fill a tile faster.  The
 // row indices are fetched by rows() one tile ahead of load(), so their
-// latency overlaps the wait for a free slot, and one fetch serves the K and V
-// tiles of the same rows.
-template <int R>
+// latency overlaps the wait for a free slot, and one fetch can serve the K and
+// V tiles of the same rows.
+template <int R, int W>
 struct Gatherer {
+  static constexpr int kRowsW = kTile / W;   // rows per warp
+  static constexpr int kLanes = kRowsW / 4;  // lanes issuing one gather4 per half
+  static_assert(kTile % (4 * W) == 0 && kLanes <= 32, "gather split");
   uint8_t* ring;
   uint64_t* full;
   uint64_t* empty;
   uint32_t use = 0;
-  // lanes 0..15: the four rows pw*64 + 4*lane .. +3 of tile t, as map rows
+  // lanes < kLanes: the four rows pw*kRowsW + 4*lane .. +3 of tile t, as map rows
   __device__ __forceinline__ void rows(const int32_t* rows_u, int B, int n, int row0, int t,
                                        int pw, int lane, int* j) const {
-    if (lane < 16) {
-      const int r = pw * 64 + 4 * lane;
+    if (lane < kLanes) {
+      const int r = pw * kRowsW + 4 * lane;
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int jj = __ldg(rows_u + min(t * kTile + r + e, B - 1));
@@ -160,10 +165,10 @@ struct Gatherer {
     if (!ok) return false;
     uint8_t* dst = ring + slot * kTileBytes;
     uint64_t* bar = &full[slot];
-    if (lane == 0) mbar_expect_tx(bar, kTileBytes / 2);
+    if (lane == 0) mbar_expect_tx(bar, kTileBytes / W);
     __syncwarp();
-    if (lane < 16) {
-      const int r = pw * 64 + 4 * lane;
+    if (lane < kLanes) {
+      const int r = pw * kRowsW + 4 * lane;
       tma_gather4(dst + r * 128, map, bar, 0, j[0], j[1], j[2], j[3]);
       tma_gather4(dst + kTileBytes / 2 + r * 128, map, bar, 64, j[0], j[1], j[2], j[3]);
     }
@@ -409,7 +414,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int32_t* src_u = a.src + (size_t)u * B;
     const int row0 = u * a.n;   // first row of this unit in the 2-D K / V maps
     const int pw = warp - 2;
-    Gatherer<kRingG> gt{sm + kOffRing, bars->ring_full, bars->ring_empty};
+    Gatherer<kRingG, 2> gt{sm + kOffRing, bars->ring_full, bars->ring_empty};
     // job k < T reads K at the slots' rows, job k >= T K and V at the positions' rows
     auto rows_of = [&](int k, int* j) {
       gt.rows(k < T ? idx_u : src_u, B, a.n, row0, k < T ? k : k - T, pw, lane, j);
@@ -932,15 +937,17 @@ __global__ void __launch_bounds__(256, 2) k_merge_solve(MArgs a) {
 }
 
 // ======================================================== k_merge_update
-// Slot order, one unit per CTA, 512 threads.  Roles: warp 0 the Q load and
-// the K_out / V_out tile stores; warp 1 MMA issue; warps 2-3 the K0 and V0
-// gathers (two-slot rings each); warps 4-7 and 8-11 two compute groups taking
-// alternate tiles (one thread per token = TMEM lane of S^T): X_G^T from S^T,
-// zero for fixed slots, written back over S^T as packed bf16 (rows 32c ..
-// 32c+31 of chunk c: high parts to columns 32c .. 32c+15, low parts to
-// 32c+16 .. 32c+31, each chunk read before it is overwritten); warps 12-15
-// the epilogue (thread = token): V_out = V0 + dV in the V0 tile, which warp 0
-// then stores.  A fixed slot has X = 0 and so dV = 0: its row is left as V0.
+// Slot order, one unit per CTA, 736 threads.  Roles: warp 0 the Q load and
+// the K_out tile stores, warp 22 the V_out tile stores; warp 1 MMA issue;
+// warps 2, 3, 16, 17 the K0 gathers and 18-21 the V0 gathers (two-slot rings
+// each, on all four SM sub-partitions); warps 4-7 and 8-11
+// two compute groups taking alternate tiles (one thread per token = TMEM lane
+// of S^T): X_G^T from S^T, zero for fixed slots, written back over S^T as
+// packed bf16 (rows 32c .. 32c+31 of chunk c: high parts to columns 32c ..
+// 32c+15, low parts to 32c+16 .. 32c+31, each chunk read before it is
+// overwritten); warps 12-15 the epilogue (thread = token): V_out = V0 + dV in
+// the V0 tile, which warp 0 then stores.  A fixed slot has X = 0 and so
+// dV = 0: its row is left as V0.
 struct UBars {
   uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
   uint64_t q_full;
@@ -978,8 +985,8 @@ __global__ void __launch_bounds__(kThreadsU, 1)
   const int32_t* idx_u = a.idx + (size_t)u * B;
   if (tid == 0) {
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&bars->k_full[i], 2);    // one expect_tx arrival per gathering warp
-      mbar_init(&bars->v_full[i], 2);
+      mbar_init(&bars->k_full[i], 4);    // one expect_tx arrival per gathering warp
+      mbar_init(&bars->v_full[i], 4);
       mbar_init(&bars->k_empty[i], 2);   // the S^T MMA and the K_out store
       mbar_init(&bars->v_empty[i], 1);   // the V_out store
       mbar_init(&bars->s_full[i], 1);
@@ -1029,17 +1036,15 @@ __global__ void __launch_bounds__(kThreadsU, 1)
     if (lane == 0) {
       prefetch_tensormap(&tmQ);
       prefetch_tensormap(&tmKo);
-      prefetch_tensormap(&tmVo);
       mbar_expect_tx(&bars->q_full, kTileBytes);
       const uint64_t pol = l2_evict_last();
       tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, 0, u, pol);
       tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
-      // K_out = K0 and V_out tile by tile (the maps clip the rows past B)
+      // K_out = K0 tile by tile (the map clips the rows past B)
       bool ok = true;
       for (int t = 0; t < T && ok; ++t) {
         const int sl = t & 1;
-        const uint32_t par = (t >> 1) & 1;
-        ok = mbar_wait(&bars->k_full[sl], par, abort_flag, kBudget);
+        ok = mbar_wait(&bars->k_full[sl], (t >> 1) & 1, abort_flag, kBudget);
         if (!ok) break;
         const uint8_t* kt = sm + kOffKU + sl * kTileBytes;
         tma_store_3d(&tmKo, kt, 0, t * kTile, u);
@@ -1047,7 +1052,18 @@ __global__ void __launch_bounds__(kThreadsU, 1)
         bulk_commit();
         bulk_wait_read<0>();
         mbar_arrive(&bars->k_empty[sl]);
-        ok = mbar_wait(&bars->vo_full[sl], par, abort_flag, kBudget);
+      }
+      bulk_wait_all();
+      if (!ok) set_status(a.status, GRKV_ERR_TIMEOUT);
+    }
+  } else if (warp == 22) {
+    if (lane == 0) {
+      prefetch_tensormap(&tmVo);
+      // V_out tile by tile, once the epilogue has written it
+      bool ok = true;
+      for (int t = 0; t < T && ok; ++t) {
+        const int sl = t & 1;
+        ok = mbar_wait(&bars->vo_full[sl], (t >> 1) & 1, abort_flag, kBudget);
         if (!ok) break;
         const uint8_t* vt = sm + kOffVU + sl * kTileBytes;
         tma_store_3d(&tmVo, vt, 0, t * kTile, u);
@@ -1059,21 +1075,23 @@ __global__ void __launch_bounds__(kThreadsU, 1)
       bulk_wait_all();
       if (!ok) set_status(a.status, GRKV_ERR_TIMEOUT);
     }
-  } else if (warp == 2 || warp == 3) {
-    const int pw = warp - 2, row0 = u * a.n;
-    Gatherer<2> gk{sm + kOffKU, bars->k_full, bars->k_empty};
-    Gatherer<2> gv{sm + kOffVU, bars->v_full, bars->v_empty};
+  } else if (warp == 2 || warp == 3 || (warp >= 16 && warp < 22)) {
+    // K0 gathers: warps 2, 3, 16, 17; V0 gathers: warps 18 - 21 (own rings, so
+    // that a K tile never waits for a V slot)
+    const bool is_v = warp >= 18;
+    const int pw = warp < 4 ? warp - 2 : (is_v ? warp - 18 : warp - 14), row0 = u * a.n;
+    Gatherer<2, 4> g{sm + (is_v ? kOffVU : kOffKU), is_v ? bars->v_full : bars->k_full,
+                     is_v ? bars->v_empty : bars->k_empty};
+    const CUtensorMap* map = is_v ? &tmV : &tmK;
     int jn[4];
-    gk.rows(idx_u, B, a.n, row0, 0, pw, lane, jn);
+    g.rows(idx_u, B, a.n, row0, 0, pw, lane, jn);
     bool ok = true;
     for (int t = 0; t < T && ok; ++t) {
       const int j[4] = {jn[0], jn[1], jn[2], jn[3]};
-      if (t + 1 < T) gk.rows(idx_u, B, a.n, row0, t + 1, pw, lane, jn);
-      ok = gk.load(&tmK, j, pw, lane, abort_flag);
-      if (ok) ok = gv.load(&tmV, j, pw, lane, abort_flag);
+      if (t + 1 < T) g.rows(idx_u, B, a.n, row0, t + 1, pw, lane, jn);
+      ok = g.load(map, j, pw, lane, abort_flag);
     }
-    gk.drain(abort_flag);
-    gv.drain(abort_flag);
+    g.drain(abort_flag);
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t id_s = idesc_bf16(kTile, kRows, 0, 0);   // S^T = K0 Q^T
@@ -1122,7 +1140,7 @@ __global__ void __launch_bounds__(kThreadsU, 1)
       mma_commit(&bars->drain);
       mbar_wait(&bars->drain, 0, abort_flag, kBudget);
     }
-  } else if (warp < 12) {
+  } else if (warp >= 4 && warp < 12) {
     // compute groups: group cg takes the tiles t with t % 2 == cg
     const int cg = (warp - 4) >> 2, q = warp & 3, tok = q * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
@@ -1158,7 +1176,7 @@ __global__ void __launch_bounds__(kThreadsU, 1)
       mbar_arrive(&bars->x_full[sl]);
     }
     if (!ok && tok == 0 && cg == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
-  } else {
+  } else if (warp >= 12 && warp < 16) {
     // epilogue: thread = token (TMEM lane of D), V_out = V0 + dV in the V tile
     const int q = warp & 3, tok = q * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
