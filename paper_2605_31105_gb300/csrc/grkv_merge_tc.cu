@@ -690,6 +690,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // so that their 32-element arrays stay in registers.
 __host__ __device__ constexpr int tri(int i) { return (i * (i + 1)) >> 1; }
 constexpr int kTri = tri(kRows) + 4;   // packed N, padded to 16 bytes
+constexpr int kSolveThreads = 256;
 
 // Factors the 32 x 32 diagonal block at k0 (right-looking; lane l holds row
 // k0 + l) and stores 1 / L_jj.  Returns true on a non-positive pivot.
@@ -741,49 +742,33 @@ __device__ __noinline__ void chol_panel_row(float* N, const float* dinv, int k0,
   for (int j = 0; j < 32; ++j) N[rb + j] = x[j];
 }
 
-// Column e of rows i0..i0+31: W = L_bb^-1 W (forward) or L_bb^-T W (backward).
-__device__ __noinline__ void trsv_fwd(const float* N, float* R, const float* dinv, int i0, int e) {
-  float z[32];
-#pragma unroll
-  for (int i = 0; i < 32; ++i) z[i] = R[(i0 + i) * kLD + e];
+// Inverts the lower-triangular 32 x 32 diagonal block at k0 in place: lane l
+// computes column l of L_bb^-1 by forward substitution (its entries above the
+// diagonal come out zero) and writes it once every lane has read the block.
+__device__ __noinline__ void tri_inv_diag(float* N, const float* dinv, int k0, int lane) {
+  float x[32];
 #pragma unroll
   for (int i = 0; i < 32; ++i) {
-    const float* li = N + tri(i0 + i) + i0;
-    float s0 = z[i], s1 = 0.f;
+    const float* li = N + tri(k0 + i) + k0;
+    float s0 = i == lane ? 1.f : 0.f, s1 = 0.f;
 #pragma unroll
-    for (int kx = 0; kx < i; ++kx) {
-      if (kx & 1) s1 += li[kx] * z[kx];
-      else s0 -= li[kx] * z[kx];
+    for (int k = 0; k < i; ++k) {
+      if (k & 1) s1 += li[k] * x[k];
+      else s0 -= li[k] * x[k];
     }
-    z[i] = (s0 - s1) * dinv[i0 + i];
+    x[i] = (s0 - s1) * dinv[k0 + i];
   }
+  __syncwarp();
 #pragma unroll
-  for (int i = 0; i < 32; ++i) R[(i0 + i) * kLD + e] = z[i];
-}
-__device__ __noinline__ void trsv_bwd(const float* N, float* R, const float* dinv, int i0, int e) {
-  float z[32];
-#pragma unroll
-  for (int i = 0; i < 32; ++i) z[i] = R[(i0 + i) * kLD + e];
-#pragma unroll
-  for (int i = 31; i >= 0; --i) {
-    float s0 = z[i], s1 = 0.f;
-#pragma unroll
-    for (int kx = i + 1; kx < 32; ++kx) {
-      const float l = N[tri(i0 + kx) + i0 + i];
-      if (kx & 1) s1 += l * z[kx];
-      else s0 -= l * z[kx];
-    }
-    z[i] = (s0 - s1) * dinv[i0 + i];
-  }
-#pragma unroll
-  for (int i = 0; i < 32; ++i) R[(i0 + i) * kLD + e] = z[i];
+  for (int i = 0; i < 32; ++i)
+    if (i >= lane) N[tri(k0 + i) + k0 + lane] = x[i];
 }
 
 // N = (G + G^T) / 2 + lambda I on the window rows (identity on padding rows),
-// Cholesky N = L L^T in 32-row blocks, then Z = L^-T L^-1 R; fp32 in shared
-// memory.  A non-positive pivot reports GRKV_ERR_NUMERIC and leaves Z = 0
+// Cholesky N = L L^T in 32-row blocks, then Z = L^-T L^-1 R by block
+// substitution with the inverted diagonal blocks; fp32 in shared memory.  A non-positive pivot reports GRKV_ERR_NUMERIC and leaves Z = 0
 // (values stay V0); lambda = +inf also gives Z = 0.
-__global__ void __launch_bounds__(256, 2) k_merge_solve(MArgs a) {
+__global__ void __launch_bounds__(kSolveThreads, 2) k_merge_solve(MArgs a) {
   extern __shared__ __align__(16) float ssm[];
   float* N = ssm;                   // packed lower triangle
   float* R = N + kTri;              // [128][kLD]: G first, then R, then Z
@@ -791,22 +776,32 @@ __global__ void __launch_bounds__(256, 2) k_merge_solve(MArgs a) {
   int* fail = (int*)(dinv + kRows);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, nt = blockDim.x;
   const int u = blockIdx.x, m = a.m;
-  const float4* G4 = (const float4*)(a.gram + (size_t)u * kRows * kRows);
   float* RZ = a.rz + (size_t)u * kRows * kD;
   if (a.lambda_inf) {
     for (int p = tid; p < kRows * kD / 4; p += nt) ((float4*)RZ)[p] = make_float4(0.f, 0.f, 0.f, 0.f);
     return;
   }
   if (tid == 0) *fail = 0;
-  // G into the R buffer, then its symmetric part into the packed triangle
-#pragma unroll 4
-  for (int p = tid; p < kRows * kRows / 4; p += nt) {
-    const float4 g = __ldg(G4 + p);
-    float* r = R + (p >> 5) * kLD + (p & 31) * 4;
-    r[0] = g.x; r[1] = g.y; r[2] = g.z; r[3] = g.w;
+  // G into the R buffer with every load of a half in flight at once (one
+  // element per lane and step: conflict-free stores into the padded rows)
+  const float* Gs = a.gram + (size_t)u * kRows * kRows;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    float g[32];
+#pragma unroll
+    for (int k = 0; k < 32; ++k) g[k] = __ldg(Gs + tid + kSolveThreads * (32 * h + k));
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      const int p = tid + kSolveThreads * (32 * h + k);
+      R[(p >> 7) * kLD + (p & 127)] = g[k];
+    }
   }
+  // R's loads are issued before the symmetric part is formed and stored after
+  float rr[64];
+#pragma unroll
+  for (int k = 0; k < 64; ++k) rr[k] = __ldg(RZ + tid + kSolveThreads * k);
   __syncthreads();
-  for (int i = warp; i < kRows; i += nt / 32)
+  for (int i = warp; i < kRows; i += kSolveThreads / 32)
     for (int j = lane; j <= i; j += 32) {
       float val;
       if (i >= m || j >= m) val = (i == j) ? 1.f : 0.f;
@@ -815,11 +810,10 @@ __global__ void __launch_bounds__(256, 2) k_merge_solve(MArgs a) {
       N[tri(i) + j] = val;
     }
   __syncthreads();
-#pragma unroll 4
-  for (int p = tid; p < kRows * kD / 4; p += nt) {
-    const float4 r4 = __ldg((const float4*)RZ + p);
-    float* r = R + (p >> 5) * kLD + (p & 31) * 4;
-    r[0] = r4.x; r[1] = r4.y; r[2] = r4.z; r[3] = r4.w;
+#pragma unroll
+  for (int k = 0; k < 64; ++k) {
+    const int p = tid + kSolveThreads * k;
+    R[(p >> 7) * kLD + (p & 127)] = rr[k];
   }
   for (int kb = 0; kb < kRows / 32; ++kb) {
     const int k0 = kb * 32;
@@ -868,10 +862,37 @@ __global__ void __launch_bounds__(256, 2) k_merge_solve(MArgs a) {
     for (int p = tid; p < kRows * kD / 4; p += nt) ((float4*)RZ)[p] = make_float4(0.f, 0.f, 0.f, 0.f);
     return;
   }
-  // forward: L W = R in 32-row blocks; one column of R per thread
+  // the diagonal blocks of L are replaced by their inverses (one warp each)
+  if (warp < kRows / 32) tri_inv_diag(N, dinv, warp * 32, lane);
+  __syncthreads();
+  // forward: L W = R in 32-row blocks, W_b = L_bb^-1 (R_b - L_b,<b W_<b);
+  // thread: rows 4 rg .. 4 rg + 3 of the block, columns e + 32 c
+  const int rg = warp, e = lane;
   for (int ib = 0; ib < kRows / 32; ++ib) {
     const int i0 = ib * 32;
-    if (tid < kD) trsv_fwd(N, R, dinv, i0, tid);
+    {
+      float acc[4][4] = {};
+      const float* lr[4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) lr[r] = N + tri(i0 + 4 * rg + r) + i0;
+#pragma unroll 4
+      for (int kx = 0; kx < 4 * rg + 4; ++kx) {
+        float l[4], z[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) l[r] = kx <= 4 * rg + r ? lr[r][kx] : 0.f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) z[c] = R[(i0 + kx) * kLD + e + 32 * c];
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) acc[r][c] += l[r] * z[c];
+      }
+      __syncthreads();
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) R[(i0 + 4 * rg + r) * kLD + e + 32 * c] = acc[r][c];
+    }
     __syncthreads();
     // rows below: 4 rows x 4 columns (stride 32) per thread
     const int i1 = i0 + 32, nb = (kRows - i1) / 4 * 32;
@@ -900,10 +921,30 @@ __global__ void __launch_bounds__(256, 2) k_merge_solve(MArgs a) {
     }
     __syncthreads();
   }
-  // backward: L^T Z = W
+  // backward: L^T Z = W, Z_b = L_bb^-T (W_b - L_>b,b^T Z_>b)
   for (int ib = kRows / 32 - 1; ib >= 0; --ib) {
     const int i0 = ib * 32;
-    if (tid < kD) trsv_bwd(N, R, dinv, i0, tid);
+    {
+      float acc[4][4] = {};
+#pragma unroll 4
+      for (int kx = 4 * rg; kx < 32; ++kx) {
+        const float* lk = N + tri(i0 + kx) + i0 + 4 * rg;
+        float l[4], z[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) l[r] = 4 * rg + r <= kx ? lk[r] : 0.f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) z[c] = R[(i0 + kx) * kLD + e + 32 * c];
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) acc[r][c] += l[r] * z[c];
+      }
+      __syncthreads();
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) R[(i0 + 4 * rg + r) * kLD + e + 32 * c] = acc[r][c];
+    }
     __syncthreads();
     // rows above: 4 rows x 4 columns (stride 32) per thread
     const int nb = i0 / 4 * 32;
@@ -1299,7 +1340,7 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
     a.gram_mode = 0;
     k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, a);
   }
-  k_merge_solve<<<s.U, 256, kSolveSmem, st>>>(a);
+  k_merge_solve<<<s.U, kSolveThreads, kSolveSmem, st>>>(a);
   k_merge_update<<<s.U, kThreadsU, kSmemBytesU, st>>>(mq, mk, mv, mko, mvo, a);
   count_launches(row_stats ? 5 : 4);
   return cudaGetLastError();

@@ -180,15 +180,20 @@ __device__ __forceinline__ int ld_acquire(const int* p) {
   return v;
 }
 
+// Three-operand maximum (one instruction on sm_100 and later).
+__device__ __forceinline__ float fmax3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
 __device__ __forceinline__ float max32(const float* v) {
-  float m[16];
+  float m[11];
 #pragma unroll
-  for (int e = 0; e < 16; ++e) m[e] = fmaxf(v[e], v[e + 16]);
-#pragma unroll
-  for (int h = 8; h >= 1; h >>= 1)
-#pragma unroll
-    for (int e = 0; e < h; ++e) m[e] = fmaxf(m[e], m[e + h]);
-  return m[0];
+  for (int e = 0; e < 10; ++e) m[e] = fmax3f(v[3 * e], v[3 * e + 1], v[3 * e + 2]);
+  m[10] = fmaxf(v[30], v[31]);
+  const float x0 = fmax3f(m[0], m[1], m[2]), x1 = fmax3f(m[3], m[4], m[5]),
+              x2 = fmax3f(m[6], m[7], m[8]), x3 = fmaxf(m[9], m[10]);
+  return fmaxf(fmax3f(x0, x1, x2), x3);
 }
 
 // Pass A on 32 logits of one row: online max / sum of exp2 in log2 units.
