@@ -86,6 +86,13 @@ SCORE_TRAFFIC = {
 }
 
 
+SCORE_KERNEL = {
+    "default": "grkv_score stage (k_score_tc: window scoring + target, two launches)",
+    "one_read": "grkv_score stage (k_score_pipe: window scoring + target, one read of K)",
+    "portable": "grkv_score stage (CUDA-core kernels: k_stats_chunk, k_stats_reduce, k_prob_chunk, k_y_reduce)",
+}
+
+
 def score_traffic(wl):
     rec = SCORE_TRAFFIC.get(wl.name)
     if rec is None:
@@ -438,7 +445,8 @@ def run_ours(a):
                    "pool_kernel": wl.pool_kernel, "l2": "inputs (K+V %.1f GB) exceed L2" %
                    (read / 1e9), "parallelism": f"units sharded, {world} rank(s)"},
         "path": a.path,
-        "roofline": {"bound": "hbm", "kernel": "grkv_score stage (k_score_tc: window scoring + target, two launches)",
+        "roofline": {"bound": "hbm",
+                     "kernel": SCORE_KERNEL["portable" if wl.dtype != "bf16" else a.path],
                      "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "traffic": score_traffic(wl) if a.path == "default" else None,
