@@ -126,7 +126,7 @@ __device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map, u
 }
 
 // Producer side of a ring of R gathered tiles, run by W warps: warp pw
-// (0 <= pw < W) gathers tile rows pw*128/W .. (pw+1)*128/W - 1 (the rows
+// (0 <= pw < W) gathers its share of the tile's 32 four-row groups (the rows
 // rows_u[t*128 + row], clamped to B-1; a row outside [0, n) reads row 0) with
 // TMA gather4 into the 128-byte-swizzled tile and arrives on the slot's full
 // barrier (initialised with W arrivals) with its share of the transaction
@@ -137,18 +137,18 @@ __device__ __forceinline__ void tma_gather4(void* dst, const CUtensorMap* map, u
 // V tiles of the same rows.
 template <int R, int W>
 struct Gatherer {
-  static constexpr int kRowsW = kTile / W;   // rows per warp
-  static constexpr int kLanes = kRowsW / 4;  // lanes issuing one gather4 per half
-  static_assert(kTile % (4 * W) == 0 && kLanes <= 32, "gather split");
+  // warp pw takes the four-row groups g0(pw) .. g0(pw + 1) - 1 of the 32 in a tile
+  static constexpr int g0(int pw) { return pw * (kTile / 4) / W; }
+  static_assert(kTile / 4 / W <= 32 && W >= 1, "gather split");
   uint8_t* ring;
   uint64_t* full;
   uint64_t* empty;
   uint32_t use = 0;
-  // lanes < kLanes: the four rows pw*kRowsW + 4*lane .. +3 of tile t, as map rows
+  // lanes < the warp's group count: the four rows of group g0(pw) + lane of tile t, as map rows
   __device__ __forceinline__ void rows(const int32_t* rows_u, int B, int n, int row0, int t,
                                        int pw, int lane, int* j) const {
-    if (lane < kLanes) {
-      const int r = pw * kRowsW + 4 * lane;
+    if (lane < g0(pw + 1) - g0(pw)) {
+      const int r = 4 * (g0(pw) + lane);
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int jj = __ldg(rows_u + min(t * kTile + r + e, B - 1));
@@ -165,10 +165,11 @@ struct Gatherer {
     if (!ok) return false;
     uint8_t* dst = ring + slot * kTileBytes;
     uint64_t* bar = &full[slot];
-    if (lane == 0) mbar_expect_tx(bar, kTileBytes / W);
+    const int ng = g0(pw + 1) - g0(pw);
+    if (lane == 0) mbar_expect_tx(bar, ng * 4 * kD * 2);
     __syncwarp();
-    if (lane < kLanes) {
-      const int r = pw * kRowsW + 4 * lane;
+    if (lane < ng) {
+      const int r = 4 * (g0(pw) + lane);
       tma_gather4(dst + r * 128, map, bar, 0, j[0], j[1], j[2], j[3]);
       tma_gather4(dst + kTileBytes / 2 + r * 128, map, bar, 64, j[0], j[1], j[2], j[3]);
     }
@@ -188,7 +189,7 @@ __device__ __forceinline__ void init_common(MBars* bars, int warp, uint32_t ring
                                             uint32_t group_count, uint32_t epi_count) {
   if (threadIdx.x == 0) {
     for (int i = 0; i < 4; ++i) {
-      mbar_init(&bars->ring_full[i], 2);   // one expect_tx arrival per gathering warp
+      mbar_init(&bars->ring_full[i], 3);   // one expect_tx arrival per gathering warp
       mbar_init(&bars->ring_empty[i], ring_empty_count);
     }
     mbar_init(&bars->q_full, 1);
@@ -370,7 +371,7 @@ __global__ void __launch_bounds__(256) k_merge_fixed(MArgs a) {
 }
 
 // ======================================================== k_merge_gram
-// Roles (384 threads): warp 0 the Q load; warp 1 MMA issue; warps 2-3 the gathers (half a tile each);
+// Roles (384 threads): warp 0 the Q load; warp 1 MMA issue; warps 0, 2, 3 the gathers;
 // warps 4-7 and 8-11 two compute groups (one thread per window row / TMEM
 // lane) taking alternate jobs.  Job k < T: statistics of slot tile k;
 // T <= k < 2T: R~ and Gram of position tile k - T.  Ring loads: K of each
@@ -401,20 +402,21 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = bars->tmem;
   volatile int* abort_flag = &bars->abort;
 
-  if (warp == 0) {
-    if (lane == 0) {
+  if (warp == 0 || warp == 2 || warp == 3) {
+    if (warp == 0 && lane == 0) {
       prefetch_tensormap(&tmQ);
       mbar_expect_tx(&bars->q_full, kTileBytes);
       const uint64_t pol = l2_evict_last();
       tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, 0, u, pol);
       tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
     }
-  } else if (warp == 2 || warp == 3) {
+    __syncwarp();
+    // the gathers: warps 0, 2 and 3 (three SM sub-partitions)
     const int32_t* idx_u = a.idx + (size_t)u * B;
     const int32_t* src_u = a.src + (size_t)u * B;
     const int row0 = u * a.n;   // first row of this unit in the 2-D K / V maps
-    const int pw = warp - 2;
-    Gatherer<kRingG, 2> gt{sm + kOffRing, bars->ring_full, bars->ring_empty};
+    const int pw = warp == 0 ? 0 : warp - 1;
+    Gatherer<kRingG, 3> gt{sm + kOffRing, bars->ring_full, bars->ring_empty};
     // job k < T reads K at the slots' rows, job k >= T K and V at the positions' rows
     auto rows_of = [&](int k, int* j) {
       gt.rows(k < T ? idx_u : src_u, B, a.n, row0, k < T ? k : k - T, pw, lane, j);
