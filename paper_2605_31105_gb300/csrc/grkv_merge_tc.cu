@@ -979,6 +979,152 @@ __global__ void __launch_bounds__(kSolveThreads, 2) k_merge_solve(MArgs a) {
   }
 }
 
+// ======================================================== k_solve_dense
+// The regression solve of the portable merge (m <= 256): N = X_G X_G^T +
+// lambda I (full symmetric, lambda included, [m][m]) and R ([m][128]) from
+// the workspace, Z = N^-1 R written over R.  The same blocked fp32 algorithm
+// as k_merge_solve, for up to 256 rows: N as a packed lower triangle in
+// shared memory (rows past m are identity), Cholesky in 32-row blocks, the
+// diagonal blocks inverted in place, then block substitution over R in two
+// passes of 64 columns.  One 512-thread CTA per unit.
+constexpr int kDenseM = 256, kDenseNT = 512, kDenseC = 64, kDenseLD = kDenseC + 1;
+constexpr int kDenseTri = tri(kDenseM) + 4;
+constexpr uint32_t kDenseSmem = (kDenseTri + kDenseM * kDenseLD + kDenseM + 32) * 4;
+
+__global__ void __launch_bounds__(kDenseNT, 1)
+    k_solve_dense(const float* __restrict__ gram, float* __restrict__ rz, int m, int* status) {
+  extern __shared__ __align__(16) float dsm[];
+  float* N = dsm;                       // packed lower triangle
+  float* R = N + kDenseTri;             // [256][kDenseLD]: one column pass of R, then of Z
+  float* dinv = R + kDenseM * kDenseLD; // [256]
+  int* fail = (int*)(dinv + kDenseM);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int u = blockIdx.x;
+  const float* Gu = gram + (size_t)u * m * m;
+  float* RZ = rz + (size_t)u * m * kD;
+  if (tid == 0) *fail = 0;
+  for (int i = warp; i < kDenseM; i += kDenseNT / 32)
+    for (int j = lane; j <= i; j += 32)
+      N[tri(i) + j] = (i < m && j < m) ? __ldg(Gu + (size_t)i * m + j) : (i == j ? 1.f : 0.f);
+  __syncthreads();
+  for (int kb = 0; kb < kDenseM / 32; ++kb) {
+    const int k0 = kb * 32;
+    if (warp == 0 && chol_diag(N, dinv, k0, lane) && lane == 0) *fail = 1;
+    __syncthreads();
+    for (int i = k0 + 32 + tid; i < kDenseM; i += kDenseNT) chol_panel_row(N, dinv, k0, i);
+    __syncthreads();
+    // trailing update of the lower triangle in 4x4 register blocks
+    const int k1 = k0 + 32, t4 = (kDenseM - k1) / 4, nb = t4 * (t4 + 1) / 2;
+    for (int t = tid; t < nb; t += kDenseNT) {
+      int bi = (int)((sqrtf(8.f * t + 1.f) - 1.f) * 0.5f);
+      while ((bi + 1) * (bi + 2) / 2 <= t) ++bi;
+      while (bi * (bi + 1) / 2 > t) --bi;
+      const int i = k1 + 4 * bi, j = k1 + 4 * (t - bi * (bi + 1) / 2);
+      float acc[4][4] = {};
+#pragma unroll 4
+      for (int pp = 0; pp < 32; ++pp) {
+        float vi[4], vj[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          vi[r] = N[tri(i + r) + k0 + pp];
+          vj[r] = N[tri(j + r) + k0 + pp];
+        }
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) acc[r][c] += vi[r] * vj[c];
+      }
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+          if (j + c <= i + r) N[tri(i + r) + j + c] -= acc[r][c];
+    }
+    __syncthreads();
+  }
+  if (*fail) {
+    if (tid == 0) set_status(status, GRKV_ERR_NUMERIC);
+    for (int p = tid; p < m * kD; p += kDenseNT) RZ[p] = 0.f;
+    return;
+  }
+  if (warp < kDenseM / 32) tri_inv_diag(N, dinv, warp * 32, lane);
+  __syncthreads();
+  // block steps: thread = rows 4 rg .. 4 rg + 3 of a 32-row block, column cc
+  const int rg = warp & 7, cc = (tid >> 8) * 32 + lane;
+  for (int c0 = 0; c0 < kD; c0 += kDenseC) {
+    for (int p = tid; p < kDenseM * kDenseC; p += kDenseNT) {
+      const int r = p / kDenseC, c = p % kDenseC;
+      R[r * kDenseLD + c] = r < m ? RZ[(size_t)r * kD + c0 + c] : 0.f;
+    }
+    __syncthreads();
+    // forward: W_b = L_bb^-1 (R_b - L_b,<b W_<b)
+    for (int ib = 0; ib < kDenseM / 32; ++ib) {
+      const int i0 = ib * 32;
+      float acc[4] = {};
+      for (int kx = 0; kx < 4 * rg + 4; ++kx) {
+        const float z = R[(i0 + kx) * kDenseLD + cc];
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+          acc[r] += (kx <= 4 * rg + r ? N[tri(i0 + 4 * rg + r) + i0 + kx] : 0.f) * z;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int r = 0; r < 4; ++r) R[(i0 + 4 * rg + r) * kDenseLD + cc] = acc[r];
+      __syncthreads();
+      // rows below: 4 rows x 1 column per task
+      const int i1 = i0 + 32, ntask = (kDenseM - i1) / 4 * kDenseC;
+      for (int t = tid; t < ntask; t += kDenseNT) {
+        const int i = i1 + 4 * (t / kDenseC), c = t % kDenseC;
+        float a4[4] = {};
+#pragma unroll 8
+        for (int kx = 0; kx < 32; ++kx) {
+          const float z = R[(i0 + kx) * kDenseLD + c];
+#pragma unroll
+          for (int r = 0; r < 4; ++r) a4[r] += N[tri(i + r) + i0 + kx] * z;
+        }
+#pragma unroll
+        for (int r = 0; r < 4; ++r) R[(i + r) * kDenseLD + c] -= a4[r];
+      }
+      __syncthreads();
+    }
+    // backward: Z_b = L_bb^-T (W_b - L_>b,b^T Z_>b)
+    for (int ib = kDenseM / 32 - 1; ib >= 0; --ib) {
+      const int i0 = ib * 32;
+      float acc[4] = {};
+      for (int kx = 4 * rg; kx < 32; ++kx) {
+        const float z = R[(i0 + kx) * kDenseLD + cc];
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+          acc[r] += (4 * rg + r <= kx ? N[tri(i0 + kx) + i0 + 4 * rg + r] : 0.f) * z;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int r = 0; r < 4; ++r) R[(i0 + 4 * rg + r) * kDenseLD + cc] = acc[r];
+      __syncthreads();
+      // rows above: 4 rows x 1 column per task
+      const int ntask = i0 / 4 * kDenseC;
+      for (int t = tid; t < ntask; t += kDenseNT) {
+        const int i = 4 * (t / kDenseC), c = t % kDenseC;
+        float a4[4] = {};
+#pragma unroll 8
+        for (int kx = 0; kx < 32; ++kx) {
+          const float z = R[(i0 + kx) * kDenseLD + c];
+#pragma unroll
+          for (int r = 0; r < 4; ++r) a4[r] += N[tri(i0 + kx) + i + r] * z;
+        }
+#pragma unroll
+        for (int r = 0; r < 4; ++r) R[(i + r) * kDenseLD + c] -= a4[r];
+      }
+      __syncthreads();
+    }
+    for (int p = tid; p < m * kDenseC; p += kDenseNT) {
+      const int r = p / kDenseC, c = p % kDenseC;
+      RZ[(size_t)r * kD + c0 + c] = R[r * kDenseLD + c];
+    }
+    __syncthreads();
+  }
+}
+
 // ======================================================== k_merge_update
 // Slot order, one unit per CTA, 736 threads.  Roles: warp 0 the Q load and
 // the K_out tile stores, warp 22 the V_out tile stores; warp 1 MMA issue;
@@ -1279,6 +1425,17 @@ size_t merge_tc_ws_bytes(const Shape& s) {
   const size_t U = (size_t)s.U;
   return U * kRows * kD * 4 + U * kRows * kRows * 4 + U * kRows * 4 + U * (size_t)s.B * 4 +
          2 * U * 4 + ((U * (size_t)s.B + 15) & ~(size_t)15);
+}
+
+cudaError_t launch_solve_dense(int U, int m, const float* gram, float* rz, int* status,
+                               cudaStream_t st) {
+  if (m > kDenseM) return cudaErrorInvalidValue;
+  cudaError_t e = cudaFuncSetAttribute(k_solve_dense, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       kDenseSmem);
+  if (e != cudaSuccess) return e;
+  k_solve_dense<<<U, kDenseNT, kDenseSmem, st>>>(gram, rz, m, status);
+  count_launches(1);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const void* v,

@@ -7,6 +7,7 @@
 // The value-step solve accumulates in double for fp32 inputs.
 #include <cfloat>
 #include <cmath>
+#include <type_traits>
 
 #include "block_select.cuh"
 #include "grkv_internal.cuh"
@@ -421,13 +422,16 @@ __global__ void __launch_bounds__(kSelThreads, 1) k_select_smem(const float* __r
 
 // ------------------------------------------------------------------ merge --
 // One CTA per unit.  A is the accumulation type of the regression (double for
-// fp32 inputs, float for bf16).
+// fp32 inputs, float for bf16).  phase 0 runs the whole value step; phase 1
+// stops once R and N are in the workspace and phase 2 starts from Z there
+// (the fp32 solve between them is k_solve_dense).
 template <typename T, typename A>
 __global__ void __launch_bounds__(512) k_merge(
     const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
     const float* __restrict__ scores, const float* __restrict__ y, const int32_t* __restrict__ idx,
     T* __restrict__ k_out, T* __restrict__ v_out, Shape s, float* __restrict__ xbuf,
-    uint8_t* __restrict__ flags, A* __restrict__ gram, A* __restrict__ rz, int* status) {
+    uint8_t* __restrict__ flags, A* __restrict__ gram, A* __restrict__ rz, int* status,
+    int phase) {
   extern __shared__ __align__(16) float sm[];
   __shared__ int hist[256];
   __shared__ int sh[48];
@@ -442,8 +446,6 @@ __global__ void __launch_bounds__(512) k_merge(
     const int j = id[i];
     return (unsigned)j < (unsigned)s.n ? j : 0;
   };
-  for (int i = tid; i < B; i += nthr)
-    if ((unsigned)id[i] >= (unsigned)s.n) set_status(status, GRKV_ERR_INVALID_ARG);
   float* X = xbuf + (size_t)u * m * B;
   uint8_t* F = flags + (size_t)u * B;
   A* N = gram + (size_t)u * m * m;
@@ -454,6 +456,10 @@ __global__ void __launch_bounds__(512) k_merge(
   T* vo = v_out + (size_t)u * B * kD;
   const float* yu = y + (size_t)u * m * kD;
   const float* cu = scores + (size_t)u * s.P;
+  if (phase == 2 && s.lambda_inf) return;   // phase 1 wrote V_out = V0
+  if (phase != 2) {
+  for (int i = tid; i < B; i += nthr)
+    if ((unsigned)id[i] >= (unsigned)s.n) set_status(status, GRKV_ERR_INVALID_ARG);
 
   for (int i = tid; i < m * kD; i += nthr)
     qs[(i / kD) * QP + i % kD] = ldv(q + (size_t)u * m * kD, i);
@@ -595,6 +601,7 @@ __global__ void __launch_bounds__(512) k_merge(
     }
   }
   __syncthreads();
+  if (phase == 1) return;
 
   // Cholesky N = L L^T in place (lower triangle), right-looking.
   for (int c = 0; c < m; ++c) {
@@ -633,6 +640,8 @@ __global__ void __launch_bounds__(512) k_merge(
     }
   }
   __syncthreads();
+
+  }   // phase != 2
 
   // V_out[G] = V0[G] + X_G^T Z, V_out[F] = V0[F].
   for (int base = 0; base < B; base += 32) {
@@ -697,11 +706,23 @@ cudaError_t merge_impl(const Shape& s, const T* q, const T* k, const T* v, const
   cudaError_t e = cudaFuncSetAttribute(k_merge<T, A>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)sm);
   if (e != cudaSuccess) return e;
-  k_merge<T, A><<<s.U, 512, sm, st>>>(q, k, v, scores, y, idx, k_out, v_out, s,
-                                      (float*)(ws + L.xbuf), (uint8_t*)(ws + L.flags),
-                                      (A*)(ws + L.gram), (A*)(ws + L.rz), (int*)(ws + L.status));
-  count_launches(1);
-  return cudaGetLastError();
+  auto run = [&](int phase) {
+    k_merge<T, A><<<s.U, 512, sm, st>>>(q, k, v, scores, y, idx, k_out, v_out, s,
+                                        (float*)(ws + L.xbuf), (uint8_t*)(ws + L.flags),
+                                        (A*)(ws + L.gram), (A*)(ws + L.rz), (int*)(ws + L.status),
+                                        phase);
+    count_launches(1);
+    return cudaGetLastError();
+  };
+  // fp32 inputs keep the double-precision solve inside the kernel; bf16 inputs
+  // take the blocked shared-memory solve between two phases
+  if (!std::is_same<A, float>::value) return run(0);
+  if ((e = run(1)) != cudaSuccess) return e;
+  if (!s.lambda_inf &&
+      (e = launch_solve_dense(s.U, s.m, (const float*)(ws + L.gram), (float*)(ws + L.rz),
+                              (int*)(ws + L.status), st)) != cudaSuccess)
+    return e;
+  return run(2);
 }
 
 }  // namespace
