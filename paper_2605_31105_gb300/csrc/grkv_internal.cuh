@@ -111,10 +111,11 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
 
 // Tensor-core value merge (bf16, m <= 128, B <= 32768).
 bool merge_tc_supported(const Shape& s);
-// The portable merge's regression solve for m <= 256 (grkv_merge_tc.cu):
-// gram [U][m][m] (N with lambda), rz [U][m][128] (R in, Z out).
-cudaError_t launch_solve_dense(int U, int m, const float* gram, float* rz, int* status,
-                               cudaStream_t st);
+// The regression solve for m <= 256 (grkv_merge_tc.cu): gram [U][ld][ld]
+// (N with lambda when sym = 0; raw Gram blocks, symmetrised with lambda added,
+// when sym = 1), rz [U][ld][128] (R in, Z out).
+cudaError_t launch_solve_dense(int U, int m, int ld, int sym, float lambda, int lambda_inf,
+                               const float* gram, float* rz, int* status, cudaStream_t st);
 size_t merge_tc_ws_bytes(const Shape& s);
 // row_stats (nullable): the full-cache row statistics; with them the Gram
 // needs one pass over the retained keys.

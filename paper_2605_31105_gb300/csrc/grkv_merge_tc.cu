@@ -89,6 +89,12 @@ struct MArgs {
   int32_t* redo;             // [U]            single-pass result unusable: run two passes
   uint8_t* fixed;            // [U][B]         1 for a fixed slot
   int gram_mode;             // 0 two passes; 1 one pass against rstats; 2 two passes for redo units
+  // Row blocks (m > 128): a launch takes the 128 window rows row0 .. row0+127
+  // of block rb (of nrb); the per-unit arrays hold ldr rows (128 or 256):
+  // rz [U][ldr][128], gram [U][ldr][ldr], lam [U][ldr], redo [U][nrb].
+  int row0, rb, nrb, ldr;
+  int upd_mode;              // update: 0 V_out = V0 + dV; 1 vpart = V0 + dV; 2 V_out = vpart + dV
+  float* vpart;              // [U][B][128] fp32, between the update's two row blocks
   int* status;
 };
 
@@ -108,6 +114,14 @@ static_assert(sizeof(MBars) <= 256, "barrier block");
 
 __device__ __forceinline__ float lo_half(uint32_t h) { return __uint_as_float(h << 16); }
 __device__ __forceinline__ float hi_half(uint32_t h) { return __uint_as_float(h & 0xFFFF0000u); }
+
+// TMEM column, within a 128-column buffer, of the packed high (lo = 0) or low
+// (lo = 1) parts of K rows 16kk .. 16kk+15 of an A operand written back in
+// place over 32-column chunks (chunk c: high parts in 32c .. 32c+15, low parts
+// in 32c+16 .. 32c+31).
+__device__ __forceinline__ uint32_t xt_col(int kk, int lo) {
+  return (kk >> 1) * 32 + lo * 16 + (kk & 1) * 8;
+}
 
 // mbar_wait for all lanes of a warp with one answer, so that warp-collective
 // instructions after a wait are reached by all lanes or by none.
@@ -392,7 +406,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   MBars* bars = (MBars*)(sm + kOffBar);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int u = blockIdx.x, B = a.B, T = (B + kTile - 1) / kTile;
-  if (a.gram_mode == 2 && __ldg(a.redo + u) == 0) return;   // the single pass was valid
+  if (a.gram_mode == 2 && __ldg(a.redo + u * a.nrb + a.rb) == 0) return;   // the single pass was valid
   const bool single = a.gram_mode == 1;
   const int k0 = single ? T : 0;   // first job
   const int ng = __ldg(a.ng + u);
@@ -407,8 +421,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tensormap(&tmQ);
       mbar_expect_tx(&bars->q_full, kTileBytes);
       const uint64_t pol = l2_evict_last();
-      tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, 0, u, pol);
-      tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
+      tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, a.row0, u, pol);
+      tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, a.row0, u, pol);
     }
     __syncwarp();
     // the gathers: warps 0, 2 and 3 (three SM sub-partitions)
@@ -503,14 +517,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= 4) {
     const int wg = (warp - 4) >> 2, q = warp & 3, row = q * 32 + lane;
-    const bool row_ok = row < a.m;
+    const int grow = a.row0 + row;   // window row of the stacked m
+    const bool row_ok = grow < a.m;
     // slots / positions past vlim are invisible to this row (and so are those >= B)
-    const int vlim = !row_ok ? -1 : (a.causal ? B - a.w + row % a.w : B - 1);
+    const int vlim = !row_ok ? -1 : (a.causal ? B - a.w + grow % a.w : B - 1);
     const int open = B - a.w;   // below this everything is visible to every window row
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
     float M = -INFINITY, L = 0.f, lam = INFINITY;
     float vmax = -INFINITY, xsum = 0.f;   // visible retained logits (raw) and sum of X
-    if (single && row_ok) lam = __ldg(a.rstats + ((size_t)u * a.m + row) * 2) * 1.4426950408889634f;
+    if (single && row_ok) lam = __ldg(a.rstats + ((size_t)u * a.m + grow) * 2) * 1.4426950408889634f;
     bool ok = true;
     for (int k = k0; k < 2 * T; ++k) {
       if (k == T && !single) {
@@ -530,7 +545,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         lam = (row_ok && L > 0.f) ? M + __log2f(L) : INFINITY;
-        if (wg == 0) a.lam[(size_t)u * kRows + row] = lam;
+        if (wg == 0) a.lam[(size_t)u * a.ldr + grow] = lam;
       }
       if (!ok) {
         if (k < T) continue;
@@ -638,16 +653,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       ci = (row_ok && lsum > 0.f) ? 1.f / lsum : 0.f;
       if (wg == 0) {
         cs[row] = ci;
-        a.lam[(size_t)u * kRows + row] = (row_ok && lsum > 0.f) ? lam + __log2f(lsum) : INFINITY;
+        a.lam[(size_t)u * a.ldr + grow] = (row_ok && lsum > 0.f) ? lam + __log2f(lsum) : INFINITY;
       }
       named_bar(4, 256);
-      if (tid == 128) a.redo[u] = bars->bad;
+      if (tid == 128) a.redo[u * a.nrb + a.rb] = bars->bad;
       if (bars->bad) ok = false;   // gram_mode 2 redoes this unit; not a failure
     }
     if (ok) {
-      float* R = a.rz + ((size_t)u * kRows + row) * kD;
-      float* G = a.gram + ((size_t)u * kRows + row) * kRows;
-      const float* yr = a.y + ((size_t)u * a.m + (row_ok ? row : 0)) * kD;
+      float* R = a.rz + ((size_t)u * a.ldr + grow) * kD;
+      float* G = a.gram + ((size_t)u * a.ldr + grow) * a.ldr + a.row0;   // the diagonal block
+      const float* yr = a.y + ((size_t)u * a.m + (row_ok ? grow : 0)) * kD;
 #pragma unroll 1
       for (int c = 2 * wg; c < 2 * wg + 2; ++c) {
         float v[32];
@@ -979,20 +994,217 @@ __global__ void __launch_bounds__(kSolveThreads, 2) k_merge_solve(MArgs a) {
   }
 }
 
+// ======================================================== k_merge_cross
+// The off-diagonal Gram block of a unit with two row blocks (128 < m <= 256):
+// G01 = X_G0 X_G1^T over the non-fixed positions, as the split products
+// Xh0 Xh1^T + Xl0 Xh1^T + Xh0 Xl1^T (the low-low term dropped, as in the
+// diagonal blocks).  X uses the final row normalisers of both blocks (from
+// the diagonal launches), so nothing is rescaled afterwards.  G01 goes to
+// gram[u][r0][128 + r1] and, transposed, to gram[u][128 + r1][r0].  Roles
+// (384 threads): warp 0 the Q loads; warps 0, 2, 3 the K0 gathers; warp 1 MMA
+// issue; warps 4-7 the rows of block 0 (X_0 high / low parts written back
+// over S_0 in TMEM, the A operands); warps 8-11 the rows of block 1 (XGh_1,
+// XGl_1 in shared memory, the B operands).  One tile in flight: the S MMAs of
+// a tile are issued after the Gram MMAs of the previous one, so s_full also
+// tells both groups that their buffers are free.
+struct CBars {
+  uint64_t ring_full[2], ring_empty[2];
+  uint64_t q_full, s_full, x0_full, x1_full, acc_done, drain;
+  uint32_t tmem;
+  int abort;
+};
+static_assert(sizeof(CBars) <= 256, "barrier block");
+constexpr uint32_t kOffQ1C = kTileBytes, kOffRingC = 2 * kTileBytes, kOffXhC = 4 * kTileBytes,
+                   kOffXlC = 5 * kTileBytes, kOffBarC = 6 * kTileBytes;
+constexpr uint32_t kSmemBytesC = kOffBarC + 256 + 1024;
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_merge_cross(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                  MArgs a) {
+  extern __shared__ __align__(1024) uint8_t smraw[];
+  uint8_t* sm = (uint8_t*)(((uintptr_t)smraw + 1023) & ~(uintptr_t)1023);
+  CBars* bars = (CBars*)(sm + kOffBarC);
+  uint8_t* xgh = sm + kOffXhC;
+  uint8_t* xgl = sm + kOffXlC;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int u = blockIdx.x, B = a.B;
+  const int ng = __ldg(a.ng + u), TG = (ng + kTile - 1) / kTile;
+  if (tid == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bars->ring_full[i], 3);   // one expect_tx arrival per gathering warp
+      mbar_init(&bars->ring_empty[i], 1);
+    }
+    mbar_init(&bars->q_full, 1);
+    mbar_init(&bars->s_full, 1);
+    mbar_init(&bars->x0_full, 128);
+    mbar_init(&bars->x1_full, 128);
+    mbar_init(&bars->acc_done, 1);
+    mbar_init(&bars->drain, 1);
+    bars->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&bars->tmem, 512);
+    tmem_relinquish();
+  }
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bars->tmem;
+  volatile int* abort_flag = &bars->abort;
+  constexpr uint32_t kColS0 = 0, kColS1 = 128, kColGC = 256;
+
+  if (warp == 0 || warp == 2 || warp == 3) {
+    if (warp == 0 && lane == 0) {
+      prefetch_tensormap(&tmQ);
+      mbar_expect_tx(&bars->q_full, 2 * kTileBytes);
+      const uint64_t pol = l2_evict_last();
+      for (int h = 0; h < 2; ++h) {
+        tma_load_3d(sm + h * kTileBytes, &tmQ, &bars->q_full, 0, h * kRows, u, pol);
+        tma_load_3d(sm + h * kTileBytes + kTileBytes / 2, &tmQ, &bars->q_full, 64, h * kRows, u, pol);
+      }
+    }
+    __syncwarp();
+    const int32_t* src_u = a.src + (size_t)u * B;
+    const int pw = warp == 0 ? 0 : warp - 1;
+    Gatherer<2, 3> gt{sm + kOffRingC, bars->ring_full, bars->ring_empty};
+    int jn[4];
+    if (TG > 0) gt.rows(src_u, B, a.n, u * a.n, 0, pw, lane, jn);
+    bool ok = true;
+    for (int t = 0; t < TG && ok; ++t) {
+      const int j[4] = {jn[0], jn[1], jn[2], jn[3]};
+      if (t + 1 < TG) gt.rows(src_u, B, a.n, u * a.n, t + 1, pw, lane, jn);
+      ok = gt.load(&tmK, j, pw, lane, abort_flag);
+    }
+    gt.drain(abort_flag);
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t id_g = idesc_bf16(kRows, kRows, 0, 0);   // G01 += A XG1^T
+      bool ok = mbar_wait(&bars->q_full, 0, abort_flag, kBudget);
+      const uint32_t qa0 = smem_u32(sm), qa1 = smem_u32(sm + kOffQ1C);
+      const uint32_t ha = smem_u32(xgh), la = smem_u32(xgl);
+      for (int t = 0; t < TG && ok; ++t) {
+        ok = mbar_wait(&bars->ring_full[t & 1], (t >> 1) & 1, abort_flag, kBudget);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t ka = smem_u32(sm + kOffRingC + (t & 1) * kTileBytes);
+        issue_s(tmem + kColS0, qa0, ka);
+        issue_s(tmem + kColS1, qa1, ka);
+        mma_commit(&bars->ring_empty[t & 1]);
+        mma_commit(&bars->s_full);
+        ok = mbar_wait(&bars->x0_full, t & 1, abort_flag, kBudget);
+        if (ok) ok = mbar_wait(&bars->x1_full, t & 1, abort_flag, kBudget);
+        if (!ok) break;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < kTile / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
+          mma_bf16_ts(tmem + kColGC, tmem + kColS0 + xt_col(kk, 0), sw128_desc(ha + off, 16, 1024),
+                      id_g, (t > 0 || kk > 0));
+        }
+#pragma unroll
+        for (int kk = 0; kk < kTile / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
+          mma_bf16_ts(tmem + kColGC, tmem + kColS0 + xt_col(kk, 1), sw128_desc(ha + off, 16, 1024),
+                      id_g, 1);
+        }
+#pragma unroll
+        for (int kk = 0; kk < kTile / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * (kTileBytes / 2) + (kk & 3) * 32;
+          mma_bf16_ts(tmem + kColGC, tmem + kColS0 + xt_col(kk, 0), sw128_desc(la + off, 16, 1024),
+                      id_g, 1);
+        }
+      }
+      mma_commit(&bars->acc_done);
+      mma_commit(&bars->drain);
+      mbar_wait(&bars->drain, 0, abort_flag, kBudget);
+    }
+  } else {
+    const int grp = (warp - 4) >> 2, q = warp & 3, row = q * 32 + lane;
+    const int grow = grp * kRows + row;
+    const float lam = grow < a.m ? a.lam[(size_t)u * a.ldr + grow] : INFINITY;
+    const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
+    const uint32_t sbase = lane_addr + (grp ? kColS1 : kColS0);
+    bool ok = true;
+    for (int t = 0; t < TG && ok; ++t) {
+      ok = mbar_wait_warp(&bars->s_full, t & 1, abort_flag);
+      if (!ok) break;
+      tc_fence_after();
+      float v[32];
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        tmem_ld32f(sbase + 32 * c, v);
+        tmem_wait32(v);
+        uint32_t hi[16], lo[16];
+        const int p0 = t * kTile + 32 * c;
+#pragma unroll
+        for (int e = 0; e < 32; e += 2) {
+          const float x0 = p0 + e < ng ? fast_exp2(fmaf(v[e], a.sl2, -lam)) : 0.f;
+          const float x1 = p0 + e + 1 < ng ? fast_exp2(fmaf(v[e + 1], a.sl2, -lam)) : 0.f;
+          const uint32_t h = pack_bf16(x0, x1);
+          hi[e / 2] = h;
+          lo[e / 2] = pack_bf16(x0 - lo_half(h), x1 - hi_half(h));
+        }
+        if (grp == 0) {
+          tmem_st16(sbase + 32 * c, hi);
+          tmem_st16(sbase + 32 * c + 16, lo);
+        } else {
+          store_row_chunk(xgh, row, c, hi);
+          store_row_chunk(xgl, row, c, lo);
+        }
+      }
+      if (grp == 0) {
+        tmem_st_wait();
+      } else {
+        fence_proxy_async_smem();
+      }
+      tc_fence_before();
+      mbar_arrive(grp == 0 ? &bars->x0_full : &bars->x1_full);
+    }
+    if (grp == 0) {
+      if (ok) ok = mbar_wait_warp(&bars->acc_done, 0, abort_flag);
+      tc_fence_after();
+      if (ok) {
+        float* up = a.gram + ((size_t)u * a.ldr + row) * a.ldr + kRows;   // row r0, columns 128 + r1
+        float* lo = a.gram + ((size_t)u * a.ldr + kRows) * a.ldr + row;    // rows 128 + r1, column r0
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          float g[32];
+          tmem_ld32f(lane_addr + kColGC + 32 * c, g);
+          tmem_wait32(g);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            const float x = TG > 0 ? g[e] : 0.f;
+            up[32 * c + e] = x;
+            lo[(size_t)(32 * c + e) * a.ldr] = x;
+          }
+        }
+      }
+    }
+    if (!ok && row == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
 // ======================================================== k_solve_dense
-// The regression solve of the portable merge (m <= 256): N = X_G X_G^T +
-// lambda I (full symmetric, lambda included, [m][m]) and R ([m][128]) from
-// the workspace, Z = N^-1 R written over R.  The same blocked fp32 algorithm
-// as k_merge_solve, for up to 256 rows: N as a packed lower triangle in
-// shared memory (rows past m are identity), Cholesky in 32-row blocks, the
-// diagonal blocks inverted in place, then block substitution over R in two
-// passes of 64 columns.  One 512-thread CTA per unit.
+// The regression solve for m <= 256: N and R ([m][128]) from the workspace,
+// Z = N^-1 R written over R.  With sym = 0, gram holds N = X_G X_G^T +
+// lambda I (the portable merge); with sym = 1 it holds the raw Gram blocks of
+// the tensor-core merge and N = (G + G^T) / 2 + lambda I.  Each unit's arrays
+// hold ld rows.  The same blocked fp32 algorithm as k_merge_solve, for up to
+// 256 rows: N as a packed lower triangle in shared memory (rows past m are
+// identity), Cholesky in 32-row blocks, the diagonal blocks inverted in place,
+// then block substitution over R in two passes of 64 columns.  lambda = +inf
+// gives Z = 0.  One 512-thread CTA per unit.
 constexpr int kDenseM = 256, kDenseNT = 512, kDenseC = 64, kDenseLD = kDenseC + 1;
 constexpr int kDenseTri = tri(kDenseM) + 4;
 constexpr uint32_t kDenseSmem = (kDenseTri + kDenseM * kDenseLD + kDenseM + 32) * 4;
 
 __global__ void __launch_bounds__(kDenseNT, 1)
-    k_solve_dense(const float* __restrict__ gram, float* __restrict__ rz, int m, int* status) {
+    k_solve_dense(const float* __restrict__ gram, float* __restrict__ rz, int m, int ld, int sym,
+                  float lambda, int lambda_inf, int* status) {
   extern __shared__ __align__(16) float dsm[];
   float* N = dsm;                       // packed lower triangle
   float* R = N + kDenseTri;             // [256][kDenseLD]: one column pass of R, then of Z
@@ -1000,12 +1212,22 @@ __global__ void __launch_bounds__(kDenseNT, 1)
   int* fail = (int*)(dinv + kDenseM);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int u = blockIdx.x;
-  const float* Gu = gram + (size_t)u * m * m;
-  float* RZ = rz + (size_t)u * m * kD;
+  const float* Gu = gram + (size_t)u * ld * ld;
+  float* RZ = rz + (size_t)u * ld * kD;
+  if (lambda_inf) {
+    for (int p = tid; p < m * kD; p += kDenseNT) RZ[p] = 0.f;
+    return;
+  }
   if (tid == 0) *fail = 0;
   for (int i = warp; i < kDenseM; i += kDenseNT / 32)
-    for (int j = lane; j <= i; j += 32)
-      N[tri(i) + j] = (i < m && j < m) ? __ldg(Gu + (size_t)i * m + j) : (i == j ? 1.f : 0.f);
+    for (int j = lane; j <= i; j += 32) {
+      float val = i == j ? 1.f : 0.f;
+      if (i < m && j < m) {
+        val = __ldg(Gu + (size_t)i * ld + j);
+        if (sym) val = 0.5f * (val + __ldg(Gu + (size_t)j * ld + i)) + (i == j ? lambda : 0.f);
+      }
+      N[tri(i) + j] = val;
+    }
   __syncthreads();
   for (int kb = 0; kb < kDenseM / 32; ++kb) {
     const int k0 = kb * 32;
@@ -1153,12 +1375,6 @@ constexpr uint32_t kOffLamU = kOffBar + 256;               // [128] row normalis
 static_assert(kOffZU + 2 * kTileBytes == kOffBar, "update shared-memory layout");
 constexpr uint32_t kSmemBytesU = kOffLamU + kRows * 4 + 1024;
 
-// TMEM column of the packed high (lo = 0) or low (lo = 1) parts of rows
-// 16kk .. 16kk+15 of X_G^T.
-__device__ __forceinline__ uint32_t xt_col(int kk, int lo) {
-  return (kk >> 1) * 32 + lo * 16 + (kk & 1) * 8;
-}
-
 __global__ void __launch_bounds__(kThreadsU, 1)
     k_merge_update(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, const __grid_constant__ CUtensorMap tmKo,
@@ -1194,11 +1410,11 @@ __global__ void __launch_bounds__(kThreadsU, 1)
     tmem_relinquish();
   }
   // rows past m have lam = +inf and give X = 0
-  if (tid < kRows) lam_s[tid] = a.lam[(size_t)u * kRows + tid];
+  if (tid < kRows) lam_s[tid] = a.lam[(size_t)u * a.ldr + a.row0 + tid];
   // Z (fp32 [row][d]) to the bf16 B operands Zh, Zl: MN-major tiles of
   // 128-byte rows (d contiguous), two blocks of 64 columns
   {
-    const float* Z = a.rz + (size_t)u * kRows * kD;
+    const float* Z = a.rz + ((size_t)u * a.ldr + a.row0) * kD;
     for (int i = tid; i < kRows * (kD / 8); i += kThreadsU) {
       const int r = i >> 4, d8 = i & 15;
       const float4 z0 = __ldg((const float4*)(Z + r * kD + d8 * 8));
@@ -1227,19 +1443,21 @@ __global__ void __launch_bounds__(kThreadsU, 1)
       prefetch_tensormap(&tmKo);
       mbar_expect_tx(&bars->q_full, kTileBytes);
       const uint64_t pol = l2_evict_last();
-      tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, 0, u, pol);
-      tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, 0, u, pol);
+      tma_load_3d(sm + kOffQ, &tmQ, &bars->q_full, 0, a.row0, u, pol);
+      tma_load_3d(sm + kOffQ + kTileBytes / 2, &tmQ, &bars->q_full, 64, a.row0, u, pol);
       // K_out = K0 tile by tile (the map clips the rows past B)
       bool ok = true;
       for (int t = 0; t < T && ok; ++t) {
         const int sl = t & 1;
         ok = mbar_wait(&bars->k_full[sl], (t >> 1) & 1, abort_flag, kBudget);
         if (!ok) break;
-        const uint8_t* kt = sm + kOffKU + sl * kTileBytes;
-        tma_store_3d(&tmKo, kt, 0, t * kTile, u);
-        tma_store_3d(&tmKo, kt + kTileBytes / 2, 64, t * kTile, u);
-        bulk_commit();
-        bulk_wait_read<0>();
+        if (a.upd_mode != 2) {   // the second row block's K_out is the first's
+          const uint8_t* kt = sm + kOffKU + sl * kTileBytes;
+          tma_store_3d(&tmKo, kt, 0, t * kTile, u);
+          tma_store_3d(&tmKo, kt + kTileBytes / 2, 64, t * kTile, u);
+          bulk_commit();
+          bulk_wait_read<0>();
+        }
         mbar_arrive(&bars->k_empty[sl]);
       }
       bulk_wait_all();
@@ -1254,11 +1472,13 @@ __global__ void __launch_bounds__(kThreadsU, 1)
         const int sl = t & 1;
         ok = mbar_wait(&bars->vo_full[sl], (t >> 1) & 1, abort_flag, kBudget);
         if (!ok) break;
-        const uint8_t* vt = sm + kOffVU + sl * kTileBytes;
-        tma_store_3d(&tmVo, vt, 0, t * kTile, u);
-        tma_store_3d(&tmVo, vt + kTileBytes / 2, 64, t * kTile, u);
-        bulk_commit();
-        bulk_wait_read<0>();
+        if (a.upd_mode != 1) {   // mode 1 leaves its result in vpart
+          const uint8_t* vt = sm + kOffVU + sl * kTileBytes;
+          tma_store_3d(&tmVo, vt, 0, t * kTile, u);
+          tma_store_3d(&tmVo, vt + kTileBytes / 2, 64, t * kTile, u);
+          bulk_commit();
+          bulk_wait_read<0>();
+        }
         mbar_arrive(&bars->v_empty[sl]);
       }
       bulk_wait_all();
@@ -1269,15 +1489,17 @@ __global__ void __launch_bounds__(kThreadsU, 1)
     // that a K tile never waits for a V slot)
     const bool is_v = warp >= 18;
     const int pw = warp < 4 ? warp - 2 : (is_v ? warp - 18 : warp - 14), row0 = u * a.n;
+    // mode 2 builds V_out from vpart: no V0 tiles
+    const int TG = is_v && a.upd_mode == 2 ? 0 : T;
     Gatherer<2, 4> g{sm + (is_v ? kOffVU : kOffKU), is_v ? bars->v_full : bars->k_full,
                      is_v ? bars->v_empty : bars->k_empty};
     const CUtensorMap* map = is_v ? &tmV : &tmK;
     int jn[4];
-    g.rows(idx_u, B, a.n, row0, 0, pw, lane, jn);
+    if (TG > 0) g.rows(idx_u, B, a.n, row0, 0, pw, lane, jn);
     bool ok = true;
-    for (int t = 0; t < T && ok; ++t) {
+    for (int t = 0; t < TG && ok; ++t) {
       const int j[4] = {jn[0], jn[1], jn[2], jn[3]};
-      if (t + 1 < T) g.rows(idx_u, B, a.n, row0, t + 1, pw, lane, jn);
+      if (t + 1 < TG) g.rows(idx_u, B, a.n, row0, t + 1, pw, lane, jn);
       ok = g.load(map, j, pw, lane, abort_flag);
     }
     g.drain(abort_flag);
@@ -1366,19 +1588,26 @@ __global__ void __launch_bounds__(kThreadsU, 1)
     }
     if (!ok && tok == 0 && cg == 0) set_status(a.status, GRKV_ERR_TIMEOUT);
   } else if (warp >= 12 && warp < 16) {
-    // epilogue: thread = token (TMEM lane of D), V_out = V0 + dV in the V tile
+    // epilogue: thread = token (TMEM lane of D).  Mode 0: V_out = V0 + dV in
+    // the V tile; mode 1: vpart = V0 + dV (fp32, every retained slot); mode 2:
+    // V_out = vpart + dV into the V tile slot (no V0 there)
     const int q = warp & 3, tok = q * 32 + lane;
     const uint32_t lane_addr = tmem + ((uint32_t)(q * 32) << 16);
+    const int mode = a.upd_mode;
     bool ok = true;
     for (int t = 0; t < T && ok; ++t) {
       const int sl = t & 1, slot = t * kTile + tok;
-      const bool live = slot < B && __ldg(a.fixed + (size_t)u * B + min(slot, B - 1)) == 0;
+      const bool in = slot < B;
+      const bool live = in && (mode != 0 || __ldg(a.fixed + (size_t)u * B + min(slot, B - 1)) == 0);
       ok = mbar_wait_warp(&bars->d_full[sl], (t >> 1) & 1, abort_flag);
-      if (ok) ok = mbar_wait_warp(&bars->v_full[sl], (t >> 1) & 1, abort_flag);
+      if (ok && mode != 2) ok = mbar_wait_warp(&bars->v_full[sl], (t >> 1) & 1, abort_flag);
+      if (ok && mode == 2 && t >= 2)
+        ok = mbar_wait_warp(&bars->v_empty[sl], ((t >> 1) - 1) & 1, abort_flag);
       if (!ok) break;
       tc_fence_after();
       uint8_t* vt = sm + kOffVU + sl * kTileBytes;
       const uint32_t dcol = lane_addr + kColD + sl * kD;
+      float* vp = mode != 0 ? a.vpart + ((size_t)u * B + min(slot, B - 1)) * kD : nullptr;
 #pragma unroll 1
       for (int c = 0; c < 4; ++c) {
         float dv[32];
@@ -1394,13 +1623,30 @@ __global__ void __launch_bounds__(kThreadsU, 1)
 #pragma unroll
           for (int h = 0; h < 4; ++h) {
             uint4* p = (uint4*)(row + sw128_offset(tok, (c & 1) * 4 + h));
-            const uint4 v0 = *p;
-            const uint32_t w[4] = {v0.x, v0.y, v0.z, v0.w};
-            uint32_t o[4];
+            float x[8];
+            if (mode == 2) {
+              const float4 p0 = *(const float4*)(vp + 32 * c + 8 * h);
+              const float4 p1 = *(const float4*)(vp + 32 * c + 8 * h + 4);
+              x[0] = p0.x; x[1] = p0.y; x[2] = p0.z; x[3] = p0.w;
+              x[4] = p1.x; x[5] = p1.y; x[6] = p1.z; x[7] = p1.w;
+            } else {
+              const uint4 v0 = *p;
+              const uint32_t w[4] = {v0.x, v0.y, v0.z, v0.w};
 #pragma unroll
-            for (int z = 0; z < 4; ++z)
-              o[z] = pack_bf16(lo_half(w[z]) + dv[8 * h + 2 * z], hi_half(w[z]) + dv[8 * h + 2 * z + 1]);
-            *p = make_uint4(o[0], o[1], o[2], o[3]);
+              for (int z = 0; z < 4; ++z) {
+                x[2 * z] = lo_half(w[z]);
+                x[2 * z + 1] = hi_half(w[z]);
+              }
+            }
+#pragma unroll
+            for (int z = 0; z < 8; ++z) x[z] += dv[8 * h + z];
+            if (mode == 1) {
+              *(float4*)(vp + 32 * c + 8 * h) = make_float4(x[0], x[1], x[2], x[3]);
+              *(float4*)(vp + 32 * c + 8 * h + 4) = make_float4(x[4], x[5], x[6], x[7]);
+            } else {
+              *p = make_uint4(pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]), pack_bf16(x[4], x[5]),
+                              pack_bf16(x[6], x[7]));
+            }
           }
         }
       }
@@ -1418,22 +1664,43 @@ __global__ void __launch_bounds__(kThreadsU, 1)
 }  // namespace
 
 bool merge_tc_supported(const Shape& s) {
-  return s.dtype == GRKV_BF16 && s.m <= kRows && s.B <= kMaxB && s.B >= 1;
+  return s.dtype == GRKV_BF16 && s.m <= 2 * kRows && s.B <= kMaxB && s.B >= 1;
 }
 
-size_t merge_tc_ws_bytes(const Shape& s) {
-  const size_t U = (size_t)s.U;
-  return U * kRows * kD * 4 + U * kRows * kRows * 4 + U * kRows * 4 + U * (size_t)s.B * 4 +
-         2 * U * 4 + ((U * (size_t)s.B + 15) & ~(size_t)15);
+// Workspace of the tensor-core merge: rz [U][ldr][128], gram [U][ldr][ldr],
+// lam [U][ldr] (fp32), src [U][B], ng [U], redo [U][nrb] (int32), fixed [U][B]
+// (bytes), and for two row blocks vpart [U][B][128] (fp32).
+struct MergeWs {
+  int ldr, nrb;
+  size_t rz, gram, lam, src, ng, redo, fixed, vpart, total;
+};
+MergeWs merge_ws(const Shape& s) {
+  MergeWs w;
+  const size_t U = (size_t)s.U, B = (size_t)s.B;
+  w.nrb = s.m > kRows ? 2 : 1;
+  w.ldr = w.nrb * kRows;
+  const size_t ldr = (size_t)w.ldr;
+  w.rz = 0;
+  w.gram = w.rz + U * ldr * kD * 4;
+  w.lam = w.gram + U * ldr * ldr * 4;
+  w.src = w.lam + U * ldr * 4;
+  w.ng = w.src + U * B * 4;
+  w.redo = w.ng + U * 4;
+  w.fixed = w.redo + U * w.nrb * 4;
+  w.vpart = (w.fixed + U * B + 15) & ~(size_t)15;
+  w.total = w.vpart + (w.nrb > 1 ? U * B * kD * 4 : 0);
+  return w;
 }
 
-cudaError_t launch_solve_dense(int U, int m, const float* gram, float* rz, int* status,
-                               cudaStream_t st) {
-  if (m > kDenseM) return cudaErrorInvalidValue;
+size_t merge_tc_ws_bytes(const Shape& s) { return merge_ws(s).total; }
+
+cudaError_t launch_solve_dense(int U, int m, int ld, int sym, float lambda, int lambda_inf,
+                               const float* gram, float* rz, int* status, cudaStream_t st) {
+  if (m > kDenseM || ld < m) return cudaErrorInvalidValue;
   cudaError_t e = cudaFuncSetAttribute(k_solve_dense, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        kDenseSmem);
   if (e != cudaSuccess) return e;
-  k_solve_dense<<<U, kDenseNT, kDenseSmem, st>>>(gram, rz, m, status);
+  k_solve_dense<<<U, kDenseNT, kDenseSmem, st>>>(gram, rz, m, ld, sym, lambda, lambda_inf, status);
   count_launches(1);
   return cudaGetLastError();
 }
@@ -1470,14 +1737,18 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
   a.k_out = (__nv_bfloat16*)k_out;
   a.v_out = (__nv_bfloat16*)v_out;
   a.rstats = row_stats;
-  const size_t U = (size_t)s.U;
-  a.rz = (float*)(ws + L.merge_tc);
-  a.gram = a.rz + U * kRows * kD;
-  a.lam = a.gram + U * kRows * kRows;
-  a.src = (int32_t*)(a.lam + U * kRows);
-  a.ng = a.src + U * s.B;
-  a.redo = a.ng + U;
-  a.fixed = (uint8_t*)(a.redo + U);
+  const MergeWs W = merge_ws(s);
+  char* mw = ws + L.merge_tc;
+  a.rz = (float*)(mw + W.rz);
+  a.gram = (float*)(mw + W.gram);
+  a.lam = (float*)(mw + W.lam);
+  a.src = (int32_t*)(mw + W.src);
+  a.ng = (int32_t*)(mw + W.ng);
+  a.redo = (int32_t*)(mw + W.redo);
+  a.fixed = (uint8_t*)(mw + W.fixed);
+  a.vpart = W.nrb > 1 ? (float*)(mw + W.vpart) : nullptr;
+  a.ldr = W.ldr;
+  a.nrb = W.nrb;
   a.status = (int*)(ws + L.status);
   cudaError_t e;
   if ((e = cudaFuncSetAttribute(k_merge_gram, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1489,19 +1760,54 @@ cudaError_t launch_merge_tc(const Shape& s, const void* q, const void* k, const 
       (e = cudaFuncSetAttribute(k_merge_fixed, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 s.B * 4)) != cudaSuccess)
     return e;
+  if (W.nrb > 1 && (e = cudaFuncSetAttribute(k_merge_cross, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kSmemBytesC)) != cudaSuccess)
+    return e;
   k_merge_fixed<<<s.U, 256, s.B * 4, st>>>(a);
-  if (row_stats) {
-    a.gram_mode = 1;
-    k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, a);
-    a.gram_mode = 2;
-    k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, a);
-  } else {
-    a.gram_mode = 0;
-    k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, a);
+  int launches = 1;
+  // the retained statistics, R and the diagonal Gram block of every row block
+  for (int rb = 0; rb < W.nrb; ++rb) {
+    a.rb = rb;
+    a.row0 = rb * kRows;
+    if (row_stats) {
+      a.gram_mode = 1;
+      k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, a);
+      a.gram_mode = 2;
+      k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, a);
+      launches += 2;
+    } else {
+      a.gram_mode = 0;
+      k_merge_gram<<<s.U, kThreads, kSmemBytes, st>>>(mq, mk, mv, a);
+      launches += 1;
+    }
   }
-  k_merge_solve<<<s.U, kSolveThreads, kSolveSmem, st>>>(a);
-  k_merge_update<<<s.U, kThreadsU, kSmemBytesU, st>>>(mq, mk, mv, mko, mvo, a);
-  count_launches(row_stats ? 5 : 4);
+  if (W.nrb == 1) {
+    a.rb = 0;
+    a.row0 = 0;
+    a.upd_mode = 0;
+    k_merge_solve<<<s.U, kSolveThreads, kSolveSmem, st>>>(a);
+    k_merge_update<<<s.U, kThreadsU, kSmemBytesU, st>>>(mq, mk, mv, mko, mvo, a);
+    launches += 2;
+  } else {
+    // two row blocks: the cross Gram block, the 256-row solve, and the value
+    // update of each row block (the first leaves V0 + dV_0 in vpart)
+    k_merge_cross<<<s.U, kThreads, kSmemBytesC, st>>>(mq, mk, a);
+    launches += 1;
+    count_launches(launches);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if ((e = launch_solve_dense(s.U, s.m, W.ldr, 1, s.lambda, s.lambda_inf, a.gram, a.rz,
+                                a.status, st)) != cudaSuccess)
+      return e;
+    launches = 0;
+    for (int rb = 0; rb < 2; ++rb) {
+      a.rb = rb;
+      a.row0 = rb * kRows;
+      a.upd_mode = rb == 0 ? 1 : 2;
+      k_merge_update<<<s.U, kThreadsU, kSmemBytesU, st>>>(mq, mk, mv, mko, mvo, a);
+      launches += 1;
+    }
+  }
+  count_launches(launches);
   return cudaGetLastError();
 }
 

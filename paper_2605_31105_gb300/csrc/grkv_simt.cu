@@ -719,8 +719,8 @@ cudaError_t merge_impl(const Shape& s, const T* q, const T* k, const T* v, const
   if (!std::is_same<A, float>::value) return run(0);
   if ((e = run(1)) != cudaSuccess) return e;
   if (!s.lambda_inf &&
-      (e = launch_solve_dense(s.U, s.m, (const float*)(ws + L.gram), (float*)(ws + L.rz),
-                              (int*)(ws + L.status), st)) != cudaSuccess)
+      (e = launch_solve_dense(s.U, s.m, s.m, 0, 0.f, 0, (const float*)(ws + L.gram),
+                              (float*)(ws + L.rz), (int*)(ws + L.status), st)) != cudaSuccess)
     return e;
   return run(2);
 }
