@@ -80,11 +80,27 @@ struct GemmSmem {
 
 // C(i, j) = sum_k a(i, k) b(k, j) for i < M, j < N; store(i, j, value).
 // 64 x 64 output tiles, 16-deep k slabs in shared memory, 4 x 4 per thread.
-template <class FA, class FB, class FS>
+// The next slab is fetched into registers while the current one is used.
+// Each thread fetches four elements of each operand; kAIFast / kBKFast pick
+// the index that runs fastest across threads (i for A, k for B), so that the
+// loads are coalesced for operands stored with that index contiguous.
+template <bool kAIFast = false, bool kBKFast = false, class FA, class FB, class FS>
 __device__ void block_gemm(GemmSmem& g, int M, int N, int K, FA a, FB b, FS store) {
+  constexpr int kAL = kTM * kTK / kKT, kBL = kTN * kTK / kKT;
+  static_assert(kAL * kKT == kTM * kTK && kBL * kKT == kTN * kTK, "slab split");
   auto& As = g.As;
   auto& Bs = g.Bs;
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  auto a_at = [&](int l, int& ii, int& kk) {
+    const int e = threadIdx.x + l * kKT;
+    ii = kAIFast ? e % kTM : e / kTK;
+    kk = kAIFast ? e / kTM : e % kTK;
+  };
+  auto b_at = [&](int l, int& jj, int& kk) {
+    const int e = threadIdx.x + l * kKT;
+    jj = kBKFast ? e / kTK : e % kTN;
+    kk = kBKFast ? e % kTK : e / kTN;
+  };
   for (int i0 = 0; i0 < M; i0 += kTM)
     for (int j0 = 0; j0 < N; j0 += kTN) {
       float acc[4][4];
@@ -92,16 +108,37 @@ __device__ void block_gemm(GemmSmem& g, int M, int N, int K, FA a, FB b, FS stor
       for (int t = 0; t < 4; ++t)
 #pragma unroll
         for (int u = 0; u < 4; ++u) acc[t][u] = 0.f;
-      for (int k0 = 0; k0 < K; k0 += kTK) {
-        for (int e = threadIdx.x; e < kTM * kTK; e += kKT) {
-          const int ii = e / kTK, kk = e % kTK;
-          As[kk][ii] = (i0 + ii < M && k0 + kk < K) ? a(i0 + ii, k0 + kk) : 0.f;
+      float ra[kAL], rb[kBL];
+      auto fetch = [&](int k0) {
+#pragma unroll
+        for (int l = 0; l < kAL; ++l) {
+          int ii, kk;
+          a_at(l, ii, kk);
+          ra[l] = (i0 + ii < M && k0 + kk < K) ? a(i0 + ii, k0 + kk) : 0.f;
         }
-        for (int e = threadIdx.x; e < kTN * kTK; e += kKT) {
-          const int jj = e % kTN, kk = e / kTN;
-          Bs[kk][jj] = (j0 + jj < N && k0 + kk < K) ? b(k0 + kk, j0 + jj) : 0.f;
+#pragma unroll
+        for (int l = 0; l < kBL; ++l) {
+          int jj, kk;
+          b_at(l, jj, kk);
+          rb[l] = (j0 + jj < N && k0 + kk < K) ? b(k0 + kk, j0 + jj) : 0.f;
+        }
+      };
+      fetch(0);
+      for (int k0 = 0; k0 < K; k0 += kTK) {
+#pragma unroll
+        for (int l = 0; l < kAL; ++l) {
+          int ii, kk;
+          a_at(l, ii, kk);
+          As[kk][ii] = ra[l];
+        }
+#pragma unroll
+        for (int l = 0; l < kBL; ++l) {
+          int jj, kk;
+          b_at(l, jj, kk);
+          Bs[kk][jj] = rb[l];
         }
         __syncthreads();
+        if (k0 + kTK < K) fetch(k0 + kTK);
 #pragma unroll
         for (int kk = 0; kk < kTK; ++kk) {
           // rows of 68 floats keep every 4-float group 16-byte aligned
@@ -220,7 +257,7 @@ template <class FK>
 __device__ void retained_softmax(const KArgs& a, const KUnit& k, GemmSmem& gs, FK kget) {
   const int m = k.m, B = k.B, dt = a.dtype;
   const float s = a.scale;
-  block_gemm(gs,
+  block_gemm<false, true>(gs,
       m, B, kD, [&](int r, int t) { return ldv(k.q, (size_t)r * kD + t, dt); },
       [&](int t, int j) { return kget(j, t); },
       [&](int r, int j, float v) { k.X[(size_t)r * B + j] = s * v; });
@@ -252,12 +289,12 @@ template <class FV>
 __device__ void key_vjp(const KArgs& a, const KUnit& k, GemmSmem& gs, const float* W, FV vget) {
   const int m = k.m, B = k.B, dt = a.dtype;
   const float s = a.scale;
-  block_gemm(gs,
+  block_gemm<false, true>(gs,
       m, B, kD, [&](int r, int t) { return W[(size_t)r * kD + t]; },
       [&](int t, int j) { return vget(j, t); },
       [&](int r, int j, float v) { k.T[(size_t)r * B + j] = v; });
   softmax_jacobian_rows(k.X, k.T, m, B);
-  block_gemm(gs,
+  block_gemm<true, false>(gs,
       B, kD, m, [&](int j, int r) { return k.T[(size_t)r * B + j]; },
       [&](int r, int t) { return ldv(k.q, (size_t)r * kD + t, dt); },
       [&](int j, int t, float v) { k.dK[(size_t)j * kD + t] = k.fixed[j] ? 0.f : s * v; });
@@ -270,7 +307,7 @@ template <class FV>
 __device__ void key_cg(const KArgs& a, const KUnit& k, GemmSmem& gs, float* red, FV vget) {
   const int m = k.m, B = k.B, dt = a.dtype, md = m * kD;
   const float s = a.scale;
-  block_gemm(gs,
+  block_gemm<false, true>(gs,
       m, m, kD, [&](int r, int t) { return ldv(k.q, (size_t)r * kD + t, dt); },
       [&](int t, int r2) { return ldv(k.q, (size_t)r2 * kD + t, dt); },
       [&](int r, int r2, float v) { k.GQ[(size_t)r * m + r2] = s * s * v; });
@@ -287,7 +324,7 @@ __device__ void key_cg(const KArgs& a, const KUnit& k, GemmSmem& gs, float* red,
     // Ap = J_G (J_G^T p) + lambda p without forming dK: with dS = X o (dA -
     // rowsum(X o dA)), dA = p V^T, the JVP of dK = s dS^T Q (free rows) is
     // s Q dK^T = (s^2 Q Q^T) dS on the free columns and 0 on the fixed ones.
-    block_gemm(gs,
+    block_gemm<false, true>(gs,
         m, B, kD, [&](int r, int t) { return k.Pd[(size_t)r * kD + t]; },
         [&](int t, int j) { return vget(j, t); },
         [&](int r, int j, float v) { k.T[(size_t)r * B + j] = v; });
@@ -408,7 +445,7 @@ __global__ void __launch_bounds__(kKT) k_alternate_step(KArgs a) {
   float* Z = a.RZ + (size_t)k.u * m * kD;
   bool solved = false;
   if (!a.lambda_inf) {
-    block_gemm(gs,
+    block_gemm<false, true>(gs,
         m, m, B, [&](int r, int j) { return k.fixed[j] ? 0.f : k.X[(size_t)r * B + j]; },
         [&](int j, int r2) { return k.fixed[j] ? 0.f : k.X[(size_t)r2 * B + j]; },
         [&](int r, int r2, float v) { G[(size_t)r * m + r2] = v + (r == r2 ? a.lambda_v : 0.f); });
@@ -442,7 +479,7 @@ __global__ void __launch_bounds__(kKT) k_alternate_step(KArgs a) {
   }
   // V^(t+1) (fp32 in dK as scratch), its largest change, then v_out / Vt
   if (solved) {
-    block_gemm(gs,
+    block_gemm<true, false>(gs,
         B, kD, m, [&](int j, int r) { return k.fixed[j] ? 0.f : k.X[(size_t)r * B + j]; },
         [&](int r, int t) { return Z[(size_t)r * kD + t]; },
         [&](int j, int t, float v) { k.dK[(size_t)j * kD + t] = v0(j, t) + v; });
@@ -471,7 +508,7 @@ __global__ void __launch_bounds__(kKT) k_alternate_step(KArgs a) {
   block_gemm(gs,
       m, kD, B, [&](int r, int j) { return k.X[(size_t)r * B + j]; }, vget,
       [&](int r, int t, float v) { k.R[(size_t)r * kD + t] = k.Y[(size_t)r * kD + t] - v; });
-  block_gemm(gs,
+  block_gemm<false, true>(gs,
       m, B, kD, [&](int r, int t) { return ldv(k.q, (size_t)r * kD + t, dt); },
       [&](int t, int j) {
         return k.fixed[j] ? 0.f : a.Kt[k.kv_off + (size_t)j * kD + t] - k0(j, t);
