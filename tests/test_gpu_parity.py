@@ -20,6 +20,9 @@ pytestmark = pytest.mark.gpu
 
 RAGGED = gi.Workload("ragged_g3_w5_n1000", 3, 3, 1000, 128, 5, 77, 5, 1e-2, "bf16", "lowrank", 777)
 M256 = gi.Workload("m256_spans_n8192", 2, 4, 8192, 128, 64, 512, 7, 1e-1, "bf16", "spans", 888)
+# 128 < m < 256: the second 128-row block of the tensor-core merge is partly padding
+M160 = gi.Workload("m160_lowrank_n3000", 2, 4, 3000, 128, 40, 300, 7, 1e-1, "bf16", "lowrank", 161)
+M200 = gi.Workload("m200_spans_n2500", 2, 5, 2500, 128, 40, 333, 7, 1e-1, "bf16", "spans", 202)
 
 CASES = {
     "c0_full": (gi.workload(0), {}),
@@ -28,6 +31,8 @@ CASES = {
     "ragged_noncausal_avgpool": (RAGGED, dict(causal=False, pool_type="avg")),
     "ragged_f32": (RAGGED.replace(dtype="f32"), {}),
     "m256_spans": (M256, {}),
+    "m160_ragged": (M160, {}),
+    "m200_noncausal": (M200, dict(causal=False)),
     "c2_recipe_n8192": (gi.workload(2).replace(units=3, n=8192, budget=1024), {}),
     "g1_w1": (RAGGED.replace(group=1, window=1, budget=40, seed=5), dict(n_sink=0, beta=0.0)),
 }
