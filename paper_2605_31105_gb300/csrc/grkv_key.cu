@@ -31,12 +31,16 @@
 
 #include "block_select.cuh"
 #include "grkv_internal.cuh"
+#include "sm100.cuh"
 
 namespace grkv {
 namespace {
 
+using namespace sm100;
+
 constexpr int kKT = 256;                  // threads per CTA
 constexpr int kTM = 64, kTN = 64, kTK = 16;
+constexpr long long kWaitBudget = 1ll << 32;   // clock cycles of a bounded wait
 
 struct KArgs {
   int n, w, m, B, P, n_sink, n_fix, causal, dtype, iters;
@@ -44,6 +48,7 @@ struct KArgs {
   float lambda_v, step_tol;
   int lambda_inf;
   int vt_valid;           // Vt holds V^(t) (false at t = 1: V^(1) is only in v_out)
+  int use_tc;             // m <= 128: the CG products run on the tensor cores
   const void* k;          // [U][n][d]  full caches (K0, V0 gathers of steps t >= 1)
   const void* v;
   float* Kt;              // [U][B][d]  fp32 K^(t) of the alternation, or null
@@ -161,6 +166,165 @@ __device__ void block_gemm(GemmSmem& g, int M, int N, int K, FA a, FB b, FS stor
         }
     }
   __syncthreads();
+}
+
+// ----------------------------------------------------- tensor-core products
+// The CG products on tcgen05.  An fp32 operand is split into three bf16 parts
+// x = h + m + l (h = bf16(x), m = bf16(x - h), l = bf16(x - h - m)); keeping
+// the six part products of combined order <= 2 (h.h, h.m, m.h, h.l, m.m, l.h)
+// reproduces the fp32 product to about 2^-24 of its terms, so CG sees fp32
+// products.  An operand exact in bf16 (V* of a bf16 cache) takes one part and
+// three products.  One 128 x 128 output tile at a time: 64-deep slabs of A
+// (K-major) and B (K-major or MN-major) staged by all threads into
+// 128-byte-swizzled shared memory, the MMAs issued by one thread into a
+// 128-column TMEM accumulator, then the tile staged through shared memory so
+// that warps write rows with coalesced stores.
+constexpr int kTP = 3;                          // parts of an fp32 operand
+constexpr uint32_t kSlab = 128 * 64 * 2;        // one part of a 128 x 64 bf16 slab
+constexpr uint32_t kTcSmem = 2 * kTP * kSlab + 1024;
+constexpr int kTLD = 129;                       // fp32 row stride of the staged output tile
+static_assert(128 * kTLD * 4 <= 2 * kTP * kSlab, "output tile fits the slabs");
+
+struct TcCtx {
+  uint8_t* sm;        // 1024-byte aligned: A parts, then B parts
+  uint32_t tmem;      // 128 fp32 columns
+  uint64_t* bar;      // MMA completion
+  uint32_t phase;
+  int* status;
+};
+
+__device__ __forceinline__ float bf_lo(uint32_t h) { return __uint_as_float(h << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t h) { return __uint_as_float(h & 0xFFFF0000u); }
+
+// Eight values into their three bf16 parts, four packed pairs each.
+__device__ __forceinline__ void split3(const float* x, uint4* part) {
+  uint32_t p[3][4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float a0 = x[2 * e], a1 = x[2 * e + 1];
+    const uint32_t h = pack_bf16(a0, a1);
+    const float r0 = a0 - bf_lo(h), r1 = a1 - bf_hi(h);
+    const uint32_t mm = pack_bf16(r0, r1);
+    p[0][e] = h;
+    p[1][e] = mm;
+    p[2][e] = pack_bf16(r0 - bf_lo(mm), r1 - bf_hi(mm));
+  }
+#pragma unroll
+  for (int q = 0; q < 3; ++q) part[q] = make_uint4(p[q][0], p[q][1], p[q][2], p[q][3]);
+}
+
+// C = A B for A [M][K] (a(i, k), M <= 128) and B [K][N] (b(k, j)), B staged
+// K-major ([N] rows of K, kBK) or MN-major ([K] rows of N); parts_b = 1 when B
+// is exact in bf16.  For every output element store(i, j, v) returns a value
+// summed per row and handed to rowsum(i, s) once per 128-column tile.  All
+// threads of the CTA call it; loads run in the order of their contiguous index.
+template <bool kBK, class FA, class FB, class FS, class FR>
+__device__ void tc_gemm(TcCtx& c, int M, int N, int K, int parts_b, FA a, FB b, FS store,
+                        FR rowsum) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  uint8_t* As = c.sm;
+  uint8_t* Bs = c.sm + kTP * kSlab;
+  const uint32_t as = smem_u32(As), bs = smem_u32(Bs);
+  const uint32_t idesc = idesc_bf16(128, 128, 0, kBK ? 0 : 1);
+  volatile int no_abort = 0;
+  for (int j0 = 0; j0 < N; j0 += 128) {
+    for (int k0 = 0; k0 < K; k0 += 64) {
+      for (int ch = tid; ch < 128 * 8; ch += kKT) {
+        const int r = ch >> 3, c8 = ch & 7;
+        float x[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const int kk = k0 + c8 * 8 + e;
+          x[e] = (r < M && kk < K) ? a(r, kk) : 0.f;
+        }
+        uint4 pt[3];
+        split3(x, pt);
+        const uint32_t off = sw128_offset(r, c8);
+#pragma unroll
+        for (int q = 0; q < kTP; ++q) *(uint4*)(As + q * kSlab + off) = pt[q];
+      }
+      if (kBK) {
+        for (int ch = tid; ch < 128 * 8; ch += kKT) {
+          const int r = ch >> 3, c8 = ch & 7;
+          float x[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int kk = k0 + c8 * 8 + e;
+            x[e] = (j0 + r < N && kk < K) ? b(kk, j0 + r) : 0.f;
+          }
+          uint4 pt[3];
+          split3(x, pt);
+          const uint32_t off = sw128_offset(r, c8);
+          for (int q = 0; q < parts_b; ++q) *(uint4*)(Bs + q * kSlab + off) = pt[q];
+        }
+      } else {
+        // [64 rows of K][128 of N] as two halves of 64 columns (8 KB each)
+        for (int ch = tid; ch < 64 * 16; ch += kKT) {
+          const int kr = ch >> 4, nc = ch & 15, hf = nc >> 3, c8 = nc & 7;
+          float x[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int jj = j0 + nc * 8 + e;
+            x[e] = (k0 + kr < K && jj < N) ? b(k0 + kr, jj) : 0.f;
+          }
+          uint4 pt[3];
+          split3(x, pt);
+          const uint32_t off = hf * (kSlab / 2) + sw128_offset(kr, c8);
+          for (int q = 0; q < parts_b; ++q) *(uint4*)(Bs + q * kSlab + off) = pt[q];
+        }
+      }
+      fence_proxy_async_smem();
+      __syncthreads();
+      if (tid == 0) {
+        tc_fence_after();
+        bool acc = k0 > 0;
+        for (int pa = 0; pa < kTP; ++pa)
+          for (int pb = 0; pb < parts_b; ++pb) {
+            if (pa + pb > 2) continue;
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk) {
+              const uint64_t ad = sw128_desc(as + pa * kSlab + kk * 32, 16, 1024);
+              const uint64_t bd = kBK ? sw128_desc(bs + pb * kSlab + kk * 32, 16, 1024)
+                                      : sw128_desc(bs + pb * kSlab + kk * 2048, kSlab / 2, 1024);
+              mma_bf16(c.tmem, ad, bd, idesc, acc ? 1u : 0u);
+              acc = true;
+            }
+          }
+        mma_commit(c.bar);
+      }
+      if (!mbar_wait(c.bar, c.phase, &no_abort, kWaitBudget) && tid == 0)
+        set_status(c.status, GRKV_ERR_TIMEOUT);
+      c.phase ^= 1;
+      tc_fence_after();
+    }
+    // the tile through shared memory (the slabs are free: every MMA has completed)
+    float* tile = (float*)c.sm;
+    if (warp < 4) {
+      const uint32_t la = c.tmem + ((uint32_t)(warp * 32) << 16);
+#pragma unroll 1
+      for (int cc = 0; cc < 4; ++cc) {
+        float v[32];
+        tmem_ld32f(la + cc * 32, v);
+        tmem_wait32(v);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) tile[(warp * 32 + lane) * kTLD + cc * 32 + e] = v[e];
+      }
+    }
+    tc_fence_before();
+    __syncthreads();
+    for (int i = warp; i < M; i += kKT / 32) {
+      float sum = 0.f;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int jj = q * 32 + lane, j = j0 + jj;
+        if (j < N) sum += store(i, j, tile[i * kTLD + jj]);
+      }
+#pragma unroll
+      for (int o = 16; o >= 1; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+      if (lane == 0) rowsum(i, sum);
+    }
+    __syncthreads();
+  }
 }
 
 // Sum over the block of one value per thread (all threads return it).
@@ -361,6 +525,110 @@ __device__ void key_cg(const KArgs& a, const KUnit& k, GemmSmem& gs, float* red,
   }
 }
 
+// key_cg with the three products of an iteration on the tensor cores
+// (m <= 128).  The softmax Jacobians are applied as the next product stages
+// its operand: the row sums rho1 = rowsum(X o T) and rho2 = rowsum(X o T2)
+// are taken in the epilogues of the products that write T and T2.
+template <class FV>
+__device__ void key_cg_tc(const KArgs& a, const KUnit& k, GemmSmem& gs, float* red, TcCtx& c,
+                          float* rho1, float* rho2, int parts_v, FV vget) {
+  const int m = k.m, B = k.B, dt = a.dtype, md = m * kD;
+  const float s = a.scale;
+  block_gemm<false, true>(gs,
+      m, m, kD, [&](int r, int t) { return ldv(k.q, (size_t)r * kD + t, dt); },
+      [&](int t, int r2) { return ldv(k.q, (size_t)r2 * kD + t, dt); },
+      [&](int r, int r2, float v) { k.GQ[(size_t)r * m + r2] = s * s * v; });
+  float rs = 0.f;
+  for (int i = threadIdx.x; i < md; i += kKT) {
+    k.Pd[i] = k.R[i];
+    k.AL[i] = 0.f;
+    rs = fmaf(k.R[i], k.R[i], rs);
+  }
+  rs = block_sum(rs, red);
+  const float stop = a.tol * a.tol * rs;
+  auto add1 = [&](int i, float v) { rho1[i] += v; };
+  auto add2 = [&](int i, float v) { rho2[i] += v; };
+  for (int it = 0; it < a.iters; ++it) {
+    if (!(rs > stop) || !(rs > 0.f)) break;
+    if (threadIdx.x < 128) rho1[threadIdx.x] = rho2[threadIdx.x] = 0.f;
+    __syncthreads();
+    // T = P V*^T
+    tc_gemm<true>(c, m, B, kD, parts_v, [&](int r, int t) { return k.Pd[(size_t)r * kD + t]; },
+        [&](int t, int j) { return vget(j, t); },
+        [&](int r, int j, float v) {
+          k.T[(size_t)r * B + j] = v;
+          return k.X[(size_t)r * B + j] * v;
+        }, add1);
+    // T2 = (s^2 Q Q^T) dS on the free columns, dS = X o (T - rho1)
+    tc_gemm<false>(c, m, B, m, kTP, [&](int r, int r2) { return k.GQ[(size_t)r * m + r2]; },
+        [&](int r2, int j) {
+          const size_t o = (size_t)r2 * B + j;
+          return k.X[o] * (k.T[o] - rho1[r2]);
+        },
+        [&](int r, int j, float v) {
+          const float t2 = k.fixed[j] ? 0.f : v;
+          k.T2[(size_t)r * B + j] = t2;
+          return k.X[(size_t)r * B + j] * t2;
+        }, add2);
+    // Ap = dS2 V* + lambda p, dS2 = X o (T2 - rho2)
+    tc_gemm<false>(c, m, kD, B, parts_v,
+        [&](int r, int j) {
+          const size_t o = (size_t)r * B + j;
+          return k.X[o] * (k.T2[o] - rho2[r]);
+        },
+        [&](int j, int t) { return vget(j, t); },
+        [&](int r, int t, float v) {
+          const size_t o = (size_t)r * kD + t;
+          k.AP[o] = v + a.lambda_k * k.Pd[o];
+          return 0.f;
+        }, [](int, float) {});
+    float pap = 0.f;
+    for (int i = threadIdx.x; i < md; i += kKT) pap = fmaf(k.Pd[i], k.AP[i], pap);
+    pap = block_sum(pap, red);
+    if (!(pap > 0.f)) break;   // the direction has vanished
+    const float al = rs / pap;
+    float rn = 0.f;
+    for (int i = threadIdx.x; i < md; i += kKT) {
+      k.AL[i] = fmaf(al, k.Pd[i], k.AL[i]);
+      const float r = fmaf(-al, k.AP[i], k.R[i]);
+      k.R[i] = r;
+      rn = fmaf(r, r, rn);
+    }
+    rn = block_sum(rn, red);
+    const float beta = rn / rs;
+    for (int i = threadIdx.x; i < md; i += kKT) k.Pd[i] = fmaf(beta, k.Pd[i], k.R[i]);
+    rs = rn;
+    __syncthreads();
+  }
+}
+
+// Tensor-core context of a key-step CTA: dynamic shared memory for the
+// slabs, a 128-column TMEM accumulator (allocated by warp 0) and the MMA
+// barrier.  tc_release frees the TMEM once every thread is done with it.
+__device__ void tc_setup(TcCtx& c, uint8_t* dyn, uint32_t* tmem_s, uint64_t* bar, int* status) {
+  c.sm = (uint8_t*)(((uintptr_t)dyn + 1023) & ~(uintptr_t)1023);
+  c.bar = bar;
+  c.phase = 0;
+  c.status = status;
+  if (threadIdx.x == 0) {
+    mbar_init(bar, 1);
+    fence_mbar_init();
+  }
+  if (threadIdx.x < 32) {
+    tmem_alloc(tmem_s, 128);
+    tmem_relinquish();
+  }
+  __syncthreads();
+  tc_fence_after();
+  c.tmem = *tmem_s;
+}
+__device__ void tc_release(const TcCtx& c) {
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (threadIdx.x < 32) tmem_dealloc(c.tmem, 128);
+}
+
 __device__ __forceinline__ void stv(void* p, size_t i, int dtype, float v) {
   if (dtype == GRKV_F32)
     ((float*)p)[i] = v;
@@ -374,8 +642,14 @@ __global__ void __launch_bounds__(kKT) k_key_step(KArgs a) {
   __shared__ int hist[256], sh[64];
   __shared__ float red[kKT / 32];
   __shared__ GemmSmem gs;
+  __shared__ float rho[2][128];
+  __shared__ uint64_t tc_bar;
+  __shared__ uint32_t tc_tmem;
+  extern __shared__ uint8_t tc_dyn[];
   const KUnit k(a, blockIdx.x);
   const int B = k.B, dt = a.dtype;
+  TcCtx tc{};
+  if (a.use_tc) tc_setup(tc, tc_dyn, &tc_tmem, &tc_bar, a.status);
   fixed_set(a, k, hist, sh);
   retained_softmax(a, k, gs, [&](int j, int t) { return ldv(a.k_out, k.kv_off + (size_t)j * kD + t, dt); });
   auto vget = [&](int j, int t) { return ldv(a.v_out, k.kv_off + (size_t)j * kD + t, dt); };
@@ -383,7 +657,12 @@ __global__ void __launch_bounds__(kKT) k_key_step(KArgs a) {
   block_gemm(gs,
       k.m, kD, B, [&](int r, int j) { return k.X[(size_t)r * B + j]; }, vget,
       [&](int r, int t, float v) { k.R[(size_t)r * kD + t] = k.Y[(size_t)r * kD + t] - v; });
-  key_cg(a, k, gs, red, vget);
+  if (a.use_tc) {
+    key_cg_tc(a, k, gs, red, tc, rho[0], rho[1], dt == GRKV_BF16 ? 1 : kTP, vget);
+    tc_release(tc);
+  } else {
+    key_cg(a, k, gs, red, vget);
+  }
   // K*_G = K0_G + J_G^T alpha; fixed rows keep K0
   key_vjp(a, k, gs, k.AL, vget);
   for (int i = threadIdx.x; i < B * kD; i += kKT) {
@@ -601,9 +880,14 @@ cudaError_t launch_key_step(const Shape& s, const void* q, const void* k, const 
     cudaError_t e = cudaMemsetAsync(a.done, 0, U * sizeof(int), st);
     if (e != cudaSuccess) return e;
   }
+  a.use_tc = s.m <= 128;
+  const uint32_t dyn = a.use_tc ? kTcSmem : 0;
+  cudaError_t e = cudaFuncSetAttribute(k_key_step, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)kTcSmem);
+  if (e != cudaSuccess) return e;
   count_launches(1);
-  k_key_step<<<s.U, kKT, 0, st>>>(a);
-  cudaError_t e = cudaGetLastError();
+  k_key_step<<<s.U, kKT, dyn, st>>>(a);
+  e = cudaGetLastError();
   for (int t = 1; t < s.steps && e == cudaSuccess; ++t) {
     a.vt_valid = t > 1;   // V^(1) exists only as written to v_out (rounded)
     count_launches(1);
