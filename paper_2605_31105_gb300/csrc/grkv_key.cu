@@ -196,6 +196,33 @@ struct TcCtx {
 __device__ __forceinline__ float bf_lo(uint32_t h) { return __uint_as_float(h << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t h) { return __uint_as_float(h & 0xFFFF0000u); }
 
+// x[0..8) = p[0..nv), zero past nv: two 16-byte loads when the chunk is whole
+// and aligned, element loads otherwise.
+__device__ __forceinline__ void ld8(const float* p, int nv, float* x) {
+  if (nv == 8 && ((uintptr_t)p & 15) == 0) {
+    const float4 a = *(const float4*)p, b = *(const float4*)(p + 4);
+    x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w;
+    x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+  } else {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) x[e] = e < nv ? p[e] : 0.f;
+  }
+}
+__device__ __forceinline__ void ld8(const __nv_bfloat16* p, int nv, float* x) {
+  if (nv == 8 && ((uintptr_t)p & 15) == 0) {
+    const uint4 a = *(const uint4*)p;
+    const uint32_t w[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      x[2 * e] = bf_lo(w[e]);
+      x[2 * e + 1] = bf_hi(w[e]);
+    }
+  } else {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) x[e] = e < nv ? __bfloat162float(p[e]) : 0.f;
+  }
+}
+
 // Eight values into their three bf16 parts, four packed pairs each.
 __device__ __forceinline__ void split3(const float* x, uint4* part) {
   uint32_t p[3][4];
@@ -213,11 +240,13 @@ __device__ __forceinline__ void split3(const float* x, uint4* part) {
   for (int q = 0; q < 3; ++q) part[q] = make_uint4(p[q][0], p[q][1], p[q][2], p[q][3]);
 }
 
-// C = A B for A [M][K] (a(i, k), M <= 128) and B [K][N] (b(k, j)), B staged
-// K-major ([N] rows of K, kBK) or MN-major ([K] rows of N); parts_b = 1 when B
-// is exact in bf16.  For every output element store(i, j, v) returns a value
-// summed per row and handed to rowsum(i, s) once per 128-column tile.  All
-// threads of the CTA call it; loads run in the order of their contiguous index.
+// C = A B for A [M][K] (M <= 128) and B [K][N], B staged K-major ([N] rows of
+// K, kBK) or MN-major ([K] rows of N); parts_b = 1 when B is exact in bf16.
+// Operands come in chunks of eight along their contiguous index:
+// a8(i, k, nv, x) fills x with A[i][k .. k+nv) (nv <= 8, zeros after), b8(k,
+// j, nv, x) with B[k .. k+nv)[j] (kBK) or B[k][j .. j+nv).  For every output
+// element store(i, j, v) returns a value summed per row and handed to
+// rowsum(i, s) once per 128-column tile.  All threads of the CTA call it.
 template <bool kBK, class FA, class FB, class FS, class FR>
 __device__ void tc_gemm(TcCtx& c, int M, int N, int K, int parts_b, FA a, FB b, FS store,
                         FR rowsum) {
@@ -230,13 +259,9 @@ __device__ void tc_gemm(TcCtx& c, int M, int N, int K, int parts_b, FA a, FB b, 
   for (int j0 = 0; j0 < N; j0 += 128) {
     for (int k0 = 0; k0 < K; k0 += 64) {
       for (int ch = tid; ch < 128 * 8; ch += kKT) {
-        const int r = ch >> 3, c8 = ch & 7;
+        const int r = ch >> 3, c8 = ch & 7, kk = k0 + c8 * 8;
         float x[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const int kk = k0 + c8 * 8 + e;
-          x[e] = (r < M && kk < K) ? a(r, kk) : 0.f;
-        }
+        a(r, kk, r < M ? max(0, min(8, K - kk)) : 0, x);
         uint4 pt[3];
         split3(x, pt);
         const uint32_t off = sw128_offset(r, c8);
@@ -245,13 +270,9 @@ __device__ void tc_gemm(TcCtx& c, int M, int N, int K, int parts_b, FA a, FB b, 
       }
       if (kBK) {
         for (int ch = tid; ch < 128 * 8; ch += kKT) {
-          const int r = ch >> 3, c8 = ch & 7;
+          const int r = ch >> 3, c8 = ch & 7, kk = k0 + c8 * 8;
           float x[8];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const int kk = k0 + c8 * 8 + e;
-            x[e] = (j0 + r < N && kk < K) ? b(kk, j0 + r) : 0.f;
-          }
+          b(kk, j0 + r, j0 + r < N ? max(0, min(8, K - kk)) : 0, x);
           uint4 pt[3];
           split3(x, pt);
           const uint32_t off = sw128_offset(r, c8);
@@ -260,13 +281,9 @@ __device__ void tc_gemm(TcCtx& c, int M, int N, int K, int parts_b, FA a, FB b, 
       } else {
         // [64 rows of K][128 of N] as two halves of 64 columns (8 KB each)
         for (int ch = tid; ch < 64 * 16; ch += kKT) {
-          const int kr = ch >> 4, nc = ch & 15, hf = nc >> 3, c8 = nc & 7;
+          const int kr = ch >> 4, nc = ch & 15, hf = nc >> 3, c8 = nc & 7, jj = j0 + nc * 8;
           float x[8];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const int jj = j0 + nc * 8 + e;
-            x[e] = (k0 + kr < K && jj < N) ? b(k0 + kr, jj) : 0.f;
-          }
+          b(k0 + kr, jj, k0 + kr < K ? max(0, min(8, N - jj)) : 0, x);
           uint4 pt[3];
           split3(x, pt);
           const uint32_t off = hf * (kSlab / 2) + sw128_offset(kr, c8);
@@ -529,9 +546,10 @@ __device__ void key_cg(const KArgs& a, const KUnit& k, GemmSmem& gs, float* red,
 // (m <= 128).  The softmax Jacobians are applied as the next product stages
 // its operand: the row sums rho1 = rowsum(X o T) and rho2 = rowsum(X o T2)
 // are taken in the epilogues of the products that write T and T2.
-template <class FV>
+template <class FV, class FV8>
 __device__ void key_cg_tc(const KArgs& a, const KUnit& k, GemmSmem& gs, float* red, TcCtx& c,
-                          float* rho1, float* rho2, int parts_v, FV vget) {
+                          float* rho1, float* rho2, int parts_v, FV vget, FV8 vget8) {
+  (void)vget;
   const int m = k.m, B = k.B, dt = a.dtype, md = m * kD;
   const float s = a.scale;
   block_gemm<false, true>(gs,
@@ -553,17 +571,24 @@ __device__ void key_cg_tc(const KArgs& a, const KUnit& k, GemmSmem& gs, float* r
     if (threadIdx.x < 128) rho1[threadIdx.x] = rho2[threadIdx.x] = 0.f;
     __syncthreads();
     // T = P V*^T
-    tc_gemm<true>(c, m, B, kD, parts_v, [&](int r, int t) { return k.Pd[(size_t)r * kD + t]; },
-        [&](int t, int j) { return vget(j, t); },
+    tc_gemm<true>(c, m, B, kD, parts_v,
+        [&](int r, int t, int nv, float* x) { ld8(k.Pd + (size_t)r * kD + t, nv, x); },
+        [&](int t, int j, int nv, float* x) { vget8(j, t, nv, x); },
         [&](int r, int j, float v) {
           k.T[(size_t)r * B + j] = v;
           return k.X[(size_t)r * B + j] * v;
         }, add1);
     // T2 = (s^2 Q Q^T) dS on the free columns, dS = X o (T - rho1)
-    tc_gemm<false>(c, m, B, m, kTP, [&](int r, int r2) { return k.GQ[(size_t)r * m + r2]; },
-        [&](int r2, int j) {
+    tc_gemm<false>(c, m, B, m, kTP,
+        [&](int r, int r2, int nv, float* x) { ld8(k.GQ + (size_t)r * m + r2, nv, x); },
+        [&](int r2, int j, int nv, float* x) {
+          float t[8];
           const size_t o = (size_t)r2 * B + j;
-          return k.X[o] * (k.T[o] - rho1[r2]);
+          ld8(k.X + o, nv, x);
+          ld8(k.T + o, nv, t);
+          const float rh = nv > 0 ? rho1[r2] : 0.f;
+#pragma unroll
+          for (int e = 0; e < 8; ++e) x[e] *= t[e] - rh;
         },
         [&](int r, int j, float v) {
           const float t2 = k.fixed[j] ? 0.f : v;
@@ -572,11 +597,16 @@ __device__ void key_cg_tc(const KArgs& a, const KUnit& k, GemmSmem& gs, float* r
         }, add2);
     // Ap = dS2 V* + lambda p, dS2 = X o (T2 - rho2)
     tc_gemm<false>(c, m, kD, B, parts_v,
-        [&](int r, int j) {
+        [&](int r, int j, int nv, float* x) {
+          float t[8];
           const size_t o = (size_t)r * B + j;
-          return k.X[o] * (k.T2[o] - rho2[r]);
+          ld8(k.X + o, nv, x);
+          ld8(k.T2 + o, nv, t);
+          const float rh = nv > 0 ? rho2[r] : 0.f;
+#pragma unroll
+          for (int e = 0; e < 8; ++e) x[e] *= t[e] - rh;
         },
-        [&](int j, int t) { return vget(j, t); },
+        [&](int j, int t, int nv, float* x) { vget8(j, t, nv, x); },
         [&](int r, int t, float v) {
           const size_t o = (size_t)r * kD + t;
           k.AP[o] = v + a.lambda_k * k.Pd[o];
@@ -658,7 +688,15 @@ __global__ void __launch_bounds__(kKT) k_key_step(KArgs a) {
       k.m, kD, B, [&](int r, int j) { return k.X[(size_t)r * B + j]; }, vget,
       [&](int r, int t, float v) { k.R[(size_t)r * kD + t] = k.Y[(size_t)r * kD + t] - v; });
   if (a.use_tc) {
-    key_cg_tc(a, k, gs, red, tc, rho[0], rho[1], dt == GRKV_BF16 ? 1 : kTP, vget);
+    // V* row j, columns t .. t+nv
+    auto vget8 = [&](int j, int t, int nv, float* x) {
+      const size_t o = k.kv_off + (size_t)j * kD + t;
+      if (dt == GRKV_BF16)
+        ld8((const __nv_bfloat16*)a.v_out + o, nv, x);
+      else
+        ld8((const float*)a.v_out + o, nv, x);
+    };
+    key_cg_tc(a, k, gs, red, tc, rho[0], rho[1], dt == GRKV_BF16 ? 1 : kTP, vget, vget8);
     tc_release(tc);
   } else {
     key_cg(a, k, gs, red, vget);
