@@ -1,5 +1,6 @@
-// Key step of Algorithm 1 at t = 0 (Sec. 3.4 "Key step", App. D.2) on CUDA
-// cores in fp32, one CTA per unit.
+// Key step of Algorithm 1 at t = 0 (Sec. 3.4 "Key step", App. D.2), one CTA
+// per unit: fp32 on CUDA cores, with the CG products on the tensor cores
+// (three-part bf16 splits of the fp32 operands) when m <= 128.
 //
 // With the merged values V* of the value step fixed, f(K) = softmax(s Q K^T) V*
 // is linearised at K0 and the local ridge problem is solved in its dual form:
@@ -15,8 +16,9 @@
 // so an iteration is three GEMMs (m x B x d, m x m x B, m x B x d).
 // Conjugate gradients start from alpha = 0 and run at most cg_iters
 // iterations, stopping once ||r|| <= cg_tol ||e|| or the search direction
-// vanishes.  Each product is a small tiled GEMM over the unit's
-// m x B, B x d and m x d matrices, staged in the workspace (L2-resident).
+// vanishes.  Each product is a tiled GEMM over the unit's m x B, B x d and
+// m x d matrices, staged in the workspace; with m <= 128 the three products
+// of a CG iteration run on tcgen05 (tc_gemm).
 //
 // V* is read from v_out as written by the value step (rounded to the input
 // dtype), K0 from k_out (the value step copies K0 there), and the fixed set is
@@ -748,6 +750,10 @@ __global__ void __launch_bounds__(kKT) k_alternate_step(KArgs a) {
   __shared__ float red[kKT / 32];
   __shared__ GemmSmem gs;
   __shared__ int flag;
+  __shared__ float rho[2][128];
+  __shared__ uint64_t tc_bar;
+  __shared__ uint32_t tc_tmem;
+  extern __shared__ uint8_t tc_dyn[];
   const KUnit k(a, blockIdx.x);
   if (a.done[k.u]) return;
   const int m = k.m, B = k.B, dt = a.dtype;
@@ -835,7 +841,17 @@ __global__ void __launch_bounds__(kKT) k_alternate_step(KArgs a) {
   block_gemm(gs,
       m, kD, B, [&](int r, int j) { return k.T[(size_t)r * B + j]; }, vget,
       [&](int r, int t, float v) { k.R[(size_t)r * kD + t] += v; });
-  key_cg(a, k, gs, red, vget);
+  if (a.use_tc) {
+    TcCtx tc{};
+    tc_setup(tc, tc_dyn, &tc_tmem, &tc_bar, a.status);
+    auto vget8 = [&](int j, int t, int nv, float* x) {
+      ld8(a.Vt + k.kv_off + (size_t)j * kD + t, nv, x);
+    };
+    key_cg_tc(a, k, gs, red, tc, rho[0], rho[1], kTP, vget, vget8);
+    tc_release(tc);
+  } else {
+    key_cg(a, k, gs, red, vget);
+  }
   key_vjp(a, k, gs, k.AL, vget);
   float dkmax = 0.f;
   for (int i = threadIdx.x; i < B * kD; i += kKT) {
@@ -922,6 +938,9 @@ cudaError_t launch_key_step(const Shape& s, const void* q, const void* k, const 
   const uint32_t dyn = a.use_tc ? kTcSmem : 0;
   cudaError_t e = cudaFuncSetAttribute(k_key_step, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kTcSmem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_alternate_step, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kTcSmem);
   if (e != cudaSuccess) return e;
   count_launches(1);
   k_key_step<<<s.U, kKT, dyn, st>>>(a);
@@ -929,7 +948,7 @@ cudaError_t launch_key_step(const Shape& s, const void* q, const void* k, const 
   for (int t = 1; t < s.steps && e == cudaSuccess; ++t) {
     a.vt_valid = t > 1;   // V^(1) exists only as written to v_out (rounded)
     count_launches(1);
-    k_alternate_step<<<s.U, kKT, 0, st>>>(a);
+    k_alternate_step<<<s.U, kKT, dyn, st>>>(a);
     e = cudaGetLastError();
   }
   return e;
