@@ -25,7 +25,7 @@ struct Shape {
   int pool_k, pool_type, n_sink, n_fix, causal, dtype;
   float lambda, scale;
   int lambda_inf; // lambda_v == +inf: values stay V0
-  int tc;         // bf16, m <= 128, not forced portable: tensor-core scoring
+  int tc;         // bf16, m <= 256, not forced portable: tensor-core scoring
   int tc_merge;   // ... and B <= 32768: tensor-core value merge
   int one_read;   // tensor-core scoring in one launch that reads K from HBM once
   int deterministic;  // Y summed in a fixed order (GRKV_DETERMINISTIC)
@@ -109,7 +109,7 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
                             float* scores, float* y, float* row_stats, char* ws,
                             const WsLayout& L, int mode, cudaStream_t st);
 
-// Tensor-core value merge (bf16, m <= 128, B <= 32768).
+// Tensor-core value merge (bf16, m <= 256 in 128-row blocks, B <= 32768).
 bool merge_tc_supported(const Shape& s);
 // The regression solve for m <= 256 (grkv_merge_tc.cu): gram [U][ld][ld]
 // (N with lambda when sym = 0; raw Gram blocks, symmetrised with lambda added,

@@ -1,4 +1,4 @@
-// GRKV value step on the tensor cores (bf16, d = 128, m <= 128, B <= 32768).
+// GRKV value step on the tensor cores (bf16, d = 128, m <= 256, B <= 32768).
 //
 // Algorithm 1's value step in dual form (Sec. 3.4, App. D.1) with the fixed
 // tokens of App. D.3, one unit per CTA:
