@@ -265,13 +265,14 @@ __global__ void __launch_bounds__(1024) k_select(const float* __restrict__ score
 }
 
 // Selection with the unit's keys resident in shared memory (n - w <= 32768):
-// one 1024-thread CTA per unit.  The scores are staged once, pooled into
-// order-preserving keys (thread t owns positions t + 1024 e, the keys stay in
-// its registers), the (B - w)-th largest key is found by four 8-bit radix
-// passes over per-warp histograms, and the positions are compacted in order
-// from contiguous segments.  Same result as k_select.  Shared-memory words are
-// padded by one per 32 (index j + j / 32) so both the strided and the
-// segmented accesses are free of bank conflicts.
+// one 1024-thread CTA per unit.  The scores are staged once; thread t owns the
+// 32 contiguous positions 32t .. 32t+31 and pools them into order-preserving
+// keys held in its registers (max pooling of width 7 as a sliding window over
+// the 38 scores around the segment); the (B - w)-th largest key is found by
+// four 8-bit radix passes over per-warp histograms, and the positions are
+// compacted in order from the same segments.  Same result as k_select.
+// Shared-memory words are padded by one per 32 (index j + j / 32) so that
+// both the strided staging and the segment reads are free of bank conflicts.
 constexpr int kSelThreads = 1024, kSelPer = 32, kSelMaxP = kSelThreads * kSelPer;
 
 __host__ __device__ __forceinline__ int sel_pad(int j) { return j + (j >> 5); }
@@ -298,35 +299,48 @@ __global__ void __launch_bounds__(kSelThreads, 1) k_select_smem(const float* __r
   }
   __syncthreads();
   auto cs = [&](int j) { return __uint_as_float(skey[sel_pad(j)]); };
+  const int lo = tid * kSelPer;   // this thread's segment lo .. lo + 31
   uint32_t kr[kSelPer];
+  if (s.pool_type == GRKV_POOL_MAX && h == 3) {
+    // w[i] = score at lo - 3 + i (cells outside [0, P) are ignored: -inf);
+    // the window max over w[e .. e + 6] from pairs and quadruples
+    float w[kSelPer + 6];
 #pragma unroll
-  for (int e = 0; e < kSelPer; ++e) {
-    const int j = tid + e * kSelThreads;
-    kr[e] = 0u;
-    if (j < P) {
-      float pv;
-      if (s.pool_type == GRKV_POOL_MAX) {
-        pv = cs(j);
-        for (int t = 1; t <= h; ++t) {
-          if (j - t >= 0) pv = fmaxf(pv, cs(j - t));
-          if (j + t < P) pv = fmaxf(pv, cs(j + t));
+    for (int i = 0; i < kSelPer + 6; ++i) {
+      const int j = lo - 3 + i;
+      w[i] = (j >= 0 && j < P) ? cs(j) : -INFINITY;
+    }
+    float m2[kSelPer + 5], m4[kSelPer + 3];
+#pragma unroll
+    for (int i = 0; i < kSelPer + 5; ++i) m2[i] = fmaxf(w[i], w[i + 1]);
+#pragma unroll
+    for (int i = 0; i < kSelPer + 3; ++i) m4[i] = fmaxf(m2[i], m2[i + 2]);
+#pragma unroll
+    for (int e = 0; e < kSelPer; ++e)
+      kr[e] = lo + e < P ? order_key(fmaxf(fmaxf(m4[e], m2[e + 4]), w[e + 6])) : 0u;
+  } else {
+#pragma unroll
+    for (int e = 0; e < kSelPer; ++e) {
+      const int j = lo + e;
+      kr[e] = 0u;
+      if (j < P) {
+        float pv;
+        if (s.pool_type == GRKV_POOL_MAX) {
+          pv = cs(j);
+          for (int t = 1; t <= h; ++t) {
+            if (j - t >= 0) pv = fmaxf(pv, cs(j - t));
+            if (j + t < P) pv = fmaxf(pv, cs(j + t));
+          }
+        } else {
+          double acc = 0.0;   // left to right, zero padding, divisor k
+          for (int t = -h; t <= h; ++t)
+            if (j + t >= 0 && j + t < P) acc += (double)cs(j + t);
+          pv = (float)(acc / (double)s.pool_k);
         }
-      } else {
-        double acc = 0.0;   // left to right, zero padding, divisor k
-        for (int t = -h; t <= h; ++t)
-          if (j + t >= 0 && j + t < P) acc += (double)cs(j + t);
-        pv = (float)(acc / (double)s.pool_k);
+        kr[e] = order_key(pv);
       }
-      kr[e] = order_key(pv);
     }
   }
-  __syncthreads();
-#pragma unroll
-  for (int e = 0; e < kSelPer; ++e) {
-    const int j = tid + e * kSelThreads;
-    if (j < P) skey[sel_pad(j)] = kr[e];
-  }
-  __syncthreads();
   if (s.kk >= P) {
     for (int j = tid; j < P; j += kSelThreads) out[j] = j;
   } else if (s.kk > 0) {
@@ -338,8 +352,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) k_select_smem(const float* __r
       __syncthreads();
 #pragma unroll
       for (int e = 0; e < kSelPer; ++e) {
-        const int j = tid + e * kSelThreads;
-        if (j < P && (kr[e] & mask) == prefix)
+        if (lo + e < P && (kr[e] & mask) == prefix)
           atomicAdd(&whist[warp * 256 + ((kr[e] >> shift) & 255u)], 1);
       }
       __syncthreads();
@@ -389,30 +402,32 @@ __global__ void __launch_bounds__(kSelThreads, 1) k_select_smem(const float* __r
     }
     const uint32_t tau = prefix;
     const int need_eq = rem;
-    // compaction in position order: thread t owns positions 32t .. 32t+31
-    const int lo = min(P, tid * kSelPer), hi = min(P, lo + kSelPer);
+    // compaction in position order over the same segments
     int eq = 0;
-    for (int i = lo; i < hi; ++i) eq += skey[sel_pad(i)] == tau;
+#pragma unroll
+    for (int e = 0; e < kSelPer; ++e) eq += (lo + e < P && kr[e] == tau);
     int tot;
     const int er0 = block_exclusive_scan(eq, sh + 8, &tot);
     int sel = 0, er = er0;
-    for (int i = lo; i < hi; ++i) {
-      const uint32_t key = skey[sel_pad(i)];
-      if (key > tau) {
+#pragma unroll
+    for (int e = 0; e < kSelPer; ++e) {
+      if (lo + e >= P) continue;
+      if (kr[e] > tau) {
         ++sel;
-      } else if (key == tau) {
+      } else if (kr[e] == tau) {
         if (er < need_eq) ++sel;
         ++er;
       }
     }
     int pos = block_exclusive_scan(sel, sh + 8, &tot);
     er = er0;
-    for (int i = lo; i < hi; ++i) {
-      const uint32_t key = skey[sel_pad(i)];
-      if (key > tau) {
-        out[pos++] = i;
-      } else if (key == tau) {
-        if (er < need_eq) out[pos++] = i;
+#pragma unroll
+    for (int e = 0; e < kSelPer; ++e) {
+      if (lo + e >= P) continue;
+      if (kr[e] > tau) {
+        out[pos++] = lo + e;
+      } else if (kr[e] == tau) {
+        if (er < need_eq) out[pos++] = lo + e;
         ++er;
       }
     }
