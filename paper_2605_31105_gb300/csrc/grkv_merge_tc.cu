@@ -1219,15 +1219,23 @@ __global__ void __launch_bounds__(kDenseNT, 1)
     return;
   }
   if (tid == 0) *fail = 0;
+  // the lower triangle row by row (with sym: halved off the diagonal, lambda
+  // added on it), then with sym the upper triangle's halves added, also read
+  // row by row: both passes load whole rows
   for (int i = warp; i < kDenseM; i += kDenseNT / 32)
     for (int j = lane; j <= i; j += 32) {
       float val = i == j ? 1.f : 0.f;
       if (i < m && j < m) {
         val = __ldg(Gu + (size_t)i * ld + j);
-        if (sym) val = 0.5f * (val + __ldg(Gu + (size_t)j * ld + i)) + (i == j ? lambda : 0.f);
+        if (sym) val = i == j ? val + lambda : 0.5f * val;
       }
       N[tri(i) + j] = val;
     }
+  if (sym) {
+    __syncthreads();
+    for (int r = warp; r < m; r += kDenseNT / 32)
+      for (int c = r + 1 + lane; c < m; c += 32) N[tri(c) + r] += 0.5f * __ldg(Gu + (size_t)r * ld + c);
+  }
   __syncthreads();
   for (int kb = 0; kb < kDenseM / 32; ++kb) {
     const int k0 = kb * 32;

@@ -64,14 +64,15 @@ constexpr uint32_t kColS = 0, kColY = 256;
 struct Args {
   int U, n, w, m, P, causal;
   int row0, mr;   // stacked rows row0 .. row0 + mr - 1 (mr <= 128) in this launch
-  int acc;        // add the prefix scores to those of an earlier launch (rows before row0)
+  int acc;        // a later row block: its prefix scores go to scores2 (added by k_add_scores)
   int tpu;        // tiles per unit
   int mode;       // 0: pass A, 1: pass B
   int gu;         // units per round (all of them)
   int rounds;     // 1
   int maxc;       // stats slots per unit
   float sl2;      // scale * log2(e)
-  float* scores;  // [U][P]
+  float* scores;   // [U][P]
+  float* scores2;  // [U][P] prefix scores of the second row block (m > 128)
   float* y;       // [U][m][128], zeroed by the host
   float* row_stats;  // [U][m][2]
   float2* pstats;    // [U][maxc][128]  (max in log2 units, sum)
@@ -724,8 +725,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const int jj = q * 32 + lane;
               const float cs = ((rb[jj] + rb[64 + jj]) + rb[128 + jj]) + rb[192 + jj];
               if (t0 + jj < a.P && 64 * wg + jj < j.len) {
-                float* dst = a.scores + (size_t)j.u * a.P + t0 + jj;
-                *dst = a.acc ? *dst + cs : cs;
+                (a.acc ? a.scores2 : a.scores)[(size_t)j.u * a.P + t0 + jj] = cs;
               }
             }
           }
@@ -752,6 +752,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
+// scores += scores2: the second row block's prefix scores (m > 128) added
+// once, instead of read-modify-written by the tiles of its pass B.
+__global__ void k_add_scores(float* __restrict__ scores, const float* __restrict__ scores2,
+                             size_t count) {
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < count;
+       i += (size_t)gridDim.x * blockDim.x)
+    scores[i] += scores2[i];
 }
 
 // Deterministic mode: Y[u] = sum over the unit's slots k = 0 .. maxc-1 of the
@@ -833,6 +842,7 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
   a.rounds = rounds;
   a.sl2 = (float)((double)s.scale * 1.4426950408889634);
   a.scores = scores;
+  a.scores2 = (float*)(ws + L.pooled);   // unused until the selection
   a.y = y;
   a.row_stats = row_stats;
   a.pstats = (float2*)(ws + L.pstats_tc);
@@ -871,6 +881,13 @@ cudaError_t launch_score_tc(const Shape& s, const void* q, const void* k, const 
     e = launch(0);
     if (e == cudaSuccess) e = launch(1);
     if (e != cudaSuccess) return e;
+  }
+  if (s.m > kRows) {
+    const size_t count = (size_t)s.U * s.P;
+    const int blocks = (int)std::min<size_t>((count + 255) / 256, (size_t)G * 8);
+    k_add_scores<<<blocks, 256, 0, st>>>(scores, a.scores2, count);
+    count_launches(1);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   if (a.ypart) {
     const size_t n4 = (size_t)s.U * s.m * kD / 4;
