@@ -81,8 +81,8 @@ SCORE_SRC = os.path.join("paper_2605_31105_gb300", "csrc", "grkv_score_tc.cu")
 # the ncu capture in profiles/score_tc_c2_llama_32k.md, keyed by the SHA-256 of the
 # kernel source it was taken on.
 SCORE_TRAFFIC = {
-    "c2_llama_32k_bf16": ("a42b3f34fc6ed4bad174cd5869ab7034001206452d4ddbf8ce655ee5bf6d456c",
-                          6533601280),
+    "c2_llama_32k_bf16": ("0ea59ba48bb5a0be128f6060b1dd07717b01f47bfca8e89e80517f105e7d52bc",
+                          6532132864),
 }
 
 
