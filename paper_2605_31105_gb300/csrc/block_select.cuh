@@ -46,10 +46,18 @@ __device__ void block_kth_largest(Get get, int count, int k, int* hist, int* sh,
   for (int shift = 24; shift >= 0; shift -= 8) {
     for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
     __syncthreads();
-    for (int i = threadIdx.x; i < count; i += blockDim.x) {
-      uint32_t key;
-      if (!get(i, &key)) continue;
-      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1);
+    // eight keys fetched per step, so that their loads are in flight together
+    for (int i0 = threadIdx.x; i0 < count; i0 += 8 * blockDim.x) {
+      uint32_t key[8];
+      bool ok[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int i = i0 + q * blockDim.x;
+        ok[q] = i < count && get(i, &key[q]);
+      }
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        if (ok[q] && (key[q] & mask) == prefix) atomicAdd(&hist[(key[q] >> shift) & 255u], 1);
     }
     __syncthreads();
     if (threadIdx.x < 32) {

@@ -205,19 +205,37 @@ __global__ void __launch_bounds__(1024) k_select(const float* __restrict__ score
   const float* c = scores + (size_t)u * P;
   float* pl = pooled + (size_t)u * P;
   int32_t* out = idx + (size_t)u * s.B;
-  for (int j = tid; j < P; j += blockDim.x) {
+  // four positions per step, the neighbour offset outermost, so that each
+  // step's loads are independent of one another
+  for (int j0 = tid; j0 < P; j0 += 4 * blockDim.x) {
+    int j[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) j[q] = j0 + q * blockDim.x;
     if (s.pool_type == GRKV_POOL_MAX) {
-      float mx = c[j];
+      float mx[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) mx[q] = j[q] < P ? c[j[q]] : 0.f;
       for (int t = 1; t <= h; ++t) {
-        if (j - t >= 0) mx = fmaxf(mx, c[j - t]);
-        if (j + t < P) mx = fmaxf(mx, c[j + t]);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          if (j[q] >= P) continue;
+          if (j[q] - t >= 0) mx[q] = fmaxf(mx[q], c[j[q] - t]);
+          if (j[q] + t < P) mx[q] = fmaxf(mx[q], c[j[q] + t]);
+        }
       }
-      pl[j] = mx;
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        if (j[q] < P) pl[j[q]] = mx[q];
     } else {
-      double a = 0.0;  // left to right, zero padding, divisor k
-      for (int t = -h; t <= h; ++t)
-        if (j + t >= 0 && j + t < P) a += (double)c[j + t];
-      pl[j] = (float)(a / (double)s.pool_k);
+      double a[4] = {0.0, 0.0, 0.0, 0.0};   // left to right, zero padding, divisor k
+      for (int t = -h; t <= h; ++t) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          if (j[q] < P && j[q] + t >= 0 && j[q] + t < P) a[q] += (double)c[j[q] + t];
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        if (j[q] < P) pl[j[q]] = (float)(a[q] / (double)s.pool_k);
     }
   }
   __syncthreads();
@@ -234,30 +252,49 @@ __global__ void __launch_bounds__(1024) k_select(const float* __restrict__ score
     uint32_t tau;
     int need_eq;
     block_kth_largest(get, P, s.kk, hist, sh, &tau, &need_eq);
+    // the segment's keys in chunks of eight loaded together
+    auto seg_keys = [&](int i0, uint32_t* kk) {
+#pragma unroll
+      for (int q = 0; q < 8; ++q) kk[q] = i0 + q < hi ? order_key(pl[i0 + q]) : 0u;
+    };
     int eq = 0;
-    for (int i = lo; i < hi; ++i)
-      if (order_key(pl[i]) == tau) ++eq;
+    for (int i0 = lo; i0 < hi; i0 += 8) {
+      uint32_t kk[8];
+      seg_keys(i0, kk);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) eq += (i0 + q < hi && kk[q] == tau);
+    }
     int tot;
     const int er0 = block_exclusive_scan(eq, sh + 8, &tot);
     int sel = 0, er = er0;
-    for (int i = lo; i < hi; ++i) {
-      const uint32_t key = order_key(pl[i]);
-      if (key > tau) {
-        ++sel;
-      } else if (key == tau) {
-        if (er < need_eq) ++sel;
-        ++er;
+    for (int i0 = lo; i0 < hi; i0 += 8) {
+      uint32_t kk[8];
+      seg_keys(i0, kk);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        if (i0 + q >= hi) continue;
+        if (kk[q] > tau) {
+          ++sel;
+        } else if (kk[q] == tau) {
+          if (er < need_eq) ++sel;
+          ++er;
+        }
       }
     }
     int pos = block_exclusive_scan(sel, sh + 8, &tot);
     er = er0;
-    for (int i = lo; i < hi; ++i) {
-      const uint32_t key = order_key(pl[i]);
-      if (key > tau) {
-        out[pos++] = i;
-      } else if (key == tau) {
-        if (er < need_eq) out[pos++] = i;
-        ++er;
+    for (int i0 = lo; i0 < hi; i0 += 8) {
+      uint32_t kk[8];
+      seg_keys(i0, kk);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        if (i0 + q >= hi) continue;
+        if (kk[q] > tau) {
+          out[pos++] = i0 + q;
+        } else if (kk[q] == tau) {
+          if (er < need_eq) out[pos++] = i0 + q;
+          ++er;
+        }
       }
     }
   }
