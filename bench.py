@@ -49,7 +49,14 @@ def args_():
     ap.add_argument("--path", choices=("default", "one_read", "portable"), default="default",
                     help="scoring kernels: default (two tensor-core launches, K read twice), "
                          "one_read (one launch that reads K from HBM once) or portable (CUDA cores)")
-    return ap.parse_args()
+    ap.add_argument("--update-k", action="store_true",
+                    help="add the key step (GRKV_UPDATE_K, CG to the library's default residual); "
+                         "no CPU baseline is timed for it")
+    ap.add_argument("--lambda-k", type=float, default=1e-2)
+    a = ap.parse_args()
+    if a.update_k:
+        a.no_cpu_baseline = True
+    return a
 
 
 def workload(a):
@@ -331,9 +338,10 @@ def run_ours(a):
     gi.fill_units(wl, view(hq), view(hk), view(hv))
     dq, dk, dv = hq.cuda(), hk.cuda(), hv.cuda()
     p = b.params(U, wl.group, n, wl.window, B, pool_kernel=wl.pool_kernel,
-                 lambda_v=wl.lambda_v, dtype=wl.dtype,
+                 lambda_v=wl.lambda_v, lambda_k=a.lambda_k, dtype=wl.dtype,
                  flags={"default": 0, "one_read": b.GRKV_ONE_READ_SCORE,
-                        "portable": b.GRKV_FORCE_SIMT}[a.path])
+                        "portable": b.GRKV_FORCE_SIMT}[a.path]
+                 | (b.GRKV_UPDATE_K if a.update_k else 0))
     ws = torch.empty(b.grkv_workspace_size(p), dtype=torch.uint8, device="cuda")
     ko = torch.empty((U, B, d), dtype=tdt, device="cuda")
     vo = torch.empty_like(ko)
@@ -443,7 +451,8 @@ def run_ours(a):
         "config": {"workload": wl.name, "units": U, "n": n, "budget": B, "window": wl.window,
                    "group": wl.group, "d": d, "lambda_v": wl.lambda_v,
                    "pool_kernel": wl.pool_kernel, "l2": "inputs (K+V %.1f GB) exceed L2" %
-                   (read / 1e9), "parallelism": f"units sharded, {world} rank(s)"},
+                   (read / 1e9), "parallelism": f"units sharded, {world} rank(s)",
+                   "key_step": bool(a.update_k)},
         "path": a.path,
         "roofline": {"bound": "hbm",
                      "kernel": SCORE_KERNEL["portable" if wl.dtype != "bf16" else a.path],
