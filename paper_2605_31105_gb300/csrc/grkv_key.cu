@@ -51,6 +51,7 @@ struct KArgs {
   int lambda_inf;
   int vt_valid;           // Vt holds V^(t) (false at t = 1: V^(1) is only in v_out)
   int use_tc;             // m <= 128: the CG products run on the tensor cores
+  int cluster;            // C: CTAs per unit in k_key_step's CG (one cluster each)
   const void* k;          // [U][n][d]  full caches (K0, V0 gathers of steps t >= 1)
   const void* v;
   float* Kt;              // [U][B][d]  fp32 K^(t) of the alternation, or null
@@ -70,7 +71,10 @@ struct KArgs {
   float* dK;              // [U][B][d]
   float* T2;              // [U][m][B]
   float* GQ;              // [U][m][m]
-  float* vec;             // [U][4][m][d]: r, p, Ap, alpha
+  float* vec;             // [U][C][5][m][d]: r, p, Ap, alpha, X V* of each CTA
+  float* app;             // [U][C][m][d]  per-CTA partial products (C > 1)
+  float* rho2p;           // [U][C][128]   per-CTA partial row sums (C > 1)
+  int* cnt;               // [U]           barrier counters (C > 1, zeroed per launch)
   uint8_t* fixed;         // [U][B]
 };
 
@@ -242,80 +246,110 @@ __device__ __forceinline__ void split3(const float* x, uint4* part) {
   for (int q = 0; q < 3; ++q) part[q] = make_uint4(p[q][0], p[q][1], p[q][2], p[q][3]);
 }
 
+// x[0..8) = p[0..nv) read through L2 only: data another CTA of the unit
+// wrote (L1 is not coherent across SMs).
+__device__ __forceinline__ void ld8cg(const float* p, int nv, float* x) {
+  if (nv == 8 && ((uintptr_t)p & 15) == 0) {
+    const float4 a = __ldcg((const float4*)p), b = __ldcg((const float4*)(p + 4));
+    x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w;
+    x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+  } else {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) x[e] = e < nv ? __ldcg(p + e) : 0.f;
+  }
+}
+
 // C = A B for A [M][K] (M <= 128) and B [K][N], B staged K-major ([N] rows of
 // K, kBK) or MN-major ([K] rows of N); parts_b = 1 when B is exact in bf16.
 // Operands come in chunks of eight along their contiguous index:
 // a8(i, k, nv, x) fills x with A[i][k .. k+nv) (nv <= 8, zeros after), b8(k,
-// j, nv, x) with B[k .. k+nv)[j] (kBK) or B[k][j .. j+nv).  For every output
-// element store(i, j, v) returns a value summed per row and handed to
+// j, nv, x) with B[k .. k+nv)[j] (kBK) or B[k][j .. j+nv).  Every thread
+// loads all its chunks of a slab before it stores any to shared memory, and
+// loads the next slab of the same output tile while the MMAs of the
+// current one run.  The epilogue takes a warp's rows four
+// at a time: pre(i, j) for all of them first, then store(i, j, v, pre(i, j))
+// for every output element, whose results are summed per row and handed to
 // rowsum(i, s) once per 128-column tile.  All threads of the CTA call it.
-template <bool kBK, class FA, class FB, class FS, class FR>
-__device__ void tc_gemm(TcCtx& c, int M, int N, int K, int parts_b, FA a, FB b, FS store,
+template <bool kBK, class FA, class FB, class FP, class FS, class FR>
+__device__ void tc_gemm(TcCtx& c, int M, int N, int K, int parts_b, FA a, FB b, FP pre, FS store,
                         FR rowsum) {
+  constexpr int kCh = 128 * 8 / kKT;     // chunks of each operand a thread stages per slab
+  constexpr int kRows = kKT / 32;        // rows apart in a warp's epilogue batch
+  static_assert(kCh * kKT == 128 * 8 && kCh * kKT == 64 * 16, "slab split");
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   uint8_t* As = c.sm;
   uint8_t* Bs = c.sm + kTP * kSlab;
   const uint32_t as = smem_u32(As), bs = smem_u32(Bs);
   const uint32_t idesc = idesc_bf16(128, 128, 0, kBK ? 0 : 1);
   volatile int no_abort = 0;
-  for (int j0 = 0; j0 < N; j0 += 128) {
-    for (int k0 = 0; k0 < K; k0 += 64) {
-      for (int ch = tid; ch < 128 * 8; ch += kKT) {
-        const int r = ch >> 3, c8 = ch & 7, kk = k0 + c8 * 8;
-        float x[8];
-        a(r, kk, r < M ? max(0, min(8, K - kk)) : 0, x);
-        uint4 pt[3];
-        split3(x, pt);
-        const uint32_t off = sw128_offset(r, c8);
+  const int nk = max(1, (K + 63) / 64), nt = (N + 127) / 128 * nk;
+  float xa[kCh][8], xb[kCh][8];
+  auto fetch = [&](int sl) {
+    const int j0 = sl / nk * 128, k0 = sl % nk * 64;
 #pragma unroll
-        for (int q = 0; q < kTP; ++q) *(uint4*)(As + q * kSlab + off) = pt[q];
-      }
+    for (int l = 0; l < kCh; ++l) {
+      const int ch = tid + l * kKT, r = ch >> 3, kk = k0 + (ch & 7) * 8;
+      a(r, kk, r < M ? max(0, min(8, K - kk)) : 0, xa[l]);
+    }
+#pragma unroll
+    for (int l = 0; l < kCh; ++l) {
+      const int ch = tid + l * kKT;
       if (kBK) {
-        for (int ch = tid; ch < 128 * 8; ch += kKT) {
-          const int r = ch >> 3, c8 = ch & 7, kk = k0 + c8 * 8;
-          float x[8];
-          b(kk, j0 + r, j0 + r < N ? max(0, min(8, K - kk)) : 0, x);
-          uint4 pt[3];
-          split3(x, pt);
-          const uint32_t off = sw128_offset(r, c8);
-          for (int q = 0; q < parts_b; ++q) *(uint4*)(Bs + q * kSlab + off) = pt[q];
-        }
+        const int r = ch >> 3, kk = k0 + (ch & 7) * 8;
+        b(kk, j0 + r, j0 + r < N ? max(0, min(8, K - kk)) : 0, xb[l]);
       } else {
         // [64 rows of K][128 of N] as two halves of 64 columns (8 KB each)
-        for (int ch = tid; ch < 64 * 16; ch += kKT) {
-          const int kr = ch >> 4, nc = ch & 15, hf = nc >> 3, c8 = nc & 7, jj = j0 + nc * 8;
-          float x[8];
-          b(k0 + kr, jj, k0 + kr < K ? max(0, min(8, N - jj)) : 0, x);
-          uint4 pt[3];
-          split3(x, pt);
-          const uint32_t off = hf * (kSlab / 2) + sw128_offset(kr, c8);
-          for (int q = 0; q < parts_b; ++q) *(uint4*)(Bs + q * kSlab + off) = pt[q];
-        }
+        const int kr = ch >> 4, jj = j0 + (ch & 15) * 8;
+        b(k0 + kr, jj, k0 + kr < K ? max(0, min(8, N - jj)) : 0, xb[l]);
       }
-      fence_proxy_async_smem();
-      __syncthreads();
-      if (tid == 0) {
-        tc_fence_after();
-        bool acc = k0 > 0;
-        for (int pa = 0; pa < kTP; ++pa)
-          for (int pb = 0; pb < parts_b; ++pb) {
-            if (pa + pb > 2) continue;
-#pragma unroll
-            for (int kk = 0; kk < 4; ++kk) {
-              const uint64_t ad = sw128_desc(as + pa * kSlab + kk * 32, 16, 1024);
-              const uint64_t bd = kBK ? sw128_desc(bs + pb * kSlab + kk * 32, 16, 1024)
-                                      : sw128_desc(bs + pb * kSlab + kk * 2048, kSlab / 2, 1024);
-              mma_bf16(c.tmem, ad, bd, idesc, acc ? 1u : 0u);
-              acc = true;
-            }
-          }
-        mma_commit(c.bar);
-      }
-      if (!mbar_wait(c.bar, c.phase, &no_abort, kWaitBudget) && tid == 0)
-        set_status(c.status, GRKV_ERR_TIMEOUT);
-      c.phase ^= 1;
-      tc_fence_after();
     }
+  };
+  if (nt > 0) fetch(0);
+  for (int sl = 0; sl < nt; ++sl) {
+    const int j0 = sl / nk * 128, kt = sl % nk;
+#pragma unroll
+    for (int l = 0; l < kCh; ++l) {
+      const int ch = tid + l * kKT;
+      uint4 pt[3];
+      split3(xa[l], pt);
+      const uint32_t off = sw128_offset(ch >> 3, ch & 7);
+#pragma unroll
+      for (int q = 0; q < kTP; ++q) *(uint4*)(As + q * kSlab + off) = pt[q];
+    }
+#pragma unroll
+    for (int l = 0; l < kCh; ++l) {
+      const int ch = tid + l * kKT;
+      uint4 pt[3];
+      split3(xb[l], pt);
+      const uint32_t off = kBK ? sw128_offset(ch >> 3, ch & 7)
+                               : ((ch & 15) >> 3) * (kSlab / 2) + sw128_offset(ch >> 4, ch & 7);
+      for (int q = 0; q < parts_b; ++q) *(uint4*)(Bs + q * kSlab + off) = pt[q];
+    }
+    fence_proxy_async_smem();
+    __syncthreads();
+    if (tid == 0) {
+      tc_fence_after();
+      bool acc = kt > 0;
+      for (int pa = 0; pa < kTP; ++pa)
+        for (int pb = 0; pb < parts_b; ++pb) {
+          if (pa + pb > 2) continue;
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk) {
+            const uint64_t ad = sw128_desc(as + pa * kSlab + kk * 32, 16, 1024);
+            const uint64_t bd = kBK ? sw128_desc(bs + pb * kSlab + kk * 32, 16, 1024)
+                                    : sw128_desc(bs + pb * kSlab + kk * 2048, kSlab / 2, 1024);
+            mma_bf16(c.tmem, ad, bd, idesc, acc ? 1u : 0u);
+            acc = true;
+          }
+        }
+      mma_commit(c.bar);
+    }
+    if (sl + 1 < nt && kt + 1 < nk) fetch(sl + 1);
+    if (!mbar_wait(c.bar, c.phase, &no_abort, kWaitBudget) && tid == 0)
+      set_status(c.status, GRKV_ERR_TIMEOUT);
+    c.phase ^= 1;
+    tc_fence_after();
+    if (kt != nk - 1) continue;
     // the tile through shared memory (the slabs are free: every MMA has completed)
     float* tile = (float*)c.sm;
     if (warp < 4) {
@@ -331,18 +365,36 @@ __device__ void tc_gemm(TcCtx& c, int M, int N, int K, int parts_b, FA a, FB b, 
     }
     tc_fence_before();
     __syncthreads();
-    for (int i = warp; i < M; i += kKT / 32) {
-      float sum = 0.f;
+    for (int i0 = warp; i0 < M; i0 += 4 * kRows) {
+      float pv[4][4], tv[4][4];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int jj = q * 32 + lane, j = j0 + jj;
-        if (j < N) sum += store(i, j, tile[i * kTLD + jj]);
+      for (int rr = 0; rr < 4; ++rr) {
+        const int i = i0 + rr * kRows;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int j = j0 + q * 32 + lane;
+          const bool ok = i < M && j < N;
+          pv[rr][q] = ok ? pre(i, j) : 0.f;
+          tv[rr][q] = ok ? tile[i * kTLD + q * 32 + lane] : 0.f;
+        }
       }
 #pragma unroll
-      for (int o = 16; o >= 1; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-      if (lane == 0) rowsum(i, sum);
+      for (int rr = 0; rr < 4; ++rr) {
+        const int i = i0 + rr * kRows;
+        if (i >= M) break;
+        float sum = 0.f;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int j = j0 + q * 32 + lane;
+          if (j < N) sum += store(i, j, tv[rr][q], pv[rr][q]);
+        }
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+        if (lane == 0) rowsum(i, sum);
+      }
     }
     __syncthreads();
+    if (sl + 1 < nt) fetch(sl + 1);
   }
 }
 
@@ -374,16 +426,18 @@ __device__ void softmax_jacobian_rows(const float* X, float* T, int m, int B) {
   __syncthreads();
 }
 
-// Per-unit working set of the key step and of the alternation.
+// Per-unit working set of the key step and of the alternation; r is the
+// CTA's rank among the unit's C CTAs, whose m x d vectors are its own.
 struct KUnit {
   int u, m, B;
   const int32_t* idx;
   const void* q;
   size_t kv_off;          // u * B * d
   const float* Y;
-  float *X, *T, *dK, *T2, *GQ, *R, *Pd, *AP, *AL;
+  float *X, *T, *dK, *T2, *GQ, *R, *Pd, *AP, *AL, *XV;
+  float* E;               // rank 0's r: the right-hand side e on entry to CG
   uint8_t* fixed;
-  __device__ KUnit(const KArgs& a, int u_) : u(u_), m(a.m), B(a.B) {
+  __device__ KUnit(const KArgs& a, int u_, int r_ = 0) : u(u_), m(a.m), B(a.B) {
     idx = a.idx + (size_t)u * B;
     q = (const char*)a.q + (size_t)u * m * kD * (a.dtype == GRKV_F32 ? 4 : 2);
     kv_off = (size_t)u * B * kD;
@@ -393,10 +447,13 @@ struct KUnit {
     dK = a.dK + kv_off;
     T2 = a.T2 + (size_t)u * m * B;
     GQ = a.GQ + (size_t)u * m * m;
-    R = a.vec + (size_t)u * 4 * m * kD;
-    Pd = R + (size_t)m * kD;
-    AP = Pd + (size_t)m * kD;
-    AL = AP + (size_t)m * kD;
+    const size_t md = (size_t)m * kD;
+    E = a.vec + (size_t)u * a.cluster * 5 * md;
+    R = E + (size_t)r_ * 5 * md;
+    Pd = R + md;
+    AP = Pd + md;
+    AL = AP + md;
+    XV = AL + md;
     fixed = a.fixed + (size_t)u * B;
   }
 };
@@ -544,91 +601,336 @@ __device__ void key_cg(const KArgs& a, const KUnit& k, GemmSmem& gs, float* red,
   }
 }
 
-// key_cg with the three products of an iteration on the tensor cores
-// (m <= 128).  The softmax Jacobians are applied as the next product stages
-// its operand: the row sums rho1 = rowsum(X o T) and rho2 = rowsum(X o T2)
-// are taken in the epilogues of the products that write T and T2.
-template <class FV, class FV8>
-__device__ void key_cg_tc(const KArgs& a, const KUnit& k, GemmSmem& gs, float* red, TcCtx& c,
-                          float* rho1, float* rho2, int parts_v, FV vget, FV8 vget8) {
-  (void)vget;
-  const int m = k.m, B = k.B, dt = a.dtype, md = m * kD;
-  const float s = a.scale;
-  block_gemm<false, true>(gs,
-      m, m, kD, [&](int r, int t) { return ldv(k.q, (size_t)r * kD + t, dt); },
-      [&](int t, int r2) { return ldv(k.q, (size_t)r2 * kD + t, dt); },
-      [&](int r, int r2, float v) { k.GQ[(size_t)r * m + r2] = s * s * v; });
-  float rs = 0.f;
-  for (int i = threadIdx.x; i < md; i += kKT) {
-    k.Pd[i] = k.R[i];
-    k.AL[i] = 0.f;
-    rs = fmaf(k.R[i], k.R[i], rs);
+// The share of a unit's CG that one CTA carries.  With C > 1 CTAs per unit
+// (launched as one cluster, so they run together), rank r takes the
+// retained columns [c0, c0 + nc) of the three products; the row sums rho2
+// and the product J_G (J_G^T p) are summed over the ranks through the
+// workspace, always in rank order, and every rank keeps its own copy of the
+// m x d vectors and updates all of it.  Every rank therefore holds the same
+// bits, takes the same branches and meets the same barriers.
+struct KPart {
+  int C, r, c0, nc;
+  float* app;       // [C][m][d] partial products, one slot per rank (k.AP when C == 1)
+  float* rho2p;     // [C][128] partial row sums (C > 1)
+  int* cnt;         // barrier counter of the unit (C > 1)
+  int nb;           // barriers passed
+  int* flag;        // shared: the last barrier completed
+};
+
+__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Barrier of the C CTAs of a unit on its counter in global memory (zeroed
+// before the launch).  Each CTA's earlier global writes are visible to the
+// others' L2 loads (__ldcg) once it returns.  The wait is bounded: when the
+// peers have not all arrived within the budget it sets the status and
+// returns false, and the caller stops exchanging.
+__device__ bool part_barrier(KPart& kp, int* status) {
+  __syncthreads();
+  ++kp.nb;
+  if (threadIdx.x == 0) {
+    int ok = 1;
+    __threadfence();
+    atomicAdd(kp.cnt, 1);
+    const int target = kp.nb * kp.C;
+    if (ld_acquire_gpu(kp.cnt) < target) {
+      const long long t0 = clock64();
+      while (ld_acquire_gpu(kp.cnt) < target)
+        if (clock64() - t0 > kWaitBudget) {
+          ok = 0;
+          set_status(status, GRKV_ERR_TIMEOUT);
+          break;
+        }
+    }
+    __threadfence();
+    *kp.flag = ok;
   }
+  __syncthreads();
+  return *kp.flag != 0;
+}
+
+// The m x d vectors of the tensor-core CG are walked by rows: warp w takes
+// rows w, w + 8, ..., lane l the four columns 4l .. 4l+3 of each (one float4).
+// Each loop loads a batch of rows before it stores anything, so that the
+// loads of a batch are in flight together.
+constexpr int kWarps = kKT / 32;
+
+__device__ __forceinline__ float dot4(float4 a, float4 b, float acc) {
+  acc = fmaf(a.x, b.x, acc);
+  acc = fmaf(a.y, b.y, acc);
+  acc = fmaf(a.z, b.z, acc);
+  return fmaf(a.w, b.w, acc);
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+// Sum of float4 i over the kC partial slots (md floats apart), in rank order.
+template <int kC>
+__device__ __forceinline__ float4 sum_parts(const float* app, size_t md, int i) {
+  float4 t[kC];
+#pragma unroll
+  for (int q = 0; q < kC; ++q) t[q] = __ldcg((const float4*)(app + (size_t)q * md) + i);
+  float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+  for (int q = 0; q < kC; ++q) {
+    v.x += t[q].x;
+    v.y += t[q].y;
+    v.z += t[q].z;
+    v.w += t[q].w;
+  }
+  return v;
+}
+
+// Start of CG: r = p = e (rank 0's r), alpha = 0 and, for a split unit
+// (kC > 1), X V* = sum of the partials and rho1 = rowsum(p o X V*); returns
+// the thread's share of ||e||^2.
+template <int kC>
+__device__ float cg_start(const KUnit& k, const KPart& kp, float* rho1) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, m = k.m;
+  const size_t md = (size_t)m * kD;
+  float rs = 0.f;
+  for (int r0 = warp; r0 < m; r0 += 2 * kWarps) {
+    float4 xv[2], e[2];
+#pragma unroll
+    for (int b = 0; b < 2; ++b) {
+      const int r = r0 + b * kWarps, i = r * 32 + lane;
+      xv[b] = kC > 1 && r < m ? sum_parts<kC>(kp.app, md, i) : make_float4(0.f, 0.f, 0.f, 0.f);
+      e[b] = r < m ? __ldcg((const float4*)k.E + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int b = 0; b < 2; ++b) {
+      const int r = r0 + b * kWarps, i = r * 32 + lane;
+      if (r >= m) break;
+      ((float4*)k.R)[i] = e[b];
+      ((float4*)k.Pd)[i] = e[b];
+      ((float4*)k.AL)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      rs = dot4(e[b], e[b], rs);
+      if (kC > 1) {
+        ((float4*)k.XV)[i] = xv[b];
+        const float d = warp_sum(dot4(e[b], xv[b], 0.f));
+        if (lane == 0) rho1[r] = d;
+      }
+    }
+  }
+  return rs;
+}
+
+// Ap = (sum of the partial products) + lambda p; returns the share of p . Ap.
+template <int kC>
+__device__ float cg_ap(const KUnit& k, const KPart& kp, float lambda) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, m = k.m;
+  const size_t md = (size_t)m * kD;
+  float pap = 0.f;
+  for (int r0 = warp; r0 < m; r0 += 2 * kWarps) {
+    float4 v[2], pd[2];
+#pragma unroll
+    for (int b = 0; b < 2; ++b) {
+      const int r = r0 + b * kWarps, i = r * 32 + lane;
+      v[b] = r < m ? sum_parts<kC>(kp.app, md, i) : make_float4(0.f, 0.f, 0.f, 0.f);
+      pd[b] = r < m ? ((const float4*)k.Pd)[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int b = 0; b < 2; ++b) {
+      const int r = r0 + b * kWarps, i = r * 32 + lane;
+      if (r >= m) break;
+      float4 ap = v[b];
+      ap.x = fmaf(lambda, pd[b].x, ap.x);
+      ap.y = fmaf(lambda, pd[b].y, ap.y);
+      ap.z = fmaf(lambda, pd[b].z, ap.z);
+      ap.w = fmaf(lambda, pd[b].w, ap.w);
+      ((float4*)k.AP)[i] = ap;
+      pap = dot4(pd[b], ap, pap);
+    }
+  }
+  return pap;
+}
+
+// alpha += al p, r -= al Ap; returns the share of ||r||^2.
+__device__ float cg_step(const KUnit& k, float al) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, m = k.m;
+  float rn = 0.f;
+  for (int r0 = warp; r0 < m; r0 += 4 * kWarps) {
+    float4 pd[4], alp[4], ap[4], rr[4];
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+      const int r = min(r0 + b * kWarps, m - 1), i = r * 32 + lane;
+      pd[b] = ((const float4*)k.Pd)[i];
+      alp[b] = ((const float4*)k.AL)[i];
+      ap[b] = ((const float4*)k.AP)[i];
+      rr[b] = ((const float4*)k.R)[i];
+    }
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+      const int r = r0 + b * kWarps, i = r * 32 + lane;
+      if (r >= m) break;
+      float4 a4 = alp[b], r4 = rr[b];
+      a4.x = fmaf(al, pd[b].x, a4.x);
+      a4.y = fmaf(al, pd[b].y, a4.y);
+      a4.z = fmaf(al, pd[b].z, a4.z);
+      a4.w = fmaf(al, pd[b].w, a4.w);
+      r4.x = fmaf(-al, ap[b].x, r4.x);
+      r4.y = fmaf(-al, ap[b].y, r4.y);
+      r4.z = fmaf(-al, ap[b].z, r4.z);
+      r4.w = fmaf(-al, ap[b].w, r4.w);
+      ((float4*)k.AL)[i] = a4;
+      ((float4*)k.R)[i] = r4;
+      rn = dot4(r4, r4, rn);
+    }
+  }
+  return rn;
+}
+
+// p = r + beta p and, for a split unit, the next iteration's rho1 =
+// rowsum(p o X V*).
+__device__ void cg_dir(const KUnit& k, float beta, float* rho1, bool split) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, m = k.m;
+  for (int r0 = warp; r0 < m; r0 += 4 * kWarps) {
+    float4 pd[4], rr[4], xv[4];
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+      const int r = min(r0 + b * kWarps, m - 1), i = r * 32 + lane;
+      pd[b] = ((const float4*)k.Pd)[i];
+      rr[b] = ((const float4*)k.R)[i];
+      xv[b] = split ? ((const float4*)k.XV)[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+      const int r = r0 + b * kWarps, i = r * 32 + lane;
+      if (r >= m) break;
+      float4 p4 = rr[b];
+      p4.x = fmaf(beta, pd[b].x, p4.x);
+      p4.y = fmaf(beta, pd[b].y, p4.y);
+      p4.z = fmaf(beta, pd[b].z, p4.z);
+      p4.w = fmaf(beta, pd[b].w, p4.w);
+      ((float4*)k.Pd)[i] = p4;
+      if (split) {
+        const float d = warp_sum(dot4(p4, xv[b], 0.f));
+        if (lane == 0) rho1[r] = d;
+      }
+    }
+  }
+}
+
+// key_cg with the three products of an iteration on the tensor cores
+// (m <= 128), over the CTA's columns of kp.  The softmax Jacobians are
+// applied as the next product stages its operand.  Their row sums are
+// rho1 = rowsum(X o T) and rho2 = rowsum(X o T2), taken in the epilogues of
+// the products that write T and T2; a unit split over C > 1 CTAs takes
+// rho1 = rowsum(P o (X V*)) instead, with X V* formed once, which needs no
+// exchange.
+template <class FV8>
+__device__ void key_cg_tc(const KArgs& a, const KUnit& k, GemmSmem& gs, float* red, TcCtx& c,
+                          KPart& kp, float* rho1, float* rho2, int parts_v, FV8 vget8) {
+  const int m = k.m, B = k.B, dt = a.dtype, md = m * kD;
+  const int C = kp.C, c0 = kp.c0, nc = kp.nc;
+  const float s = a.scale;
+  float* mine = kp.app + (size_t)kp.r * md;
+  if (kp.r == 0)
+    block_gemm<false, true>(gs,
+        m, m, kD, [&](int r, int t) { return ldv(k.q, (size_t)r * kD + t, dt); },
+        [&](int t, int r2) { return ldv(k.q, (size_t)r2 * kD + t, dt); },
+        [&](int r, int r2, float v) { k.GQ[(size_t)r * m + r2] = s * s * v; });
+  const bool split = C > 1;
+  bool ok = !split || part_barrier(kp, a.status);
+  if (split) {
+    // X V* over the CTA's columns, summed over the ranks in cg_start
+    tc_gemm<false>(c, m, kD, nc, parts_v,
+        [&](int r, int j, int nv, float* x) { ld8cg(k.X + (size_t)r * B + c0 + j, nv, x); },
+        [&](int j, int t, int nv, float* x) { vget8(c0 + j, t, nv, x); },
+        [](int, int) { return 0.f; },
+        [&](int r, int t, float v, float) {
+          mine[(size_t)r * kD + t] = v;
+          return 0.f;
+        }, [](int, float) {});
+    if (ok) ok = part_barrier(kp, a.status);
+  }
+  float rs = C == 8 ? cg_start<8>(k, kp, rho1)
+           : C == 4 ? cg_start<4>(k, kp, rho1)
+           : C == 2 ? cg_start<2>(k, kp, rho1) : cg_start<1>(k, kp, rho1);
   rs = block_sum(rs, red);
   const float stop = a.tol * a.tol * rs;
   auto add1 = [&](int i, float v) { rho1[i] += v; };
   auto add2 = [&](int i, float v) { rho2[i] += v; };
-  for (int it = 0; it < a.iters; ++it) {
+  for (int it = 0; it < a.iters && ok; ++it) {
     if (!(rs > stop) || !(rs > 0.f)) break;
-    if (threadIdx.x < 128) rho1[threadIdx.x] = rho2[threadIdx.x] = 0.f;
+    if (threadIdx.x < 128) {
+      rho2[threadIdx.x] = 0.f;
+      if (!split) rho1[threadIdx.x] = 0.f;
+    }
     __syncthreads();
-    // T = P V*^T
-    tc_gemm<true>(c, m, B, kD, parts_v,
+    // T = P V*^T (and rho1 = rowsum(X o T) for an unsplit unit)
+    tc_gemm<true>(c, m, nc, kD, parts_v,
         [&](int r, int t, int nv, float* x) { ld8(k.Pd + (size_t)r * kD + t, nv, x); },
-        [&](int t, int j, int nv, float* x) { vget8(j, t, nv, x); },
-        [&](int r, int j, float v) {
-          k.T[(size_t)r * B + j] = v;
-          return k.X[(size_t)r * B + j] * v;
+        [&](int t, int j, int nv, float* x) { vget8(c0 + j, t, nv, x); },
+        [&](int r, int j) { return split ? 0.f : __ldcg(k.X + (size_t)r * B + c0 + j); },
+        [&](int r, int j, float v, float x) {
+          k.T[(size_t)r * B + c0 + j] = v;
+          return x * v;
         }, add1);
     // T2 = (s^2 Q Q^T) dS on the free columns, dS = X o (T - rho1)
-    tc_gemm<false>(c, m, B, m, kTP,
-        [&](int r, int r2, int nv, float* x) { ld8(k.GQ + (size_t)r * m + r2, nv, x); },
+    tc_gemm<false>(c, m, nc, m, kTP,
+        [&](int r, int r2, int nv, float* x) { ld8cg(k.GQ + (size_t)r * m + r2, nv, x); },
         [&](int r2, int j, int nv, float* x) {
           float t[8];
-          const size_t o = (size_t)r2 * B + j;
-          ld8(k.X + o, nv, x);
+          const size_t o = (size_t)r2 * B + c0 + j;
+          ld8cg(k.X + o, nv, x);
           ld8(k.T + o, nv, t);
           const float rh = nv > 0 ? rho1[r2] : 0.f;
 #pragma unroll
           for (int e = 0; e < 8; ++e) x[e] *= t[e] - rh;
         },
-        [&](int r, int j, float v) {
-          const float t2 = k.fixed[j] ? 0.f : v;
-          k.T2[(size_t)r * B + j] = t2;
-          return k.X[(size_t)r * B + j] * t2;
+        // X (a probability, >= 0) of a free column, -1 for a fixed one
+        [&](int r, int j) {
+          return __ldcg(k.fixed + c0 + j) ? -1.f : __ldcg(k.X + (size_t)r * B + c0 + j);
+        },
+        [&](int r, int j, float v, float x) {
+          const float t2 = x < 0.f ? 0.f : v;
+          k.T2[(size_t)r * B + c0 + j] = t2;
+          return x < 0.f ? 0.f : x * t2;
         }, add2);
-    // Ap = dS2 V* + lambda p, dS2 = X o (T2 - rho2)
-    tc_gemm<false>(c, m, kD, B, parts_v,
+    if (C > 1) {
+      if (threadIdx.x < m) kp.rho2p[(size_t)kp.r * 128 + threadIdx.x] = rho2[threadIdx.x];
+      ok = part_barrier(kp, a.status);
+      if (threadIdx.x < m) {
+        float v = 0.f;
+        for (int q = 0; q < C; ++q) v += __ldcg(kp.rho2p + (size_t)q * 128 + threadIdx.x);
+        rho2[threadIdx.x] = v;
+      }
+      __syncthreads();
+      if (!ok) break;
+    }
+    // the CTA's share of J_G (J_G^T p) = dS2 V*, dS2 = X o (T2 - rho2)
+    tc_gemm<false>(c, m, kD, nc, parts_v,
         [&](int r, int j, int nv, float* x) {
           float t[8];
-          const size_t o = (size_t)r * B + j;
-          ld8(k.X + o, nv, x);
+          const size_t o = (size_t)r * B + c0 + j;
+          ld8cg(k.X + o, nv, x);
           ld8(k.T2 + o, nv, t);
           const float rh = nv > 0 ? rho2[r] : 0.f;
 #pragma unroll
           for (int e = 0; e < 8; ++e) x[e] *= t[e] - rh;
         },
-        [&](int j, int t, int nv, float* x) { vget8(j, t, nv, x); },
-        [&](int r, int t, float v) {
-          const size_t o = (size_t)r * kD + t;
-          k.AP[o] = v + a.lambda_k * k.Pd[o];
+        [&](int j, int t, int nv, float* x) { vget8(c0 + j, t, nv, x); },
+        [](int, int) { return 0.f; },
+        [&](int r, int t, float v, float) {
+          mine[(size_t)r * kD + t] = v;
           return 0.f;
         }, [](int, float) {});
-    float pap = 0.f;
-    for (int i = threadIdx.x; i < md; i += kKT) pap = fmaf(k.Pd[i], k.AP[i], pap);
+    if (C > 1 && !(ok = part_barrier(kp, a.status))) break;
+    // Ap = J_G (J_G^T p) + lambda p
+    float pap = C == 8 ? cg_ap<8>(k, kp, a.lambda_k)
+              : C == 4 ? cg_ap<4>(k, kp, a.lambda_k)
+              : C == 2 ? cg_ap<2>(k, kp, a.lambda_k) : cg_ap<1>(k, kp, a.lambda_k);
     pap = block_sum(pap, red);
     if (!(pap > 0.f)) break;   // the direction has vanished
     const float al = rs / pap;
-    float rn = 0.f;
-    for (int i = threadIdx.x; i < md; i += kKT) {
-      k.AL[i] = fmaf(al, k.Pd[i], k.AL[i]);
-      const float r = fmaf(-al, k.AP[i], k.R[i]);
-      k.R[i] = r;
-      rn = fmaf(r, r, rn);
-    }
-    rn = block_sum(rn, red);
-    const float beta = rn / rs;
-    for (int i = threadIdx.x; i < md; i += kKT) k.Pd[i] = fmaf(beta, k.Pd[i], k.R[i]);
+    const float rn = block_sum(cg_step(k, al), red);
+    cg_dir(k, rn / rs, rho1, split);
     rs = rn;
     __syncthreads();
   }
@@ -670,25 +972,29 @@ __device__ __forceinline__ void stv(void* p, size_t i, int dtype, float v) {
 
 // Key step of Algorithm 1 at t = 0: linearised at K0 (k_out on entry) with
 // V* = v_out; K* to k_out (and, for an alternation, in fp32 to Kt).
-__global__ void __launch_bounds__(kKT) k_key_step(KArgs a) {
+__global__ void __launch_bounds__(kKT, 2) k_key_step(KArgs a) {
   __shared__ int hist[256], sh[64];
   __shared__ float red[kKT / 32];
   __shared__ GemmSmem gs;
   __shared__ float rho[2][128];
   __shared__ uint64_t tc_bar;
   __shared__ uint32_t tc_tmem;
+  __shared__ int part_flag;
   extern __shared__ uint8_t tc_dyn[];
-  const KUnit k(a, blockIdx.x);
+  const int C = a.cluster, u = blockIdx.x / C, rank = blockIdx.x - u * C;
+  const KUnit k(a, u, rank);
   const int B = k.B, dt = a.dtype;
   TcCtx tc{};
   if (a.use_tc) tc_setup(tc, tc_dyn, &tc_tmem, &tc_bar, a.status);
-  fixed_set(a, k, hist, sh);
-  retained_softmax(a, k, gs, [&](int j, int t) { return ldv(a.k_out, k.kv_off + (size_t)j * kD + t, dt); });
   auto vget = [&](int j, int t) { return ldv(a.v_out, k.kv_off + (size_t)j * kD + t, dt); };
-  // e = Y - X V*
-  block_gemm(gs,
-      k.m, kD, B, [&](int r, int j) { return k.X[(size_t)r * B + j]; }, vget,
-      [&](int r, int t, float v) { k.R[(size_t)r * kD + t] = k.Y[(size_t)r * kD + t] - v; });
+  if (rank == 0) {
+    fixed_set(a, k, hist, sh);
+    retained_softmax(a, k, gs, [&](int j, int t) { return ldv(a.k_out, k.kv_off + (size_t)j * kD + t, dt); });
+    // e = Y - X V*
+    block_gemm(gs,
+        k.m, kD, B, [&](int r, int j) { return k.X[(size_t)r * B + j]; }, vget,
+        [&](int r, int t, float v) { k.R[(size_t)r * kD + t] = k.Y[(size_t)r * kD + t] - v; });
+  }
   if (a.use_tc) {
     // V* row j, columns t .. t+nv
     auto vget8 = [&](int j, int t, int nv, float* x) {
@@ -698,8 +1004,20 @@ __global__ void __launch_bounds__(kKT) k_key_step(KArgs a) {
       else
         ld8((const float*)a.v_out + o, nv, x);
     };
-    key_cg_tc(a, k, gs, red, tc, rho[0], rho[1], dt == GRKV_BF16 ? 1 : kTP, vget, vget8);
+    // rank r carries columns [r * Bc, r * Bc + Bc) (the last rank the rest)
+    const int Bc = ((B + C - 1) / C + 7) / 8 * 8;
+    KPart kp{};
+    kp.C = C;
+    kp.r = rank;
+    kp.c0 = min(B, rank * Bc);
+    kp.nc = min(B, kp.c0 + Bc) - kp.c0;
+    kp.app = C > 1 ? a.app + (size_t)u * C * k.m * kD : k.AP;
+    kp.rho2p = C > 1 ? a.rho2p + (size_t)u * C * 128 : nullptr;
+    kp.cnt = C > 1 ? a.cnt + u : nullptr;
+    kp.flag = &part_flag;
+    key_cg_tc(a, k, gs, red, tc, kp, rho[0], rho[1], dt == GRKV_BF16 ? 1 : kTP, vget8);
     tc_release(tc);
+    if (rank != 0) return;
   } else {
     key_cg(a, k, gs, red, vget);
   }
@@ -745,7 +1063,7 @@ __device__ bool block_cholesky(float* G, int m, int* flag) {
 // step linearised at K^(t) (right-hand side e + J_G (K^(t) - K0)).  Writes
 // V^(t+1), K^(t+1) to v_out / k_out (rounded) and to Vt / Kt (fp32), and
 // marks the unit done once both changes are <= step_tol.
-__global__ void __launch_bounds__(kKT) k_alternate_step(KArgs a) {
+__global__ void __launch_bounds__(kKT, 2) k_alternate_step(KArgs a) {
   __shared__ int hist[256], sh[64];
   __shared__ float red[kKT / 32];
   __shared__ GemmSmem gs;
@@ -847,7 +1165,12 @@ __global__ void __launch_bounds__(kKT) k_alternate_step(KArgs a) {
     auto vget8 = [&](int j, int t, int nv, float* x) {
       ld8(a.Vt + k.kv_off + (size_t)j * kD + t, nv, x);
     };
-    key_cg_tc(a, k, gs, red, tc, rho[0], rho[1], kTP, vget, vget8);
+    KPart kp{};
+    kp.C = 1;
+    kp.nc = B;
+    kp.app = k.AP;
+    kp.flag = &flag;
+    key_cg_tc(a, k, gs, red, tc, kp, rho[0], rho[1], kTP, vget8);
     tc_release(tc);
   } else {
     key_cg(a, k, gs, red, vget);
@@ -878,19 +1201,57 @@ __global__ void __launch_bounds__(kKT) k_alternate_step(KArgs a) {
 
 }  // namespace
 
-size_t key_ws_bytes(const Shape& s) {
-  const size_t U = (size_t)s.U, m = (size_t)s.m, B = (size_t)s.B, d = (size_t)kD;
-  size_t bytes = U * (3 * m * B * 4 + B * d * 4 + 4 * m * d * 4 + m * m * 4 + B) + 1024;
-  if (s.steps > 1) bytes += U * (2 * B * d * 4 + m * m * 4 + m * d * 4 + 4) + 1024;
-  return bytes;
+// CTAs per unit in k_key_step: with few units, a unit's CG products are split
+// over up to 8 CTAs (at least 64 retained columns each) while the units
+// times the split stay within one CTA per SM of a GB300 (152 SMs).
+constexpr int kKeySms = 152;
+int key_cluster(const Shape& s) {
+  if (s.m > 128) return 1;   // the fp32 CUDA-core CG runs one CTA per unit
+  int c = 1;
+  while (c < 8 && (long long)s.U * 2 * c <= kKeySms && s.B >= 2 * c * 64) c *= 2;
+  return c;
 }
+
+namespace {
+size_t a256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// Regions of the key step's workspace (offsets from its base, 256-aligned).
+struct KeyLayout {
+  size_t vec, app, rho2p, cnt, X, T, dK, T2, GQ, fixed, alt, total;
+};
+KeyLayout key_layout(const Shape& s, int C) {
+  const size_t U = (size_t)s.U, m = (size_t)s.m, B = (size_t)s.B, d = (size_t)kD;
+  KeyLayout l{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off = a256(off + bytes);
+    return o;
+  };
+  l.vec = take(U * C * 5 * m * d * 4);
+  l.app = take(C > 1 ? U * C * m * d * 4 : 0);
+  l.rho2p = take(C > 1 ? U * C * 128 * 4 : 0);
+  l.cnt = take(C > 1 ? U * 4 : 0);
+  l.X = take(U * m * B * 4);
+  l.T = take(U * m * B * 4);
+  l.dK = take(U * B * d * 4);
+  l.T2 = take(U * m * B * 4);
+  l.GQ = take(U * m * m * 4);
+  l.fixed = take(U * B);
+  l.alt = take(s.steps > 1 ? U * (2 * B * d * 4 + m * m * 4 + m * d * 4 + 4) + 1024 : 0);
+  l.total = off;
+  return l;
+}
+}  // namespace
+
+size_t key_ws_bytes(const Shape& s) { return key_layout(s, key_cluster(s)).total + 256; }
 
 cudaError_t launch_key_step(const Shape& s, const void* q, const void* k, const void* v,
                             const float* y, const float* scores, const int32_t* idx,
                             void* v_out, void* k_out, char* ws, const WsLayout& L,
                             cudaStream_t st) {
   const size_t U = (size_t)s.U, m = (size_t)s.m, B = (size_t)s.B, d = (size_t)kD;
-  char* base = ws + L.key;
+  char* base = (char*)(((uintptr_t)(ws + L.key) + 255) & ~(uintptr_t)255);
   KArgs a{};
   a.n = s.n;
   a.w = s.w;
@@ -917,23 +1278,6 @@ cudaError_t launch_key_step(const Shape& s, const void* q, const void* k, const 
   a.v_out = v_out;
   a.k_out = k_out;
   a.status = (int*)(ws + L.status);
-  a.X = (float*)base;
-  a.T = a.X + U * m * B;
-  a.dK = a.T + U * m * B;
-  a.vec = a.dK + U * B * d;
-  a.T2 = a.vec + U * 4 * m * d;
-  a.GQ = a.T2 + U * m * B;
-  a.fixed = (uint8_t*)(a.GQ + U * m * m);
-  if (s.steps > 1) {
-    char* alt = (char*)(((uintptr_t)(a.fixed + U * B) + 255) & ~(uintptr_t)255);
-    a.Kt = (float*)alt;
-    a.Vt = a.Kt + U * B * d;
-    a.G = a.Vt + U * B * d;
-    a.RZ = a.G + U * m * m;
-    a.done = (int*)(a.RZ + U * m * d);
-    cudaError_t e = cudaMemsetAsync(a.done, 0, U * sizeof(int), st);
-    if (e != cudaSuccess) return e;
-  }
   a.use_tc = s.m <= 128;
   const uint32_t dyn = a.use_tc ? kTcSmem : 0;
   cudaError_t e = cudaFuncSetAttribute(k_key_step, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -942,9 +1286,61 @@ cudaError_t launch_key_step(const Shape& s, const void* q, const void* k, const 
     e = cudaFuncSetAttribute(k_alternate_step, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)kTcSmem);
   if (e != cudaSuccess) return e;
+  // the split the workspace was sized for, halved while the device cannot
+  // hold a cluster of that many CTAs
+  int C = key_cluster(s);
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  cfg.blockDim = dim3(kKT);
+  cfg.dynamicSmemBytes = dyn;
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  for (; C > 1; C /= 2) {
+    cfg.gridDim = dim3((unsigned)(U * C));
+    attr[0].val.clusterDim.x = C;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    int nclusters = 0;
+    if (cudaOccupancyMaxActiveClusters(&nclusters, k_key_step, &cfg) == cudaSuccess &&
+        nclusters > 0)
+      break;
+    (void)cudaGetLastError();
+  }
+  const KeyLayout kl = key_layout(s, C);
+  a.cluster = C;
+  a.vec = (float*)(base + kl.vec);
+  a.app = (float*)(base + kl.app);
+  a.rho2p = (float*)(base + kl.rho2p);
+  a.cnt = (int*)(base + kl.cnt);
+  a.X = (float*)(base + kl.X);
+  a.T = (float*)(base + kl.T);
+  a.dK = (float*)(base + kl.dK);
+  a.T2 = (float*)(base + kl.T2);
+  a.GQ = (float*)(base + kl.GQ);
+  a.fixed = (uint8_t*)(base + kl.fixed);
+  if (s.steps > 1) {
+    char* alt = base + kl.alt;
+    a.Kt = (float*)alt;
+    a.Vt = a.Kt + U * B * d;
+    a.G = a.Vt + U * B * d;
+    a.RZ = a.G + U * m * m;
+    a.done = (int*)(a.RZ + U * m * d);
+    e = cudaMemsetAsync(a.done, 0, U * sizeof(int), st);
+    if (e != cudaSuccess) return e;
+  }
   count_launches(1);
-  k_key_step<<<s.U, kKT, dyn, st>>>(a);
-  e = cudaGetLastError();
+  if (C > 1) {
+    e = cudaMemsetAsync(a.cnt, 0, U * sizeof(int), st);
+    if (e != cudaSuccess) return e;
+    cfg.gridDim = dim3((unsigned)(U * C));
+    attr[0].val.clusterDim.x = C;
+    e = cudaLaunchKernelEx(&cfg, k_key_step, a);
+  } else {
+    k_key_step<<<s.U, kKT, dyn, st>>>(a);
+    e = cudaGetLastError();
+  }
   for (int t = 1; t < s.steps && e == cudaSuccess; ++t) {
     a.vt_valid = t > 1;   // V^(1) exists only as written to v_out (rounded)
     count_launches(1);

@@ -328,12 +328,16 @@ def test_full_size_c4_sweep_point(grkv_lib, wl):
 
 # --------------------------------------------------------------- key step --
 EDGE_KEY = gi.Workload("edge_n600", 2, 2, 600, 128, 8, 64, 7, 1e-2, "bf16", "lowrank", 4242)
+# B = 300 with m = 128: the CG products of a unit are split over 4 CTAs with
+# 80, 80, 80 and 60 retained columns (a ragged last share)
+SPLIT_KEY = gi.Workload("split_b300", 2, 4, 3000, 128, 32, 300, 7, 1e-2, "bf16", "lowrank", 4343)
 KEY_CASES = {
     # workload, path flags, lambda_k (1e-2 Llama default, 1e-1 Mistral default)
     "c0_f32_portable": (gi.workload(0), 0, 1e-2),
     "c1_bf16_default": (gi.workload(1).replace(units=2), 0, 1e-1),
     "c1_bf16_portable": (gi.workload(1).replace(units=2), b.GRKV_FORCE_SIMT, 1e-1),
     "edge_bf16_default": (EDGE_KEY, 0, 1e-2),
+    "split_ragged_bf16": (SPLIT_KEY, 0, 1e-2),
 }
 
 
