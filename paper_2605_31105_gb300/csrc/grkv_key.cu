@@ -246,19 +246,6 @@ __device__ __forceinline__ void split3(const float* x, uint4* part) {
   for (int q = 0; q < 3; ++q) part[q] = make_uint4(p[q][0], p[q][1], p[q][2], p[q][3]);
 }
 
-// x[0..8) = p[0..nv) read through L2 only: data another CTA of the unit
-// wrote (L1 is not coherent across SMs).
-__device__ __forceinline__ void ld8cg(const float* p, int nv, float* x) {
-  if (nv == 8 && ((uintptr_t)p & 15) == 0) {
-    const float4 a = __ldcg((const float4*)p), b = __ldcg((const float4*)(p + 4));
-    x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w;
-    x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
-  } else {
-#pragma unroll
-    for (int e = 0; e < 8; ++e) x[e] = e < nv ? __ldcg(p + e) : 0.f;
-  }
-}
-
 // C = A B for A [M][K] (M <= 128) and B [K][N], B staged K-major ([N] rows of
 // K, kBK) or MN-major ([K] rows of N); parts_b = 1 when B is exact in bf16.
 // Operands come in chunks of eight along their contiguous index:
@@ -686,9 +673,8 @@ __device__ __forceinline__ float4 sum_parts(const float* app, size_t md, int i) 
   return v;
 }
 
-// Start of CG: r = p = e (rank 0's r), alpha = 0 and, for a split unit
-// (kC > 1), X V* = sum of the partials and rho1 = rowsum(p o X V*); returns
-// the thread's share of ||e||^2.
+// Start of CG: X V* = sum of the partials, r = p = e (rank 0's r), alpha = 0,
+// rho1 = rowsum(p o X V*); returns the thread's share of ||e||^2.
 template <int kC>
 __device__ float cg_start(const KUnit& k, const KPart& kp, float* rho1) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, m = k.m;
@@ -699,7 +685,7 @@ __device__ float cg_start(const KUnit& k, const KPart& kp, float* rho1) {
 #pragma unroll
     for (int b = 0; b < 2; ++b) {
       const int r = r0 + b * kWarps, i = r * 32 + lane;
-      xv[b] = kC > 1 && r < m ? sum_parts<kC>(kp.app, md, i) : make_float4(0.f, 0.f, 0.f, 0.f);
+      xv[b] = r < m ? sum_parts<kC>(kp.app, md, i) : make_float4(0.f, 0.f, 0.f, 0.f);
       e[b] = r < m ? __ldcg((const float4*)k.E + i) : make_float4(0.f, 0.f, 0.f, 0.f);
     }
 #pragma unroll
@@ -710,11 +696,9 @@ __device__ float cg_start(const KUnit& k, const KPart& kp, float* rho1) {
       ((float4*)k.Pd)[i] = e[b];
       ((float4*)k.AL)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
       rs = dot4(e[b], e[b], rs);
-      if (kC > 1) {
-        ((float4*)k.XV)[i] = xv[b];
-        const float d = warp_sum(dot4(e[b], xv[b], 0.f));
-        if (lane == 0) rho1[r] = d;
-      }
+      ((float4*)k.XV)[i] = xv[b];
+      const float d = warp_sum(dot4(e[b], xv[b], 0.f));
+      if (lane == 0) rho1[r] = d;
     }
   }
   return rs;
@@ -785,9 +769,8 @@ __device__ float cg_step(const KUnit& k, float al) {
   return rn;
 }
 
-// p = r + beta p and, for a split unit, the next iteration's rho1 =
-// rowsum(p o X V*).
-__device__ void cg_dir(const KUnit& k, float beta, float* rho1, bool split) {
+// p = r + beta p and the next iteration's rho1 = rowsum(p o X V*).
+__device__ void cg_dir(const KUnit& k, float beta, float* rho1) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, m = k.m;
   for (int r0 = warp; r0 < m; r0 += 4 * kWarps) {
     float4 pd[4], rr[4], xv[4];
@@ -796,7 +779,7 @@ __device__ void cg_dir(const KUnit& k, float beta, float* rho1, bool split) {
       const int r = min(r0 + b * kWarps, m - 1), i = r * 32 + lane;
       pd[b] = ((const float4*)k.Pd)[i];
       rr[b] = ((const float4*)k.R)[i];
-      xv[b] = split ? ((const float4*)k.XV)[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+      xv[b] = ((const float4*)k.XV)[i];
     }
 #pragma unroll
     for (int b = 0; b < 4; ++b) {
@@ -808,10 +791,8 @@ __device__ void cg_dir(const KUnit& k, float beta, float* rho1, bool split) {
       p4.z = fmaf(beta, pd[b].z, p4.z);
       p4.w = fmaf(beta, pd[b].w, p4.w);
       ((float4*)k.Pd)[i] = p4;
-      if (split) {
-        const float d = warp_sum(dot4(p4, xv[b], 0.f));
-        if (lane == 0) rho1[r] = d;
-      }
+      const float d = warp_sum(dot4(p4, xv[b], 0.f));
+      if (lane == 0) rho1[r] = d;
     }
   }
 }
@@ -819,10 +800,13 @@ __device__ void cg_dir(const KUnit& k, float beta, float* rho1, bool split) {
 // key_cg with the three products of an iteration on the tensor cores
 // (m <= 128), over the CTA's columns of kp.  The softmax Jacobians are
 // applied as the next product stages its operand.  Their row sums are
-// rho1 = rowsum(X o T) and rho2 = rowsum(X o T2), taken in the epilogues of
-// the products that write T and T2; a unit split over C > 1 CTAs takes
-// rho1 = rowsum(P o (X V*)) instead, with X V* formed once, which needs no
-// exchange.
+//   rho1 = rowsum(X o (P V*^T)) = rowsum(P o (X V*)),  with X V* formed once,
+//   rho2 = rowsum(X o T2), taken in the epilogue of the product writing T2,
+// so that rho1 needs neither a pass over X nor, for a split unit, an exchange.
+// X, the query Gram and the fixed flags are written by rank 0 before the
+// first barrier and never again, and no other SM has read them before it,
+// so plain (L1-cached) loads see them; the partials, rewritten every
+// iteration by other CTAs, are read through L2 (__ldcg).
 template <class FV8>
 __device__ void key_cg_tc(const KArgs& a, const KUnit& k, GemmSmem& gs, float* red, TcCtx& c,
                           KPart& kp, float* rho1, float* rho2, int parts_v, FV8 vget8) {
@@ -837,48 +821,42 @@ __device__ void key_cg_tc(const KArgs& a, const KUnit& k, GemmSmem& gs, float* r
         [&](int r, int r2, float v) { k.GQ[(size_t)r * m + r2] = s * s * v; });
   const bool split = C > 1;
   bool ok = !split || part_barrier(kp, a.status);
-  if (split) {
-    // X V* over the CTA's columns, summed over the ranks in cg_start
-    tc_gemm<false>(c, m, kD, nc, parts_v,
-        [&](int r, int j, int nv, float* x) { ld8cg(k.X + (size_t)r * B + c0 + j, nv, x); },
-        [&](int j, int t, int nv, float* x) { vget8(c0 + j, t, nv, x); },
-        [](int, int) { return 0.f; },
-        [&](int r, int t, float v, float) {
-          mine[(size_t)r * kD + t] = v;
-          return 0.f;
-        }, [](int, float) {});
-    if (ok) ok = part_barrier(kp, a.status);
-  }
+  // X V* over the CTA's columns, summed over the ranks in cg_start
+  tc_gemm<false>(c, m, kD, nc, parts_v,
+      [&](int r, int j, int nv, float* x) { ld8(k.X + (size_t)r * B + c0 + j, nv, x); },
+      [&](int j, int t, int nv, float* x) { vget8(c0 + j, t, nv, x); },
+      [](int, int) { return 0.f; },
+      [&](int r, int t, float v, float) {
+        mine[(size_t)r * kD + t] = v;
+        return 0.f;
+      }, [](int, float) {});
+  if (split && ok) ok = part_barrier(kp, a.status);
   float rs = C == 8 ? cg_start<8>(k, kp, rho1)
            : C == 4 ? cg_start<4>(k, kp, rho1)
            : C == 2 ? cg_start<2>(k, kp, rho1) : cg_start<1>(k, kp, rho1);
   rs = block_sum(rs, red);
   const float stop = a.tol * a.tol * rs;
-  auto add1 = [&](int i, float v) { rho1[i] += v; };
   auto add2 = [&](int i, float v) { rho2[i] += v; };
   for (int it = 0; it < a.iters && ok; ++it) {
     if (!(rs > stop) || !(rs > 0.f)) break;
-    if (threadIdx.x < 128) {
-      rho2[threadIdx.x] = 0.f;
-      if (!split) rho1[threadIdx.x] = 0.f;
-    }
+    if (threadIdx.x < 128) rho2[threadIdx.x] = 0.f;
     __syncthreads();
-    // T = P V*^T (and rho1 = rowsum(X o T) for an unsplit unit)
+    // T = P V*^T
     tc_gemm<true>(c, m, nc, kD, parts_v,
         [&](int r, int t, int nv, float* x) { ld8(k.Pd + (size_t)r * kD + t, nv, x); },
         [&](int t, int j, int nv, float* x) { vget8(c0 + j, t, nv, x); },
-        [&](int r, int j) { return split ? 0.f : __ldcg(k.X + (size_t)r * B + c0 + j); },
-        [&](int r, int j, float v, float x) {
+        [](int, int) { return 0.f; },
+        [&](int r, int j, float v, float) {
           k.T[(size_t)r * B + c0 + j] = v;
-          return x * v;
-        }, add1);
+          return 0.f;
+        }, [](int, float) {});
     // T2 = (s^2 Q Q^T) dS on the free columns, dS = X o (T - rho1)
     tc_gemm<false>(c, m, nc, m, kTP,
-        [&](int r, int r2, int nv, float* x) { ld8cg(k.GQ + (size_t)r * m + r2, nv, x); },
+        [&](int r, int r2, int nv, float* x) { ld8(k.GQ + (size_t)r * m + r2, nv, x); },
         [&](int r2, int j, int nv, float* x) {
           float t[8];
           const size_t o = (size_t)r2 * B + c0 + j;
-          ld8cg(k.X + o, nv, x);
+          ld8(k.X + o, nv, x);
           ld8(k.T + o, nv, t);
           const float rh = nv > 0 ? rho1[r2] : 0.f;
 #pragma unroll
@@ -886,7 +864,7 @@ __device__ void key_cg_tc(const KArgs& a, const KUnit& k, GemmSmem& gs, float* r
         },
         // X (a probability, >= 0) of a free column, -1 for a fixed one
         [&](int r, int j) {
-          return __ldcg(k.fixed + c0 + j) ? -1.f : __ldcg(k.X + (size_t)r * B + c0 + j);
+          return k.fixed[c0 + j] ? -1.f : k.X[(size_t)r * B + c0 + j];
         },
         [&](int r, int j, float v, float x) {
           const float t2 = x < 0.f ? 0.f : v;
@@ -909,7 +887,7 @@ __device__ void key_cg_tc(const KArgs& a, const KUnit& k, GemmSmem& gs, float* r
         [&](int r, int j, int nv, float* x) {
           float t[8];
           const size_t o = (size_t)r * B + c0 + j;
-          ld8cg(k.X + o, nv, x);
+          ld8(k.X + o, nv, x);
           ld8(k.T2 + o, nv, t);
           const float rh = nv > 0 ? rho2[r] : 0.f;
 #pragma unroll
@@ -930,7 +908,7 @@ __device__ void key_cg_tc(const KArgs& a, const KUnit& k, GemmSmem& gs, float* r
     if (!(pap > 0.f)) break;   // the direction has vanished
     const float al = rs / pap;
     const float rn = block_sum(cg_step(k, al), red);
-    cg_dir(k, rn / rs, rho1, split);
+    cg_dir(k, rn / rs, rho1);
     rs = rn;
     __syncthreads();
   }
