@@ -63,7 +63,7 @@ struct WsLayout {
   size_t scores;  // float [U][P]
   size_t y;       // float [U][m][d]
   size_t rstats;  // float2 [U][m]
-  size_t key;     // key step: X, T [U][m][B], dK [U][B][d], CG vectors [U][4][m][d], fixed [U][B]
+  size_t key;     // key step: CG vectors [U][C][5][m][d], X, T, T2 [U][m][B], dK [U][B][d], fixed [U][B]
   size_t total;
 };
 

@@ -1,6 +1,8 @@
-// Key step of Algorithm 1 at t = 0 (Sec. 3.4 "Key step", App. D.2), one CTA
-// per unit: fp32 on CUDA cores, with the CG products on the tensor cores
-// (three-part bf16 splits of the fp32 operands) when m <= 128.
+// Key step of Algorithm 1 at t = 0 (Sec. 3.4 "Key step", App. D.2): fp32 on
+// CUDA cores, with the CG products on the tensor cores (three-part bf16
+// splits of the fp32 operands) when m <= 128.  One CTA per unit, or, when
+// units are few, a cluster of up to 8 CTAs per unit that split the CG
+// products by retained columns (KPart).
 //
 // With the merged values V* of the value step fixed, f(K) = softmax(s Q K^T) V*
 // is linearised at K0 and the local ridge problem is solved in its dual form:
